@@ -1,0 +1,57 @@
+"""Packing of retained units into contiguous INT8 panels (Sec. 3.3, Appendix
+"Backing-store semantics"). Test infrastructure only.
+
+The paper packs each mask's retained heads and channels into contiguous
+tensors over one shared INT8 store. The panel layout the build uses (and
+which the library's panels must match byte for byte) is:
+
+* ``qkv``  [(m_q + 2 m_kv) d_h, d]: for each kept group j in ascending order,
+  the d_h rows of each of its g query heads (heads j g .. j g + g - 1), then
+  the d_h rows of K head j, then the d_h rows of V head j.
+* ``o``    [d, m_q d_h]: the O-projection columns of the kept query heads in
+  ascending head order; scales are the dense per-row scales [d].
+* ``gu``   [2 c, d]: for each kept channel c_i in ascending order, the gate
+  row c_i then the up row c_i.
+* ``down`` [d, c]: the down-projection columns of the kept channels; scales
+  are the dense per-row scales [d].
+
+The all-keep mask packs to the shared store itself.
+
+Pin: the compacted forward (oracle.forward, ``compact=True``) consumes these
+panels and must equal the mask-as-zero forward; a permuted or misaligned
+panel fails that test.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def qkv_rows(shape, keep_groups):
+    """Dense-matrix row sources of the qkv panel: list of (proj, row)."""
+    rows = []
+    g, dh = shape.g, shape.dh
+    for j in keep_groups:
+        for h in range(j * g, (j + 1) * g):
+            rows += [("q", h * dh + i) for i in range(dh)]
+        rows += [("k", j * dh + i) for i in range(dh)]
+        rows += [("v", j * dh + i) for i in range(dh)]
+    return rows
+
+
+def pack_layer(shape, lq, keep_groups, keep_chans) -> dict:
+    g, dh = shape.g, shape.dh
+    src = qkv_rows(shape, keep_groups)
+    qkv_w = np.stack([lq.q[p][r] for p, r in src]) if src else np.zeros((0, shape.d), np.int8)
+    qkv_s = np.array([lq.s[p][r] for p, r in src], dtype=np.float32)
+    ocols = [h * dh + i for j in keep_groups for h in range(j * g, (j + 1) * g) for i in range(dh)]
+    o_w = np.ascontiguousarray(lq.q["o"][:, ocols])
+    kc = np.asarray(keep_chans, dtype=np.int64)
+    gu_w = np.empty((2 * len(kc), shape.d), dtype=np.int8)
+    gu_w[0::2] = lq.q["gate"][kc]
+    gu_w[1::2] = lq.q["up"][kc]
+    gu_s = np.empty(2 * len(kc), dtype=np.float32)
+    gu_s[0::2] = lq.s["gate"][kc]
+    gu_s[1::2] = lq.s["up"][kc]
+    down_w = np.ascontiguousarray(lq.q["down"][:, kc])
+    return dict(qkv_w=qkv_w, qkv_s=qkv_s, o_w=o_w, o_s=lq.s["o"].copy(), gu_w=gu_w, gu_s=gu_s,
+                down_w=down_w, down_s=lq.s["down"].copy())
