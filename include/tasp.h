@@ -1,0 +1,232 @@
+/*
+ * tasp.h - C ABI of the TASP compiled sparse execution path on one GB300 (sm_103a).
+ *
+ * The path (paper Sec. 3.3 and Appendix "Backing-store semantics"): one shared,
+ * immutable INT8 weight store per model; a mask is a dependency-closed set of
+ * retained GQA groups and SwiGLU channel units, compiled into a plan (retained
+ * index lists + packed panels + launch geometry) that owns no weights it does
+ * not need; one plan is chosen per user turn and stays fixed through prefill
+ * and every decode step; a KV cache is never reused across plans.
+ *
+ * Conventions for every function below:
+ *  - Return value: TASP_OK (0) or a negative tasp_status. Nothing aborts. On
+ *    failure tasp_last_error() returns a thread-local description.
+ *  - Pointers named d_* are DEVICE pointers owned by the caller; h_* are HOST
+ *    pointers owned by the caller. All other objects (store, plans, sessions
+ *    and their device memory) are owned by the library and freed with
+ *    tasp_release().
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Functions marked "async" enqueue work on it and return without
+ *    synchronizing; their device outputs are valid once the stream reaches
+ *    that point. Functions marked "sync" synchronize the device before return.
+ *  - BF16 buffers hold IEEE bfloat16 bit patterns (uint16); FP32 buffers hold
+ *    float. Matrices are row-major.
+ *  - All sizes are element counts unless the name says bytes.
+ */
+#ifndef TASP_H
+#define TASP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum tasp_status {
+    TASP_OK = 0,
+    TASP_EINVAL = -1, /* bad shape, pointer, mask (closure violated, budget exceeded, empty layer) */
+    TASP_EMASK = -2,  /* sessions of different plans in one decode call (KV reuse across masks, Sec. 3.3) */
+    TASP_ECAP = -3,   /* KV-cache capacity of a session exhausted */
+    TASP_ENOMEM = -4, /* device or host allocation failed */
+    TASP_EBUSY = -5,  /* plan released while sessions still reference it */
+    TASP_ECUDA = -6,  /* a CUDA call failed; tasp_last_error() holds the CUDA error string */
+    TASP_EUNSUP = -7  /* valid request this build does not implement */
+} tasp_status;
+
+/* Shape of a Llama-style decoder (Sec. 3.3 / Table 1) and the seed of its
+ * synthetic weights. Requirements: Hq % Hkv == 0, dh even and a multiple of 16
+ * (dh <= 128), d % 16 == 0, df % chan_unit == 0, vocab >= 0 (0 = no LM head).
+ * The library regenerates the weights from `seed` with its counter-based
+ * generator (N(0, 0.02), quantized per output row to INT8 with FP32 scales). */
+typedef struct tasp_model_desc {
+    int32_t L, d, Hq, Hkv, dh, df, vocab;
+    int32_t chan_unit; /* SwiGLU channels per mask unit (1,024 in Table 1) */
+    float rms_eps;     /* RMSNorm epsilon (1e-5) */
+    float rope_theta;  /* rotary base (500000) */
+    uint64_t seed;
+} tasp_model_desc;
+
+enum tasp_mask_kind {
+    TASP_MASK_ALL_KEEP = 0, /* dense fallback: every unit retained; panels are the store itself */
+    TASP_MASK_GREEDY = 1,   /* budgeted greedy by score per active FLOP with closure (Sec. 3.3) */
+    TASP_MASK_EXPLICIT = 2  /* caller-given retained groups / channel units per layer */
+};
+
+enum tasp_panel_mode {
+    TASP_PANELS_COMPACT = 0,    /* all four panels are packed copies (contiguous retained tensors) */
+    TASP_PANELS_ROW_INDEXED = 1 /* Q/K/V and gate/up rows index the shared store (zero copy);
+                                   O and down columns are packed copies. Same bytes are read. */
+};
+
+/* Mask request. For kind GREEDY: `scores` is host uint32 [L][Hkv + df/chan_unit]
+ * (stand-ins for the predictor scores s_h of Sec. 3.3; groups first, then
+ * channel units), `target_u24` is host uint32 [L] with per-layer retention
+ * draws in [0, 2^24), `flop_budget` the active-FLOP target (0.57) and
+ * [r_lo, r_hi] the per-layer retention range. For kind EXPLICIT:
+ * keep_groups / keep_units are host int32 lists concatenated over layers with
+ * n_groups / n_units [L] giving each layer's count (indices ascending).
+ * Unused fields may be NULL / 0. */
+typedef struct tasp_mask_desc {
+    int32_t kind;
+    int32_t panel_mode;
+    double flop_budget, r_lo, r_hi;
+    const uint32_t* scores;
+    const uint32_t* target_u24;
+    const int32_t* keep_groups;
+    const int32_t* n_groups;
+    const int32_t* keep_units;
+    const int32_t* n_units;
+} tasp_mask_desc;
+
+typedef struct tasp_plan tasp_plan;
+typedef struct tasp_session tasp_session;
+
+/* ---------------------------------------------------------------------------
+ * The four entry points of the path.
+ * ------------------------------------------------------------------------- */
+
+/* Compile one mask into a plan (Sec. 3.3 "packed into contiguous tensors and
+ * compiled as static launch plans over one shared INT8 weight store";
+ * Appendix "Backing-store semantics"). Creates the model's shared store on
+ * first use (generated and quantized on the device; later plans with an
+ * identical model_desc share it), runs the host mask compiler, packs the
+ * panels on the device. sync. *out receives the plan.
+ * Errors: EINVAL (bad desc, mask violates closure/budget, empty layer),
+ * ENOMEM, ECUDA. */
+int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out);
+
+/* Prefill one prompt with a plan (Sec. 3.3: the plan chosen for a turn serves
+ * its prefill; Fig. 1 "one launch plan for prefill"): d_embeds_bf16 is a device
+ * BF16 [T][d] buffer of input embeddings. Creates a session whose KV cache
+ * (retained KV heads only, capacity T + max_new_tokens) holds the prompt's
+ * keys/values. If d_logits_last != NULL it receives FP32 [vocab] logits of the
+ * last prompt position. async on `stream`. *out receives the session.
+ * Errors: EINVAL, ENOMEM, ECUDA, EUNSUP (vocab == 0 with d_logits_last). */
+int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t max_new_tokens, void* stream,
+                 tasp_session** out, float* d_logits_last);
+
+/* One decode step for n >= 1 sessions that share one plan (Fig. 1 "same plan
+ * for every decode step"). d_x_bf16 is device BF16 [n][d] (the step's input
+ * vectors, session order). Outputs, each optional (NULL skips it):
+ * d_hidden_out FP32 [n][d] = the residual stream after the last decoder layer
+ * (before the final norm); d_logits FP32 [n][vocab]. Each session's KV grows by
+ * one position. The step is replayed from a CUDA graph captured on first use
+ * for this (sessions, buffers) combination; call it outside any stream capture.
+ * async on `stream`.
+ * Errors: EMASK (sessions on different plans), ECAP (a session is full),
+ * EINVAL, ENOMEM, ECUDA. */
+int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,
+                     float* d_logits, void* stream);
+
+/* Release a plan or a session (the handle's type is recorded inside). A plan
+ * still referenced by live sessions returns EBUSY and stays valid. The shared
+ * store is freed with its last plan. sync. NULL is a no-op. */
+int tasp_release(void* handle);
+
+/* ---------------------------------------------------------------------------
+ * Sessions without prefill, host-buffer decode, host-only mask compilation.
+ * ------------------------------------------------------------------------- */
+
+/* Empty session on a plan with KV capacity max_tokens (position 0). sync. */
+int tasp_session_create(tasp_plan* plan, int32_t max_tokens, tasp_session** out);
+
+/* Fill positions [0, t_prior) of a session's KV cache with the synthetic
+ * N(0,1) BF16 "prior tokens" keyed by kv_seed (the keys are taken as already
+ * rotated) and set its position to t_prior. async. Errors: ECAP, EINVAL. */
+int tasp_session_fill_synthetic(tasp_session* s, int32_t t_prior, uint64_t kv_seed, void* stream);
+
+/* Current position (number of cached tokens) as tracked on the host. */
+int tasp_session_position(const tasp_session* s, int32_t* pos);
+
+/* tasp_decode_step with HOST buffers: h_x_bf16 [n][d] is copied to the device
+ * (should be pinned memory), the step runs, and the requested outputs are
+ * copied back to h_hidden_out [n][d] / h_logits [n][vocab] (either may be
+ * NULL). Synchronizes `stream` before returning. */
+int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* h_x_bf16, float* h_hidden_out,
+                          float* h_logits, void* stream);
+
+/* Host-only mask compilation (no GPU work): the retained index lists the plan
+ * would use. Outputs (host, caller-sized): keep_groups [L*Hkv] and keep_units
+ * [L*(df/chan_unit)] concatenated per layer with counts n_groups [L],
+ * n_units [L]; flops [L + 3] = per-layer retained FLOPs (Eqs. flop-attn +
+ * flop-mlp), the total, the global budget B and the dense total. */
+int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
+                     int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops);
+
+/* ---------------------------------------------------------------------------
+ * Introspection and measurement (tests and benchmark).
+ * ------------------------------------------------------------------------- */
+
+typedef struct tasp_plan_info {
+    int32_t L;
+    int64_t panel_bytes;   /* device bytes owned by the plan (packed panels, maps, scales) */
+    int64_t store_bytes;   /* device bytes of the shared store (INT8, scales, gains, LM head) */
+    int64_t weight_bytes_per_token; /* INT8 panel bytes + FP32 scales + BF16 LM head read per decode token */
+    int64_t flops_retained, flops_dense; /* layer FLOPs per token, Eqs. flop-attn + flop-mlp */
+    int64_t launched_flops; /* 2 x rows x cols over the packed panels (Appendix ledger check) */
+} tasp_plan_info;
+
+int tasp_plan_info_get(const tasp_plan* plan, tasp_plan_info* out);
+
+/* Per-layer retained sizes: out[0] = m_kv (kept groups), out[1] = c (kept channels). */
+int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2);
+
+enum tasp_export_item {
+    TASP_EXPORT_KEEP_GROUPS = 0, /* int32 [m_kv] */
+    TASP_EXPORT_KEEP_CHANS = 1,  /* int32 [c] */
+    TASP_EXPORT_QKV_W = 2,       /* int8 [(m_q + 2 m_kv) dh][d] */
+    TASP_EXPORT_QKV_S = 3,       /* float [(m_q + 2 m_kv) dh] */
+    TASP_EXPORT_O_W = 4,         /* int8 [d][m_q dh] */
+    TASP_EXPORT_O_S = 5,         /* float [d] */
+    TASP_EXPORT_GU_W = 6,        /* int8 [2c][d], gate row then up row per kept channel */
+    TASP_EXPORT_GU_S = 7,        /* float [2c] */
+    TASP_EXPORT_DOWN_W = 8,      /* int8 [d][c] */
+    TASP_EXPORT_DOWN_S = 9       /* float [d] */
+};
+
+/* Copy one packed panel (logical layout, no padding) or index list of a layer
+ * to host memory h_dst of `bytes` bytes (must equal the item's size). sync. */
+int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h_dst, size_t bytes);
+
+/* Run one decoder layer of a session's plan in isolation on a given FP32
+ * residual d_x_in [d] at the session's current position, writing d_x_out [d]
+ * (K/V of that position are written into the layer's cache; the position is
+ * not advanced). For per-layer parity checks. async. */
+int tasp_layer_step(tasp_session* s, int32_t layer, const float* d_x_in, float* d_x_out, void* stream);
+
+/* Run one decode step eagerly (no graph, no programmatic overlap) with CUDA
+ * events around every kernel, then synchronize. h_ms[k] / h_count[k] receive
+ * the total time and launch count of kernel kind k over the step:
+ * 0 qkv (RMSNorm + QKV GEMV + RoPE + KV append), 1 attention (split-KV + combine),
+ * 2 o-proj + residual, 3 gate/up + SiLU*up, 4 down + residual, 5 final norm +
+ * LM head, 6 other. Arrays have TASP_KERNEL_KINDS entries. */
+#define TASP_KERNEL_KINDS 7
+int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_logits,
+                      void* stream, float* h_ms, int32_t* h_count);
+
+/* Number of library kernel launches one decode step of these sessions makes
+ * (graph nodes). */
+int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_logits, int32_t* out);
+
+/* Thread-local description of the last failure on this thread ("" if none). */
+const char* tasp_last_error(void);
+
+/* Library version string. */
+const char* tasp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TASP_H */

@@ -1,0 +1,763 @@
+// C ABI of the TASP runtime: shared store registry, plan compilation and packing,
+// sessions with plan-bound KV caches, CUDA-graph decode steps, introspection.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "tasp_internal.h"
+
+namespace tasp {
+
+int attn_splits(int m_kv, int max_tokens, int sms);
+int attn_supported(int dh, int g);
+
+// ---------------------------------------------------------------- errors
+static thread_local std::string g_err;
+
+void set_error(const std::string& msg) { g_err = msg; }
+int fail(int code, const std::string& msg) {
+    g_err = msg;
+    return code;
+}
+int cuda_fail(cudaError_t e, const char* what) {
+    g_err = std::string(what) + ": " + cudaGetErrorString(e);
+    return e == cudaErrorMemoryAllocation ? TASP_ENOMEM : TASP_ECUDA;
+}
+
+// ---------------------------------------------------------------- device info
+int device_info(DevInfo& out) {
+    static DevInfo cached;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lk(mu);
+    int dev = 0;
+    TASP_CUDA(cudaGetDevice(&dev));
+    if (cached.dev != dev) {
+        cudaDeviceProp pr;
+        TASP_CUDA(cudaGetDeviceProperties(&pr, dev));
+        cached.dev = dev;
+        cached.sms = pr.multiProcessorCount;
+        cached.smem_optin = (int)pr.sharedMemPerBlockOptin;
+    }
+    out = cached;
+    return TASP_OK;
+}
+
+// ---------------------------------------------------------------- arena
+int Arena::reserve(size_t bytes) {
+    cap = (bytes + 255) & ~size_t(255);
+    used = 0;
+    if (cap == 0) return TASP_OK;
+    cudaError_t e = cudaMalloc((void**)&base, cap);
+    if (e != cudaSuccess) {
+        base = nullptr;
+        cap = 0;
+        return cuda_fail(e, "cudaMalloc");
+    }
+    return TASP_OK;
+}
+void* Arena::take(size_t bytes) {
+    size_t b = (bytes + 255) & ~size_t(255);
+    if (used + b > cap) return nullptr;
+    void* p = base + used;
+    used += b;
+    return p;
+}
+void Arena::release() {
+    if (base) cudaFree(base);
+    base = nullptr;
+    cap = used = 0;
+}
+
+// Sizing pass helper: records sizes then hands out pointers from a reserved arena.
+struct Layout {
+    std::vector<size_t> sizes;
+    size_t total = 0;
+    void add(size_t b) {
+        sizes.push_back(b);
+        total += (b + 255) & ~size_t(255);
+    }
+};
+
+static int round16(int v) { return (v + 15) & ~15; }
+
+// ---------------------------------------------------------------- store registry
+static std::mutex g_mu;
+static std::vector<Store*> g_stores;
+
+static int validate_shape(const tasp_model_desc* m, Shape& s, bool device = true) {
+    if (!m) return fail(TASP_EINVAL, "model_desc is NULL");
+    s.L = m->L; s.d = m->d; s.Hq = m->Hq; s.Hkv = m->Hkv; s.dh = m->dh; s.df = m->df; s.vocab = m->vocab;
+    s.cu = m->chan_unit; s.eps = m->rms_eps; s.theta = m->rope_theta; s.seed = m->seed;
+    if (s.L < 1 || s.d < 16 || s.d % 16 || s.Hq < 1 || s.Hkv < 1 || s.Hq % s.Hkv || s.dh < 16 || s.dh % 16 ||
+        s.dh > 128 || s.df < 1 || s.df % 16 || s.cu < 1 || s.df % s.cu || s.vocab < 0 || !(s.eps > 0.f) ||
+        !(s.theta > 0.f))
+        return fail(TASP_EINVAL, "invalid model shape (need d, df, dh multiples of 16, dh <= 128, Hq % Hkv == 0, "
+                                 "df % chan_unit == 0)");
+    if (!device) return TASP_OK;
+    if (!attn_supported(s.dh, s.g()))
+        return fail(TASP_EUNSUP, "attention kernel not built for this (head_dim, query heads per group)");
+    if ((int64_t)s.d * 4 > 200 * 1024 || (int64_t)s.df * 4 > 200 * 1024)
+        return fail(TASP_EUNSUP, "hidden or SwiGLU width too large for the shared-memory activation stage");
+    return TASP_OK;
+}
+
+static int store_acquire(const Shape& sh, Store** out) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (Store* st : g_stores)
+        if (st->sh.same(sh)) {
+            st->refs++;
+            *out = st;
+            return TASP_OK;
+        }
+    auto st = std::make_unique<Store>();
+    st->sh = sh;
+    const size_t d = sh.d, qkv = (size_t)sh.qkv_rows_dense(), hq = (size_t)sh.Hq * sh.dh, df = sh.df;
+    Layout lay;
+    for (int l = 0; l < sh.L; ++l) {
+        lay.add(qkv * d); lay.add(d * hq); lay.add(2 * df * d); lay.add(d * df);
+        lay.add(qkv * 4); lay.add(d * 4); lay.add(2 * df * 4); lay.add(d * 4); lay.add(d * 4); lay.add(d * 4);
+    }
+    lay.add(d * 4);
+    lay.add((size_t)sh.vocab * d * 2);
+    int rc = st->arena.reserve(lay.total);
+    if (rc) return rc;
+    st->layers.resize(sh.L);
+    for (int l = 0; l < sh.L; ++l) {
+        LayerStore& ls = st->layers[l];
+        ls.qkv = (int8_t*)st->arena.take(qkv * d);
+        ls.o = (int8_t*)st->arena.take(d * hq);
+        ls.gu = (int8_t*)st->arena.take(2 * df * d);
+        ls.down = (int8_t*)st->arena.take(d * df);
+        ls.qkv_s = (float*)st->arena.take(qkv * 4);
+        ls.o_s = (float*)st->arena.take(d * 4);
+        ls.gu_s = (float*)st->arena.take(2 * df * 4);
+        ls.down_s = (float*)st->arena.take(d * 4);
+        ls.g_attn = (float*)st->arena.take(d * 4);
+        ls.g_mlp = (float*)st->arena.take(d * 4);
+    }
+    st->g_final = (float*)st->arena.take(d * 4);
+    st->lm_head = sh.vocab ? (uint16_t*)st->arena.take((size_t)sh.vocab * d * 2) : nullptr;
+    st->bytes = lay.total;
+    cudaStream_t s;
+    TASP_CUDA(cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking));
+    rc = store_generate(*st, s);
+    cudaError_t e = cudaStreamSynchronize(s);
+    cudaStreamDestroy(s);
+    if (rc) {
+        st->arena.release();
+        return rc;
+    }
+    if (e != cudaSuccess) {
+        st->arena.release();
+        return cuda_fail(e, "store generation");
+    }
+    st->refs = 1;
+    *out = st.get();
+    g_stores.push_back(st.release());
+    return TASP_OK;
+}
+
+static void store_release(Store* st) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (--st->refs > 0) return;
+    st->arena.release();
+    g_stores.erase(std::remove(g_stores.begin(), g_stores.end(), st), g_stores.end());
+    delete st;
+}
+
+// ---------------------------------------------------------------- plan compilation
+static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep) {
+    Store& st = *p.store;
+    const Shape& sh = st.sh;
+    const int g = sh.g(), dh = sh.dh, d = sh.d;
+    p.layers.resize(sh.L);
+    for (int l = 0; l < sh.L; ++l) {
+        LayerPlan& lp = p.layers[l];
+        lp.keep_groups = sel.groups[l];
+        lp.keep_chans.clear();
+        for (int u : sel.units[l])
+            for (int i = 0; i < sh.cu; ++i) lp.keep_chans.push_back(u * sh.cu + i);
+        lp.m_kv = (int)lp.keep_groups.size();
+        lp.c = (int)lp.keep_chans.size();
+        lp.qkv_rows = lp.m_kv * (g + 2) * dh;
+        lp.gu_rows = 2 * lp.c;
+        lp.o_K = lp.m_kv * g * dh;
+        lp.dn_K = lp.c;
+        lp.g_attn = st.layers[l].g_attn;
+        lp.g_mlp = st.layers[l].g_mlp;
+    }
+    p.all_keep = all_keep;
+    p.panel_mode = panel_mode;
+    if (all_keep) {
+        for (int l = 0; l < sh.L; ++l) {
+            LayerPlan& lp = p.layers[l];
+            const LayerStore& ls = st.layers[l];
+            lp.qkv_w = ls.qkv; lp.qkv_s = ls.qkv_s;
+            lp.o_w = ls.o; lp.o_s = ls.o_s; lp.o_ld = sh.Hq * dh;
+            lp.gu_w = ls.gu; lp.gu_s = ls.gu_s;
+            lp.dn_w = ls.down; lp.dn_s = ls.down_s; lp.dn_ld = sh.df;
+        }
+        return TASP_OK;
+    }
+    const bool rowidx = panel_mode == TASP_PANELS_ROW_INDEXED;
+    // sizing pass
+    Layout lay;
+    for (int l = 0; l < sh.L; ++l) {
+        const LayerPlan& lp = p.layers[l];
+        const size_t ol = round16(lp.o_K), dl = round16(lp.dn_K);
+        lay.add((size_t)lp.qkv_rows * 4); lay.add((size_t)lp.qkv_rows * 4);  // map, scales
+        lay.add((size_t)lp.gu_rows * 4); lay.add((size_t)lp.gu_rows * 4);
+        lay.add(ol * 4); lay.add(dl * 4);                                       // column maps
+        if (!rowidx) { lay.add((size_t)lp.qkv_rows * d); lay.add((size_t)lp.gu_rows * d); }
+        lay.add((size_t)d * ol); lay.add((size_t)d * dl);
+    }
+    int rc = p.arena.reserve(lay.total);
+    if (rc) return rc;
+    cudaStream_t s;
+    TASP_CUDA(cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking));
+    std::vector<int32_t> hq, hg, ho, hd;
+    for (int l = 0; l < sh.L && !rc; ++l) {
+        LayerPlan& lp = p.layers[l];
+        const LayerStore& ls = st.layers[l];
+        const int ol = round16(lp.o_K), dl = round16(lp.dn_K);
+        hq.clear(); hg.clear(); ho.clear(); hd.clear();
+        for (int j : lp.keep_groups)
+            for (int r = 0; r < (g + 2) * dh; ++r) hq.push_back(j * (g + 2) * dh + r);
+        for (int c : lp.keep_chans) { hg.push_back(2 * c); hg.push_back(2 * c + 1); }
+        for (int j : lp.keep_groups)
+            for (int c = 0; c < g * dh; ++c) ho.push_back(j * g * dh + c);
+        ho.resize(ol, 0);
+        hd = std::vector<int32_t>(lp.keep_chans.begin(), lp.keep_chans.end());
+        hd.resize(dl, 0);
+        int32_t* dq = (int32_t*)p.arena.take(hq.size() * 4);
+        float* sq = (float*)p.arena.take(hq.size() * 4);
+        int32_t* dg = (int32_t*)p.arena.take(hg.size() * 4);
+        float* sg = (float*)p.arena.take(hg.size() * 4);
+        int32_t* dco = (int32_t*)p.arena.take(ho.size() * 4);
+        int32_t* dcd = (int32_t*)p.arena.take(hd.size() * 4);
+        if (hq.size()) TASP_CUDA(cudaMemcpyAsync(dq, hq.data(), hq.size() * 4, cudaMemcpyHostToDevice, s));
+        if (hg.size()) TASP_CUDA(cudaMemcpyAsync(dg, hg.data(), hg.size() * 4, cudaMemcpyHostToDevice, s));
+        if (ho.size()) TASP_CUDA(cudaMemcpyAsync(dco, ho.data(), ho.size() * 4, cudaMemcpyHostToDevice, s));
+        if (hd.size()) TASP_CUDA(cudaMemcpyAsync(dcd, hd.data(), hd.size() * 4, cudaMemcpyHostToDevice, s));
+        if ((rc = gather_f32(sq, ls.qkv_s, dq, (int)hq.size(), s))) break;
+        if ((rc = gather_f32(sg, ls.gu_s, dg, (int)hg.size(), s))) break;
+        lp.qkv_s = sq;
+        lp.gu_s = sg;
+        if (rowidx) {
+            lp.qkv_w = ls.qkv; lp.qkv_map = dq;
+            lp.gu_w = ls.gu; lp.gu_map = dg;
+        } else {
+            int8_t* wq = (int8_t*)p.arena.take((size_t)lp.qkv_rows * d);
+            int8_t* wg = (int8_t*)p.arena.take((size_t)lp.gu_rows * d);
+            if ((rc = gather_rows(wq, ls.qkv, dq, lp.qkv_rows, d, s))) break;
+            if ((rc = gather_rows(wg, ls.gu, dg, lp.gu_rows, d, s))) break;
+            lp.qkv_w = wq;
+            lp.gu_w = wg;
+        }
+        int8_t* wo = (int8_t*)p.arena.take((size_t)d * ol);
+        int8_t* wd = (int8_t*)p.arena.take((size_t)d * dl);
+        if ((rc = gather_cols(wo, ol, ls.o, sh.Hq * dh, dco, d, lp.o_K, s))) break;
+        if ((rc = gather_cols(wd, dl, ls.down, sh.df, dcd, d, lp.dn_K, s))) break;
+        lp.o_w = wo; lp.o_ld = ol; lp.o_s = ls.o_s;
+        lp.dn_w = wd; lp.dn_ld = dl; lp.dn_s = ls.down_s;
+        // host vectors must outlive the async copies
+        cudaError_t e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) { rc = cuda_fail(e, "plan packing"); break; }
+    }
+    cudaStreamDestroy(s);
+    return rc;
+}
+
+static void plan_ledger(Plan& p) {
+    const Shape& sh = p.store->sh;
+    int64_t fl = 0, launched = 0, bytes = 0;
+    for (const LayerPlan& lp : p.layers) {
+        fl += layer_flops(sh, (int64_t)lp.m_kv * sh.g(), lp.m_kv, lp.c);
+        launched += 2 * (int64_t)lp.qkv_rows * sh.d + 2 * (int64_t)sh.d * lp.o_K + 2 * (int64_t)lp.gu_rows * sh.d +
+                    2 * (int64_t)sh.d * lp.dn_K;
+        bytes += (int64_t)lp.qkv_rows * sh.d + (int64_t)sh.d * lp.o_K + (int64_t)lp.gu_rows * sh.d +
+                 (int64_t)sh.d * lp.dn_K;
+        bytes += 4 * ((int64_t)lp.qkv_rows + (lp.m_kv ? sh.d : 0) + lp.gu_rows + (lp.c ? sh.d : 0));
+        bytes += 2 * 4 * (int64_t)sh.d;  // norm gains
+    }
+    bytes += (int64_t)sh.vocab * sh.d * 2 + 4 * (int64_t)sh.d;
+    p.flops_retained = fl;
+    p.flops_dense = dense_layer_flops(sh) * sh.L;
+    p.launched_flops = launched;
+    p.weight_bytes_per_token = bytes;
+}
+
+static Plan* as_plan(void* h) {
+    Plan* p = (Plan*)h;
+    return (p && p->magic == PLAN_MAGIC) ? p : nullptr;
+}
+static Session* as_session(void* h) {
+    Session* s = (Session*)h;
+    return (s && s->magic == SESSION_MAGIC) ? s : nullptr;
+}
+
+// ---------------------------------------------------------------- sessions
+static int session_alloc(Plan* p, int max_tokens, Session** out) {
+    const Shape& sh = p->store->sh;
+    DevInfo di;
+    int rc = device_info(di);
+    if (rc) return rc;
+    auto se = std::make_unique<Session>();
+    se->plan = p;
+    se->max_tokens = max_tokens;
+    int smax = 1;
+    for (const LayerPlan& lp : p->layers) smax = std::max(smax, attn_splits(lp.m_kv, max_tokens, di.sms));
+    se->att_splits_max = smax;
+    Layout lay;
+    for (const LayerPlan& lp : p->layers) {
+        lay.add((size_t)lp.m_kv * max_tokens * sh.dh * 2);
+        lay.add((size_t)lp.m_kv * max_tokens * sh.dh * 2);
+    }
+    const size_t half = sh.dh / 2;
+    lay.add((size_t)max_tokens * half * sizeof(float2));
+    lay.add(sizeof(int));
+    lay.add((size_t)sh.d * 4);
+    lay.add((size_t)sh.Hq * sh.dh * 2);
+    lay.add((size_t)sh.Hq * sh.dh * 2);
+    lay.add((size_t)sh.df * 2);
+    const size_t part = (size_t)sh.Hkv * smax * sh.g() * (sh.dh + 2) * 4;
+    lay.add(part);
+    lay.add((size_t)sh.Hkv * 4);
+    lay.add((size_t)sh.d * 2);
+    lay.add((size_t)sh.vocab * 4);
+    lay.add((size_t)sh.d * 4);
+    if ((rc = se->arena.reserve(lay.total))) return rc;
+    for (const LayerPlan& lp : p->layers) {
+        se->K.push_back((uint16_t*)se->arena.take((size_t)lp.m_kv * max_tokens * sh.dh * 2));
+        se->V.push_back((uint16_t*)se->arena.take((size_t)lp.m_kv * max_tokens * sh.dh * 2));
+    }
+    se->rope = (float2*)se->arena.take((size_t)max_tokens * half * sizeof(float2));
+    se->d_pos = (int*)se->arena.take(sizeof(int));
+    se->x = (float*)se->arena.take((size_t)sh.d * 4);
+    se->q = (uint16_t*)se->arena.take((size_t)sh.Hq * sh.dh * 2);
+    se->o = (uint16_t*)se->arena.take((size_t)sh.Hq * sh.dh * 2);
+    se->h = (uint16_t*)se->arena.take((size_t)sh.df * 2);
+    se->part = (float*)se->arena.take(part);
+    se->cnt = (int*)se->arena.take((size_t)sh.Hkv * 4);
+    se->x_stage = (uint16_t*)se->arena.take((size_t)sh.d * 2);
+    se->logits_stage = sh.vocab ? (float*)se->arena.take((size_t)sh.vocab * 4) : nullptr;
+    se->hidden_stage = (float*)se->arena.take((size_t)sh.d * 4);
+    // zero the whole arena: empty caches, position 0, attention tickets 0
+    TASP_CUDA(cudaMemset(se->arena.base, 0, se->arena.cap));
+    if ((rc = rope_table(*se, 0))) return rc;
+    TASP_CUDA(cudaDeviceSynchronize());
+    *out = se.release();
+    return TASP_OK;
+}
+
+static void session_free(Session* se) {
+    if (se->graph.exec) cudaGraphExecDestroy(se->graph.exec);
+    se->arena.release();
+    se->magic = 0;
+    delete se;
+}
+
+// Record (or re-record) the step graph of a session for a set of caller buffers.
+static int session_graph(Session& se, const StepTarget& t) {
+    StepGraph& g = se.graph;
+    if (g.exec && g.x == t.x_in && g.hidden == t.hidden_out && g.logits == t.logits) return TASP_OK;
+    if (g.exec) {
+        cudaGraphExecDestroy(g.exec);
+        g.exec = nullptr;
+    }
+    cudaStream_t cs;
+    TASP_CUDA(cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking));
+    cudaError_t e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed);
+    if (e != cudaSuccess) {
+        cudaStreamDestroy(cs);
+        return cuda_fail(e, "cudaStreamBeginCapture");
+    }
+    int launches = 0;
+    int rc = enqueue_step(se, t, cs, -1, nullptr, nullptr, &launches);
+    cudaGraph_t graph = nullptr;
+    e = cudaStreamEndCapture(cs, &graph);
+    cudaStreamDestroy(cs);
+    if (rc) {
+        if (graph) cudaGraphDestroy(graph);
+        return rc;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamEndCapture");
+    e = cudaGraphInstantiate(&g.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+        g.exec = nullptr;
+        return cuda_fail(e, "cudaGraphInstantiate");
+    }
+    g.x = t.x_in;
+    g.hidden = t.hidden_out;
+    g.logits = t.logits;
+    g.launches = launches;
+    return TASP_OK;
+}
+
+static int check_sessions(tasp_session* const* ss, int n, Plan** plan) {
+    if (!ss || n < 1) return fail(TASP_EINVAL, "need at least one session");
+    Plan* p = nullptr;
+    for (int i = 0; i < n; ++i) {
+        Session* se = as_session(ss[i]);
+        if (!se) return fail(TASP_EINVAL, "invalid session handle");
+        if (!p) p = se->plan;
+        if (se->plan != p) return fail(TASP_EMASK, "sessions of different plans in one decode step (a KV cache is "
+                                                   "never reused across masks)");
+        if (se->pos + 1 > se->max_tokens) return fail(TASP_ECAP, "session KV capacity exhausted");
+        for (int j = 0; j < i; ++j)
+            if (ss[j] == ss[i]) return fail(TASP_EINVAL, "a session appears twice in one decode step");
+    }
+    *plan = p;
+    return TASP_OK;
+}
+
+}  // namespace tasp
+
+using namespace tasp;
+
+// ==================================================================== C ABI
+extern "C" {
+
+const char* tasp_last_error(void) { return g_err.c_str(); }
+const char* tasp_version(void) { return "tasp-gb300 0.1 (sm_103a)"; }
+
+int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
+                     int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops) {
+    Shape sh;
+    int rc = validate_shape(model, sh, false);
+    if (rc) return rc;
+    if (!mask) return fail(TASP_EINVAL, "mask_desc is NULL");
+    MaskSel sel;
+    if ((rc = select_mask(sh, *mask, sel))) return rc;
+    size_t og = 0, ou = 0;
+    for (int l = 0; l < sh.L; ++l) {
+        if (n_groups) n_groups[l] = (int32_t)sel.groups[l].size();
+        if (n_units) n_units[l] = (int32_t)sel.units[l].size();
+        for (int j : sel.groups[l]) if (keep_groups) keep_groups[og++] = j;
+        for (int u : sel.units[l]) if (keep_units) keep_units[ou++] = u;
+        if (flops) flops[l] = sel.layer_flops[l];
+    }
+    if (flops) {
+        flops[sh.L] = sel.total;
+        flops[sh.L + 1] = sel.budget;
+        flops[sh.L + 2] = sel.dense;
+    }
+    return TASP_OK;
+}
+
+int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out) {
+    if (!out) return fail(TASP_EINVAL, "out is NULL");
+    *out = nullptr;
+    Shape sh;
+    int rc = validate_shape(model, sh);
+    if (rc) return rc;
+    if (!mask) return fail(TASP_EINVAL, "mask_desc is NULL");
+    if (mask->panel_mode != TASP_PANELS_COMPACT && mask->panel_mode != TASP_PANELS_ROW_INDEXED)
+        return fail(TASP_EINVAL, "unknown panel mode");
+    MaskSel sel;
+    if ((rc = select_mask(sh, *mask, sel))) return rc;
+    for (int l = 0; l < sh.L; ++l)
+        if (sel.groups[l].empty() && sel.units[l].empty())
+            return fail(TASP_EINVAL, "mask leaves a layer empty (layer " + std::to_string(l) + ")");
+    Store* st = nullptr;
+    if ((rc = store_acquire(sh, &st))) return rc;
+    auto p = std::make_unique<Plan>();
+    p->store = st;
+    if ((rc = build_plan(*p, sel, mask->panel_mode, mask->kind == TASP_MASK_ALL_KEEP))) {
+        p->arena.release();
+        store_release(st);
+        return rc;
+    }
+    plan_ledger(*p);
+    *out = (tasp_plan*)p.release();
+    return TASP_OK;
+}
+
+int tasp_session_create(tasp_plan* plan, int32_t max_tokens, tasp_session** out) {
+    if (!out) return fail(TASP_EINVAL, "out is NULL");
+    *out = nullptr;
+    Plan* p = as_plan(plan);
+    if (!p) return fail(TASP_EINVAL, "invalid plan handle");
+    if (max_tokens < 1) return fail(TASP_EINVAL, "max_tokens must be positive");
+    Session* se = nullptr;
+    int rc = session_alloc(p, max_tokens, &se);
+    if (rc) return rc;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        p->live_sessions++;
+    }
+    *out = (tasp_session*)se;
+    return TASP_OK;
+}
+
+int tasp_session_fill_synthetic(tasp_session* s, int32_t t_prior, uint64_t kv_seed, void* stream) {
+    Session* se = as_session(s);
+    if (!se) return fail(TASP_EINVAL, "invalid session handle");
+    if (t_prior < 0 || t_prior > se->max_tokens) return fail(TASP_ECAP, "t_prior exceeds the session capacity");
+    int rc = kv_fill_synthetic(*se, t_prior, kv_seed, (cudaStream_t)stream);
+    if (rc) return rc;
+    se->pos = t_prior;
+    return TASP_OK;
+}
+
+int tasp_session_position(const tasp_session* s, int32_t* pos) {
+    Session* se = as_session((void*)s);
+    if (!se || !pos) return fail(TASP_EINVAL, "invalid session handle or NULL output");
+    *pos = se->pos;
+    return TASP_OK;
+}
+
+int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,
+                     float* d_logits, void* stream) {
+    Plan* p = nullptr;
+    int rc = check_sessions(sessions, n, &p);
+    if (rc) return rc;
+    if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");
+    const Shape& sh = p->store->sh;
+    if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
+    for (int i = 0; i < n; ++i) {
+        Session* se = (Session*)sessions[i];
+        StepTarget t;
+        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i * sh.d;
+        t.hidden_out = d_hidden_out ? d_hidden_out + (size_t)i * sh.d : nullptr;
+        t.logits = d_logits ? d_logits + (size_t)i * sh.vocab : nullptr;
+        if ((rc = session_graph(*se, t))) return rc;
+        TASP_CUDA(cudaGraphLaunch(se->graph.exec, (cudaStream_t)stream));
+        se->pos += 1;
+    }
+    return TASP_OK;
+}
+
+int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* h_x_bf16, float* h_hidden_out,
+                          float* h_logits, void* stream) {
+    Plan* p = nullptr;
+    int rc = check_sessions(sessions, n, &p);
+    if (rc) return rc;
+    if (!h_x_bf16) return fail(TASP_EINVAL, "h_x_bf16 is NULL");
+    const Shape& sh = p->store->sh;
+    if (h_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
+    cudaStream_t st = (cudaStream_t)stream;
+    for (int i = 0; i < n; ++i) {
+        Session* se = (Session*)sessions[i];
+        TASP_CUDA(cudaMemcpyAsync(se->x_stage, (const uint16_t*)h_x_bf16 + (size_t)i * sh.d, (size_t)sh.d * 2,
+                                  cudaMemcpyHostToDevice, st));
+        StepTarget t;
+        t.x_in = se->x_stage;
+        t.hidden_out = h_hidden_out ? se->hidden_stage : nullptr;
+        t.logits = h_logits ? se->logits_stage : nullptr;
+        if ((rc = session_graph(*se, t))) return rc;
+        TASP_CUDA(cudaGraphLaunch(se->graph.exec, st));
+        se->pos += 1;
+        if (h_hidden_out)
+            TASP_CUDA(cudaMemcpyAsync(h_hidden_out + (size_t)i * sh.d, se->hidden_stage, (size_t)sh.d * 4,
+                                      cudaMemcpyDeviceToHost, st));
+        if (h_logits)
+            TASP_CUDA(cudaMemcpyAsync(h_logits + (size_t)i * sh.vocab, se->logits_stage, (size_t)sh.vocab * 4,
+                                      cudaMemcpyDeviceToHost, st));
+    }
+    TASP_CUDA(cudaStreamSynchronize(st));
+    return TASP_OK;
+}
+
+int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t max_new_tokens, void* stream,
+                 tasp_session** out, float* d_logits_last) {
+    (void)plan; (void)d_embeds_bf16; (void)T; (void)max_new_tokens; (void)stream; (void)d_logits_last;
+    if (out) *out = nullptr;
+    return fail(TASP_EUNSUP, "prefill is not built yet");
+}
+
+int tasp_release(void* handle) {
+    if (!handle) return TASP_OK;
+    if (Session* se = as_session(handle)) {
+        cudaError_t e = cudaDeviceSynchronize();
+        {
+            std::lock_guard<std::mutex> lk(g_mu);
+            se->plan->live_sessions--;
+        }
+        session_free(se);
+        if (e != cudaSuccess) return cuda_fail(e, "tasp_release");
+        return TASP_OK;
+    }
+    if (Plan* p = as_plan(handle)) {
+        {
+            std::lock_guard<std::mutex> lk(g_mu);
+            if (p->live_sessions > 0) return fail(TASP_EBUSY, "plan still has live sessions");
+        }
+        cudaError_t e = cudaDeviceSynchronize();
+        p->arena.release();
+        store_release(p->store);
+        p->magic = 0;
+        delete p;
+        if (e != cudaSuccess) return cuda_fail(e, "tasp_release");
+        return TASP_OK;
+    }
+    return fail(TASP_EINVAL, "unknown handle");
+}
+
+int tasp_plan_info_get(const tasp_plan* plan, tasp_plan_info* out) {
+    Plan* p = as_plan((void*)plan);
+    if (!p || !out) return fail(TASP_EINVAL, "invalid plan handle or NULL output");
+    out->L = p->store->sh.L;
+    out->panel_bytes = (int64_t)p->arena.cap;
+    out->store_bytes = (int64_t)p->store->bytes;
+    out->weight_bytes_per_token = p->weight_bytes_per_token;
+    out->flops_retained = p->flops_retained;
+    out->flops_dense = p->flops_dense;
+    out->launched_flops = p->launched_flops;
+    return TASP_OK;
+}
+
+int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2) {
+    Plan* p = as_plan((void*)plan);
+    if (!p || !out2 || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan or layer");
+    out2[0] = p->layers[layer].m_kv;
+    out2[1] = p->layers[layer].c;
+    return TASP_OK;
+}
+
+int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h_dst, size_t bytes) {
+    Plan* p = as_plan((void*)plan);
+    if (!p || !h_dst || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan, layer or dst");
+    const LayerPlan& lp = p->layers[layer];
+    const Shape& sh = p->store->sh;
+    const size_t d = sh.d;
+    auto need = [&](size_t b) { return b == bytes ? TASP_OK : fail(TASP_EINVAL, "export size mismatch: expected " +
+                                                                                std::to_string(b)); };
+    auto rows_out = [&](const int8_t* w, const int32_t* map, int rows) -> int {
+        if (int rc = need((size_t)rows * d)) return rc;
+        if (!map) {
+            TASP_CUDA(cudaMemcpy(h_dst, w, (size_t)rows * d, cudaMemcpyDeviceToHost));
+            return TASP_OK;
+        }
+        int8_t* tmp = nullptr;
+        TASP_CUDA(cudaMalloc((void**)&tmp, std::max<size_t>(16, (size_t)rows * d)));
+        int rc = gather_rows(tmp, w, map, rows, (int)d, 0);
+        cudaError_t e = cudaMemcpy(h_dst, tmp, (size_t)rows * d, cudaMemcpyDeviceToHost);
+        cudaFree(tmp);
+        if (rc) return rc;
+        if (e != cudaSuccess) return cuda_fail(e, "export");
+        return TASP_OK;
+    };
+    auto cols_out = [&](const int8_t* w, int ld, int K) -> int {
+        if (int rc = need(d * (size_t)K)) return rc;
+        if (K == 0) return TASP_OK;
+        TASP_CUDA(cudaMemcpy2D(h_dst, K, w, ld, K, d, cudaMemcpyDeviceToHost));
+        return TASP_OK;
+    };
+    auto f32_out = [&](const float* v, size_t n) -> int {
+        if (int rc = need(n * 4)) return rc;
+        if (n) TASP_CUDA(cudaMemcpy(h_dst, v, n * 4, cudaMemcpyDeviceToHost));
+        return TASP_OK;
+    };
+    switch (item) {
+        case TASP_EXPORT_KEEP_GROUPS: {
+            if (int rc = need(lp.keep_groups.size() * 4)) return rc;
+            std::memcpy(h_dst, lp.keep_groups.data(), bytes);
+            return TASP_OK;
+        }
+        case TASP_EXPORT_KEEP_CHANS: {
+            if (int rc = need(lp.keep_chans.size() * 4)) return rc;
+            std::memcpy(h_dst, lp.keep_chans.data(), bytes);
+            return TASP_OK;
+        }
+        case TASP_EXPORT_QKV_W: return rows_out(lp.qkv_w, lp.qkv_map, lp.qkv_rows);
+        case TASP_EXPORT_QKV_S: return f32_out(lp.qkv_s, lp.qkv_rows);
+        case TASP_EXPORT_O_W: return cols_out(lp.o_w, lp.o_ld, lp.o_K);
+        case TASP_EXPORT_O_S: return f32_out(lp.o_s, d);
+        case TASP_EXPORT_GU_W: return rows_out(lp.gu_w, lp.gu_map, lp.gu_rows);
+        case TASP_EXPORT_GU_S: return f32_out(lp.gu_s, lp.gu_rows);
+        case TASP_EXPORT_DOWN_W: return cols_out(lp.dn_w, lp.dn_ld, lp.dn_K);
+        case TASP_EXPORT_DOWN_S: return f32_out(lp.dn_s, d);
+        default: return fail(TASP_EINVAL, "unknown export item");
+    }
+}
+
+int tasp_layer_step(tasp_session* s, int32_t layer, const float* d_x_in, float* d_x_out, void* stream) {
+    Session* se = as_session(s);
+    if (!se || !d_x_in || !d_x_out) return fail(TASP_EINVAL, "invalid session or NULL buffers");
+    const Shape& sh = se->plan->store->sh;
+    if (layer < 0 || layer >= sh.L) return fail(TASP_EINVAL, "layer out of range");
+    if (se->pos + 1 > se->max_tokens) return fail(TASP_ECAP, "session KV capacity exhausted");
+    cudaStream_t st = (cudaStream_t)stream;
+    TASP_CUDA(cudaMemcpyAsync(se->x, d_x_in, (size_t)sh.d * 4, cudaMemcpyDeviceToDevice, st));
+    StepTarget t;
+    t.advance = false;
+    int rc = enqueue_step(*se, t, st, layer, nullptr, nullptr, nullptr);
+    if (rc) return rc;
+    TASP_CUDA(cudaMemcpyAsync(d_x_out, se->x, (size_t)sh.d * 4, cudaMemcpyDeviceToDevice, st));
+    return TASP_OK;
+}
+
+struct ProfCtx {
+    cudaStream_t s;
+    std::vector<cudaEvent_t> ev;
+    std::vector<int> kind;
+    int err = 0;
+};
+
+static void prof_hook(void* c, int kind, bool before) {
+    ProfCtx* pc = (ProfCtx*)c;
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+        pc->err = 1;
+        return;
+    }
+    cudaEventRecord(e, pc->s);
+    pc->ev.push_back(e);
+    pc->kind.push_back(before ? -1 : kind);
+}
+
+int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_logits, void* stream,
+                      float* h_ms, int32_t* h_count) {
+    Plan* p = nullptr;
+    int rc = check_sessions(sessions, n, &p);
+    if (rc) return rc;
+    if (!h_ms || !h_count || !d_x_bf16) return fail(TASP_EINVAL, "NULL buffers");
+    const Shape& sh = p->store->sh;
+    for (int k = 0; k < TASP_KERNEL_KINDS; ++k) { h_ms[k] = 0.f; h_count[k] = 0; }
+    for (int i = 0; i < n; ++i) {
+        Session* se = (Session*)sessions[i];
+        ProfCtx pc;
+        pc.s = (cudaStream_t)stream;
+        StepTarget t;
+        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i * sh.d;
+        t.logits = d_logits ? d_logits + (size_t)i * sh.vocab : nullptr;
+        rc = enqueue_step(*se, t, pc.s, -1, prof_hook, &pc, nullptr);
+        cudaError_t e = cudaStreamSynchronize(pc.s);
+        if (!rc && e == cudaSuccess && !pc.err) {
+            for (size_t j = 0; j + 1 < pc.ev.size(); j += 2) {
+                float ms = 0.f;
+                cudaEventElapsedTime(&ms, pc.ev[j], pc.ev[j + 1]);
+                int k = pc.kind[j + 1];
+                h_ms[k] += ms;
+                h_count[k] += 1;
+            }
+            se->pos += 1;
+        }
+        for (cudaEvent_t ev : pc.ev) cudaEventDestroy(ev);
+        if (rc) return rc;
+        if (e != cudaSuccess) return cuda_fail(e, "profile step");
+        if (pc.err) return fail(TASP_ECUDA, "event creation failed");
+    }
+    return TASP_OK;
+}
+
+int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_logits, int32_t* out) {
+    Plan* p = nullptr;
+    int rc = check_sessions(sessions, n, &p);
+    if (rc) return rc;
+    if (!out) return fail(TASP_EINVAL, "NULL output");
+    int per = 0;
+    for (const LayerPlan& lp : p->layers) per += 1 + (lp.m_kv ? 2 : 0) + (lp.c ? 2 : 0);
+    per += (with_logits && p->store->sh.vocab ? 1 : 0) + 1;
+    *out = per * n;
+    return TASP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,180 @@
+// Internal structures of the TASP runtime: shared store, plans, sessions, kernel parameters.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/tasp.h"
+
+namespace tasp {
+
+// ---------------------------------------------------------------- errors
+void set_error(const std::string& msg);
+int fail(int code, const std::string& msg);
+int cuda_fail(cudaError_t e, const char* what);
+
+#define TASP_CUDA(call)                                   \
+    do {                                                  \
+        cudaError_t e_ = (call);                          \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+    } while (0)
+
+// ---------------------------------------------------------------- shape
+struct Shape {
+    int L = 0, d = 0, Hq = 0, Hkv = 0, dh = 0, df = 0, vocab = 0, cu = 1;
+    float eps = 1e-5f, theta = 500000.f;
+    uint64_t seed = 0;
+    int g() const { return Hq / Hkv; }
+    int n_units() const { return df / cu; }
+    int qkv_rows_dense() const { return (Hq + 2 * Hkv) * dh; }
+    bool same(const Shape& o) const;
+};
+
+// Active-FLOP ledger (Appendix, Eqs. flop-attn and flop-mlp).
+int64_t layer_flops(const Shape& s, int64_t m_q, int64_t m_kv, int64_t c);
+inline int64_t dense_layer_flops(const Shape& s) { return layer_flops(s, s.Hq, s.Hkv, s.df); }
+
+// Host mask compiler result: per layer kept groups and channel units (ascending).
+struct MaskSel {
+    std::vector<std::vector<int>> groups, units;
+    std::vector<int64_t> layer_flops;
+    int64_t total = 0, budget = 0, dense = 0;
+};
+int select_mask(const Shape& s, const tasp_mask_desc& m, MaskSel& out);
+
+// ---------------------------------------------------------------- device memory arena
+struct Arena {
+    char* base = nullptr;
+    size_t cap = 0, used = 0;
+    int reserve(size_t bytes);  // cudaMalloc of the whole arena
+    void* take(size_t bytes);   // 256-byte aligned sub-allocation
+    void release();
+};
+
+// ---------------------------------------------------------------- shared store
+// Each projection once, INT8 with one FP32 scale per output row; QKV rows group-major
+// (per KV group: its g query heads, then K, then V) and gate/up rows interleaved per
+// channel, i.e. the packed layout of the all-keep mask.
+struct LayerStore {
+    int8_t *qkv, *o, *gu, *down;
+    float *qkv_s, *o_s, *gu_s, *down_s, *g_attn, *g_mlp;
+};
+
+struct Store {
+    Shape sh;
+    int refs = 0;
+    Arena arena;
+    std::vector<LayerStore> layers;
+    float* g_final = nullptr;
+    uint16_t* lm_head = nullptr;  // BF16 [vocab][d]
+    size_t bytes = 0;
+};
+
+// ---------------------------------------------------------------- plans
+struct LayerPlan {
+    int m_kv = 0, c = 0;
+    std::vector<int> keep_groups, keep_chans;
+    // qkv panel: rows (m_q + 2 m_kv) dh of K = d; row i at qkv_w + (qkv_map ? qkv_map[i] : i) * d
+    const int8_t* qkv_w = nullptr;
+    const int32_t* qkv_map = nullptr;
+    const float* qkv_s = nullptr;
+    int qkv_rows = 0;
+    // o panel: d rows of K = m_q dh (stride o_ld >= K, multiple of 16, zero padded)
+    const int8_t* o_w = nullptr;
+    const float* o_s = nullptr;
+    int o_K = 0, o_ld = 0;
+    // gate/up panel: 2c rows of K = d
+    const int8_t* gu_w = nullptr;
+    const int32_t* gu_map = nullptr;
+    const float* gu_s = nullptr;
+    int gu_rows = 0;
+    // down panel: d rows of K = c (stride dn_ld)
+    const int8_t* dn_w = nullptr;
+    const float* dn_s = nullptr;
+    int dn_K = 0, dn_ld = 0;
+    const float *g_attn = nullptr, *g_mlp = nullptr;
+};
+
+constexpr uint32_t PLAN_MAGIC = 0x7A5B1A01u;
+constexpr uint32_t SESSION_MAGIC = 0x7A5B5E55u;
+
+struct Plan {
+    uint32_t magic = PLAN_MAGIC;
+    Store* store = nullptr;
+    int live_sessions = 0;
+    int panel_mode = 0;
+    bool all_keep = false;
+    std::vector<LayerPlan> layers;
+    Arena arena;
+    int64_t flops_retained = 0, flops_dense = 0, launched_flops = 0;
+    int64_t weight_bytes_per_token = 0;
+};
+
+// ---------------------------------------------------------------- sessions
+struct StepGraph {
+    cudaGraphExec_t exec = nullptr;
+    const void* x = nullptr;
+    float* hidden = nullptr;
+    float* logits = nullptr;
+    int launches = 0;
+};
+
+struct Session {
+    uint32_t magic = SESSION_MAGIC;
+    Plan* plan = nullptr;
+    int max_tokens = 0;
+    int pos = 0;  // host mirror of the device position
+    Arena arena;
+    std::vector<uint16_t*> K, V;  // per layer BF16 [m_kv][max_tokens][dh]
+    float2* rope = nullptr;       // [max_tokens][dh/2] (cos, sin)
+    int* d_pos = nullptr;
+    // workspace of one decode step
+    float* x = nullptr;     // FP32 residual [d]
+    uint16_t* q = nullptr;  // BF16 [Hq dh]
+    uint16_t* o = nullptr;  // BF16 [Hq dh]
+    uint16_t* h = nullptr;  // BF16 [df]
+    float* part = nullptr;  // attention split partials
+    int* cnt = nullptr;     // attention split counters [Hkv]
+    int att_splits_max = 0;
+    uint16_t* x_stage = nullptr;  // BF16 [d] host-buffer staging
+    float* logits_stage = nullptr;
+    float* hidden_stage = nullptr;
+    StepGraph graph;
+};
+
+// ---------------------------------------------------------------- device info
+struct DevInfo {
+    int dev = -1, sms = 0, smem_optin = 0;
+};
+int device_info(DevInfo& out);
+
+// ---------------------------------------------------------------- kernels (launchers)
+// store.cu
+int store_generate(Store& st, cudaStream_t s);
+int kv_fill_synthetic(Session& se, int t_prior, uint64_t kv_seed, cudaStream_t s);
+int rope_table(Session& se, cudaStream_t s);
+int gather_rows(int8_t* dst, const int8_t* src, const int32_t* map, int rows, int K, cudaStream_t s);
+int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const int32_t* cmap, int rows, int Kc,
+                cudaStream_t s);
+int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
+
+// decode.cu
+enum KernelKind { K_QKV = 0, K_ATTN = 1, K_O = 2, K_GU = 3, K_DOWN = 4, K_LM = 5, K_OTHER = 6 };
+
+struct StepTarget {
+    const uint16_t* x_in = nullptr;  // BF16 [d] step input (first layer) or nullptr (use residual)
+    float* hidden_out = nullptr;
+    float* logits = nullptr;
+    bool advance = true;
+};
+
+using KernelHook = void (*)(void* ctx, int kind, bool before);
+
+// Enqueue one decode step (or one isolated layer when only_layer >= 0) on `s`.
+int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
+                 int* launches);
+
+}  // namespace tasp

@@ -1,0 +1,291 @@
+"""Thin Python binding of the TASP C ABI (include/tasp.h).
+
+Argument marshalling only: every step of the path runs in the CUDA library
+``libtasp.so`` built in-tree by ``paper_2609_29499_gb300.build``. There is no
+fallback: if the library is missing or cannot be loaded, ``load()`` raises.
+PyTorch supplies device buffers and streams (``tensor.data_ptr()``,
+``torch.cuda.current_stream().cuda_stream``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_float, c_int32, c_int64, c_size_t, c_uint32, c_uint64, c_void_p
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libtasp.so")
+
+OK, EINVAL, EMASK, ECAP, ENOMEM, EBUSY, ECUDA, EUNSUP = 0, -1, -2, -3, -4, -5, -6, -7
+MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT = 0, 1, 2
+PANELS_COMPACT, PANELS_ROW_INDEXED = 0, 1
+(EXPORT_KEEP_GROUPS, EXPORT_KEEP_CHANS, EXPORT_QKV_W, EXPORT_QKV_S, EXPORT_O_W, EXPORT_O_S, EXPORT_GU_W,
+ EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S) = range(10)
+KERNEL_KINDS = 7
+KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "other")
+
+# Symbols declared in include/tasp.h (the CPU test checks they are all exported).
+EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
+            "tasp_session_fill_synthetic", "tasp_session_position", "tasp_decode_step_host", "tasp_mask_select",
+            "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
+            "tasp_profile_step", "tasp_step_launches", "tasp_last_error", "tasp_version")
+
+
+class ModelDesc(ctypes.Structure):
+    _fields_ = [("L", c_int32), ("d", c_int32), ("Hq", c_int32), ("Hkv", c_int32), ("dh", c_int32),
+                ("df", c_int32), ("vocab", c_int32), ("chan_unit", c_int32), ("rms_eps", c_float),
+                ("rope_theta", c_float), ("seed", c_uint64)]
+
+
+class MaskDesc(ctypes.Structure):
+    _fields_ = [("kind", c_int32), ("panel_mode", c_int32), ("flop_budget", c_double), ("r_lo", c_double),
+                ("r_hi", c_double), ("scores", POINTER(c_uint32)), ("target_u24", POINTER(c_uint32)),
+                ("keep_groups", POINTER(c_int32)), ("n_groups", POINTER(c_int32)),
+                ("keep_units", POINTER(c_int32)), ("n_units", POINTER(c_int32))]
+
+
+class PlanInfo(ctypes.Structure):
+    _fields_ = [("L", c_int32), ("panel_bytes", c_int64), ("store_bytes", c_int64),
+                ("weight_bytes_per_token", c_int64), ("flops_retained", c_int64), ("flops_dense", c_int64),
+                ("launched_flops", c_int64)]
+
+
+class TaspError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"tasp error {code}: {msg}")
+        self.code = code
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load libtasp.so (raises if it is missing: there is no CPU fallback)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with paper_2609_29499_gb300.build.build()")
+    try:  # make the CUDA runtime that PyTorch ships visible first, when torch is installed
+        import torch  # noqa: F401
+    except Exception:
+        pass
+    lib = ctypes.CDLL(path)
+    P = c_void_p
+    sig = {
+        "tasp_compile_mask": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), POINTER(P)]),
+        "tasp_prefill": (c_int32, [P, P, c_int32, c_int32, P, POINTER(P), P]),
+        "tasp_decode_step": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
+        "tasp_release": (c_int32, [P]),
+        "tasp_session_create": (c_int32, [P, c_int32, POINTER(P)]),
+        "tasp_session_fill_synthetic": (c_int32, [P, c_int32, c_uint64, P]),
+        "tasp_session_position": (c_int32, [P, POINTER(c_int32)]),
+        "tasp_decode_step_host": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
+        "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
+        "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
+        "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
+        "tasp_plan_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
+        "tasp_layer_step": (c_int32, [P, c_int32, P, P, P]),
+        "tasp_profile_step": (c_int32, [POINTER(P), c_int32, P, P, P, P, P]),
+        "tasp_step_launches": (c_int32, [POINTER(P), c_int32, c_int32, POINTER(c_int32)]),
+        "tasp_last_error": (ctypes.c_char_p, []),
+        "tasp_version": (ctypes.c_char_p, []),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(rc):
+    if rc != OK:
+        raise TaspError(rc, load().tasp_last_error().decode())
+
+
+def model_desc(shape) -> ModelDesc:
+    """ModelDesc from any object with L, d, Hq, Hkv, dh, df, vocab, chan_unit, eps, rope_theta, seed."""
+    return ModelDesc(shape.L, shape.d, shape.Hq, shape.Hkv, shape.dh, shape.df, shape.vocab, shape.chan_unit,
+                     shape.eps, shape.rope_theta, shape.seed)
+
+
+class _MaskArgs:
+    """Owns the numpy buffers a MaskDesc points to."""
+
+    def __init__(self, kind, panel_mode=PANELS_COMPACT, budget=0.57, r_lo=0.35, r_hi=0.85, scores=None,
+                 target_u24=None, groups=None, units=None):
+        self.keep = []
+        d = MaskDesc()
+        d.kind, d.panel_mode, d.flop_budget, d.r_lo, d.r_hi = kind, panel_mode, budget, r_lo, r_hi
+        if scores is not None:
+            s = np.ascontiguousarray(scores, dtype=np.uint32)
+            t = np.ascontiguousarray(target_u24, dtype=np.uint32)
+            self.keep += [s, t]
+            d.scores = s.ctypes.data_as(POINTER(c_uint32))
+            d.target_u24 = t.ctypes.data_as(POINTER(c_uint32))
+        if groups is not None:
+            kg = np.ascontiguousarray(np.concatenate([np.asarray(g, np.int32) for g in groups] + [np.zeros(0, np.int32)]))
+            ng = np.ascontiguousarray([len(g) for g in groups], dtype=np.int32)
+            ku = np.ascontiguousarray(np.concatenate([np.asarray(u, np.int32) for u in units] + [np.zeros(0, np.int32)]))
+            nu = np.ascontiguousarray([len(u) for u in units], dtype=np.int32)
+            self.keep += [kg, ng, ku, nu]
+            d.keep_groups = kg.ctypes.data_as(POINTER(c_int32))
+            d.n_groups = ng.ctypes.data_as(POINTER(c_int32))
+            d.keep_units = ku.ctypes.data_as(POINTER(c_int32))
+            d.n_units = nu.ctypes.data_as(POINTER(c_int32))
+        self.desc = d
+
+
+def greedy_mask(scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85, panel_mode=PANELS_COMPACT):
+    return _MaskArgs(MASK_GREEDY, panel_mode, budget, r_lo, r_hi, scores=scores, target_u24=target_u24)
+
+
+def explicit_mask(groups, units, panel_mode=PANELS_COMPACT):
+    return _MaskArgs(MASK_EXPLICIT, panel_mode, groups=groups, units=units)
+
+
+def all_keep_mask():
+    return _MaskArgs(MASK_ALL_KEEP)
+
+
+def mask_select(shape, mask: _MaskArgs):
+    """Host-only mask compilation: (groups per layer, channel units per layer, flops array)."""
+    lib = load()
+    L, G, U = shape.L, shape.Hkv, shape.df // shape.chan_unit
+    kg = np.zeros(L * G, np.int32)
+    ng = np.zeros(L, np.int32)
+    ku = np.zeros(L * U, np.int32)
+    nu = np.zeros(L, np.int32)
+    fl = np.zeros(L + 3, np.int64)
+    md = model_desc(shape)
+    _check(lib.tasp_mask_select(ctypes.byref(md), ctypes.byref(mask.desc), kg.ctypes.data, ng.ctypes.data,
+                                ku.ctypes.data, nu.ctypes.data, fl.ctypes.data))
+    groups, units, og, ou = [], [], 0, 0
+    for layer in range(L):
+        groups.append(kg[og:og + ng[layer]].tolist())
+        units.append(ku[ou:ou + nu[layer]].tolist())
+        og += ng[layer]
+        ou += nu[layer]
+    return groups, units, fl
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return int(stream)
+
+
+class Plan:
+    def __init__(self, shape, mask: _MaskArgs):
+        lib = load()
+        self.shape = shape
+        self.handle = c_void_p()
+        md = model_desc(shape)
+        _check(lib.tasp_compile_mask(ctypes.byref(md), ctypes.byref(mask.desc), ctypes.byref(self.handle)))
+
+    def info(self) -> dict:
+        pi = PlanInfo()
+        _check(load().tasp_plan_info_get(self.handle, ctypes.byref(pi)))
+        return {name: getattr(pi, name) for name, _ in PlanInfo._fields_}
+
+    def layer_dims(self, layer):
+        out = np.zeros(2, np.int32)
+        _check(load().tasp_plan_layer_dims(self.handle, layer, out.ctypes.data))
+        return int(out[0]), int(out[1])
+
+    def export(self, layer, item):
+        sh = self.shape
+        m_kv, c = self.layer_dims(layer)
+        m_q = m_kv * (sh.Hq // sh.Hkv)
+        spec = {
+            EXPORT_KEEP_GROUPS: (np.int32, (m_kv,)),
+            EXPORT_KEEP_CHANS: (np.int32, (c,)),
+            EXPORT_QKV_W: (np.int8, ((m_q + 2 * m_kv) * sh.dh, sh.d)),
+            EXPORT_QKV_S: (np.float32, ((m_q + 2 * m_kv) * sh.dh,)),
+            EXPORT_O_W: (np.int8, (sh.d, m_q * sh.dh)),
+            EXPORT_O_S: (np.float32, (sh.d,)),
+            EXPORT_GU_W: (np.int8, (2 * c, sh.d)),
+            EXPORT_GU_S: (np.float32, (2 * c,)),
+            EXPORT_DOWN_W: (np.int8, (sh.d, c)),
+            EXPORT_DOWN_S: (np.float32, (sh.d,)),
+        }[item]
+        out = np.zeros(spec[1], dtype=spec[0])
+        _check(load().tasp_plan_export(self.handle, layer, item, out.ctypes.data, out.nbytes))
+        return out
+
+    def release(self):
+        if self.handle:
+            _check(load().tasp_release(self.handle))
+            self.handle = c_void_p()
+
+
+class Session:
+    def __init__(self, plan: Plan, max_tokens: int, handle=None):
+        self.plan = plan
+        self.handle = c_void_p() if handle is None else handle
+        if handle is None:
+            _check(load().tasp_session_create(plan.handle, max_tokens, ctypes.byref(self.handle)))
+
+    def fill_synthetic(self, t_prior: int, kv_seed: int, stream=None):
+        _check(load().tasp_session_fill_synthetic(self.handle, t_prior, kv_seed, _stream_ptr(stream)))
+
+    @property
+    def position(self) -> int:
+        v = c_int32()
+        _check(load().tasp_session_position(self.handle, ctypes.byref(v)))
+        return v.value
+
+    def layer_step(self, layer, x_in, x_out, stream=None):
+        _check(load().tasp_layer_step(self.handle, layer, x_in.data_ptr(), x_out.data_ptr(), _stream_ptr(stream)))
+
+    def release(self):
+        if self.handle:
+            _check(load().tasp_release(self.handle))
+            self.handle = c_void_p()
+
+
+def _handles(sessions):
+    arr = (c_void_p * len(sessions))(*[s.handle.value for s in sessions])
+    return ctypes.cast(arr, POINTER(c_void_p)), arr
+
+
+def decode_step(sessions, x_bf16, hidden=None, logits=None, stream=None):
+    """One decode step; x_bf16 is a CUDA bfloat16 tensor [n, d]; hidden / logits float32 CUDA tensors or None."""
+    p, keep = _handles(sessions)
+    _check(load().tasp_decode_step(p, len(sessions), x_bf16.data_ptr(),
+                                   hidden.data_ptr() if hidden is not None else None,
+                                   logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
+
+
+def decode_step_host(sessions, x_bf16_host, hidden_host=None, logits_host=None, stream=None):
+    """Decode step with host buffers (torch CPU tensors, ideally pinned); synchronizes the stream."""
+    p, keep = _handles(sessions)
+    _check(load().tasp_decode_step_host(p, len(sessions), x_bf16_host.data_ptr(),
+                                        hidden_host.data_ptr() if hidden_host is not None else None,
+                                        logits_host.data_ptr() if logits_host is not None else None,
+                                        _stream_ptr(stream)))
+
+
+def profile_step(sessions, x_bf16, logits=None, stream=None):
+    """Eager step with CUDA events around each kernel: {kind: (ms, launches)}."""
+    p, keep = _handles(sessions)
+    ms = np.zeros(KERNEL_KINDS, np.float32)
+    cnt = np.zeros(KERNEL_KINDS, np.int32)
+    _check(load().tasp_profile_step(p, len(sessions), x_bf16.data_ptr(),
+                                    logits.data_ptr() if logits is not None else None, _stream_ptr(stream),
+                                    ms.ctypes.data, cnt.ctypes.data))
+    return {KERNEL_NAMES[k]: (float(ms[k]), int(cnt[k])) for k in range(KERNEL_KINDS)}
+
+
+def step_launches(sessions, with_logits=True) -> int:
+    p, keep = _handles(sessions)
+    v = c_int32()
+    _check(load().tasp_step_launches(p, len(sessions), int(with_logits), ctypes.byref(v)))
+    return v.value
+
+
+def version() -> str:
+    return load().tasp_version().decode()

@@ -1,0 +1,97 @@
+"""CPU checks of the C-ABI library: it loads, exports every declared symbol, and its
+host mask compiler matches the oracle's bit for bit (no GPU work)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import ledger, maskc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_29499_gb300 import build
+    build.build()
+    from paper_2609_29499_gb300 import tasp
+    return tasp
+
+
+def _declared_symbols():
+    src = open(os.path.join(ROOT, "include", "tasp.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:int|const char\*)\s+(tasp_\w+)\s*\(", src, re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared_symbols()
+    assert len(names) >= 15
+    so = ctypes.CDLL(lib.LIB_PATH)
+    for n in names:
+        assert hasattr(so, n), n
+    assert set(names) == set(lib.EXPORTED)
+    assert "sm_103a" in lib.version()
+
+
+CASES = [(synth.LAYER1, (1000, 1001, 77)), (synth.LLAMA3_8B, synth.MASK_SEEDS), (synth.LLAMA3_70B, synth.MASK_SEEDS),
+         (synth.tiny_shape(L=7), (3, 4, 5))]
+
+
+@pytest.mark.parametrize("shape,seeds", CASES)
+def test_host_mask_compiler_matches_oracle(lib, shape, seeds):
+    for seed in seeds:
+        sc = synth.mask_scores_u32(seed, shape.L, shape.n_units)
+        tg = synth.layer_target_u24(seed, shape.L)
+        want = maskc.compile_mask(shape, sc, tg, 0.57, 0.35, 0.85)
+        groups, units, fl = lib.mask_select(shape, lib.greedy_mask(sc, tg, 0.57, 0.35, 0.85))
+        assert groups == want.keep_groups
+        assert units == want.keep_units
+        assert fl[:shape.L].tolist() == want.info["layer_flops"]
+        assert fl[shape.L] == want.info["total_flops"]
+        assert fl[shape.L + 1] == want.info["budget_flops"]
+        assert fl[shape.L + 2] == shape.L * ledger.dense_layer_flops(shape)
+
+
+def test_other_budgets_match_oracle(lib):
+    sh = synth.LLAMA3_8B
+    for budget, lo, hi in ((0.3, 0.2, 0.5), (0.7, 0.5, 0.9), (0.57, 0.57, 0.57)):
+        sc = synth.mask_scores_u32(9, sh.L, sh.n_units)
+        tg = synth.layer_target_u24(9, sh.L)
+        want = maskc.compile_mask(sh, sc, tg, budget, lo, hi)
+        groups, units, _ = lib.mask_select(sh, lib.greedy_mask(sc, tg, budget, lo, hi))
+        assert groups == want.keep_groups and units == want.keep_units
+
+
+def test_explicit_and_all_keep(lib):
+    sh = synth.tiny_shape(L=2)
+    g = [[0], [1]]
+    u = [[0, 3, 5], [2]]
+    groups, units, fl = lib.mask_select(sh, lib.explicit_mask(g, u))
+    assert groups == g and units == u
+    m = maskc.explicit(sh, g, u)
+    assert fl[sh.L] == ledger.mask_flops(sh, m.keep_groups, m.keep_chans)
+    groups, units, fl = lib.mask_select(sh, lib.all_keep_mask())
+    assert groups == [list(range(sh.Hkv))] * sh.L
+    assert fl[sh.L] == fl[sh.L + 2]
+
+
+def test_invalid_requests_are_rejected(lib):
+    sh = synth.tiny_shape(L=2)
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select(sh, lib.explicit_mask([[1, 0], [0]], [[0], [0]]))  # not ascending
+    assert e.value.code == lib.EINVAL
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select(sh, lib.explicit_mask([[0], [5]], [[0], [0]]))  # group out of range
+    assert e.value.code == lib.EINVAL
+    sc = synth.mask_scores_u32(1, sh.L, sh.n_units)
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select(sh, lib.greedy_mask(sc, synth.layer_target_u24(1, sh.L), budget=1.5))
+    assert e.value.code == lib.EINVAL
+    bad = synth.tiny_shape(d=100)  # d not a multiple of 16
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select(bad, lib.all_keep_mask())
+    assert e.value.code == lib.EINVAL
+    assert "multiples of 16" in str(e.value)
