@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--dense", action="store_true", help="time the dense fallback plan instead of the mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="keep the workload's widths but only this many layers (small cases for ncu captures)")
     return ap.parse_args()
 
 
@@ -139,7 +141,11 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ workload
 def workload(args):
+    import dataclasses
     wl = synth.CONFIGS[args.config]
+    if args.layers:
+        sh = dataclasses.replace(wl.shape, L=args.layers)
+        wl = dataclasses.replace(wl, shape=sh, name=f"{wl.name}_{args.layers}layers")
     return wl, wl.shape, wl.masks[0]
 
 
@@ -155,12 +161,12 @@ def gemv_bytes(shape, plan_dims):
     b = {"qkv": 0, "o_proj": 0, "gate_up": 0, "down": 0}
     for m_kv, c in plan_dims:
         rows = m_kv * (g + 2) * dh
-        b["qkv"] += rows * d + rows * 4 + d * 4 + d * 4 + rows * 2
+        b["qkv"] += rows * d + rows * 4 + d * 4 + d * 4 + m_kv * g * dh * 4 + m_kv * 2 * dh * 2
         if m_kv:
-            b["o_proj"] += d * m_kv * g * dh + d * 4 + m_kv * g * dh * 2 + 2 * d * 4
+            b["o_proj"] += d * m_kv * g * dh + d * 4 + m_kv * g * dh * 4 + 2 * d * 4
         if c:
-            b["gate_up"] += 2 * c * d + 2 * c * 4 + d * 4 + d * 4 + c * 2
-            b["down"] += d * c + d * 4 + c * 2 + 2 * d * 4
+            b["gate_up"] += 2 * c * d + 2 * c * 4 + d * 4 + d * 4 + c * 4
+            b["down"] += d * c + d * 4 + c * 4 + 2 * d * 4
     b["lm_head"] = shape.vocab * d * 2 + d * 4 + shape.vocab * 4
     return b
 
@@ -344,7 +350,7 @@ def run_ours(args):
         out = {
             "metric": METRIC, "value": round(ms, 4), "unit": "ms/token", "n_gpus": world, "steps": K, "warmup": Wm,
             "ms_per_step": round(ms, 4), "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
-            "dtype": "int8w-bf16", "data": "synthetic",
+            "dtype": "int8w-f32", "data": "synthetic",
             "config": {"workload": wl.name + ("_dense" if args.dense else ""),
                        "mask": "all-keep dense fallback" if args.dense else
                        f"greedy dependency-closed, active-FLOP ratio {info['flops_retained'] / info['flops_dense']:.4f}",

@@ -149,6 +149,12 @@ int tasp_session_fill_synthetic(tasp_session* s, int32_t t_prior, uint64_t kv_se
 /* Current position (number of cached tokens) as tracked on the host. */
 int tasp_session_position(const tasp_session* s, int32_t* pos);
 
+/* Device-side status of a session's kernels: *device_error = 0 when no kernel
+ * reported a failure; bit 0 set when a bounded wait inside a kernel gave up
+ * (the step's outputs are then invalid). Synchronizes the device; clears the word
+ * when `clear` is nonzero. */
+int tasp_session_status(tasp_session* s, int32_t clear, int32_t* device_error);
+
 /* tasp_decode_step with HOST buffers: h_x_bf16 [n][d] is copied to the device
  * (should be pinned memory), the step runs, and the requested outputs are
  * copied back to h_hidden_out [n][d] / h_logits [n][vocab] (either may be

@@ -8,16 +8,16 @@
 //    group keeps R x CPT 128-bit streaming loads in flight per thread;
 //  * the next group is loaded into a second register buffer and the one after is
 //    prefetched into L2 with cp.async.bulk.prefetch while the current one is reduced;
-//  * the activation vector (BF16 values) sits in shared memory as FP32 with an XOR
-//    swizzle that makes the per-chunk 128-bit reads conflict-free;
+//  * the activation vector sits in shared memory as FP32 with an XOR swizzle that
+//    makes the per-chunk 128-bit reads conflict-free (activations stay FP32 inside a
+//    step; the KV cache, step inputs and LM head are BF16);
 //  * INT8 -> FP32 is exact: byte ^ 0x80 is placed in the mantissa of 2^23 with PRMT and
 //    2^23 + 128 is subtracted (packed f32x2 add), then packed f32x2 FMAs accumulate;
 //    the row scale is applied once after the reduction;
 //  * the previous kernel's tail is overlapped with programmatic dependent launch:
 //    weights (which never depend on the previous kernel) are fetched before
 //    griddepcontrol.wait, activations after it.
-// Attention is a split-KV (flash-decoding) kernel over the retained KV heads only; the
-// last CTA of each KV group (atomic ticket, no waiting) merges the splits.
+// Attention (attention.cu) is a split-KV kernel over the retained KV heads only.
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -30,10 +30,8 @@ namespace tasp {
 
 namespace {
 
-constexpr int NT = 256;
+constexpr int NT = 512;  // consumer threads of a GEMV CTA
 constexpr int NWARP = NT / 32;
-constexpr int ATT_THREADS = 256;
-constexpr int ATT_SPLITS_MAX = 64;
 
 enum GemvMode { M_QKV = 0, M_O = 1, M_GU = 2, M_DOWN = 3, M_LM = 4 };
 
@@ -48,31 +46,23 @@ struct GemvParams {
     float* x_resid_init;
     const float* gamma;
     float eps;
-    const uint16_t* act;
+    const float* act;
     float* resid_out;
     float* hidden_out;
-    uint16_t* q_out;
+    float* q_out;
     uint16_t* k_cache;
     uint16_t* v_cache;
     int max_tokens;
     const float2* rope;
     const int* pos;
     int g, dh;
-    uint16_t* h_out;
+    float* h_out;
     float* logits;
+    int* err;       // device error word (bounded waits that gave up)
+    int smem_cap;   // dynamic shared memory available to the launch
 };
 
-struct AttnParams {
-    const uint16_t* q;
-    const uint16_t* K;
-    const uint16_t* V;
-    const int* pos;
-    int max_tokens;
-    float qscale;  // 1/sqrt(dh) * log2(e)
-    float* part;
-    int* cnt;
-    uint16_t* o;
-};
+
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
@@ -124,7 +114,6 @@ __device__ __forceinline__ int swz(int f) {
 }
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
-__device__ __forceinline__ float round_bf16(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
 __device__ __forceinline__ uint16_t f32_to_bf16_bits(float v) {
     __nv_bfloat16 b = __float2bfloat16_rn(v);
     return *reinterpret_cast<uint16_t*>(&b);
@@ -136,8 +125,17 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
+constexpr int CW = NWARP;                // consumer warps
+constexpr int CT = CW * 32;              // consumer threads
+constexpr int GEMV_THREADS = CT + 32;    // + producer warp
+constexpr int MAX_STAGES = 8;
+constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s) before a wait gives up
+constexpr int ERR_WAIT_TIMEOUT = 1;
+
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(CT) : "memory"); }
+
 // ---------------------------------------------------------------- activation prologues
-// x^ = bf16(x * (1/sqrt(mean(x^2) + eps)) * gamma) into swizzled FP32 shared memory.
+// x^ = x * (1/sqrt(mean(x^2) + eps)) * gamma (FP32) into swizzled shared memory.
 // Every CTA reduces in the same fixed order, so all CTAs see identical x^.
 template <int F>
 __device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __restrict__ x_in, float* x_init,
@@ -163,7 +161,7 @@ __device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __rest
     }
     ss = warp_sum(ss);
     if ((tid & 31) == 0) stat[tid >> 5] = ss;
-    __syncthreads();
+    consumer_sync();
     float tot = 0.f;
 #pragma unroll
     for (int w = 0; w < NWARP; ++w) tot += stat[w];
@@ -181,30 +179,34 @@ __device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __rest
                 v = reinterpret_cast<const float4*>(x)[f];
             }
             float4 gm = reinterpret_cast<const float4*>(gamma)[f];
-            o.x = round_bf16((v.x * inv) * gm.x);
-            o.y = round_bf16((v.y * inv) * gm.y);
-            o.z = round_bf16((v.z * inv) * gm.z);
-            o.w = round_bf16((v.w * inv) * gm.w);
+            o.x = (v.x * inv) * gm.x;
+            o.y = (v.y * inv) * gm.y;
+            o.z = (v.z * inv) * gm.z;
+            o.w = (v.w * inv) * gm.w;
         }
         xs[swz<F>(f)] = o;
     }
-    __syncthreads();
+    consumer_sync();
 }
 
-// BF16 activation vector [K] -> swizzled FP32 shared memory (zero padded to nchunks*16)
-__device__ void bf16_to_smem(const uint16_t* __restrict__ a, int K, int nchunks, float4* xs) {
+// FP32 activation vector [K] -> swizzled shared memory (zero padded to nchunks*16)
+__device__ void f32_to_smem(const float* __restrict__ a, int K, int nchunks, float4* xs) {
     const int tid = threadIdx.x;
     const int ntot4 = nchunks * 4;
     for (int f = tid; f < ntot4; f += NT) {
         float4 o;
-        int e = 4 * f;
-        o.x = (e + 0 < K) ? bf16_to_f32(a[e + 0]) : 0.f;
-        o.y = (e + 1 < K) ? bf16_to_f32(a[e + 1]) : 0.f;
-        o.z = (e + 2 < K) ? bf16_to_f32(a[e + 2]) : 0.f;
-        o.w = (e + 3 < K) ? bf16_to_f32(a[e + 3]) : 0.f;
+        const int e = 4 * f;
+        if (e + 3 < K) {
+            o = *reinterpret_cast<const float4*>(a + e);
+        } else {
+            o.x = (e + 0 < K) ? a[e + 0] : 0.f;
+            o.y = (e + 1 < K) ? a[e + 1] : 0.f;
+            o.z = (e + 2 < K) ? a[e + 2] : 0.f;
+            o.w = (e + 3 < K) ? a[e + 3] : 0.f;
+        }
         xs[swz<4>(f)] = o;
     }
-    __syncthreads();
+    consumer_sync();
 }
 
 // ---------------------------------------------------------------- row addressing
@@ -228,82 +230,113 @@ __device__ __forceinline__ const int8_t* row_ptr(const GemvParams& p, int w) {
 }
 
 // ---------------------------------------------------------------- the GEMV core
-template <int R, int CPT>
-struct WRegs {
-    int4 v[R][CPT];
-};
+// One persistent CTA per SM: warp CW is the producer, warps 0..CW-1 consume.
+// The producer streams row groups (R rows, one bulk copy per row) into an NS-stage
+// shared-memory ring; stage s has a "full" mbarrier (transaction bytes) and an
+// "empty" mbarrier (released by the consumers after their last read of the stage).
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
-template <int MODE, int R, int CPT>
-__device__ __forceinline__ void load_group(WRegs<R, CPT>& wr, const GemvParams& p, int gi, int tid) {
-    const int8_t* rp[R];
-#pragma unroll
-    for (int r = 0; r < R; ++r) rp[r] = row_ptr<MODE>(p, gi * R + r);
-#pragma unroll
-    for (int i = 0; i < CPT; ++i) {
-        const int c = tid + i * NT;
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            if (c < p.nchunks)
-                wr.v[r][i] = ld_stream16(rp[r] + (int64_t)c * 16);
-            else
-                wr.v[r][i] = make_int4(0, 0, 0, 0);
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: gives up after WAIT_LIMIT cycles, records the failure in the device
+// error word and makes every later wait of this CTA return at once (abort), so a lost
+// transfer can never hang the GPU; the host reports the error word.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
+                                          bool honor_abort = true) {
+    if (honor_abort && *(volatile int*)abort_flag) return;
+    if (mbar_try(bar, parity)) return;
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity)) {
+        if (clock64() - t0 > WAIT_LIMIT) {
+            *(volatile int*)abort_flag = 1;
+            if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
+            return;
         }
     }
 }
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
 
-template <int MODE, int R>
-__device__ __forceinline__ void prefetch_group(const GemvParams& p, int gi, int g1, int tid) {
-    if (tid < R && gi < g1) {
-        const int w = gi * R + tid;
-        if (w < p.rows) prefetch_l2(row_ptr<MODE>(p, w), (uint32_t)(p.nchunks * 16));
+// This thread's slice of the activation vector, kept in registers for the whole
+// kernel: chunk j of the thread is c = tid + j * CT (16 weight bytes per chunk).
+template <int XC, int F>
+struct XRegs {
+    float4 v[XC][F];
+};
+
+template <int XC, int F>
+__device__ __forceinline__ void load_x(XRegs<XC, F>& xr, const float4* xs, int nchunks, int tid) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+#pragma unroll
+        for (int e = 0; e < F; ++e)
+            xr.v[j][e] = c < nchunks ? xs[swz<F>(F * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 }
 
-// INT8 chunk dot products: acc[r] (packed pairs) += w[r] . x
-template <int R, int CPT>
-__device__ __forceinline__ void dot_i8(const WRegs<R, CPT>& wr, const float4* __restrict__ xs, int nchunks, int tid,
-                                       u64 (&acc)[R]) {
+// INT8 rows of one stage . x: acc[r] (packed pairs) += w[r] . x
+template <int R, int XC>
+__device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XRegs<XC, 4>& xr,
+                                       int nchunks, int tid, u64 (&acc)[R]) {
     const u64 magic = pk(-8388736.0f, -8388736.0f);  // -(2^23 + 128)
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
-        const int c = tid + i * NT;
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
         if (c < nchunks) {
-            float4 xv[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) xv[j] = xs[swz<4>(4 * c + j)];
 #pragma unroll
             for (int r = 0; r < R; ++r) {
-                const uint32_t wd[4] = {(uint32_t)wr.v[r][i].x, (uint32_t)wr.v[r][i].y, (uint32_t)wr.v[r][i].z,
-                                        (uint32_t)wr.v[r][i].w};
+                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
+                const uint32_t wd[4] = {(uint32_t)wv.x, (uint32_t)wv.y, (uint32_t)wv.z, (uint32_t)wv.w};
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const uint32_t u = wd[j] ^ 0x80808080u;
+                for (int k = 0; k < 4; ++k) {
+                    const uint32_t u = wd[k] ^ 0x80808080u;
                     u64 p01 = pk(__uint_as_float(prmt(u, 0x4B000000u, 0x7540u)),
                                  __uint_as_float(prmt(u, 0x4B000000u, 0x7541u)));
                     u64 p23 = pk(__uint_as_float(prmt(u, 0x4B000000u, 0x7542u)),
                                  __uint_as_float(prmt(u, 0x4B000000u, 0x7543u)));
                     p01 = add2(p01, magic);
                     p23 = add2(p23, magic);
-                    acc[r] = fma2(p01, pk(xv[j].x, xv[j].y), acc[r]);
-                    acc[r] = fma2(p23, pk(xv[j].z, xv[j].w), acc[r]);
+                    acc[r] = fma2(p01, pk(xr.v[j][k].x, xr.v[j][k].y), acc[r]);
+                    acc[r] = fma2(p23, pk(xr.v[j][k].z, xr.v[j][k].w), acc[r]);
                 }
             }
         }
     }
 }
 
-// BF16 chunk dot products (LM head): 8 weights per 16-byte chunk
-template <int R, int CPT>
-__device__ __forceinline__ void dot_bf16(const WRegs<R, CPT>& wr, const float4* __restrict__ xs, int nchunks, int tid,
-                                         u64 (&acc)[R]) {
+// BF16 rows (LM head): 8 weights per 16-byte chunk
+template <int R, int XC>
+__device__ __forceinline__ void dot_bf16(const uint8_t* __restrict__ stage, int ld, const XRegs<XC, 2>& xr,
+                                         int nchunks, int tid, u64 (&acc)[R]) {
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
-        const int c = tid + i * NT;
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
         if (c < nchunks) {
-            const float4 x0 = xs[swz<2>(2 * c)], x1 = xs[swz<2>(2 * c + 1)];
+            const float4 x0 = xr.v[j][0], x1 = xr.v[j][1];
 #pragma unroll
             for (int r = 0; r < R; ++r) {
-                const uint32_t w0 = wr.v[r][i].x, w1 = wr.v[r][i].y, w2 = wr.v[r][i].z, w3 = wr.v[r][i].w;
+                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
+                const uint32_t w0 = wv.x, w1 = wv.y, w2 = wv.z, w3 = wv.w;
                 acc[r] = fma2(pk(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xffff0000u)), pk(x0.x, x0.y), acc[r]);
                 acc[r] = fma2(pk(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xffff0000u)), pk(x0.z, x0.w), acc[r]);
                 acc[r] = fma2(pk(__uint_as_float(w2 << 16), __uint_as_float(w2 & 0xffff0000u)), pk(x1.x, x1.y), acc[r]);
@@ -313,40 +346,44 @@ __device__ __forceinline__ void dot_bf16(const WRegs<R, CPT>& wr, const float4* 
     }
 }
 
-// Reduce, then the mode's epilogue for one row group.
-template <int MODE, int R, int CPT>
-__device__ __forceinline__ void finish_group(const GemvParams& p, const WRegs<R, CPT>& wr, const float4* xs, int gi,
-                                             float (*red)[NWARP][R], int parity, int tid) {
-    u64 acc[R];
+// Warp reduction of R row sums at once: each butterfly level halves the vector a lane
+// carries, so lane l ends with the full sum of row l / (32 / R).
+template <int R>
+__device__ __forceinline__ float row_reduce(float (&v)[R], int lane) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) acc[r] = 0ull;
-    if (MODE == M_LM)
-        dot_bf16<R, CPT>(wr, xs, p.nchunks, tid, acc);
-    else
-        dot_i8<R, CPT>(wr, xs, p.nchunks, tid, acc);
-    const int lane = tid & 31, warp = tid >> 5;
+    for (int n = R, o = 16; n > 1; n >>= 1, o >>= 1) {
+        const bool up = (lane & o) != 0;
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-        float2 a = upk(acc[r]);
-        float v = warp_sum(a.x + a.y);
-        if (lane == 0) red[parity][warp][r] = v;
+        for (int i = 0; i < n / 2; ++i) {
+            const float send = up ? v[i] : v[i + n / 2];
+            const float keep = up ? v[i + n / 2] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
     }
-    __syncthreads();
+    float s = v[0];
+#pragma unroll
+    for (int o = 16 / R; o >= 1; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    return s;
+}
+
+// Epilogue of one row group from the per-warp partial sums red[w][r].
+template <int MODE, int R>
+__device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)[R], int gi, int tid) {
     const int w0 = gi * R;
     if (MODE == M_QKV || MODE == M_GU) {
         if (tid < R / 2) {
             float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-            for (int w = 0; w < NWARP; ++w) {
-                s0 += red[parity][w][2 * tid];
-                s1 += red[parity][w][2 * tid + 1];
+            for (int w = 0; w < CW; ++w) {
+                s0 += red[w][2 * tid];
+                s1 += red[w][2 * tid + 1];
             }
             const int wa = w0 + 2 * tid;
             if (wa < p.rows) {
                 if (MODE == M_GU) {
                     const float a = p.scale[wa] * s0, b = p.scale[wa + 1] * s1;
                     const float silu = a / (1.0f + expf(-a));
-                    p.h_out[wa >> 1] = f32_to_bf16_bits(silu * b);
+                    p.h_out[wa >> 1] = silu * b;
                 } else {
                     const int half = p.dh >> 1;
                     const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
@@ -361,52 +398,99 @@ __device__ __forceinline__ void finish_group(const GemvParams& p, const WRegs<R,
                         y0 = a;
                         y1 = b;
                     }
-                    uint16_t* dst;
-                    if (hh < p.g)
-                        dst = p.q_out + (int64_t)(jl * p.g + hh) * p.dh;
-                    else if (hh == p.g)
-                        dst = p.k_cache + ((int64_t)jl * p.max_tokens + pos) * p.dh;
-                    else
-                        dst = p.v_cache + ((int64_t)jl * p.max_tokens + pos) * p.dh;
-                    dst[i] = f32_to_bf16_bits(y0);
-                    dst[i + half] = f32_to_bf16_bits(y1);
+                    if (hh < p.g) {
+                        float* dq = p.q_out + (int64_t)(jl * p.g + hh) * p.dh;
+                        dq[i] = y0;
+                        dq[i + half] = y1;
+                    } else {
+                        uint16_t* dst = (hh == p.g ? p.k_cache : p.v_cache) + ((int64_t)jl * p.max_tokens + pos) * p.dh;
+                        dst[i] = f32_to_bf16_bits(y0);  // the KV cache is BF16
+                        dst[i + half] = f32_to_bf16_bits(y1);
+                    }
                 }
             }
         }
-    } else {
-        if (tid < R) {
-            float s = 0.f;
+    } else if (tid < R) {
+        float s = 0.f;
 #pragma unroll
-            for (int w = 0; w < NWARP; ++w) s += red[parity][w][tid];
-            const int row = w0 + tid;
-            if (row < p.rows) {
-                if (MODE == M_LM) {
-                    p.logits[row] = s;
-                } else {
-                    const float v = p.resid_out[row] + p.scale[row] * s;
-                    p.resid_out[row] = v;
-                    if (p.hidden_out) p.hidden_out[row] = v;
-                }
+        for (int w = 0; w < CW; ++w) s += red[w][tid];
+        const int row = w0 + tid;
+        if (row < p.rows) {
+            if (MODE == M_LM) {
+                p.logits[row] = s;
+            } else {
+                const float v = p.resid_out[row] + p.scale[row] * s;
+                p.resid_out[row] = v;
+                if (p.hidden_out) p.hidden_out[row] = v;
             }
         }
     }
 }
 
-template <int MODE, int R, int CPT>
-__global__ void __launch_bounds__(NT) gemv_kernel(const GemvParams p) {
-    extern __shared__ __align__(16) float4 xs[];
-    __shared__ float red[2][NWARP][R];
-    __shared__ float stat[NWARP];
-    const int tid = threadIdx.x;
+// Shared-memory plan of one launch (host and device agree on it).
+struct GemvSmem {
+    int x_bytes, stage_bytes, nstages, total;
+};
+__host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap) {
+    GemvSmem g;
+    g.x_bytes = ((nchunks * F * 16) + 127) & ~127;
+    g.stage_bytes = ((R * ld) + 127) & ~127;
+    const int bar_bytes = 2 * MAX_STAGES * 8 + 16;
+    int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
+    g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
+    g.total = g.x_bytes + g.nstages * g.stage_bytes + bar_bytes;
+    return g;
+}
+
+template <int MODE, int R, int XC>
+__global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams p) {
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ float red[2][CW][R];
+    __shared__ float stat[CW];
+    __shared__ int abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    const int NS = L.nstages;
+    float4* xs = reinterpret_cast<float4*>(sm);
+    uint8_t* stages = sm + L.x_bytes;
+    const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
+    const uint32_t empty0 = full0 + 8 * MAX_STAGES;
     const int NG = (p.rows + R - 1) / R;
     const int g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
     const int g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
 
-    // weights never depend on the previous kernel: start streaming them now
-    prefetch_group<MODE, R>(p, g0 + 1, g1, tid);
-    WRegs<R, CPT> A, B;
-    if (g0 < g1) load_group<MODE, R, CPT>(A, p, g0, tid);
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
 
+    if (warp == CW) {
+        // ---- producer: weights never depend on the previous kernel, so start at once
+        pdl_trigger();
+        if (lane == 0) {
+            for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
+                const int s = i % NS, k = i / NS;
+                if (k > 0) mbar_wait(empty0 + 8 * s, (k - 1) & 1, &abort_flag, p.err);
+                const int nrow = min(R, p.rows - gi * R);
+                mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
+                for (int r = 0; r < nrow; ++r)
+                    bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)r * p.ld),
+                             row_ptr<MODE>(p, gi * R + r), (uint32_t)p.ld, full0 + 8 * s);
+            }
+            // never leave while copies into this CTA's shared memory are in flight (even
+            // after an abort: this second wait is bounded on its own)
+            for (int gi = max(g0, g1 - NS), i = gi - g0; gi < g1; ++gi, ++i)
+                mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, false);
+        }
+        return;
+    }
+
+    // ---- consumers
     pdl_wait();
     pdl_trigger();
     if (MODE == M_QKV || MODE == M_GU)
@@ -414,160 +498,34 @@ __global__ void __launch_bounds__(NT) gemv_kernel(const GemvParams p) {
     else if (MODE == M_LM)
         norm_to_smem<2>(p.x_resid, nullptr, nullptr, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
     else
-        bf16_to_smem(p.act, p.K, p.nchunks, xs);
+        f32_to_smem(p.act, p.K, p.nchunks, xs);
 
-    for (int gi = g0; gi < g1; gi += 2) {
-        if (gi + 1 < g1) load_group<MODE, R, CPT>(B, p, gi + 1, tid);
-        prefetch_group<MODE, R>(p, gi + 2, g1, tid);
-        finish_group<MODE, R, CPT>(p, A, xs, gi, red, 0, tid);
-        if (gi + 1 < g1) {
-            if (gi + 2 < g1) load_group<MODE, R, CPT>(A, p, gi + 2, tid);
-            prefetch_group<MODE, R>(p, gi + 3, g1, tid);
-            finish_group<MODE, R, CPT>(p, B, xs, gi + 1, red, 1, tid);
+    constexpr int F = MODE == M_LM ? 2 : 4;
+    XRegs<XC, F> xr;
+    load_x<XC, F>(xr, xs, p.nchunks, tid);
+    for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
+        const int s = i % NS, k = i / NS;
+        mbar_wait(full0 + 8 * s, k & 1, &abort_flag, p.err);
+        const uint8_t* st = stages + (size_t)s * L.stage_bytes;
+        u64 acc[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) acc[r] = 0ull;
+        if constexpr (MODE == M_LM)
+            dot_bf16<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
+        else
+            dot_i8<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
+        float v[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const float2 a = upk(acc[r]);
+            v[r] = a.x + a.y;
         }
+        const float rs = row_reduce<R>(v, lane);
+        if ((lane & (32 / R - 1)) == 0) red[i & 1][warp][lane / (32 / R)] = rs;
+        consumer_sync();  // every consumer is done reading stage s, partial sums are visible
+        if (tid == 0) mbar_arrive(empty0 + 8 * s);
+        epilogue<MODE, R>(p, red[i & 1], gi, tid);
     }
-}
-
-// ---------------------------------------------------------------- attention
-template <int DH, int G>
-__global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const AttnParams p) {
-    constexpr int DPL = DH / 32;
-    __shared__ float sm_m[NWARP][G], sm_l[NWARP][G];
-    __shared__ float sm_acc[NWARP][G][DH];
-    __shared__ int is_last;
-    const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-    // The prior cache does not depend on the previous kernel (only position T-1 does,
-    // and L2 is coherent): pull this CTA's K/V range into L2 before waiting.
-    const int T = *p.pos + 1;  // written by the previous step, which has completed
-    const int chunk = (T + S - 1) / S;
-    const int p0 = split * chunk, p1 = min(T, p0 + chunk);
-    const uint16_t* Kg = p.K + (int64_t)jl * p.max_tokens * DH;
-    const uint16_t* Vg = p.V + (int64_t)jl * p.max_tokens * DH;
-    if (tid == 0 && p1 > p0) prefetch_l2(Kg + (int64_t)p0 * DH, (uint32_t)((p1 - p0) * DH * 2));
-    if (tid == 32 && p1 > p0) prefetch_l2(Vg + (int64_t)p0 * DH, (uint32_t)((p1 - p0) * DH * 2));
-    pdl_wait();
-    pdl_trigger();
-
-    float q[G][DPL];
-#pragma unroll
-    for (int h = 0; h < G; ++h)
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) q[h][e] = bf16_to_f32(p.q[(int64_t)(jl * G + h) * DH + lane * DPL + e]) * p.qscale;
-    float m[G], l[G], acc[G][DPL];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        m[h] = -INFINITY;
-        l[h] = 0.f;
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) acc[h][e] = 0.f;
-    }
-    constexpr int UNR = 4;
-    for (int t0 = p0 + warp; t0 < p1; t0 += UNR * NWARP) {
-        float k[UNR][DPL], v[UNR][DPL];
-#pragma unroll
-        for (int u = 0; u < UNR; ++u) {
-            const int t = t0 + u * NWARP;
-            if (t < p1) {
-                const uint16_t* kp = Kg + (int64_t)t * DH + lane * DPL;
-                const uint16_t* vp = Vg + (int64_t)t * DH + lane * DPL;
-                if constexpr (DPL == 4) {
-                    const uint2 kb = *reinterpret_cast<const uint2*>(kp);
-                    const uint2 vb = *reinterpret_cast<const uint2*>(vp);
-                    k[u][0] = __uint_as_float(kb.x << 16);
-                    k[u][1] = __uint_as_float(kb.x & 0xffff0000u);
-                    k[u][2] = __uint_as_float(kb.y << 16);
-                    k[u][3] = __uint_as_float(kb.y & 0xffff0000u);
-                    v[u][0] = __uint_as_float(vb.x << 16);
-                    v[u][1] = __uint_as_float(vb.x & 0xffff0000u);
-                    v[u][2] = __uint_as_float(vb.y << 16);
-                    v[u][3] = __uint_as_float(vb.y & 0xffff0000u);
-                } else {
-                    const uint32_t kb = *reinterpret_cast<const uint32_t*>(kp);
-                    const uint32_t vb = *reinterpret_cast<const uint32_t*>(vp);
-                    k[u][0] = __uint_as_float(kb << 16);
-                    k[u][1] = __uint_as_float(kb & 0xffff0000u);
-                    v[u][0] = __uint_as_float(vb << 16);
-                    v[u][1] = __uint_as_float(vb & 0xffff0000u);
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < UNR; ++u) {
-            if (t0 + u * NWARP < p1) {
-                float sc[G];
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    float a = 0.f;
-#pragma unroll
-                    for (int e = 0; e < DPL; ++e) a = fmaf(q[h][e], k[u][e], a);
-                    sc[h] = warp_sum(a);
-                }
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    const float mn = fmaxf(m[h], sc[h]);
-                    const float c = exp2f(m[h] - mn);  // m = -inf before the first key gives 0
-                    const float pe = exp2f(sc[h] - mn);
-                    l[h] = l[h] * c + pe;
-#pragma unroll
-                    for (int e = 0; e < DPL; ++e) acc[h][e] = fmaf(acc[h][e], c, pe * v[u][e]);
-                    m[h] = mn;
-                }
-            }
-        }
-    }
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        if (lane == 0) {
-            sm_m[warp][h] = m[h];
-            sm_l[warp][h] = l[h];
-        }
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) sm_acc[warp][h][lane * DPL + e] = acc[h][e];
-    }
-    __syncthreads();
-    float* part = p.part + (int64_t)(jl * S + split) * G * (DH + 2);
-    for (int it = tid; it < G * DH; it += ATT_THREADS) {
-        const int h = it / DH, dim = it - h * DH;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < NWARP; ++w) M = fmaxf(M, sm_m[w][h]);
-        float Ls = 0.f, As = 0.f;
-#pragma unroll
-        for (int w = 0; w < NWARP; ++w) {
-            const float sc = (sm_m[w][h] == -INFINITY) ? 0.f : exp2f(sm_m[w][h] - M);
-            Ls = fmaf(sm_l[w][h], sc, Ls);
-            As = fmaf(sm_acc[w][h][dim], sc, As);
-        }
-        part[h * (DH + 2) + dim] = As;
-        if (dim == 0) {
-            part[h * (DH + 2) + DH] = M;
-            part[h * (DH + 2) + DH + 1] = Ls;
-        }
-    }
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) is_last = (atomicAdd(p.cnt + jl, 1) == S - 1);
-    __syncthreads();
-    if (!is_last) return;
-    __threadfence();
-    const float* pg = p.part + (int64_t)jl * S * G * (DH + 2);
-    for (int it = tid; it < G * DH; it += ATT_THREADS) {
-        const int h = it / DH, dim = it - h * DH;
-        float M = -INFINITY;
-        for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(pg + (sp * G + h) * (DH + 2) + DH));
-        float Ls = 0.f, As = 0.f;
-        for (int sp = 0; sp < S; ++sp) {
-            const float* e = pg + (sp * G + h) * (DH + 2);
-            const float ms = __ldcg(e + DH);
-            const float sc = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-            Ls = fmaf(__ldcg(e + DH + 1), sc, Ls);
-            As = fmaf(__ldcg(e + dim), sc, As);
-        }
-        p.o[(int64_t)(jl * G + h) * DH + dim] = f32_to_bf16_bits(As / Ls);
-    }
-    if (tid == 0) p.cnt[jl] = 0;
 }
 
 __global__ void advance_kernel(int* pos) {
@@ -595,88 +553,78 @@ int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const
 
 typedef void (*GemvFn)(const GemvParams);
 
-struct GemvVariant {
-    GemvFn fn;
-    int R, CPT;
-};
-
 template <int MODE>
-GemvVariant pick_variant(int nchunks) {
-    const int cpt = (nchunks + NT - 1) / NT;
-    if (cpt <= 1) return {gemv_kernel<MODE, 8, 1>, 8, 1};
-    if (cpt <= 2) return {gemv_kernel<MODE, 4, 2>, 4, 2};
-    if (cpt <= 4) return {gemv_kernel<MODE, 2, 4>, 2, 4};
-    return {gemv_kernel<MODE, 2, 8>, 2, 8};
-}
-
-GemvVariant pick(int mode, int nchunks) {
-    switch (mode) {
-        case M_QKV: return pick_variant<M_QKV>(nchunks);
-        case M_O: return pick_variant<M_O>(nchunks);
-        case M_GU: return pick_variant<M_GU>(nchunks);
-        case M_DOWN: return pick_variant<M_DOWN>(nchunks);
-        default: return pick_variant<M_LM>(nchunks);
+GemvFn gemv_fn(int R, int XC) {
+    if (XC <= 1) {
+        if (R >= 8) return gemv_kernel<MODE, 8, 1>;
+        if (R >= 4) return gemv_kernel<MODE, 4, 1>;
+        return gemv_kernel<MODE, 2, 1>;
     }
-}
-
-std::mutex g_occ_mu;
-std::map<std::pair<const void*, size_t>, int> g_occ;
-
-int resident_ctas(const void* fn, int threads, size_t smem, int* out) {
-    std::lock_guard<std::mutex> lk(g_occ_mu);
-    auto key = std::make_pair(fn, smem);
-    auto it = g_occ.find(key);
-    if (it != g_occ.end()) {
-        *out = it->second;
-        return TASP_OK;
+    if (XC <= 2) {
+        if (R >= 4) return gemv_kernel<MODE, 4, 2>;
+        return gemv_kernel<MODE, 2, 2>;
     }
-    TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
-    int n = 0;
-    TASP_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, smem));
-    if (n < 1) return fail(TASP_EINVAL, "GEMV configuration does not fit on an SM");
-    g_occ[key] = n;
-    *out = n;
-    return TASP_OK;
-}
-
-int launch_gemv(int mode, const GemvParams& p, cudaStream_t s) {
-    if (p.rows == 0) return TASP_OK;
-    GemvVariant v = pick(mode, p.nchunks);
-    const int F = (mode == M_LM) ? 2 : 4;
-    const size_t smem = (size_t)p.nchunks * F * sizeof(float4);
-    if (smem > 200 * 1024) return fail(TASP_EINVAL, "activation vector too long for shared memory");
-    DevInfo di;
-    int rc = device_info(di);
-    if (rc) return rc;
-    int occ = 0;
-    if ((rc = resident_ctas((const void*)v.fn, NT, smem, &occ))) return rc;
-    const int NG = (p.rows + v.R - 1) / v.R;
-    const int grid = std::max(1, std::min(NG, di.sms * occ));
-    return launch_pdl(v.fn, dim3(grid), dim3(NT), smem, s, p);
-}
-
-typedef void (*AttnFn)(const AttnParams);
-
-AttnFn pick_attn(int dh, int g) {
-#define TASP_ATT(D, GG) \
-    if (dh == D && g == GG) return attn_kernel<D, GG>;
-    TASP_ATT(64, 1) TASP_ATT(64, 2) TASP_ATT(64, 4) TASP_ATT(64, 8)
-    TASP_ATT(128, 1) TASP_ATT(128, 2) TASP_ATT(128, 4) TASP_ATT(128, 8)
-#undef TASP_ATT
+    if (XC <= 4) {
+        if (R >= 2) return gemv_kernel<MODE, 2, 4>;
+        if constexpr (MODE == M_QKV || MODE == M_GU)
+            return nullptr;  // rotary / SwiGLU pairs need two rows per stage
+        else
+            return gemv_kernel<MODE, 1, 4>;
+    }
     return nullptr;
 }
 
-}  // namespace
-
-int attn_splits(int m_kv, int max_tokens, int sms) {
-    if (m_kv <= 0) return 1;
-    int s = (2 * sms + m_kv - 1) / m_kv;
-    s = std::min(s, ATT_SPLITS_MAX);
-    s = std::min(s, std::max(1, (max_tokens + 15) / 16));
-    return std::max(1, s);
+GemvFn pick(int mode, int R, int XC) {
+    switch (mode) {
+        case M_QKV: return gemv_fn<M_QKV>(R, XC);
+        case M_O: return gemv_fn<M_O>(R, XC);
+        case M_GU: return gemv_fn<M_GU>(R, XC);
+        case M_DOWN: return gemv_fn<M_DOWN>(R, XC);
+        default: return gemv_fn<M_LM>(R, XC);
+    }
 }
 
-int attn_supported(int dh, int g) { return pick_attn(dh, g) != nullptr; }
+// Rows per stage: the largest power of two with R * row_bytes <= 32 KB (pairs need R >= 2).
+int rows_per_stage(int mode, int64_t ld) {
+    int R = 8;
+    while (R > 1 && (int64_t)R * ld > 32768) R >>= 1;
+    if ((mode == M_QKV || mode == M_GU) && R < 2) R = 2;
+    return R;
+}
+
+std::mutex g_attr_mu;
+std::map<const void*, bool> g_attr;
+
+int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
+    if (p.rows == 0) return TASP_OK;
+    DevInfo di;
+    int rc = device_info(di);
+    if (rc) return rc;
+    int R = rows_per_stage(mode, p.ld);
+    int XC = 1;
+    while (XC * CT < p.nchunks) XC <<= 1;
+    if (XC > 4) return fail(TASP_EUNSUP, "row too long for the register-resident activation slice");
+    if (XC == 2 && R > 4) R = 4;
+    if (XC == 4 && R > 2) R = 2;
+    GemvFn fn = pick(mode, R, XC);
+    if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
+    p.err = err;
+    p.smem_cap = di.smem_optin - 2048;  // static shared memory of the kernel stays below 2 KB
+    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
+    {
+        std::lock_guard<std::mutex> lk(g_attr_mu);
+        if (!g_attr[(const void*)fn]) {
+            TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem_cap));
+            g_attr[(const void*)fn] = true;
+        }
+    }
+    const int NG = (p.rows + R - 1) / R;
+    const int grid = std::max(1, std::min(NG, di.sms));
+    return launch_pdl(fn, dim3(grid), dim3(GEMV_THREADS), (size_t)L.total, s, p);
+}
+
+}  // namespace
 
 int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
                  int* launches) {
@@ -716,7 +664,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
         p.g = sh.g();
         p.dh = sh.dh;
         pre(K_QKV);
-        if ((rc = launch_gemv(M_QKV, p, s))) return rc;
+        if ((rc = launch_gemv(M_QKV, p, se.err, s))) return rc;
         post(K_QKV);
         // K2: split-KV attention over the retained KV heads
         if (lp.m_kv > 0) {
@@ -728,11 +676,12 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             a.max_tokens = se.max_tokens;
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
             a.part = se.part;
+            a.ml = se.ml;
             a.cnt = se.cnt;
             a.o = se.o;
             const int S = attn_splits(lp.m_kv, se.max_tokens, di.sms);
             pre(K_ATTN);
-            if ((rc = launch_pdl(pick_attn(sh.dh, sh.g()), dim3(S, lp.m_kv), dim3(ATT_THREADS), 0, s, a))) return rc;
+            if ((rc = launch_attention(a, sh.dh, sh.g(), lp.m_kv, S, s))) return rc;
             post(K_ATTN);
         }
         // K3: O-projection + residual
@@ -747,7 +696,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             o.act = se.o;
             o.resid_out = se.x;
             pre(K_O);
-            if ((rc = launch_gemv(M_O, o, s))) return rc;
+            if ((rc = launch_gemv(M_O, o, se.err, s))) return rc;
             post(K_O);
         }
         // K4: RMSNorm + gate/up GEMV + SiLU(gate) * up
@@ -766,7 +715,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             gu.eps = sh.eps;
             gu.h_out = se.h;
             pre(K_GU);
-            if ((rc = launch_gemv(M_GU, gu, s))) return rc;
+            if ((rc = launch_gemv(M_GU, gu, se.err, s))) return rc;
             post(K_GU);
             // K5: down projection + residual
             GemvParams dn{};
@@ -780,7 +729,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             dn.resid_out = se.x;
             dn.hidden_out = last ? t.hidden_out : nullptr;
             pre(K_DOWN);
-            if ((rc = launch_gemv(M_DOWN, dn, s))) return rc;
+            if ((rc = launch_gemv(M_DOWN, dn, se.err, s))) return rc;
             post(K_DOWN);
         } else if (last && t.hidden_out) {
             TASP_CUDA(cudaMemcpyAsync(t.hidden_out, se.x, sizeof(float) * sh.d, cudaMemcpyDeviceToDevice, s));
@@ -799,7 +748,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             lm.eps = sh.eps;
             lm.logits = t.logits;
             pre(K_LM);
-            if ((rc = launch_gemv(M_LM, lm, s))) return rc;
+            if ((rc = launch_gemv(M_LM, lm, se.err, s))) return rc;
             post(K_LM);
         }
         if (t.advance) {

@@ -13,8 +13,6 @@
 
 namespace tasp {
 
-int attn_splits(int m_kv, int max_tokens, int sms);
-int attn_supported(int dh, int g);
 
 // ---------------------------------------------------------------- errors
 static thread_local std::string g_err;
@@ -322,12 +320,15 @@ static int session_alloc(Plan* p, int max_tokens, Session** out) {
     lay.add((size_t)max_tokens * half * sizeof(float2));
     lay.add(sizeof(int));
     lay.add((size_t)sh.d * 4);
-    lay.add((size_t)sh.Hq * sh.dh * 2);
-    lay.add((size_t)sh.Hq * sh.dh * 2);
-    lay.add((size_t)sh.df * 2);
-    const size_t part = (size_t)sh.Hkv * smax * sh.g() * (sh.dh + 2) * 4;
+    lay.add((size_t)sh.Hq * sh.dh * 4);
+    lay.add((size_t)sh.Hq * sh.dh * 4);
+    lay.add((size_t)sh.df * 4);
+    const size_t part = (size_t)sh.Hkv * smax * sh.g() * sh.dh * 4;
+    const size_t mlb = (size_t)sh.Hkv * smax * sh.g() * 2 * 4;
     lay.add(part);
+    lay.add(mlb);
     lay.add((size_t)sh.Hkv * 4);
+    lay.add(sizeof(int));
     lay.add((size_t)sh.d * 2);
     lay.add((size_t)sh.vocab * 4);
     lay.add((size_t)sh.d * 4);
@@ -339,11 +340,13 @@ static int session_alloc(Plan* p, int max_tokens, Session** out) {
     se->rope = (float2*)se->arena.take((size_t)max_tokens * half * sizeof(float2));
     se->d_pos = (int*)se->arena.take(sizeof(int));
     se->x = (float*)se->arena.take((size_t)sh.d * 4);
-    se->q = (uint16_t*)se->arena.take((size_t)sh.Hq * sh.dh * 2);
-    se->o = (uint16_t*)se->arena.take((size_t)sh.Hq * sh.dh * 2);
-    se->h = (uint16_t*)se->arena.take((size_t)sh.df * 2);
+    se->q = (float*)se->arena.take((size_t)sh.Hq * sh.dh * 4);
+    se->o = (float*)se->arena.take((size_t)sh.Hq * sh.dh * 4);
+    se->h = (float*)se->arena.take((size_t)sh.df * 4);
     se->part = (float*)se->arena.take(part);
+    se->ml = (float*)se->arena.take(mlb);
     se->cnt = (int*)se->arena.take((size_t)sh.Hkv * 4);
+    se->err = (int*)se->arena.take(sizeof(int));
     se->x_stage = (uint16_t*)se->arena.take((size_t)sh.d * 2);
     se->logits_stage = sh.vocab ? (float*)se->arena.take((size_t)sh.vocab * 4) : nullptr;
     se->hidden_stage = (float*)se->arena.take((size_t)sh.d * 4);
@@ -510,6 +513,17 @@ int tasp_session_position(const tasp_session* s, int32_t* pos) {
     Session* se = as_session((void*)s);
     if (!se || !pos) return fail(TASP_EINVAL, "invalid session handle or NULL output");
     *pos = se->pos;
+    return TASP_OK;
+}
+
+int tasp_session_status(tasp_session* s, int32_t clear, int32_t* device_error) {
+    Session* se = as_session(s);
+    if (!se || !device_error) return fail(TASP_EINVAL, "invalid session handle or NULL output");
+    TASP_CUDA(cudaDeviceSynchronize());
+    int v = 0;
+    TASP_CUDA(cudaMemcpy(&v, se->err, sizeof(int), cudaMemcpyDeviceToHost));
+    if (clear) TASP_CUDA(cudaMemset(se->err, 0, sizeof(int)));
+    *device_error = v;
     return TASP_OK;
 }
 

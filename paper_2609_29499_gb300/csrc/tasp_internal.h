@@ -132,12 +132,14 @@ struct Session {
     float2* rope = nullptr;       // [max_tokens][dh/2] (cos, sin)
     int* d_pos = nullptr;
     // workspace of one decode step
-    float* x = nullptr;     // FP32 residual [d]
-    uint16_t* q = nullptr;  // BF16 [Hq dh]
-    uint16_t* o = nullptr;  // BF16 [Hq dh]
-    uint16_t* h = nullptr;  // BF16 [df]
-    float* part = nullptr;  // attention split partials
-    int* cnt = nullptr;     // attention split counters [Hkv]
+    float* x = nullptr;  // FP32 residual [d]
+    float* q = nullptr;  // FP32 rotated queries [Hq dh]
+    float* o = nullptr;  // FP32 attention output [Hq dh]
+    float* h = nullptr;  // FP32 SiLU(gate) * up [df]
+    float* part = nullptr;  // attention split partials [Hkv][splits][g][dh]
+    float* ml = nullptr;    // attention split (max, sum) [Hkv][splits][g][2]
+    int* cnt = nullptr;     // attention split tickets [Hkv]
+    int* err = nullptr;     // device error word (0 = no kernel reported a failure)
     int att_splits_max = 0;
     uint16_t* x_stage = nullptr;  // BF16 [d] host-buffer staging
     float* logits_stage = nullptr;
@@ -160,6 +162,24 @@ int gather_rows(int8_t* dst, const int8_t* src, const int32_t* map, int rows, in
 int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const int32_t* cmap, int rows, int Kc,
                 cudaStream_t s);
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
+
+// attention.cu
+struct AttnParams {
+    const float* q;      // FP32 rotated queries [m_q][dh] (kept heads, group-major)
+    const uint16_t* K;   // BF16 [m_kv][max_tokens][dh] of this layer
+    const uint16_t* V;
+    const int* pos;      // device position: the step attends to positions 0..pos
+    int max_tokens;
+    float qscale;        // log2(e) / sqrt(dh)
+    float* part;
+    float* ml;
+    int* cnt;            // zero between launches
+    float* o;            // FP32 [m_q][dh]
+};
+int attn_supported(int dh, int g);
+int attn_splits(int m_kv, int max_tokens, int sms);
+int attn_splits_max();
+int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, cudaStream_t s);
 
 // decode.cu
 enum KernelKind { K_QKV = 0, K_ATTN = 1, K_O = 2, K_GU = 3, K_DOWN = 4, K_LM = 5, K_OTHER = 6 };

@@ -27,7 +27,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 
 # Symbols declared in include/tasp.h (the CPU test checks they are all exported).
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
-            "tasp_session_fill_synthetic", "tasp_session_position", "tasp_decode_step_host", "tasp_mask_select",
+            "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_last_error", "tasp_version")
 
@@ -81,6 +81,7 @@ def load(path: str = LIB_PATH):
         "tasp_session_create": (c_int32, [P, c_int32, POINTER(P)]),
         "tasp_session_fill_synthetic": (c_int32, [P, c_int32, c_uint64, P]),
         "tasp_session_position": (c_int32, [P, POINTER(c_int32)]),
+        "tasp_session_status": (c_int32, [P, c_int32, POINTER(c_int32)]),
         "tasp_decode_step_host": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
         "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
@@ -236,6 +237,12 @@ class Session:
     def position(self) -> int:
         v = c_int32()
         _check(load().tasp_session_position(self.handle, ctypes.byref(v)))
+        return v.value
+
+    def device_error(self, clear=True) -> int:
+        """Device error word of this session's kernels (0 = none); synchronizes."""
+        v = c_int32()
+        _check(load().tasp_session_status(self.handle, int(clear), ctypes.byref(v)))
         return v.value
 
     def layer_step(self, layer, x_in, x_out, stream=None):

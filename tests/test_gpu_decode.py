@@ -69,6 +69,7 @@ def test_layer1_decode_16_steps(tasp, layer1):
     xb = synth.step_inputs_bf16(wl.x_seed, wl.steps, 1, sh.d)
     got, _ = _run_steps(tasp, sess, xb)
     assert sess.position == wl.t_prior + wl.steps
+    assert sess.device_error() == 0
     ref = forward.decode(sh, mask, synth.bf16_to_f32(xb[:, 0]), wl.t_prior, wl.kv_seed)
     assert within(got[:, 0], ref).all()
     assert rel_l2(got[:, 0], ref) <= TOL_E2E
@@ -237,6 +238,7 @@ def test_8b_end_to_end_8_steps(tasp, llama8b):
     sess.fill_synthetic(wl.t_prior, wl.kv_seed)
     xb = synth.step_inputs_bf16(wl.x_seed, steps, 1, sh.d)
     got, logits = _run_steps(tasp, sess, xb, with_logits=True, vocab=sh.vocab)
+    assert sess.device_error() == 0
     sess.release()
     ref = forward.decode(sh, masks[0], synth.bf16_to_f32(xb[:, 0]), wl.t_prior, wl.kv_seed)
     assert rel_l2(got[:, 0], ref) <= TOL_E2E
@@ -312,5 +314,6 @@ def test_70b_full_step_runs_and_is_finite(tasp, llama70b):
     got, logits = _run_steps(tasp, sess, synth.step_inputs_bf16(wl.x_seed, 4, 1, sh.d), True, sh.vocab)
     assert np.isfinite(got).all() and np.isfinite(logits).all()
     assert sess.position == wl.t_prior + 4
+    assert sess.device_error() == 0
     sess.release()
     torch.cuda.synchronize()
