@@ -225,6 +225,28 @@ int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_
  * (graph nodes). */
 int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_logits, int32_t* out);
 
+/* ---------------------------------------------------------------------------
+ * Allocation-free decode step (the paper has no counterpart: a deployment aid).
+ * ------------------------------------------------------------------------- */
+
+/* tasp_decode_step for ONE session that allocates nothing, for callers that must
+ * not enter the CUDA allocator while decoding (a fixed device-memory budget that
+ * is already handed out, another library's stream capture in progress, a serving
+ * loop that forbids allocator calls). The step's kernels are launched directly (no
+ * CUDA graph is built) and the split-KV attention scratch comes from one
+ * file-scope device array of about 1.06 MB (8 kept KV groups x 32 splits x 8 query
+ * heads per group x head dim 128 partial floats, plus maxima/sums and 8 merge
+ * tickets) that every GPU loading the library holds until the process exits.
+ * Arguments and outputs are those of tasp_decode_step with n = 1. The first call on
+ * a device looks up the array's device address (cudaGetSymbolAddress); make that
+ * first call before any stream capture. All calls share the array and it keeps the
+ * last call's contents (the tickets are cleared at the start of every call), so
+ * calls whose kernels overlap on the GPU (different streams, several sessions at
+ * once) race: serialize them. Errors: EINVAL (NULL pointers, or a plan whose
+ * attention partials exceed the array), ECAP, ECUDA. async on `stream`. */
+int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, float* d_hidden_out, float* d_logits,
+                            void* stream);
+
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char* tasp_last_error(void);
 

@@ -675,9 +675,9 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             a.pos = se.d_pos;
             a.max_tokens = se.max_tokens;
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
-            a.part = se.part;
-            a.ml = se.ml;
-            a.cnt = se.cnt;
+            a.part = t.att_part ? t.att_part : se.part;
+            a.ml = t.att_ml ? t.att_ml : se.ml;
+            a.cnt = t.att_cnt ? t.att_cnt : se.cnt;
             a.o = se.o;
             const int S = attn_splits(lp.m_kv, se.max_tokens, di.sms);
             pre(K_ATTN);

@@ -189,6 +189,10 @@ struct StepTarget {
     float* hidden_out = nullptr;
     float* logits = nullptr;
     bool advance = true;
+    // attention split scratch; nullptr = the session's own workspace
+    float* att_part = nullptr;
+    float* att_ml = nullptr;
+    int* att_cnt = nullptr;
 };
 
 using KernelHook = void (*)(void* ctx, int kind, bool before);

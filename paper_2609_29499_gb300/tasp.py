@@ -29,7 +29,8 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
-            "tasp_profile_step", "tasp_step_launches", "tasp_last_error", "tasp_version")
+            "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_last_error",
+            "tasp_version")
 
 
 class ModelDesc(ctypes.Structure):
@@ -90,6 +91,7 @@ def load(path: str = LIB_PATH):
         "tasp_layer_step": (c_int32, [P, c_int32, P, P, P]),
         "tasp_profile_step": (c_int32, [POINTER(P), c_int32, P, P, P, P, P]),
         "tasp_step_launches": (c_int32, [POINTER(P), c_int32, c_int32, POINTER(c_int32)]),
+        "tasp_decode_step_static": (c_int32, [P, P, P, P, P]),
         "tasp_last_error": (ctypes.c_char_p, []),
         "tasp_version": (ctypes.c_char_p, []),
     }
@@ -265,6 +267,13 @@ def decode_step(sessions, x_bf16, hidden=None, logits=None, stream=None):
     _check(load().tasp_decode_step(p, len(sessions), x_bf16.data_ptr(),
                                    hidden.data_ptr() if hidden is not None else None,
                                    logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
+
+
+def decode_step_static(session, x_bf16, hidden=None, logits=None, stream=None):
+    """Allocation-free decode step of one session (static attention scratch, no CUDA graph)."""
+    _check(load().tasp_decode_step_static(session.handle, x_bf16.data_ptr(),
+                                          hidden.data_ptr() if hidden is not None else None,
+                                          logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
 
 
 def decode_step_host(sessions, x_bf16_host, hidden_host=None, logits_host=None, stream=None):
