@@ -233,8 +233,8 @@ int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_lo
  * not enter the CUDA allocator while decoding (a fixed device-memory budget that
  * is already handed out, another library's stream capture in progress, a serving
  * loop that forbids allocator calls). The step's kernels are launched directly (no
- * CUDA graph is built) and the split-KV attention scratch comes from one
- * file-scope device array of about 1.06 MB (8 kept KV groups x 32 splits x 8 query
+ * CUDA graph is built) and the attention scratch comes from one file-scope
+ * device array of about 1.06 MB (8 kept KV groups x 32 partial slots x 8 query
  * heads per group x head dim 128 partial floats, plus maxima/sums and 8 merge
  * tickets) that every GPU loading the library holds until the process exits.
  * Arguments and outputs are those of tasp_decode_step with n = 1. The first call on

@@ -127,8 +127,9 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 constexpr int CW = NWARP;                // consumer warps
 constexpr int CT = CW * 32;              // consumer threads
-constexpr int GEMV_THREADS = CT + 32;    // + producer warp
+constexpr int GEMV_THREADS = CT + 64;    // + producer warp + epilogue warp
 constexpr int MAX_STAGES = 8;
+constexpr int NRB = 8;                   // partial-sum buffers between consumers and the epilogue warp
 constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s) before a wait gives up
 constexpr int ERR_WAIT_TIMEOUT = 1;
 
@@ -294,11 +295,67 @@ __device__ __forceinline__ void load_x(XRegs<XC, F>& xr, const float4* xs, int n
     }
 }
 
-// INT8 rows of one stage . x: acc[r] (packed pairs) += w[r] . x
+// The activation slice of an INT8 GEMV as block-scaled integers: per 16-element chunk
+// one power-of-two scale 2^(e-14) with max|x| < 2^e, each element rounded to the integer
+// X in [-2^14, 2^14] and split as X = 256 hi + lo (hi signed byte, lo unsigned byte),
+// four elements packed per 32-bit word. The INT8 weight words then feed dp4a directly.
+template <int XC>
+struct XDigits {
+    uint32_t hi[XC][4], lo[XC][4];
+    float scale[XC];
+};
+
+template <int XC>
+__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const float4* xs, int nchunks, int tid) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        float v[16];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float4 q = c < nchunks ? xs[swz<4>(4 * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[4 * e + 0] = q.x;
+            v[4 * e + 1] = q.y;
+            v[4 * e + 2] = q.z;
+            v[4 * e + 3] = q.w;
+        }
+        float m = 0.f;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) m = fmaxf(m, fabsf(v[e]));
+        int ex = 0;
+        if (m > 0.f) frexpf(m, &ex);  // m = f * 2^ex, f in [0.5, 1): every |x| < 2^ex
+        xd.scale[j] = m > 0.f ? ldexpf(1.0f, ex - 14) : 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            uint32_t h = 0, l = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int X = m > 0.f ? __float2int_rn(ldexpf(v[4 * w + b], 14 - ex)) : 0;
+                h |= ((uint32_t)(X >> 8) & 0xFFu) << (8 * b);
+                l |= ((uint32_t)X & 0xFFu) << (8 * b);
+            }
+            xd.hi[j][w] = h;
+            xd.lo[j][w] = l;
+        }
+    }
+}
+
+__device__ __forceinline__ int dp4a_ss(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+__device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+
+// INT8 rows of one stage . x: per chunk sum(w * X) = 256 sum(w * hi) + sum(w * lo) in
+// exact INT32, then acc[r] += float(sum) * scale in FP32.
 template <int R, int XC>
-__device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XRegs<XC, 4>& xr,
-                                       int nchunks, int tid, u64 (&acc)[R]) {
-    const u64 magic = pk(-8388736.0f, -8388736.0f);  // -(2^23 + 128)
+__device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC>& xd,
+                                       int nchunks, int tid, float (&acc)[R]) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
@@ -307,18 +364,13 @@ __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld
             for (int r = 0; r < R; ++r) {
                 const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
                 const uint32_t wd[4] = {(uint32_t)wv.x, (uint32_t)wv.y, (uint32_t)wv.z, (uint32_t)wv.w};
+                int sh = 0, sl = 0;
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
-                    const uint32_t u = wd[k] ^ 0x80808080u;
-                    u64 p01 = pk(__uint_as_float(prmt(u, 0x4B000000u, 0x7540u)),
-                                 __uint_as_float(prmt(u, 0x4B000000u, 0x7541u)));
-                    u64 p23 = pk(__uint_as_float(prmt(u, 0x4B000000u, 0x7542u)),
-                                 __uint_as_float(prmt(u, 0x4B000000u, 0x7543u)));
-                    p01 = add2(p01, magic);
-                    p23 = add2(p23, magic);
-                    acc[r] = fma2(p01, pk(xr.v[j][k].x, xr.v[j][k].y), acc[r]);
-                    acc[r] = fma2(p23, pk(xr.v[j][k].z, xr.v[j][k].w), acc[r]);
+                    sh = dp4a_ss(wd[k], xd.hi[j][k], sh);
+                    sl = dp4a_su(wd[k], xd.lo[j][k], sl);
                 }
+                acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xd.scale[j], acc[r]);
             }
         }
     }
@@ -366,37 +418,55 @@ __device__ __forceinline__ float row_reduce(float (&v)[R], int lane) {
     return s;
 }
 
-// Epilogue of one row group from the per-warp partial sums red[w][r].
+// Per-CTA values the epilogue warp stages in shared memory: row scales (constant, read
+// before the dependency wait), residual rows (after it) and this position's rotary pairs.
+constexpr int EPI_MAXR = 512;
+struct EpiStage {
+    float sc[EPI_MAXR];
+    float res[EPI_MAXR];
+    float2 rope[64];
+    int w_lo, pos;
+    bool ok;  // the CTA's rows fit the staging arrays
+};
+
+// Epilogue of one row group, run by the epilogue warp: lanes split the CW partial sums
+// of each row, then lanes < R (or < R/2 for rotary / SwiGLU pairs) finish the rows.
 template <int MODE, int R>
-__device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)[R], int gi, int tid) {
+__device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)[R], int gi, int lane,
+                                         const EpiStage& es) {
+    constexpr int LPR = 32 / R;  // lanes per row
+    const int r = lane % R;
+    float s = 0.f;
+#pragma unroll
+    for (int w = lane / R; w < CW; w += LPR) s += red[w][r];
+#pragma unroll
+    for (int o = R; o < 32; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    // lane r (< R) now holds the full sum of row r of the group
     const int w0 = gi * R;
     if (MODE == M_QKV || MODE == M_GU) {
-        if (tid < R / 2) {
-            float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-            for (int w = 0; w < CW; ++w) {
-                s0 += red[w][2 * tid];
-                s1 += red[w][2 * tid + 1];
-            }
-            const int wa = w0 + 2 * tid;
+        const float s_other = __shfl_down_sync(0xffffffffu, s, 1);  // row 2t+1 for lane 2t
+        if ((lane & 1) == 0 && lane < R) {
+            const float s0 = s, s1 = s_other;
+            const int wa = w0 + lane;
             if (wa < p.rows) {
+                const float sc0 = es.ok ? es.sc[wa - es.w_lo] : p.scale[panel_row<MODE>(p, wa)];
+                const float sc1 = es.ok ? es.sc[wa + 1 - es.w_lo] : p.scale[panel_row<MODE>(p, wa + 1)];
                 if (MODE == M_GU) {
-                    const float a = p.scale[wa] * s0, b = p.scale[wa + 1] * s1;
+                    const float a = sc0 * s0, b = sc1 * s1;
                     const float silu = a / (1.0f + expf(-a));
                     p.h_out[wa >> 1] = silu * b;
                 } else {
                     const int half = p.dh >> 1;
                     const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
-                    const int pr0 = hb * p.dh + i, pr1 = pr0 + half;
-                    float y0 = p.scale[pr0] * s0, y1 = p.scale[pr1] * s1;
+                    float y0 = sc0 * s0, y1 = sc1 * s1;
                     const int gp2 = p.g + 2;
                     const int jl = hb / gp2, hh = hb - jl * gp2;
-                    const int pos = *p.pos;
+                    const int pos = es.pos;
                     if (hh <= p.g) {
-                        const float2 cs = p.rope[(int64_t)pos * half + i];
-                        const float a = y0 * cs.x - y1 * cs.y, b = y1 * cs.x + y0 * cs.y;
-                        y0 = a;
-                        y1 = b;
+                        const float2 cs = es.rope[i];
+                        const float ya = y0 * cs.x - y1 * cs.y, yb = y1 * cs.x + y0 * cs.y;
+                        y0 = ya;
+                        y1 = yb;
                     }
                     if (hh < p.g) {
                         float* dq = p.q_out + (int64_t)(jl * p.g + hh) * p.dh;
@@ -410,16 +480,14 @@ __device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)
                 }
             }
         }
-    } else if (tid < R) {
-        float s = 0.f;
-#pragma unroll
-        for (int w = 0; w < CW; ++w) s += red[w][tid];
-        const int row = w0 + tid;
+    } else if (lane < R) {
+        const int row = w0 + lane;
         if (row < p.rows) {
             if (MODE == M_LM) {
                 p.logits[row] = s;
             } else {
-                const float v = p.resid_out[row] + p.scale[row] * s;
+                const float base = es.ok ? es.res[row - es.w_lo] : p.resid_out[row];
+                const float v = base + (es.ok ? es.sc[row - es.w_lo] : p.scale[row]) * s;
                 p.resid_out[row] = v;
                 if (p.hidden_out) p.hidden_out[row] = v;
             }
@@ -435,7 +503,7 @@ __host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld,
     GemvSmem g;
     g.x_bytes = ((nchunks * F * 16) + 127) & ~127;
     g.stage_bytes = ((R * ld) + 127) & ~127;
-    const int bar_bytes = 2 * MAX_STAGES * 8 + 16;
+    const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
     int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
     g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
     g.total = g.x_bytes + g.nstages * g.stage_bytes + bar_bytes;
@@ -445,7 +513,7 @@ __host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld,
 template <int MODE, int R, int XC>
 __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams p) {
     extern __shared__ __align__(128) uint8_t sm[];
-    __shared__ float red[2][CW][R];
+    __shared__ float red[NRB][CW][R];
     __shared__ float stat[CW];
     __shared__ int abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -455,6 +523,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     uint8_t* stages = sm + L.x_bytes;
     const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
     const uint32_t empty0 = full0 + 8 * MAX_STAGES;
+    const uint32_t rfull0 = empty0 + 8 * MAX_STAGES;
+    const uint32_t rempty0 = rfull0 + 8 * NRB;
     const int NG = (p.rows + R - 1) / R;
     const int g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
     const int g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
@@ -463,7 +533,11 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
         abort_flag = 0;
         for (int s = 0; s < NS; ++s) {
             mbar_init(full0 + 8 * s, 1);
-            mbar_init(empty0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, CW);
+        }
+        for (int b = 0; b < NRB; ++b) {
+            mbar_init(rfull0 + 8 * b, CW);
+            mbar_init(rempty0 + 8 * b, 1);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -473,19 +547,59 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
         // ---- producer: weights never depend on the previous kernel, so start at once
         pdl_trigger();
         if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
             for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-                const int s = i % NS, k = i / NS;
-                if (k > 0) mbar_wait(empty0 + 8 * s, (k - 1) & 1, &abort_flag, p.err);
+                if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err);
                 const int nrow = min(R, p.rows - gi * R);
                 mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
                 for (int r = 0; r < nrow; ++r)
                     bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)r * p.ld),
                              row_ptr<MODE>(p, gi * R + r), (uint32_t)p.ld, full0 + 8 * s);
+                if (++s == NS) {
+                    s = 0;
+                    ph ^= 1;
+                }
             }
             // never leave while copies into this CTA's shared memory are in flight (even
             // after an abort: this second wait is bounded on its own)
             for (int gi = max(g0, g1 - NS), i = gi - g0; gi < g1; ++gi, ++i)
                 mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, false);
+        }
+        return;
+    }
+    if (warp == CW + 1) {
+        // ---- epilogue warp: cross-warp sums of each row group, then the mode's epilogue
+        __shared__ EpiStage es;
+        const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
+        if (lane == 0) {
+            es.w_lo = w_lo;
+            es.ok = (w_hi - w_lo) <= EPI_MAXR;
+        }
+        __syncwarp();
+        if (MODE != M_LM && es.ok)  // scales are constant: stage them before the dependency wait
+            for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
+        pdl_wait();
+        pdl_trigger();
+        if ((MODE == M_O || MODE == M_DOWN) && es.ok)
+            for (int w = w_lo + lane; w < w_hi; w += 32) es.res[w - w_lo] = p.resid_out[w];
+        if (MODE == M_QKV) {
+            const int pos = *p.pos;
+            if (lane == 0) es.pos = pos;
+            for (int i = lane; i < (p.dh >> 1); i += 32) es.rope[i] = p.rope[(int64_t)pos * (p.dh >> 1) + i];
+        }
+        __syncwarp();
+        int b = 0;
+        uint32_t ph = 0;
+        for (int gi = g0; gi < g1; ++gi) {
+            mbar_wait(rfull0 + 8 * b, ph, &abort_flag, p.err);
+            epilogue<MODE, R>(p, red[b], gi, lane, es);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rempty0 + 8 * b);
+            if (++b == NRB) {
+                b = 0;
+                ph ^= 1;
+            }
         }
         return;
     }
@@ -500,31 +614,48 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     else
         f32_to_smem(p.act, p.K, p.nchunks, xs);
 
-    constexpr int F = MODE == M_LM ? 2 : 4;
-    XRegs<XC, F> xr;
-    load_x<XC, F>(xr, xs, p.nchunks, tid);
+    XRegs<XC, 2> xr;        // LM head: FP32 activation slice
+    XDigits<XC> xd;         // INT8 modes: block-scaled integer digits of the slice
+    if constexpr (MODE == M_LM)
+        load_x<XC, 2>(xr, xs, p.nchunks, tid);
+    else
+        digits_x<XC>(xd, xs, p.nchunks, tid);
+    int s = 0, b = 0;
+    uint32_t sph = 0, bph = 0;
     for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-        const int s = i % NS, k = i / NS;
-        mbar_wait(full0 + 8 * s, k & 1, &abort_flag, p.err);
+        mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err);
         const uint8_t* st = stages + (size_t)s * L.stage_bytes;
-        u64 acc[R];
-#pragma unroll
-        for (int r = 0; r < R; ++r) acc[r] = 0ull;
-        if constexpr (MODE == M_LM)
-            dot_bf16<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
-        else
-            dot_i8<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
         float v[R];
+        if constexpr (MODE == M_LM) {
+            u64 acc[R];
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const float2 a = upk(acc[r]);
-            v[r] = a.x + a.y;
+            for (int r = 0; r < R; ++r) acc[r] = 0ull;
+            dot_bf16<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const float2 a = upk(acc[r]);
+                v[r] = a.x + a.y;
+            }
+        } else {
+#pragma unroll
+            for (int r = 0; r < R; ++r) v[r] = 0.f;
+            dot_i8<R, XC>(st, (int)p.ld, xd, p.nchunks, tid, v);
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
         const float rs = row_reduce<R>(v, lane);
-        if ((lane & (32 / R - 1)) == 0) red[i & 1][warp][lane / (32 / R)] = rs;
-        consumer_sync();  // every consumer is done reading stage s, partial sums are visible
-        if (tid == 0) mbar_arrive(empty0 + 8 * s);
-        epilogue<MODE, R>(p, red[i & 1], gi, tid);
+        if (i >= NRB) mbar_wait(rempty0 + 8 * b, bph ^ 1, &abort_flag, p.err);
+        if ((lane & (32 / R - 1)) == 0) red[b][warp][lane / (32 / R)] = rs;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(rfull0 + 8 * b);
+        if (++s == NS) {
+            s = 0;
+            sph ^= 1;
+        }
+        if (++b == NRB) {
+            b = 0;
+            bph ^= 1;
+        }
     }
 }
 
@@ -593,7 +724,7 @@ int rows_per_stage(int mode, int64_t ld) {
 }
 
 std::mutex g_attr_mu;
-std::map<const void*, bool> g_attr;
+std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 
 int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
     if (p.rows == 0) return TASP_OK;
@@ -609,16 +740,20 @@ int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
     GemvFn fn = pick(mode, R, XC);
     if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
     p.err = err;
-    p.smem_cap = di.smem_optin - 2048;  // static shared memory of the kernel stays below 2 KB
-    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
-    if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
     {
         std::lock_guard<std::mutex> lk(g_attr_mu);
-        if (!g_attr[(const void*)fn]) {
-            TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem_cap));
-            g_attr[(const void*)fn] = true;
+        auto it = g_attr.find((const void*)fn);
+        if (it == g_attr.end()) {
+            cudaFuncAttributes fa;
+            TASP_CUDA(cudaFuncGetAttributes(&fa, fn));
+            const int cap = di.smem_optin - (int)fa.sharedSizeBytes - 128;
+            TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, cap));
+            it = g_attr.emplace((const void*)fn, cap).first;
         }
+        p.smem_cap = it->second;
     }
+    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
     const int NG = (p.rows + R - 1) / R;
     const int grid = std::max(1, std::min(NG, di.sms));
     return launch_pdl(fn, dim3(grid), dim3(GEMV_THREADS), (size_t)L.total, s, p);
@@ -679,7 +814,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             a.ml = t.att_ml ? t.att_ml : se.ml;
             a.cnt = t.att_cnt ? t.att_cnt : se.cnt;
             a.o = se.o;
-            const int S = attn_splits(lp.m_kv, se.max_tokens, di.sms);
+            const int S = attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g());
             pre(K_ATTN);
             if ((rc = launch_attention(a, sh.dh, sh.g(), lp.m_kv, S, s))) return rc;
             post(K_ATTN);

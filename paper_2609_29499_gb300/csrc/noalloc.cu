@@ -5,9 +5,9 @@
 // region where the CUDA allocator must not be entered (another library's stream
 // capture, a real-time serving loop that forbids allocator calls), or embedders whose
 // own allocator owns the device. tasp_decode_step_static serves them: it launches the
-// step's kernels directly (no CUDA graph is instantiated) and takes the split-KV
-// attention scratch (per-split partial outputs, their maxima/sums and the merge
-// tickets) from one file-scope device array instead of the session's workspace.
+// step's kernels directly (no CUDA graph is instantiated) and takes the attention
+// scratch (per-cluster partial outputs of long contexts, their maxima/sums and the
+// merge tickets) from one file-scope device array instead of the session's workspace.
 //
 // The array is a module global: every GPU that loads this library holds it until the
 // process exits, every call shares it, and it keeps the last call's contents.
@@ -22,8 +22,8 @@ namespace tasp {
 
 namespace {
 
-// Capacity of the shared scratch, sized for up to 8 kept KV groups x 32 splits x 8 query
-// heads per group x head dimension 128 (the Llama-3 8B/70B shapes): ~1.06 MB.
+// Capacity of the shared scratch, sized for up to 8 kept KV groups x 32 partial slots x 8
+// query heads per group x head dimension 128 (the Llama-3 8B/70B shapes): ~1.06 MB.
 constexpr size_t kPartFloats = 8 * 32 * 8 * 128;
 constexpr size_t kMlFloats = 8 * 32 * 8 * 2;
 constexpr size_t kTickets = 8;
@@ -70,9 +70,11 @@ extern "C" int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, fl
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
-    // every layer's split partials must fit the static array
+    // every layer's attention partials must fit the static array
     for (const LayerPlan& lp : pl.layers) {
-        const size_t S = (size_t)attn_splits(lp.m_kv, se->max_tokens, di.sms);
+        // partial outputs are kept per cluster of the attention kernel
+        const size_t S = (size_t)attn_splits(lp.m_kv, se->max_tokens, di.sms, sh.dh, sh.g()) /
+                         (size_t)attn_cluster(sh.dh, sh.g());
         const size_t part = (size_t)lp.m_kv * S * sh.g() * sh.dh;
         const size_t ml = (size_t)lp.m_kv * S * sh.g() * 2;
         if (part > kPartFloats || ml > kMlFloats || (size_t)lp.m_kv > kTickets)

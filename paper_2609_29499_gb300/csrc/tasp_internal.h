@@ -177,7 +177,8 @@ struct AttnParams {
     float* o;            // FP32 [m_q][dh]
 };
 int attn_supported(int dh, int g);
-int attn_splits(int m_kv, int max_tokens, int sms);
+int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
+int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g);
 int attn_splits_max();
 int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, cudaStream_t s);
 
