@@ -34,6 +34,11 @@ import numpy as np  # noqa: E402
 import synth  # noqa: E402
 
 METRIC = "decode ms/token (70B-shape, 43% mask, bs1); achieved HBM GB/s vs ~8 TB/s"
+# DRAM traffic over algorithmic bytes of one launch, from one ncu capture of the kernel
+# (dram__bytes_read.sum + dram__bytes_write.sum of a 70B-width gate/up launch with 12,288
+# kept channels: 205,311,744 B against 201,539,584 algorithmic). Must be re-taken (or set
+# to None) whenever the kernel changes.
+TRAFFIC_PER_ALGORITHMIC = {"gate_up": 205311744 / 201539584}
 PAPER_CONTEXT = {"ms_per_token_sparse": 31.3, "ms_per_token_dense": 45.2,
                  "hardware": "1x A100 80GB SXM, real Llama-3-70B, groupwise INT8, ~2k context"}
 
@@ -313,7 +318,9 @@ def run_ours(args):
                 "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4) if achieved else None,
                 "peak_source": f"{peak_kind} hbm_gbs (copy bandwidth)",
                 "bytes_per_launch": int(per_launch_bytes), "launch_us": round(dur_ms / launches * 1e3, 2),
-                "traffic": None}
+                "traffic": (int(per_launch_bytes * TRAFFIC_PER_ALGORITHMIC[dominant])
+                            if dominant in TRAFFIC_PER_ALGORITHMIC else None),
+                "traffic_source": "ncu capture of a 70B-width launch, scaled by algorithmic bytes"}
     step_gbs = step_bytes / (ms * 1e-3) / 1e9
     kernels = {k: {"ms": round(v[0], 4), "launches": v[1],
                    "GB/s": round(gb[k] / (v[0] * 1e-3) / 1e9, 1) if k in gb and v[0] > 0 else None}
