@@ -221,6 +221,11 @@ int tasp_layer_step(tasp_session* s, int32_t layer, const float* d_x_in, float* 
 int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_logits,
                       void* stream, float* h_ms, int32_t* h_count);
 
+/* Copy the cached keys (which = 0) or values (which = 1) of one layer, BF16
+ * [m_kv][position][dh] for positions 0 .. current position - 1, to host memory of
+ * exactly that many bytes. sync. */
+int tasp_session_kv_export(const tasp_session* s, int32_t layer, int32_t which, void* h_dst, size_t bytes);
+
 /* Number of library kernel launches one decode step of these sessions makes
  * (graph nodes). */
 int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_logits, int32_t* out);

@@ -148,7 +148,7 @@ def prior_cache(shape, layer, kv_seed, t_prior, groups=None, dtype=np.float32):
 
 
 def decode(shape, mask, x_steps, t_prior, kv_seed, compact=False, dtype=np.float32,
-           layers=None, x_in=None):
+           layers=None, x_in=None, prior=None):
     """Teacher-forced batch-1 decode of len(x_steps) steps.
 
     x_steps [S, d] float inputs (the BF16 step vectors widened). Processes the
@@ -156,18 +156,23 @@ def decode(shape, mask, x_steps, t_prior, kv_seed, compact=False, dtype=np.float
     output, so the loop order does not change the result). Returns the residual
     stream after the last processed layer [S, d].
     ``layers`` restricts to a sub-range; ``x_in`` then supplies its input.
+    ``prior`` (optional) maps a layer to its dense cache (K, V) [H_kv, t_prior, d_h] (for
+    decoding after a prefill) instead of the synthetic prior tokens.
     """
     X = np.array(x_steps if x_in is None else x_in, dtype=dtype)
     S = X.shape[0]
     for layer in (range(shape.L) if layers is None else layers):
         lq = wts.gen_layer(shape, layer)
         kg, kc = mask.keep_groups[layer], mask.keep_chans[layer]
+        if prior is not None:
+            Kd, Vd = prior(layer)
+            Kd, Vd = np.asarray(Kd, dtype), np.asarray(Vd, dtype)
         if compact:
             W = compact_weights(shape, lq, kg, kc, dtype)
-            Kc, Vc = prior_cache(shape, layer, kv_seed, t_prior, kg, dtype)
+            Kc, Vc = (Kd[kg], Vd[kg]) if prior is not None else prior_cache(shape, layer, kv_seed, t_prior, kg, dtype)
         else:
             W = wts.dense_zeroed(shape, lq, kg, kc, dtype)
-            Kc, Vc = prior_cache(shape, layer, kv_seed, t_prior, None, dtype)
+            Kc, Vc = (Kd, Vd) if prior is not None else prior_cache(shape, layer, kv_seed, t_prior, None, dtype)
         nkv = Kc.shape[0]
         Kall = np.zeros((nkv, t_prior + S, shape.dh), dtype)
         Vall = np.zeros_like(Kall)

@@ -67,17 +67,7 @@ struct GemvParams {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
-__device__ __forceinline__ int4 ld_stream16(const void* p) {
-    int4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.s32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
 
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 
 typedef unsigned long long u64;
 
@@ -91,19 +81,9 @@ __device__ __forceinline__ float2 upk(u64 v) {
     asm("mov.b64 {%0,%1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
     return r;
 }
-__device__ __forceinline__ u64 add2(u64 a, u64 b) {
-    u64 d;
-    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-    return d;
-}
 __device__ __forceinline__ u64 fma2(u64 a, u64 b, u64 c) {
     u64 d;
     asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-    return d;
-}
-__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
-    uint32_t d;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
     return d;
 }
 
@@ -113,7 +93,6 @@ __device__ __forceinline__ int swz(int f) {
     return f ^ ((f >> 3) & (F - 1));
 }
 
-__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 __device__ __forceinline__ uint16_t f32_to_bf16_bits(float v) {
     __nv_bfloat16 b = __float2bfloat16_rn(v);
     return *reinterpret_cast<uint16_t*>(&b);
@@ -659,6 +638,10 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     }
 }
 
+__global__ void set_pos_kernel(int* pos, int v) {
+    if (threadIdx.x == 0) *pos = v;
+}
+
 __global__ void advance_kernel(int* pos) {
     pdl_wait();
     pdl_trigger();
@@ -893,6 +876,28 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
         }
     }
     if (launches) *launches = nl;
+    return TASP_OK;
+}
+
+int enqueue_lm_head(Session& se, float* logits, cudaStream_t s) {
+    const Shape& sh = se.plan->store->sh;
+    if (sh.vocab == 0) return fail(TASP_EINVAL, "model has no LM head");
+    GemvParams lm{};
+    lm.w = reinterpret_cast<const int8_t*>(se.plan->store->lm_head);
+    lm.ld = (int64_t)sh.d * 2;
+    lm.rows = sh.vocab;
+    lm.K = sh.d;
+    lm.nchunks = sh.d / 8;
+    lm.x_resid = se.x;
+    lm.gamma = se.plan->store->g_final;
+    lm.eps = sh.eps;
+    lm.logits = logits;
+    return launch_gemv(M_LM, lm, se.err, s);
+}
+
+int enqueue_set_pos(Session& se, int pos, cudaStream_t s) {
+    set_pos_kernel<<<1, 32, 0, s>>>(se.d_pos, pos);
+    TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }
 

@@ -1,0 +1,635 @@
+// Prefill of one prompt with a compiled plan (Fig. 1 "one launch plan for prefill"), sm_103a.
+//
+// Per layer: row RMSNorm -> QKV GEMM -> rotary + KV-cache write -> causal GQA attention
+// over the kept heads -> O GEMM (+ residual) -> row RMSNorm -> gate/up GEMM with fused
+// SiLU(gate) * up -> down GEMM (+ residual). The projections are dense GEMMs over the
+// plan's compacted panels on the 5th-generation tensor cores:
+//  * operands FP16 (INT8 weights are exact in FP16; activations keep 11 significant
+//    bits), FP32 accumulators in tensor memory, per-weight-row scales in the epilogue;
+//  * a CTA computes a 128 x 256 output tile: warp 0 streams 128 x 64 and 256 x 64 operand
+//    tiles with TMA (128-byte swizzle) into a 4-stage ring, warp 1 allocates 256 TMEM
+//    columns and issues tcgen05.mma (M = 128, N = 256, K = 16 per instruction), warps 2-5
+//    read the accumulator back with tcgen05.ld and apply the epilogue;
+//  * every mbarrier wait is bounded and reports to the session's device error word.
+// Attention is a causal flash-attention on mma.sync (BF16 K/V from the cache, queries
+// and probabilities split into BF16 high/low halves as in the decode kernel).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "tasp_internal.h"
+
+namespace tasp {
+
+namespace {
+
+// ------------------------------------------------------------------ PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s)
+// Bounded wait: after WAIT_LIMIT cycles it records the failure and makes the CTA's later
+// waits return at once, so a lost transfer can never hang the GPU.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
+                                          bool honor_abort = true) {
+    if (honor_abort && *(volatile int*)abort_flag) return;
+    if (mbar_try(bar, parity)) return;
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity)) {
+        if (clock64() - t0 > WAIT_LIMIT) {
+            *(volatile int*)abort_flag = 1;
+            if (err) atomicOr(err, 1);
+            return;
+        }
+    }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// UMMA shared-memory descriptor of a K-major operand tile written by TMA with 128-byte
+// swizzle: 8-row x 128-byte swizzle atoms stacked along the rows (stride 1024 bytes).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address / 16
+    d |= (uint64_t)1 << 16;                     // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;           // stride byte offset: 8 rows x 128 bytes
+    d |= (uint64_t)1 << 46;                     // descriptor version of the 5th-generation tensor core
+    d |= (uint64_t)2 << 61;                     // swizzle: 128 bytes
+    return d;
+}
+// Instruction descriptor of kind::f16: D FP32, A and B FP16, both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
+    return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ------------------------------------------------------------------ GEMM
+constexpr int BM = 128, BN = 256, BK = 64;
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int GEMM_THREADS = 192;
+constexpr int GEMM_SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+constexpr uint32_t TMEM_COLS = 256;
+constexpr uint32_t IDESC = idesc_f16(BM, BN);
+
+enum EpiMode { EP_STORE = 0, EP_RESID = 1, EP_SWIGLU = 2 };
+
+struct GemmArgs {
+    int M, N, K;
+    const float* scale;  // [N] scale of each weight row
+    float* out;          // STORE: out[m][n] = s_n acc; RESID: out[m][n] += s_n acc
+    int ldo;
+    __half* hout;        // SWIGLU: hout[m][n/2] = SiLU(s_g gate) * (s_u up), n even = gate
+    int ldh;
+    int mode;
+    int* err;
+};
+
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmArgs g) {
+    extern __shared__ uint8_t smraw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_acc;
+    __shared__ uint32_t tmem_base;
+    __shared__ int abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+    const int nk = (g.K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(&bar_full[s]), 1);
+            mbar_init(smem_u32(&bar_empty[s]), 1);
+        }
+        mbar_init(smem_u32(&bar_acc), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {  // ---- TMA producer
+            for (int kb = 0; kb < nk; ++kb) {
+                const int s = kb % STAGES;
+                if (kb >= STAGES) mbar_wait(smem_u32(&bar_empty[s]), ((kb / STAGES) - 1) & 1, &abort_flag, g.err);
+                const uint32_t fb = smem_u32(&bar_full[s]);
+                mbar_expect_tx(fb, STAGE_BYTES);
+                const uint32_t a = smem_u32(sm + s * STAGE_BYTES);
+                tma_load_2d(a, &tmA, kb * BK, m0, fb);
+                tma_load_2d(a + A_BYTES, &tmB, kb * BK, n0, fb);
+            }
+            for (int kb = max(0, nk - STAGES); kb < nk; ++kb)  // no copy may outlive the CTA
+                mbar_wait(smem_u32(&bar_full[kb % STAGES]), (kb / STAGES) & 1, &abort_flag, g.err, false);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // ---- MMA issuer
+            for (int kb = 0; kb < nk; ++kb) {
+                const int s = kb % STAGES;
+                mbar_wait(smem_u32(&bar_full[s]), (kb / STAGES) & 1, &abort_flag, g.err);
+                tc_fence_after();
+                const uint32_t a = smem_u32(sm + s * STAGE_BYTES), b = a + A_BYTES;
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    const uint64_t ad = sw128_desc(a + kk * 32), bd = sw128_desc(b + kk * 32);
+                    const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
+                    asm volatile(
+                        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+                        "l"(ad), "l"(bd), "r"(IDESC), "r"(accum)
+                        : "memory");
+                }
+                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                                 smem_u32(&bar_empty[s]))
+                             : "memory");
+            }
+            asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                             smem_u32(&bar_acc))
+                         : "memory");
+        }
+    } else {  // ---- epilogue: warps 2..5, warp w reads TMEM lanes 32 (w % 4) ..
+        mbar_wait(smem_u32(&bar_acc), 0, &abort_flag, g.err);
+        tc_fence_after();
+        const int q = warp & 3;
+        const int row = m0 + 32 * q + lane;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+            uint32_t r[32];
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+                "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+                  "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+                  "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+                  "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+                  "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+                : "r"(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0));
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            if (row >= g.M) continue;
+            const int nb = n0 + c0;
+            if (g.mode == EP_SWIGLU) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 2) {
+                    const int n = nb + j;
+                    if (n + 1 < g.N) {
+                        const float a = __uint_as_float(r[j]) * g.scale[n];
+                        const float b = __uint_as_float(r[j + 1]) * g.scale[n + 1];
+                        g.hout[(int64_t)row * g.ldh + (n >> 1)] = __float2half_rn(a / (1.0f + expf(-a)) * b);
+                    }
+                }
+            } else {
+                float* o = g.out + (int64_t)row * g.ldo;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    const int n = nb + j;
+                    if (n < g.N) {
+                        const float v = __uint_as_float(r[j]) * g.scale[n];
+                        if (g.mode == EP_RESID)
+                            o[n] += v;
+                        else
+                            o[n] = v;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+}
+
+// ------------------------------------------------------------------ elementwise kernels
+// x^ = half(x / sqrt(mean(x^2) + eps) * gamma) per row; row 0 source may be BF16 input embeddings.
+__global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const float* __restrict__ X, const uint16_t* x_bf16,
+                                                            float* X_init, int d, const float* __restrict__ gamma,
+                                                            float eps, __half* out, int ldo) {
+    __shared__ float red[8];
+    const int t = blockIdx.x, tid = threadIdx.x;
+    const float* xr = X + (int64_t)t * d;
+    float ss = 0.f;
+    for (int i = tid; i < d; i += 256) {
+        float v;
+        if (x_bf16) {
+            v = __uint_as_float((uint32_t)x_bf16[(int64_t)t * d + i] << 16);
+            X_init[(int64_t)t * d + i] = v;
+        } else {
+            v = xr[i];
+        }
+        ss = fmaf(v, v, ss);
+    }
+    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if ((tid & 31) == 0) red[tid >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)d) + eps);
+    for (int i = tid; i < d; i += 256) {
+        const float v = x_bf16 ? __uint_as_float((uint32_t)x_bf16[(int64_t)t * d + i] << 16) : xr[i];
+        out[(int64_t)t * ldo + i] = __float2half_rn((v * inv) * gamma[i]);
+    }
+}
+
+// Projected rows Y [T][qkv rows] (group-major panel order, scaled) -> rotated queries (FP32,
+// [m_q][T][dh]) and the plan-bound KV cache (BF16 keys rotated, values as is) at 0..T-1.
+__global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int g, int dh,
+                               const float2* __restrict__ rope, float* Qf, uint16_t* Kc, uint16_t* Vc,
+                               int max_tokens) {
+    const int t = blockIdx.x, jl = blockIdx.y;
+    const int half = dh >> 1;
+    for (int w = threadIdx.x; w < (g + 2) * half; w += blockDim.x) {
+        const int hh = w / half, i = w - hh * half;
+        const int col = (jl * (g + 2) + hh) * dh + i;
+        float y0 = Y[(int64_t)t * ldy + col], y1 = Y[(int64_t)t * ldy + col + half];
+        if (hh <= g) {
+            const float2 cs = rope[(int64_t)t * half + i];
+            const float a = y0 * cs.x - y1 * cs.y, b = y1 * cs.x + y0 * cs.y;
+            y0 = a;
+            y1 = b;
+        }
+        if (hh < g) {
+            float* q = Qf + ((int64_t)(jl * g + hh) * T + t) * dh;
+            q[i] = y0;
+            q[i + half] = y1;
+        } else {
+            uint16_t* dst = (hh == g ? Kc : Vc) + ((int64_t)jl * max_tokens + t) * dh;
+            __nv_bfloat16 b0 = __float2bfloat16_rn(y0), b1 = __float2bfloat16_rn(y1);
+            dst[i] = *reinterpret_cast<uint16_t*>(&b0);
+            dst[i + half] = *reinterpret_cast<uint16_t*>(&b1);
+        }
+    }
+}
+
+// INT8 panel rows (optionally through a row map) -> FP16 rows with a padded stride
+__global__ void i8_to_f16_kernel(const int8_t* __restrict__ src, const int32_t* map, int64_t lds, int K,
+                                 __half* dst, int ldd) {
+    const int r = blockIdx.x;
+    const int8_t* s = src + (int64_t)(map ? map[r] : r) * lds;
+    __half* d = dst + (int64_t)r * ldd;
+    for (int k = threadIdx.x; k < ldd; k += blockDim.x) d[k] = __int2half_rn(k < K ? (int)s[k] : 0);
+}
+
+// ------------------------------------------------------------------ causal attention
+constexpr int PA_WARPS = 8;
+constexpr int PA_QB = PA_WARPS * 8;  // queries per CTA (8 per warp)
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t a, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(a));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t a, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(a));
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+    const float2 hf = __bfloat1622float2(h);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+    hi = *reinterpret_cast<const uint32_t*>(&h);
+    lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// One CTA: one kept query head, 64 consecutive queries (8 per warp). The A operand rows
+// 0-7 hold the warp's 8 queries (BF16 high part), rows 8-15 the low parts.
+template <int DH>
+__global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float* __restrict__ Qf, const uint16_t* K,
+                                                                     const uint16_t* V, int T, int max_tokens, int g,
+                                                                     float qscale, __half* O, int ldo) {
+    constexpr int ROWB = DH * 2 + 16, TILEB = 16 * ROWB, KS = DH / 16, NT = DH / 8, CPR = DH * 2 / 16;
+    __shared__ __align__(128) uint8_t tiles[2][2][TILEB];
+    const int h = blockIdx.y, jl = h / g;
+    const int q0 = (gridDim.x - 1 - blockIdx.x) * PA_QB;  // the longest blocks start first
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int qw = q0 + warp * 8;                 // this warp's first query
+    const int row_q = qw + (lane >> 2);           // query of this lane's fragment rows
+    const int qc = (lane & 3) * 2;
+    const uint16_t* Kg = K + (int64_t)jl * max_tokens * DH;
+    const uint16_t* Vg = V + (int64_t)jl * max_tokens * DH;
+    const int kend = min(T, q0 + PA_QB);  // keys needed by this CTA: 0 .. kend-1
+    const int ntile = (kend + 15) / 16;
+
+    uint32_t qa[KS][4];
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks)
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+            const int col = ks * 16 + hf * 8 + qc;
+            float x0 = 0.f, x1 = 0.f;
+            if (row_q < T) {
+                const float* qp = Qf + ((int64_t)h * T + row_q) * DH + col;
+                x0 = qp[0] * qscale;
+                x1 = qp[1] * qscale;
+            }
+            split_pack(x0, x1, qa[ks][2 * hf], qa[ks][2 * hf + 1]);
+        }
+    float acc[NT][4];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+    float m_run = -INFINITY, l_run = 0.f;
+
+    auto issue = [&](int kt, int st) {
+        uint8_t* kt_s = &tiles[st][0][0];
+        uint8_t* vt_s = &tiles[st][1][0];
+        for (int c = tid; c < 16 * CPR; c += PA_WARPS * 32) {
+            const int r = c / CPR, cc = c - r * CPR;
+            const int pos = kt * 16 + r;
+            const bool ok = pos < kend;
+            const int64_t off = (int64_t)(ok ? pos : 0) * DH + cc * 8;
+            cp_async16(smem_u32(kt_s + r * ROWB + cc * 16), Kg + off, ok ? 16 : 0);
+            cp_async16(smem_u32(vt_s + r * ROWB + cc * 16), Vg + off, ok ? 16 : 0);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    if (ntile > 0) issue(0, 0);
+    for (int kt = 0; kt < ntile; ++kt) {
+        const int st = kt & 1;
+        if (kt + 1 < ntile) {
+            issue(kt + 1, st ^ 1);
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        } else {
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        }
+        __syncthreads();
+        const int base = kt * 16;
+        if (base <= qw + 7) {  // some key of the tile is visible to this warp's queries
+            const uint8_t* kt_s = &tiles[st][0][0];
+            const uint8_t* vt_s = &tiles[st][1][0];
+            float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+            const uint32_t krow =
+                smem_u32(kt_s + (8 * ((lane >> 4) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 3) & 1));
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                uint32_t b00, b01, b10, b11;
+                ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
+                mma16816(s0, qa[ks], b00, b01);
+                mma16816(s1, qa[ks], b10, b11);
+            }
+            float sc[4] = {s0[0] + s0[2], s0[1] + s0[3], s1[0] + s1[2], s1[1] + s1[3]};
+            const int kp[4] = {base + qc, base + qc + 1, base + 8 + qc, base + 9 + qc};
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if (kp[e] > row_q || kp[e] >= kend) sc[e] = -INFINITY;  // causal
+            float mt = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+            mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
+            mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
+            const float m_new = fmaxf(m_run, mt);
+            if (m_new != -INFINITY) {  // key 0 is visible to every query: finite from the first tile on
+                const float corr = exp2f(m_run - m_new);
+                float pv[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) pv[e] = exp2f(sc[e] - m_new);
+                l_run = l_run * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
+                m_run = m_new;
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    acc[nt][0] *= corr;
+                    acc[nt][1] *= corr;
+                    acc[nt][2] *= corr;
+                    acc[nt][3] *= corr;
+                }
+                uint32_t pa[4];
+                split_pack(pv[0], pv[1], pa[0], pa[1]);
+                split_pack(pv[2], pv[3], pa[2], pa[3]);
+                const uint32_t vrow =
+                    smem_u32(vt_s + (8 * ((lane >> 3) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 4) & 1));
+#pragma unroll
+                for (int nt = 0; nt < NT; nt += 2) {
+                    uint32_t v0, v1, v2, v3;
+                    ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
+                    mma16816(acc[nt], pa, v0, v1);
+                    mma16816(acc[nt + 1], pa, v2, v3);
+                }
+            }
+        }
+        __syncthreads();  // the stage is refilled two tiles later
+    }
+    l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
+    l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
+    if (row_q < T) {
+        const float inv = 1.0f / l_run;
+        __half* o = O + (int64_t)row_q * ldo + h * DH;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            const int dim = nt * 8 + qc;
+            o[dim] = __float2half_rn((acc[nt][0] + acc[nt][2]) * inv);
+            o[dim + 1] = __float2half_rn((acc[nt][1] + acc[nt][3]) * inv);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::mutex g_enc_mu;
+
+int encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
+    std::lock_guard<std::mutex> lk(g_enc_mu);
+    if (!g_encode) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+            return fail(TASP_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    *out = g_encode;
+    return TASP_OK;
+}
+
+// 2-D FP16 tensor map of a row-major [rows][ld] buffer (cols used), box = box_rows x 64.
+int make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc;
+    int rc = encoder(&enc);
+    if (rc) return rc;
+    if ((reinterpret_cast<uintptr_t>(base) & 15) || (ld * 2) % 16)
+        return fail(TASP_EINVAL, "TMA operand not 16-byte aligned");
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(TASP_ECUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+    return TASP_OK;
+}
+
+int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, const GemmArgs& ga,
+                cudaStream_t s) {
+    if (M == 0 || N == 0) return TASP_OK;
+    CUtensorMap ta, tb;
+    int rc = make_map(&ta, A, M, K, lda, BM);
+    if (rc) return rc;
+    if ((rc = make_map(&tb, B, N, K, ldb, BN))) return rc;
+    static bool attr = false;
+    if (!attr) {
+        TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMM_SMEM));
+        attr = true;
+    }
+    dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM);
+    gemm_tc_kernel<<<grid, GEMM_THREADS, GEMM_SMEM, s>>>(ta, tb, ga);
+    TASP_CUDA(cudaGetLastError());
+    return TASP_OK;
+}
+
+int round8(int v) { return (v + 7) & ~7; }
+
+// FP16 copies of a plan's panels for the prefill GEMMs (made on first use, kept by the plan).
+int ensure_f16_panels(Plan& p, cudaStream_t s) {
+    if (p.f16_ready) return TASP_OK;
+    const Shape& sh = p.store->sh;
+    size_t total = 0;
+    for (const LayerPlan& lp : p.layers) {
+        total += ((size_t)lp.qkv_rows * round8(sh.d) + (size_t)sh.d * round8(lp.o_K) + (size_t)lp.gu_rows * round8(sh.d) +
+                  (size_t)sh.d * round8(lp.dn_K)) * 2 + 4 * 256;
+    }
+    int rc = p.f16_arena.reserve(total);
+    if (rc) return rc;
+    p.f16.resize(sh.L);
+    for (int l = 0; l < sh.L; ++l) {
+        const LayerPlan& lp = p.layers[l];
+        F16Panels& f = p.f16[l];
+        f.ld_d = round8(sh.d);
+        f.ld_o = round8(lp.o_K);
+        f.ld_dn = round8(lp.dn_K);
+        f.qkv = (__half*)p.f16_arena.take((size_t)lp.qkv_rows * f.ld_d * 2);
+        f.o = (__half*)p.f16_arena.take((size_t)sh.d * f.ld_o * 2);
+        f.gu = (__half*)p.f16_arena.take((size_t)lp.gu_rows * f.ld_d * 2);
+        f.dn = (__half*)p.f16_arena.take((size_t)sh.d * f.ld_dn * 2);
+        if (lp.qkv_rows) i8_to_f16_kernel<<<lp.qkv_rows, 256, 0, s>>>(lp.qkv_w, lp.qkv_map, sh.d, sh.d, f.qkv, f.ld_d);
+        if (lp.o_K) i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.o_w, nullptr, lp.o_ld, lp.o_K, f.o, f.ld_o);
+        if (lp.gu_rows) i8_to_f16_kernel<<<lp.gu_rows, 256, 0, s>>>(lp.gu_w, lp.gu_map, sh.d, sh.d, f.gu, f.ld_d);
+        if (lp.dn_K) i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.dn_w, nullptr, lp.dn_ld, lp.dn_K, f.dn, f.ld_dn);
+        TASP_CUDA(cudaGetLastError());
+    }
+    TASP_CUDA(cudaStreamSynchronize(s));
+    p.f16_ready = true;
+    return TASP_OK;
+}
+
+}  // namespace
+
+int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
+    Plan& pl = *se.plan;
+    const Shape& sh = pl.store->sh;
+    int rc = ensure_f16_panels(pl, s);
+    if (rc) return rc;
+    int max_rows = 0, max_c = 0, max_oK = 0;
+    for (const LayerPlan& lp : pl.layers) {
+        max_rows = std::max(max_rows, lp.qkv_rows);
+        max_c = std::max(max_c, lp.c);
+        max_oK = std::max(max_oK, lp.o_K);
+    }
+    const int ld_x = round8(sh.d), ld_y = std::max(4, (max_rows + 3) & ~3), ld_o = round8(std::max(8, sh.Hq * sh.dh)),
+              ld_h = round8(std::max(8, max_c));
+    // workspace (stream-ordered, released at the end of the prefill)
+    float *X = nullptr, *Y = nullptr, *Qf = nullptr;
+    __half *Xh = nullptr, *O = nullptr, *H = nullptr;
+    TASP_CUDA(cudaMallocAsync((void**)&X, (size_t)T * sh.d * 4, s));
+    TASP_CUDA(cudaMallocAsync((void**)&Xh, (size_t)T * ld_x * 2, s));
+    TASP_CUDA(cudaMallocAsync((void**)&Y, (size_t)T * ld_y * 4, s));
+    TASP_CUDA(cudaMallocAsync((void**)&Qf, (size_t)T * sh.Hq * sh.dh * 4, s));
+    TASP_CUDA(cudaMallocAsync((void**)&O, (size_t)T * ld_o * 2, s));
+    TASP_CUDA(cudaMallocAsync((void**)&H, (size_t)T * ld_h * 2, s));
+    TASP_CUDA(cudaMemsetAsync(O, 0, (size_t)T * ld_o * 2, s));
+    TASP_CUDA(cudaMemsetAsync(H, 0, (size_t)T * ld_h * 2, s));
+    const float qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
+    for (int l = 0; l < sh.L && !rc; ++l) {
+        const LayerPlan& lp = pl.layers[l];
+        const F16Panels& f = pl.f16[l];
+        rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, l == 0 ? d_embeds : nullptr, X, sh.d, lp.g_attn, sh.eps, Xh, ld_x);
+        TASP_CUDA(cudaGetLastError());
+        if (lp.m_kv > 0) {
+            GemmArgs ga{};
+            ga.M = T; ga.N = lp.qkv_rows; ga.K = sh.d; ga.scale = lp.qkv_s; ga.out = Y; ga.ldo = ld_y;
+            ga.mode = EP_STORE; ga.err = se.err;
+            if ((rc = launch_gemm(Xh, ld_x, T, f.qkv, f.ld_d, lp.qkv_rows, sh.d, ga, s))) break;
+            rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, Qf, se.K[l], se.V[l],
+                                                            se.max_tokens);
+            const int qb = (T + PA_QB - 1) / PA_QB;
+            if (sh.dh == 128)
+                attn_prefill_kernel<128><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, 0, s>>>(
+                    Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
+            else
+                attn_prefill_kernel<64><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, 0, s>>>(
+                    Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
+            TASP_CUDA(cudaGetLastError());
+            GemmArgs go{};
+            go.M = T; go.N = sh.d; go.K = lp.o_K; go.scale = lp.o_s; go.out = X; go.ldo = sh.d;
+            go.mode = EP_RESID; go.err = se.err;
+            if ((rc = launch_gemm(O, ld_o, T, f.o, f.ld_o, sh.d, lp.o_K, go, s))) break;
+        }
+        if (lp.c > 0) {
+            rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, nullptr, nullptr, sh.d, lp.g_mlp, sh.eps, Xh, ld_x);
+            TASP_CUDA(cudaGetLastError());
+            GemmArgs gg{};
+            gg.M = T; gg.N = lp.gu_rows; gg.K = sh.d; gg.scale = lp.gu_s; gg.hout = H; gg.ldh = ld_h;
+            gg.mode = EP_SWIGLU; gg.err = se.err;
+            if ((rc = launch_gemm(Xh, ld_x, T, f.gu, f.ld_d, lp.gu_rows, sh.d, gg, s))) break;
+            GemmArgs gd{};
+            gd.M = T; gd.N = sh.d; gd.K = lp.c; gd.scale = lp.dn_s; gd.out = X; gd.ldo = sh.d;
+            gd.mode = EP_RESID; gd.err = se.err;
+            if ((rc = launch_gemm(H, ld_h, T, f.dn, f.ld_dn, sh.d, lp.c, gd, s))) break;
+        }
+    }
+    if (!rc) {
+        // the last prompt position's residual seeds the session (final norm + LM head read it)
+        cudaError_t e = cudaMemcpyAsync(se.x, X + (size_t)(T - 1) * sh.d, (size_t)sh.d * 4, cudaMemcpyDeviceToDevice, s);
+        if (e != cudaSuccess) rc = cuda_fail(e, "prefill residual copy");
+    }
+    cudaFreeAsync(X, s);
+    cudaFreeAsync(Xh, s);
+    cudaFreeAsync(Y, s);
+    cudaFreeAsync(Qf, s);
+    cudaFreeAsync(O, s);
+    cudaFreeAsync(H, s);
+    return rc;
+}
+
+}  // namespace tasp

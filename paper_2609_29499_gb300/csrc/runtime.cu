@@ -582,9 +582,50 @@ int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* 
 
 int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t max_new_tokens, void* stream,
                  tasp_session** out, float* d_logits_last) {
-    (void)plan; (void)d_embeds_bf16; (void)T; (void)max_new_tokens; (void)stream; (void)d_logits_last;
-    if (out) *out = nullptr;
-    return fail(TASP_EUNSUP, "prefill is not built yet");
+    if (!out) return fail(TASP_EINVAL, "out is NULL");
+    *out = nullptr;
+    Plan* p = as_plan(plan);
+    if (!p) return fail(TASP_EINVAL, "invalid plan handle");
+    if (!d_embeds_bf16 || T < 1 || max_new_tokens < 0) return fail(TASP_EINVAL, "bad prompt (NULL or T < 1)");
+    const Shape& sh = p->store->sh;
+    if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
+    if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
+    Session* se = nullptr;
+    int rc = session_alloc(p, T + max_new_tokens, &se);
+    if (rc) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    rc = prefill_run(*se, (const uint16_t*)d_embeds_bf16, T, st);
+    if (!rc) rc = enqueue_set_pos(*se, T, st);
+    if (!rc && d_logits_last) rc = enqueue_lm_head(*se, d_logits_last, st);
+    if (rc) {
+        cudaStreamSynchronize(st);
+        session_free(se);
+        return rc;
+    }
+    se->pos = T;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        p->live_sessions++;
+    }
+    *out = (tasp_session*)se;
+    return TASP_OK;
+}
+
+int tasp_session_kv_export(const tasp_session* s, int32_t layer, int32_t which, void* h_dst, size_t bytes) {
+    Session* se = as_session((void*)s);
+    if (!se || !h_dst) return fail(TASP_EINVAL, "invalid session or NULL destination");
+    const Shape& sh = se->plan->store->sh;
+    if (layer < 0 || layer >= sh.L || (which != 0 && which != 1)) return fail(TASP_EINVAL, "bad layer or item");
+    const int m = se->plan->layers[layer].m_kv;
+    const size_t row = (size_t)sh.dh * 2;
+    if (bytes != (size_t)m * se->pos * row)
+        return fail(TASP_EINVAL, "kv export size mismatch: expected " + std::to_string((size_t)m * se->pos * row));
+    if (bytes == 0) return TASP_OK;
+    TASP_CUDA(cudaDeviceSynchronize());
+    const uint16_t* src = which == 0 ? se->K[layer] : se->V[layer];
+    TASP_CUDA(cudaMemcpy2D(h_dst, (size_t)se->pos * row, src, (size_t)se->max_tokens * row, (size_t)se->pos * row, m,
+                           cudaMemcpyDeviceToHost));
+    return TASP_OK;
 }
 
 int tasp_release(void* handle) {
@@ -606,6 +647,7 @@ int tasp_release(void* handle) {
         }
         cudaError_t e = cudaDeviceSynchronize();
         p->arena.release();
+        p->f16_arena.release();
         store_release(p->store);
         p->magic = 0;
         delete p;

@@ -1,6 +1,7 @@
 // Internal structures of the TASP runtime: shared store, plans, sessions, kernel parameters.
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -98,6 +99,12 @@ struct LayerPlan {
     const float *g_attn = nullptr, *g_mlp = nullptr;
 };
 
+// FP16 copies of a layer's panels (row strides padded to 8 elements) for the prefill GEMMs.
+struct F16Panels {
+    __half *qkv = nullptr, *o = nullptr, *gu = nullptr, *dn = nullptr;
+    int ld_d = 0, ld_o = 0, ld_dn = 0;
+};
+
 constexpr uint32_t PLAN_MAGIC = 0x7A5B1A01u;
 constexpr uint32_t SESSION_MAGIC = 0x7A5B5E55u;
 
@@ -111,6 +118,9 @@ struct Plan {
     Arena arena;
     int64_t flops_retained = 0, flops_dense = 0, launched_flops = 0;
     int64_t weight_bytes_per_token = 0;
+    bool f16_ready = false;  // FP16 panels made on the first prefill
+    Arena f16_arena;
+    std::vector<F16Panels> f16;
 };
 
 // ---------------------------------------------------------------- sessions
@@ -201,5 +211,13 @@ using KernelHook = void (*)(void* ctx, int kind, bool before);
 // Enqueue one decode step (or one isolated layer when only_layer >= 0) on `s`.
 int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
                  int* launches);
+// Final RMSNorm + LM head on the session's residual (se.x) into logits [vocab].
+int enqueue_lm_head(Session& se, float* logits, cudaStream_t s);
+// Device position of a session := pos.
+int enqueue_set_pos(Session& se, int pos, cudaStream_t s);
+
+// prefill.cu: run the prompt [T][d] (BF16) through the plan, filling KV positions 0..T-1
+// and leaving the last position's residual in se.x.
+int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s);
 
 }  // namespace tasp

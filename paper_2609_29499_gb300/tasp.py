@@ -29,7 +29,8 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
-            "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_last_error",
+            "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
+            "tasp_last_error",
             "tasp_version")
 
 
@@ -92,6 +93,7 @@ def load(path: str = LIB_PATH):
         "tasp_profile_step": (c_int32, [POINTER(P), c_int32, P, P, P, P, P]),
         "tasp_step_launches": (c_int32, [POINTER(P), c_int32, c_int32, POINTER(c_int32)]),
         "tasp_decode_step_static": (c_int32, [P, P, P, P, P]),
+        "tasp_session_kv_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
         "tasp_last_error": (ctypes.c_char_p, []),
         "tasp_version": (ctypes.c_char_p, []),
     }
@@ -240,6 +242,23 @@ class Session:
         v = c_int32()
         _check(load().tasp_session_position(self.handle, ctypes.byref(v)))
         return v.value
+
+    @classmethod
+    def prefill(cls, plan: "Plan", embeds_bf16, max_new_tokens: int, logits=None, stream=None) -> "Session":
+        """Prefill a prompt (CUDA bfloat16 tensor [T, d]) into a new session bound to `plan`."""
+        h = c_void_p()
+        _check(load().tasp_prefill(plan.handle, embeds_bf16.data_ptr(), int(embeds_bf16.shape[0]), max_new_tokens,
+                                   _stream_ptr(stream), ctypes.byref(h),
+                                   logits.data_ptr() if logits is not None else None))
+        return cls(plan, 0, handle=h)
+
+    def kv(self, layer: int, which: int) -> np.ndarray:
+        """Cached keys (which=0) or values (1) of a layer: BF16 bits [m_kv, position, dh]."""
+        m_kv, _ = self.plan.layer_dims(layer)
+        pos = self.position
+        out = np.zeros((m_kv, pos, self.plan.shape.dh), np.uint16)
+        _check(load().tasp_session_kv_export(self.handle, layer, which, out.ctypes.data, out.nbytes))
+        return out
 
     def device_error(self, clear=True) -> int:
         """Device error word of this session's kernels (0 = none); synchronizes."""
