@@ -53,6 +53,9 @@ def parse():
     ap.add_argument("--dense", action="store_true", help="time the dense fallback plan instead of the mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--workload", choices=["decode", "prefill"], default="decode",
+                    help="decode (the headline metric) or the prefill of one prompt on the 8B shape")
+    ap.add_argument("--prompt", type=int, default=2048, help="prefill prompt length")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep the workload's widths but only this many layers (small cases for ncu captures)")
     return ap.parse_args()
@@ -382,10 +385,77 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def measured_tensor_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def run_prefill(args):
+    """Prefill of one prompt on the 8B shape with a 43% mask; reports ms and tensor TFLOP/s."""
+    import dataclasses
+
+    import torch
+    from paper_2609_29499_gb300 import build
+    build.build()
+    from paper_2609_29499_gb300 import tasp
+    tasp.load()
+    wl = synth.CFG4
+    sh = wl.shape if not args.layers else dataclasses.replace(wl.shape, L=args.layers)
+    recipe = wl.masks[0]
+    T = args.prompt
+    sc = synth.mask_scores_u32(recipe.mask_seed, sh.L, sh.n_units)
+    tg = synth.layer_target_u24(recipe.mask_seed, sh.L)
+    plan = tasp.Plan(sh, tasp.greedy_mask(sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi))
+    info = plan.info()
+    dims = [plan.layer_dims(l) for l in range(sh.L)]
+    sess = tasp.Session(plan, T + wl.steps)
+    emb = torch.from_numpy(synth.prompt_bf16(wl.x_seed, 0, T, sh.d).view(np.int16)).view(torch.bfloat16).cuda()
+    logits = torch.empty(sh.vocab, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        sess.prefill_into(emb, logits)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    for _ in range(args.steps):
+        sess.prefill_into(emb, logits)
+    ev1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    gemm_flops = info["launched_flops"] * T
+    g = sh.Hq // sh.Hkv
+    attn_flops = sum(2 * 2 * m * g * sh.dh * T * (T + 1) // 2 for m, _ in dims)
+    peak, kind = measured_tensor_peak()
+    tflops = (gemm_flops + attn_flops) / (ms * 1e-3) / 1e12
+    err = sess.device_error()
+    sess.release()
+    plan.release()
+    out = {"metric": f"prefill ms/prompt (8B-shape, 43% mask, {T} tokens)", "value": round(ms, 3), "unit": "ms",
+           "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+           "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f16xint8-f32acc",
+           "data": "synthetic",
+           "config": {"workload": f"llama3_8b_prefill_{T}" + (f"_{args.layers}layers" if args.layers else ""),
+                      "tokens_per_s": round(T / (ms * 1e-3), 1)},
+           "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": peak, "unit": "TFLOP/s",
+                        "frac": round(tflops / peak, 4), "peak_source": f"{kind} bf16_tflops (FP16 runs at the same rate)",
+                        "flops_gemm": gemm_flops, "flops_attention": attn_flops, "traffic": None},
+           "clocks": clocks, "device_error": err,
+           "paper_context": {"prefill_ms_2048_sparse": 1326, "prefill_ms_2048_dense": 1814, "hardware": "A100, 70B"}}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "prefill":
+        run_prefill(args)
     else:
         run_ours(args)
 

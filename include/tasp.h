@@ -141,6 +141,12 @@ int tasp_release(void* handle);
 /* Empty session on a plan with KV capacity max_tokens (position 0). sync. */
 int tasp_session_create(tasp_plan* plan, int32_t max_tokens, tasp_session** out);
 
+/* Prefill a prompt into an existing session (its previous contents are
+ * overwritten from position 0; capacity must be >= T): the same computation as
+ * tasp_prefill without allocating the session. async. Errors: EINVAL, ECAP,
+ * EUNSUP, ECUDA. */
+int tasp_session_prefill(tasp_session* s, const void* d_embeds_bf16, int32_t T, void* stream, float* d_logits_last);
+
 /* Fill positions [0, t_prior) of a session's KV cache with the synthetic
  * N(0,1) BF16 "prior tokens" keyed by kv_seed (the keys are taken as already
  * rotated) and set its position to t_prior. async. Errors: ECAP, EINVAL. */

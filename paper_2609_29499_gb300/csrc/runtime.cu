@@ -611,6 +611,23 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
     return TASP_OK;
 }
 
+int tasp_session_prefill(tasp_session* s, const void* d_embeds_bf16, int32_t T, void* stream, float* d_logits_last) {
+    Session* se = as_session(s);
+    if (!se) return fail(TASP_EINVAL, "invalid session handle");
+    const Shape& sh = se->plan->store->sh;
+    if (!d_embeds_bf16 || T < 1) return fail(TASP_EINVAL, "bad prompt (NULL or T < 1)");
+    if (T > se->max_tokens) return fail(TASP_ECAP, "prompt longer than the session capacity");
+    if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
+    if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
+    cudaStream_t st = (cudaStream_t)stream;
+    int rc = prefill_run(*se, (const uint16_t*)d_embeds_bf16, T, st);
+    if (!rc) rc = enqueue_set_pos(*se, T, st);
+    if (!rc && d_logits_last) rc = enqueue_lm_head(*se, d_logits_last, st);
+    if (rc) return rc;
+    se->pos = T;
+    return TASP_OK;
+}
+
 int tasp_session_kv_export(const tasp_session* s, int32_t layer, int32_t which, void* h_dst, size_t bytes) {
     Session* se = as_session((void*)s);
     if (!se || !h_dst) return fail(TASP_EINVAL, "invalid session or NULL destination");

@@ -30,6 +30,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
+            "tasp_session_prefill",
             "tasp_last_error",
             "tasp_version")
 
@@ -94,6 +95,7 @@ def load(path: str = LIB_PATH):
         "tasp_step_launches": (c_int32, [POINTER(P), c_int32, c_int32, POINTER(c_int32)]),
         "tasp_decode_step_static": (c_int32, [P, P, P, P, P]),
         "tasp_session_kv_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
+        "tasp_session_prefill": (c_int32, [P, P, c_int32, P, P]),
         "tasp_last_error": (ctypes.c_char_p, []),
         "tasp_version": (ctypes.c_char_p, []),
     }
@@ -251,6 +253,11 @@ class Session:
                                    _stream_ptr(stream), ctypes.byref(h),
                                    logits.data_ptr() if logits is not None else None))
         return cls(plan, 0, handle=h)
+
+    def prefill_into(self, embeds_bf16, logits=None, stream=None):
+        """Prefill a prompt into this (existing) session from position 0."""
+        _check(load().tasp_session_prefill(self.handle, embeds_bf16.data_ptr(), int(embeds_bf16.shape[0]),
+                                           _stream_ptr(stream), logits.data_ptr() if logits is not None else None))
 
     def kv(self, layer: int, which: int) -> np.ndarray:
         """Cached keys (which=0) or values (1) of a layer: BF16 bits [m_kv, position, dh]."""
