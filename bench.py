@@ -35,10 +35,9 @@ import synth  # noqa: E402
 
 METRIC = "decode ms/token (70B-shape, 43% mask, bs1); achieved HBM GB/s vs ~8 TB/s"
 # DRAM traffic over algorithmic bytes of one launch, from one ncu capture of the kernel
-# (dram__bytes_read.sum + dram__bytes_write.sum of a 70B-width gate/up launch with 12,288
-# kept channels: 205,311,744 B against 201,539,584 algorithmic). Must be re-taken (or set
-# to None) whenever the kernel changes.
-TRAFFIC_PER_ALGORITHMIC = {"gate_up": 205311744 / 201539584}
+# (dram__bytes_read.sum + dram__bytes_write.sum of a 70B-width launch). Empty until the
+# current kernel has been captured; re-taken whenever the kernel changes.
+TRAFFIC_PER_ALGORITHMIC = {}
 PAPER_CONTEXT = {"ms_per_token_sparse": 31.3, "ms_per_token_dense": 45.2,
                  "hardware": "1x A100 80GB SXM, real Llama-3-70B, groupwise INT8, ~2k context"}
 
@@ -53,8 +52,12 @@ def parse():
     ap.add_argument("--dense", action="store_true", help="time the dense fallback plan instead of the mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", choices=["decode", "prefill"], default="decode",
-                    help="decode (the headline metric) or the prefill of one prompt on the 8B shape")
+    ap.add_argument("--workload", choices=["decode", "prefill", "mixed"], default="decode",
+                    help="decode (the headline metric), the prefill of one prompt on the 8B shape, or "
+                         "mixed-turn serving (70B shape, 16 turns over the dense plan and five masks)")
+    ap.add_argument("--panels", choices=["row-indexed", "compact"], default="row-indexed",
+                    help="mixed workload: Q/K/V and gate/up panels as row maps into the shared store "
+                         "(zero copy) or materialized copies")
     ap.add_argument("--prompt", type=int, default=2048, help="prefill prompt length")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep the workload's widths but only this many layers (small cases for ncu captures)")
@@ -450,12 +453,162 @@ def run_prefill(args):
     print(json.dumps(out), flush=True)
 
 
+def run_mixed(args):
+    """Mixed-turn serving on the 70B shape: 16 turns, each bound to the dense plan (p = 0.1)
+    or one of five masks (seeded), prompts of U[256, 2048] synthetic prior tokens; every
+    step decodes one token for every turn, grouped per plan (up to four sessions share a
+    weight pass). Reports aggregate tokens/s."""
+    import dataclasses
+
+    import torch
+    from paper_2609_29499_gb300 import build
+    build.build()
+    from paper_2609_29499_gb300 import tasp
+    tasp.load()
+    wl = synth.CFG5
+    sh = wl.shape if not args.layers else dataclasses.replace(wl.shape, L=args.layers)
+    K, Wm = args.steps, args.warmup
+    turns = synth.turn_assignment(wl.x_seed, wl.n_turns, len(wl.masks), wl.p_dense, *wl.prompt_lens)
+    n = len(turns)
+    mode = tasp.PANELS_ROW_INDEXED if args.panels == "row-indexed" else tasp.PANELS_COMPACT
+    t0 = time.perf_counter()
+    plans = {}
+    for pi, _ in turns:
+        if pi in plans:
+            continue
+        if pi == len(wl.masks):
+            plans[pi] = tasp.Plan(sh, tasp.all_keep_mask())
+        else:
+            r = wl.masks[pi]
+            sc = synth.mask_scores_u32(r.mask_seed, sh.L, sh.n_units)
+            tg = synth.layer_target_u24(r.mask_seed, sh.L)
+            plans[pi] = tasp.Plan(sh, tasp.greedy_mask(sc, tg, r.budget, r.r_lo, r.r_hi, mode))
+    setup_s = time.perf_counter() - t0
+    e2e_steps = 0 if args.no_e2e else K
+    sessions = []
+    for i, (pi, T) in enumerate(turns):
+        s = tasp.Session(plans[pi], T + Wm + K + e2e_steps + 2)
+        s.fill_synthetic(T, wl.kv_seed + i)
+        sessions.append(s)
+    groups = {}
+    for i, (pi, _) in enumerate(turns):
+        groups.setdefault(pi, []).append(i)
+    xb = synth.step_inputs_bf16(wl.x_seed, Wm + K + 1, n, sh.d)
+    xg = {pi: torch.from_numpy(np.ascontiguousarray(xb[:, idx]).view(np.int16)).view(torch.bfloat16).cuda()
+          for pi, idx in groups.items()}
+    lg = {pi: torch.empty((len(idx), sh.vocab), dtype=torch.float32, device="cuda") for pi, idx in groups.items()}
+    gs = {pi: [sessions[i] for i in idx] for pi, idx in groups.items()}
+    stream = torch.cuda.current_stream()
+
+    def step(t):
+        for pi in groups:
+            tasp.decode_step(gs[pi], xg[pi][t], None, lg[pi])
+
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    for t in range(Wm):
+        step(t)
+    torch.cuda.synchronize()
+    ctx0 = [s.position for s in sessions]
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for t in range(K):
+        step(Wm + t)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1) / K
+    tok_s = n / (ms * 1e-3)
+    errs = sum(s.device_error() for s in sessions)
+
+    # roofline: per-kernel times of one eager step of every group, bytes from each plan's ledger
+    prof_tot, bytes_tot = {}, {}
+    step_bytes = 0
+    per_group = {}
+    for pi, idx in groups.items():
+        dims = [plans[pi].layer_dims(l) for l in range(sh.L)]
+        passes = (len(idx) + 3) // 4
+        gb = gemv_bytes(sh, dims)
+        prof = tasp.profile_step(gs[pi], xg[pi][Wm + K], lg[pi])
+        for k, (msk, cnt) in prof.items():
+            a = prof_tot.setdefault(k, [0.0, 0])
+            a[0] += msk
+            a[1] += cnt
+            if k in gb:
+                bytes_tot[k] = bytes_tot.get(k, 0) + gb[k] * passes
+        wbytes = plans[pi].info()["weight_bytes_per_token"] * passes
+        kvb = sum(kv_bytes(dims, sh.dh, ctx0[i] + K // 2 + 1) for i in idx)
+        step_bytes += wbytes + kvb
+        per_group[("dense" if pi == len(wl.masks) else f"mask{pi}")] = {"sessions": len(idx),
+                                                                         "weight_passes": passes}
+    peak, peak_kind = measured_peak()
+    kinds = {k: v for k, v in prof_tot.items() if v[1] > 0}
+    dominant = max(kinds, key=lambda k: kinds[k][0])
+    dur_ms, launches = kinds[dominant]
+    per_launch = bytes_tot.get(dominant, 0) / max(1, launches)
+    achieved = per_launch / (dur_ms / launches * 1e-3) / 1e9 if dominant in bytes_tot else None
+    roofline = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1) if achieved else None,
+                "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4) if achieved else None,
+                "peak_source": f"{peak_kind} hbm_gbs (copy bandwidth)", "bytes_per_launch": int(per_launch),
+                "launch_us": round(dur_ms / launches * 1e3, 2), "traffic": None}
+    step_gbs = step_bytes / (ms * 1e-3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        xh = {pi: torch.from_numpy(np.ascontiguousarray(xb[:, idx]).view(np.int16)).view(torch.bfloat16).pin_memory()
+              for pi, idx in groups.items()}
+        lh = {pi: torch.empty((len(idx), sh.vocab), dtype=torch.float32).pin_memory() for pi, idx in groups.items()}
+        for pi in groups:
+            tasp.decode_step_host(gs[pi], xh[pi][0], None, lh[pi])  # records the host-path graphs once
+        te = time.perf_counter()
+        for t in range(1, K):
+            for pi in groups:
+                tasp.decode_step_host(gs[pi], xh[pi][t], None, lh[pi])
+        e2e_ms = (time.perf_counter() - te) * 1e3 / max(1, K - 1)
+        e2e = {"value": round(n / (e2e_ms * 1e-3), 2), "unit": "tokens/s", "h2d_bytes_per_step": n * sh.d * 2,
+               "d2h_bytes_per_step": n * sh.vocab * 4}
+    launches = sum(tasp.step_launches(gs[pi], with_logits=True) for pi in groups)
+    for s in sessions:
+        s.release()
+    for p in plans.values():
+        p.release()
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        mean_T = int(round(np.mean([T for _, T in turns])))
+        wl_c = dataclasses.replace(wl, t_prior=mean_T)
+        per_step, cinfo = cpu_oracle_sample(sh, wl.masks[0], wl_c, 3)
+        cinfo["value"] = round(1e3 / float(np.mean(per_step)), 4)
+        cinfo["unit"] = "tokens/s"
+        cinfo["sample"] += "; the oracle decodes the turns one after another, so tokens/s = 1 / (s per token)"
+        cpu = cinfo
+
+    out = {"metric": "mixed-turn decode tokens/s (70B-shape, 16 turns over dense + 5 masks, grouped per plan)",
+           "value": round(tok_s, 2), "unit": "tokens/s", "n_gpus": 1, "steps": K, "warmup": Wm,
+           "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "int8w-f32", "data": "synthetic",
+           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else ""), "turns": n,
+                      "plans": {("dense" if pi == len(wl.masks) else f"mask{pi}"): len(idx)
+                                for pi, idx in groups.items()},
+                      "prompt_tokens": [T for _, T in turns], "panels": args.panels,
+                      "l2": "inputs larger than L2 (each step streams every plan's weights)"},
+           "groups": per_group,
+           "roofline": roofline,
+           "step_roofline": {"bytes_per_step": int(step_bytes), "achieved": round(step_gbs, 1), "peak": peak,
+                             "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
+           "e2e": e2e, "gpu_launches": launches * K, "clocks": clocks, "cpu_baseline": cpu,
+           "device_error": errs, "setup_s": round(setup_s, 1)}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
     elif args.workload == "prefill":
         run_prefill(args)
+    elif args.workload == "mixed":
+        run_mixed(args)
     else:
         run_ours(args)
 

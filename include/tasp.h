@@ -121,9 +121,15 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
  * vectors, session order). Outputs, each optional (NULL skips it):
  * d_hidden_out FP32 [n][d] = the residual stream after the last decoder layer
  * (before the final norm); d_logits FP32 [n][vocab]. Each session's KV grows by
- * one position. The step is replayed from a CUDA graph captured on first use
- * for this (sessions, buffers) combination; call it outside any stream capture.
- * async on `stream`.
+ * one position. Sessions are taken in groups of up to 4 (session order): the
+ * GEMVs of a group read every weight byte once for all of its sessions and one
+ * attention grid covers them, each on its own KV cache and position (the decode
+ * step groups the turns that share a mask). A group of 2-4 sessions keeps a step
+ * workspace (~ n x (d + 2 H_q d_h + d_f + vocab) x 4 bytes plus attention
+ * partials) until one of its sessions is released. Results per session do not
+ * depend on the group (up to FP32 summation order). The step is replayed from a
+ * CUDA graph captured on first use for this (sessions, buffers) combination;
+ * call it outside any stream capture. async on `stream`.
  * Errors: EMASK (sessions on different plans), ECAP (a session is full),
  * EINVAL, ENOMEM, ECUDA. */
 int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,
@@ -222,7 +228,8 @@ int tasp_layer_step(tasp_session* s, int32_t layer, const float* d_x_in, float* 
  * the total time and launch count of kernel kind k over the step:
  * 0 qkv (RMSNorm + QKV GEMV + RoPE + KV append), 1 attention (split-KV + combine),
  * 2 o-proj + residual, 3 gate/up + SiLU*up, 4 down + residual, 5 final norm +
- * LM head, 6 other. Arrays have TASP_KERNEL_KINDS entries. */
+ * LM head, 6 other. Arrays have TASP_KERNEL_KINDS entries. Sessions are grouped
+ * as in tasp_decode_step. */
 #define TASP_KERNEL_KINDS 7
 int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_logits,
                       void* stream, float* h_ms, int32_t* h_count);
@@ -233,7 +240,7 @@ int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_
 int tasp_session_kv_export(const tasp_session* s, int32_t layer, int32_t which, void* h_dst, size_t bytes);
 
 /* Number of library kernel launches one decode step of these sessions makes
- * (graph nodes). */
+ * (graph nodes): one launch sequence per group of up to 4 sessions. */
 int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_logits, int32_t* out);
 
 /* ---------------------------------------------------------------------------

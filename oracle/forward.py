@@ -186,6 +186,34 @@ def decode(shape, mask, x_steps, t_prior, kv_seed, compact=False, dtype=np.float
     return X
 
 
+def decode_sessions(shape, mask, x_steps, t_priors, kv_seeds, dtype=np.float32):
+    """Teacher-forced decode of several independent sessions on one mask (Sec. 3.3: the
+    turns that share a mask share its plan; each keeps its own KV cache and position).
+
+    x_steps [S, n, d]; session i starts from its synthetic prior cache of t_priors[i]
+    tokens keyed by kv_seeds[i]. Each session is exactly ``decode`` of its own inputs;
+    the loop visits layers outermost only so that a layer's weights are made once.
+    Returns [S, n, d].
+    """
+    X = np.array(x_steps, dtype=dtype)
+    S, n = X.shape[0], X.shape[1]
+    for layer in range(shape.L):
+        lq = wts.gen_layer(shape, layer)
+        W = wts.dense_zeroed(shape, lq, mask.keep_groups[layer], mask.keep_chans[layer], dtype)
+        for i in range(n):
+            tp = int(t_priors[i])
+            Kc, Vc = prior_cache(shape, layer, kv_seeds[i], tp, None, dtype)
+            Kall = np.zeros((Kc.shape[0], tp + S, shape.dh), dtype)
+            Vall = np.zeros_like(Kall)
+            Kall[:, :tp], Vall[:, :tp] = Kc, Vc
+            for t in range(S):
+                T = tp + t
+                X[t, i], k, v = layer_step(shape, W, X[t, i], Kall[:, :T], Vall[:, :T], T)
+                Kall[:, T], Vall[:, T] = k, v
+        del W
+    return X
+
+
 def final_logits(shape, x, dtype=np.float32, rows=None, chunk=8192):
     """logits = W_lm RMSNorm(x) gamma_final for x [S, d]; ``rows`` selects vocabulary rows."""
     xn = rmsnorm(np.asarray(x, dtype=dtype), wts.gamma_final(shape).astype(dtype), shape.eps)

@@ -108,16 +108,23 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     __shared__ __align__(16) float cacc[8][DH];  // this CTA's merged unnormalized output
     __shared__ float Mh[8], Lh[8], wts[CLUSTERS_MAX][8];
     __shared__ int is_last;
-    const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x;
+    const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x, bz = blockIdx.z;
     const int NC = S / CS, cid = split / CS;
+    // session bz of the batch
+    const float* const q_in = p.q + bz * p.q_stride;
+    float* const o_out = p.o + bz * p.q_stride;
+    float* const part = p.part + bz * p.part_stride;
+    float* const ml = p.ml + bz * p.ml_stride;
+    int* const cnt = p.cnt + bz * p.cnt_stride;
+    const int max_tokens = p.max_tokens[bz];
     const uint32_t rank = cluster_rank();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-    const int T = *p.pos + 1;  // written by the previous step, which has completed
+    const int T = *p.pos[bz] + 1;  // written by the previous step, which has completed
     const int chunk = (((T + S - 1) / S) + TILE - 1) / TILE * TILE;
     const int p0 = min(T, split * chunk), p1 = min(T, p0 + chunk);
-    const uint16_t* Kg = p.K + (int64_t)jl * p.max_tokens * DH;
-    const uint16_t* Vg = p.V + (int64_t)jl * p.max_tokens * DH;
+    const uint16_t* Kg = p.K[bz] + (int64_t)jl * max_tokens * DH;
+    const uint16_t* Vg = p.V[bz] + (int64_t)jl * max_tokens * DH;
     const int ntiles = (p1 - p0 + TILE - 1) / TILE;
     const int dep_tile = (p1 == T && ntiles > 0) ? ntiles - 1 : -1;  // holds this step's new token
 
@@ -156,7 +163,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             const int col = ks * 16 + half * 8 + qc;
             float x0 = 0.f, x1 = 0.f;
             if (h < G) {
-                const float* qp = p.q + (int64_t)(jl * G + h) * DH + col;
+                const float* qp = q_in + (int64_t)(jl * G + h) * DH + col;
                 x0 = qp[0] * p.qscale;
                 x1 = qp[1] * p.qscale;
             }
@@ -294,12 +301,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             As = fmaf(ld_cluster(map_to_rank(ca_a + 4 * (hh * DH + dim), r)), e, As);
         }
         if (NC == 1) {
-            p.o[(int64_t)(jl * G + hh) * DH + dim] = As / Ls;
+            o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Ls;
         } else {
-            p.part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
+            part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
             if (dim == 0) {
-                p.ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = M;
-                p.ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Ls;
+                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = M;
+                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Ls;
             }
         }
     }
@@ -309,11 +316,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
 
     // ---- several clusters per group: the last one (ticket) merges their partials
     if (rank != 0) return;
-    if (tid == 0) is_last = (atomicAdd(p.cnt + jl, 1) == NC - 1);
+    if (tid == 0) is_last = (atomicAdd(cnt + jl, 1) == NC - 1);
     __syncthreads();
     if (!is_last) return;
     __threadfence();
-    const float* mlg = p.ml + (int64_t)jl * NC * G * 2;
+    const float* mlg = ml + (int64_t)jl * NC * G * 2;
     if (tid < G) {
         float M = -INFINITY;
         for (int c = 0; c < NC; ++c) M = fmaxf(M, __ldcg(mlg + 2 * (c * G + tid)));
@@ -328,7 +335,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
         Lh[tid] = L;
     }
     __syncthreads();
-    const float* pg = p.part + (int64_t)jl * NC * G * DH;
+    const float* pg = part + (int64_t)jl * NC * G * DH;
     for (int it = tid; it < G * DH / 4; it += AT_THREADS) {
         const int hh = it / (DH / 4), d4 = it - hh * (DH / 4);
         float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -340,9 +347,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             o.z = fmaf(a.z, w, o.z);
             o.w = fmaf(a.w, w, o.w);
         }
-        reinterpret_cast<float4*>(p.o + (int64_t)(jl * G + hh) * DH)[d4] = o;
+        reinterpret_cast<float4*>(o_out + (int64_t)(jl * G + hh) * DH)[d4] = o;
     }
-    if (tid == 0) p.cnt[jl] = 0;
+    if (tid == 0) cnt[jl] = 0;
 }
 
 typedef void (*AttnFn)(const AttnParams);
@@ -411,7 +418,7 @@ int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g) {
 
 int attn_splits_max() { return CLUSTERS_MAX * 16; }
 
-int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, cudaStream_t s) {
+int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s) {
     const int cs = attn_cluster(dh, g);
     AttnFn fn = pick(dh, g, cs);
     if (!fn) return fail(TASP_EUNSUP, "attention kernel not built for this (head_dim, query heads per group)");
@@ -424,7 +431,8 @@ int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, c
     }
     if (splits % cs) return fail(TASP_EINVAL, "attention splits must be a multiple of the cluster size");
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(splits, m_kv);
+    if (nb < 1 || nb > MAX_BATCH) return fail(TASP_EINVAL, "attention batch of 1 to 4 sessions");
+    cfg.gridDim = dim3(splits, m_kv, nb);
     cfg.blockDim = dim3(AT_THREADS);
     cfg.dynamicSmemBytes = smem_of(dh);
     cfg.stream = s;

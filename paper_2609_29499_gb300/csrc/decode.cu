@@ -1,651 +1,43 @@
-// Decode kernels of the compiled sparse path (batch 1 per plan step), sm_103a.
+// Decode step of the compiled sparse path (Sec. 3.3, Fig. 1): the launch sequence of
+// one token for n <= 4 sessions of one plan, sm_103a.
 //
-// Every projection is an HBM-bound GEMV over the retained rows of an INT8 panel with
-// one FP32 scale per output row (the paper's INT8-weight / BF16-compute runtime,
-// Sec. 4 and Table 1). Design:
-//  * persistent grid (SMs x resident CTAs), each CTA owns a contiguous range of row
-//    groups (R rows) and splits K across its 256 threads in 16-byte chunks, so a row
-//    group keeps R x CPT 128-bit streaming loads in flight per thread;
-//  * the next group is loaded into a second register buffer and the one after is
-//    prefetched into L2 with cp.async.bulk.prefetch while the current one is reduced;
-//  * the activation vector sits in shared memory as FP32 with an XOR swizzle that
-//    makes the per-chunk 128-bit reads conflict-free (activations stay FP32 inside a
-//    step; the KV cache, step inputs and LM head are BF16);
-//  * INT8 -> FP32 is exact: byte ^ 0x80 is placed in the mantissa of 2^23 with PRMT and
-//    2^23 + 128 is subtracted (packed f32x2 add), then packed f32x2 FMAs accumulate;
-//    the row scale is applied once after the reduction;
-//  * the previous kernel's tail is overlapped with programmatic dependent launch:
-//    weights (which never depend on the previous kernel) are fetched before
-//    griddepcontrol.wait, activations after it.
-// Attention (attention.cu) is a split-KV kernel over the retained KV heads only.
+// Per layer: K1 RMSNorm + QKV GEMV + RoPE + KV append, K2 GQA attention over the kept
+// KV groups (attention.cu), K3 O GEMV + residual, K4 RMSNorm + gate/up GEMV +
+// SiLU(gate) * up, K5 down GEMV + residual; then the final RMSNorm + dense LM head and the
+// position advance. The GEMVs (gemv.cuh) read every weight byte once for all sessions of
+// the batch; attention runs one grid over all of them, each on its own KV cache and
+// position. Consecutive kernels overlap through programmatic dependent launch, and the
+// runtime replays the whole sequence as one CUDA graph.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cmath>
 #include <map>
 #include <mutex>
+#include <vector>
 
+#include "gemv.cuh"
 #include "tasp_internal.h"
 
 namespace tasp {
 
 namespace {
 
-constexpr int NT = 512;  // consumer threads of a GEMV CTA
-constexpr int NWARP = NT / 32;
-
-enum GemvMode { M_QKV = 0, M_O = 1, M_GU = 2, M_DOWN = 3, M_LM = 4 };
-
-struct GemvParams {
-    const int8_t* w;
-    const int32_t* map;
-    const float* scale;
-    int64_t ld;
-    int rows, K, nchunks;
-    const float* x_resid;
-    const uint16_t* x_in;
-    float* x_resid_init;
-    const float* gamma;
-    float eps;
-    const float* act;
-    float* resid_out;
-    float* hidden_out;
-    float* q_out;
-    uint16_t* k_cache;
-    uint16_t* v_cache;
-    int max_tokens;
-    const float2* rope;
-    const int* pos;
-    int g, dh;
-    float* h_out;
-    float* logits;
-    int* err;       // device error word (bounded waits that gave up)
-    int smem_cap;   // dynamic shared memory available to the launch
-};
-
-
-
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-
-
-
-typedef unsigned long long u64;
-
-__device__ __forceinline__ u64 pk(float a, float b) {
-    u64 r;
-    asm("mov.b64 %0, {%1,%2};" : "=l"(r) : "f"(a), "f"(b));
-    return r;
-}
-__device__ __forceinline__ float2 upk(u64 v) {
-    float2 r;
-    asm("mov.b64 {%0,%1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
-    return r;
-}
-__device__ __forceinline__ u64 fma2(u64 a, u64 b, u64 c) {
-    u64 d;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-    return d;
-}
-
-// float4 index swizzle: F = float4s per 16-byte weight chunk (4 for INT8, 2 for BF16)
-template <int F>
-__device__ __forceinline__ int swz(int f) {
-    return f ^ ((f >> 3) & (F - 1));
-}
-
-__device__ __forceinline__ uint16_t f32_to_bf16_bits(float v) {
-    __nv_bfloat16 b = __float2bfloat16_rn(v);
-    return *reinterpret_cast<uint16_t*>(&b);
-}
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-
-constexpr int CW = NWARP;                // consumer warps
-constexpr int CT = CW * 32;              // consumer threads
-constexpr int GEMV_THREADS = CT + 64;    // + producer warp + epilogue warp
-constexpr int MAX_STAGES = 8;
-constexpr int NRB = 8;                   // partial-sum buffers between consumers and the epilogue warp
-constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s) before a wait gives up
-constexpr int ERR_WAIT_TIMEOUT = 1;
-
-__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(CT) : "memory"); }
-
-// ---------------------------------------------------------------- activation prologues
-// x^ = x * (1/sqrt(mean(x^2) + eps)) * gamma (FP32) into swizzled shared memory.
-// Every CTA reduces in the same fixed order, so all CTAs see identical x^.
-template <int F>
-__device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __restrict__ x_in, float* x_init,
-                             const float* __restrict__ gamma, int d, float eps, int nchunks, float4* xs,
-                             float* stat) {
-    const int tid = threadIdx.x;
-    const int n4 = d / 4;
-    float ss = 0.f;
-    for (int f = tid; f < n4; f += NT) {
-        float4 v;
-        if (x_in) {
-            uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
-            v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
-                            __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
-            if (x_init && blockIdx.x == 0) reinterpret_cast<float4*>(x_init)[f] = v;
-        } else {
-            v = reinterpret_cast<const float4*>(x)[f];
-        }
-        ss = fmaf(v.x, v.x, ss);
-        ss = fmaf(v.y, v.y, ss);
-        ss = fmaf(v.z, v.z, ss);
-        ss = fmaf(v.w, v.w, ss);
-    }
-    ss = warp_sum(ss);
-    if ((tid & 31) == 0) stat[tid >> 5] = ss;
-    consumer_sync();
-    float tot = 0.f;
-#pragma unroll
-    for (int w = 0; w < NWARP; ++w) tot += stat[w];
-    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)d) + eps);
-    const int ntot4 = nchunks * F;  // float4 slots including zero padding
-    for (int f = tid; f < ntot4; f += NT) {
-        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (f < n4) {
-            float4 v;
-            if (x_in) {
-                uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
-                v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
-                                __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
-            } else {
-                v = reinterpret_cast<const float4*>(x)[f];
-            }
-            float4 gm = reinterpret_cast<const float4*>(gamma)[f];
-            o.x = (v.x * inv) * gm.x;
-            o.y = (v.y * inv) * gm.y;
-            o.z = (v.z * inv) * gm.z;
-            o.w = (v.w * inv) * gm.w;
-        }
-        xs[swz<F>(f)] = o;
-    }
-    consumer_sync();
-}
-
-// FP32 activation vector [K] -> swizzled shared memory (zero padded to nchunks*16)
-__device__ void f32_to_smem(const float* __restrict__ a, int K, int nchunks, float4* xs) {
-    const int tid = threadIdx.x;
-    const int ntot4 = nchunks * 4;
-    for (int f = tid; f < ntot4; f += NT) {
-        float4 o;
-        const int e = 4 * f;
-        if (e + 3 < K) {
-            o = *reinterpret_cast<const float4*>(a + e);
-        } else {
-            o.x = (e + 0 < K) ? a[e + 0] : 0.f;
-            o.y = (e + 1 < K) ? a[e + 1] : 0.f;
-            o.z = (e + 2 < K) ? a[e + 2] : 0.f;
-            o.w = (e + 3 < K) ? a[e + 3] : 0.f;
-        }
-        xs[swz<4>(f)] = o;
-    }
-    consumer_sync();
-}
-
-// ---------------------------------------------------------------- row addressing
-// QKV work rows are ordered so that each even/odd pair holds rows i and i + dh/2 of
-// one head (a rotary pair); all other modes use the panel order.
-template <int MODE>
-__device__ __forceinline__ int panel_row(const GemvParams& p, int w) {
-    if (MODE == M_QKV) {
-        int hb = w / p.dh, iw = w - hb * p.dh;
-        return hb * p.dh + (iw >> 1) + (iw & 1) * (p.dh >> 1);
-    }
-    return w;
-}
-
-template <int MODE>
-__device__ __forceinline__ const int8_t* row_ptr(const GemvParams& p, int w) {
-    if (w >= p.rows) w = 0;  // padding row of a ragged last group: loaded, never stored
-    int pr = panel_row<MODE>(p, w);
-    int src = p.map ? __ldg(p.map + pr) : pr;
-    return p.w + (int64_t)src * p.ld;
-}
-
-// ---------------------------------------------------------------- the GEMV core
-// One persistent CTA per SM: warp CW is the producer, warps 0..CW-1 consume.
-// The producer streams row groups (R rows, one bulk copy per row) into an NS-stage
-// shared-memory ring; stage s has a "full" mbarrier (transaction bytes) and an
-// "empty" mbarrier (released by the consumers after their last read of the stage).
-__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Bounded wait: gives up after WAIT_LIMIT cycles, records the failure in the device
-// error word and makes every later wait of this CTA return at once (abort), so a lost
-// transfer can never hang the GPU; the host reports the error word.
-__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
-                                          bool honor_abort = true) {
-    if (honor_abort && *(volatile int*)abort_flag) return;
-    if (mbar_try(bar, parity)) return;
-    const long long t0 = clock64();
-    while (!mbar_try(bar, parity)) {
-        if (clock64() - t0 > WAIT_LIMIT) {
-            *(volatile int*)abort_flag = 1;
-            if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
-            return;
-        }
-    }
-}
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
-
-// This thread's slice of the activation vector, kept in registers for the whole
-// kernel: chunk j of the thread is c = tid + j * CT (16 weight bytes per chunk).
-template <int XC, int F>
-struct XRegs {
-    float4 v[XC][F];
-};
-
-template <int XC, int F>
-__device__ __forceinline__ void load_x(XRegs<XC, F>& xr, const float4* xs, int nchunks, int tid) {
-#pragma unroll
-    for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-#pragma unroll
-        for (int e = 0; e < F; ++e)
-            xr.v[j][e] = c < nchunks ? xs[swz<F>(F * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-}
-
-// The activation slice of an INT8 GEMV as block-scaled integers: per 16-element chunk
-// one power-of-two scale 2^(e-14) with max|x| < 2^e, each element rounded to the integer
-// X in [-2^14, 2^14] and split as X = 256 hi + lo (hi signed byte, lo unsigned byte),
-// four elements packed per 32-bit word. The INT8 weight words then feed dp4a directly.
-template <int XC>
-struct XDigits {
-    uint32_t hi[XC][4], lo[XC][4];
-    float scale[XC];
-};
-
-template <int XC>
-__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const float4* xs, int nchunks, int tid) {
-#pragma unroll
-    for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-        float v[16];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float4 q = c < nchunks ? xs[swz<4>(4 * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
-            v[4 * e + 0] = q.x;
-            v[4 * e + 1] = q.y;
-            v[4 * e + 2] = q.z;
-            v[4 * e + 3] = q.w;
-        }
-        float m = 0.f;
-#pragma unroll
-        for (int e = 0; e < 16; ++e) m = fmaxf(m, fabsf(v[e]));
-        int ex = 0;
-        if (m > 0.f) frexpf(m, &ex);  // m = f * 2^ex, f in [0.5, 1): every |x| < 2^ex
-        xd.scale[j] = m > 0.f ? ldexpf(1.0f, ex - 14) : 0.f;
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-            uint32_t h = 0, l = 0;
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-                const int X = m > 0.f ? __float2int_rn(ldexpf(v[4 * w + b], 14 - ex)) : 0;
-                h |= ((uint32_t)(X >> 8) & 0xFFu) << (8 * b);
-                l |= ((uint32_t)X & 0xFFu) << (8 * b);
-            }
-            xd.hi[j][w] = h;
-            xd.lo[j][w] = l;
-        }
-    }
-}
-
-__device__ __forceinline__ int dp4a_ss(uint32_t a, uint32_t b, int c) {
-    int d;
-    asm("dp4a.s32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
-    return d;
-}
-__device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
-    int d;
-    asm("dp4a.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
-    return d;
-}
-
-// INT8 rows of one stage . x: per chunk sum(w * X) = 256 sum(w * hi) + sum(w * lo) in
-// exact INT32, then acc[r] += float(sum) * scale in FP32.
-template <int R, int XC>
-__device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC>& xd,
-                                       int nchunks, int tid, float (&acc)[R]) {
-#pragma unroll
-    for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-        if (c < nchunks) {
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
-                const uint32_t wd[4] = {(uint32_t)wv.x, (uint32_t)wv.y, (uint32_t)wv.z, (uint32_t)wv.w};
-                int sh = 0, sl = 0;
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    sh = dp4a_ss(wd[k], xd.hi[j][k], sh);
-                    sl = dp4a_su(wd[k], xd.lo[j][k], sl);
-                }
-                acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xd.scale[j], acc[r]);
-            }
-        }
-    }
-}
-
-// BF16 rows (LM head): 8 weights per 16-byte chunk
-template <int R, int XC>
-__device__ __forceinline__ void dot_bf16(const uint8_t* __restrict__ stage, int ld, const XRegs<XC, 2>& xr,
-                                         int nchunks, int tid, u64 (&acc)[R]) {
-#pragma unroll
-    for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-        if (c < nchunks) {
-            const float4 x0 = xr.v[j][0], x1 = xr.v[j][1];
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
-                const uint32_t w0 = wv.x, w1 = wv.y, w2 = wv.z, w3 = wv.w;
-                acc[r] = fma2(pk(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xffff0000u)), pk(x0.x, x0.y), acc[r]);
-                acc[r] = fma2(pk(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xffff0000u)), pk(x0.z, x0.w), acc[r]);
-                acc[r] = fma2(pk(__uint_as_float(w2 << 16), __uint_as_float(w2 & 0xffff0000u)), pk(x1.x, x1.y), acc[r]);
-                acc[r] = fma2(pk(__uint_as_float(w3 << 16), __uint_as_float(w3 & 0xffff0000u)), pk(x1.z, x1.w), acc[r]);
-            }
-        }
-    }
-}
-
-// Warp reduction of R row sums at once: each butterfly level halves the vector a lane
-// carries, so lane l ends with the full sum of row l / (32 / R).
-template <int R>
-__device__ __forceinline__ float row_reduce(float (&v)[R], int lane) {
-#pragma unroll
-    for (int n = R, o = 16; n > 1; n >>= 1, o >>= 1) {
-        const bool up = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < n / 2; ++i) {
-            const float send = up ? v[i] : v[i + n / 2];
-            const float keep = up ? v[i + n / 2] : v[i];
-            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-    float s = v[0];
-#pragma unroll
-    for (int o = 16 / R; o >= 1; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    return s;
-}
-
-// Per-CTA values the epilogue warp stages in shared memory: row scales (constant, read
-// before the dependency wait), residual rows (after it) and this position's rotary pairs.
-constexpr int EPI_MAXR = 512;
-struct EpiStage {
-    float sc[EPI_MAXR];
-    float res[EPI_MAXR];
-    float2 rope[64];
-    int w_lo, pos;
-    bool ok;  // the CTA's rows fit the staging arrays
-};
-
-// Epilogue of one row group, run by the epilogue warp: lanes split the CW partial sums
-// of each row, then lanes < R (or < R/2 for rotary / SwiGLU pairs) finish the rows.
-template <int MODE, int R>
-__device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)[R], int gi, int lane,
-                                         const EpiStage& es) {
-    constexpr int LPR = 32 / R;  // lanes per row
-    const int r = lane % R;
-    float s = 0.f;
-#pragma unroll
-    for (int w = lane / R; w < CW; w += LPR) s += red[w][r];
-#pragma unroll
-    for (int o = R; o < 32; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    // lane r (< R) now holds the full sum of row r of the group
-    const int w0 = gi * R;
-    if (MODE == M_QKV || MODE == M_GU) {
-        const float s_other = __shfl_down_sync(0xffffffffu, s, 1);  // row 2t+1 for lane 2t
-        if ((lane & 1) == 0 && lane < R) {
-            const float s0 = s, s1 = s_other;
-            const int wa = w0 + lane;
-            if (wa < p.rows) {
-                const float sc0 = es.ok ? es.sc[wa - es.w_lo] : p.scale[panel_row<MODE>(p, wa)];
-                const float sc1 = es.ok ? es.sc[wa + 1 - es.w_lo] : p.scale[panel_row<MODE>(p, wa + 1)];
-                if (MODE == M_GU) {
-                    const float a = sc0 * s0, b = sc1 * s1;
-                    const float silu = a / (1.0f + expf(-a));
-                    p.h_out[wa >> 1] = silu * b;
-                } else {
-                    const int half = p.dh >> 1;
-                    const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
-                    float y0 = sc0 * s0, y1 = sc1 * s1;
-                    const int gp2 = p.g + 2;
-                    const int jl = hb / gp2, hh = hb - jl * gp2;
-                    const int pos = es.pos;
-                    if (hh <= p.g) {
-                        const float2 cs = es.rope[i];
-                        const float ya = y0 * cs.x - y1 * cs.y, yb = y1 * cs.x + y0 * cs.y;
-                        y0 = ya;
-                        y1 = yb;
-                    }
-                    if (hh < p.g) {
-                        float* dq = p.q_out + (int64_t)(jl * p.g + hh) * p.dh;
-                        dq[i] = y0;
-                        dq[i + half] = y1;
-                    } else {
-                        uint16_t* dst = (hh == p.g ? p.k_cache : p.v_cache) + ((int64_t)jl * p.max_tokens + pos) * p.dh;
-                        dst[i] = f32_to_bf16_bits(y0);  // the KV cache is BF16
-                        dst[i + half] = f32_to_bf16_bits(y1);
-                    }
-                }
-            }
-        }
-    } else if (lane < R) {
-        const int row = w0 + lane;
-        if (row < p.rows) {
-            if (MODE == M_LM) {
-                p.logits[row] = s;
-            } else {
-                const float base = es.ok ? es.res[row - es.w_lo] : p.resid_out[row];
-                const float v = base + (es.ok ? es.sc[row - es.w_lo] : p.scale[row]) * s;
-                p.resid_out[row] = v;
-                if (p.hidden_out) p.hidden_out[row] = v;
-            }
-        }
-    }
-}
-
-// Shared-memory plan of one launch (host and device agree on it).
-struct GemvSmem {
-    int x_bytes, stage_bytes, nstages, total;
-};
-__host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap) {
-    GemvSmem g;
-    g.x_bytes = ((nchunks * F * 16) + 127) & ~127;
-    g.stage_bytes = ((R * ld) + 127) & ~127;
-    const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
-    int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
-    g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
-    g.total = g.x_bytes + g.nstages * g.stage_bytes + bar_bytes;
-    return g;
-}
-
-template <int MODE, int R, int XC>
-__global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams p) {
-    extern __shared__ __align__(128) uint8_t sm[];
-    __shared__ float red[NRB][CW][R];
-    __shared__ float stat[CW];
-    __shared__ int abort_flag;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
-    const int NS = L.nstages;
-    float4* xs = reinterpret_cast<float4*>(sm);
-    uint8_t* stages = sm + L.x_bytes;
-    const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
-    const uint32_t empty0 = full0 + 8 * MAX_STAGES;
-    const uint32_t rfull0 = empty0 + 8 * MAX_STAGES;
-    const uint32_t rempty0 = rfull0 + 8 * NRB;
-    const int NG = (p.rows + R - 1) / R;
-    const int g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
-    const int g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
-
-    if (tid == 0) {
-        abort_flag = 0;
-        for (int s = 0; s < NS; ++s) {
-            mbar_init(full0 + 8 * s, 1);
-            mbar_init(empty0 + 8 * s, CW);
-        }
-        for (int b = 0; b < NRB; ++b) {
-            mbar_init(rfull0 + 8 * b, CW);
-            mbar_init(rempty0 + 8 * b, 1);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-
-    if (warp == CW) {
-        // ---- producer: weights never depend on the previous kernel, so start at once
-        pdl_trigger();
-        if (lane == 0) {
-            int s = 0;
-            uint32_t ph = 0;
-            for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-                if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err);
-                const int nrow = min(R, p.rows - gi * R);
-                mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
-                for (int r = 0; r < nrow; ++r)
-                    bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)r * p.ld),
-                             row_ptr<MODE>(p, gi * R + r), (uint32_t)p.ld, full0 + 8 * s);
-                if (++s == NS) {
-                    s = 0;
-                    ph ^= 1;
-                }
-            }
-            // never leave while copies into this CTA's shared memory are in flight (even
-            // after an abort: this second wait is bounded on its own)
-            for (int gi = max(g0, g1 - NS), i = gi - g0; gi < g1; ++gi, ++i)
-                mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, false);
-        }
-        return;
-    }
-    if (warp == CW + 1) {
-        // ---- epilogue warp: cross-warp sums of each row group, then the mode's epilogue
-        __shared__ EpiStage es;
-        const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
-        if (lane == 0) {
-            es.w_lo = w_lo;
-            es.ok = (w_hi - w_lo) <= EPI_MAXR;
-        }
-        __syncwarp();
-        if (MODE != M_LM && es.ok)  // scales are constant: stage them before the dependency wait
-            for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
-        pdl_wait();
-        pdl_trigger();
-        if ((MODE == M_O || MODE == M_DOWN) && es.ok)
-            for (int w = w_lo + lane; w < w_hi; w += 32) es.res[w - w_lo] = p.resid_out[w];
-        if (MODE == M_QKV) {
-            const int pos = *p.pos;
-            if (lane == 0) es.pos = pos;
-            for (int i = lane; i < (p.dh >> 1); i += 32) es.rope[i] = p.rope[(int64_t)pos * (p.dh >> 1) + i];
-        }
-        __syncwarp();
-        int b = 0;
-        uint32_t ph = 0;
-        for (int gi = g0; gi < g1; ++gi) {
-            mbar_wait(rfull0 + 8 * b, ph, &abort_flag, p.err);
-            epilogue<MODE, R>(p, red[b], gi, lane, es);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(rempty0 + 8 * b);
-            if (++b == NRB) {
-                b = 0;
-                ph ^= 1;
-            }
-        }
-        return;
-    }
-
-    // ---- consumers
-    pdl_wait();
-    pdl_trigger();
-    if (MODE == M_QKV || MODE == M_GU)
-        norm_to_smem<4>(p.x_resid, p.x_in, p.x_resid_init, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
-    else if (MODE == M_LM)
-        norm_to_smem<2>(p.x_resid, nullptr, nullptr, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
-    else
-        f32_to_smem(p.act, p.K, p.nchunks, xs);
-
-    XRegs<XC, 2> xr;        // LM head: FP32 activation slice
-    XDigits<XC> xd;         // INT8 modes: block-scaled integer digits of the slice
-    if constexpr (MODE == M_LM)
-        load_x<XC, 2>(xr, xs, p.nchunks, tid);
-    else
-        digits_x<XC>(xd, xs, p.nchunks, tid);
-    int s = 0, b = 0;
-    uint32_t sph = 0, bph = 0;
-    for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-        mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err);
-        const uint8_t* st = stages + (size_t)s * L.stage_bytes;
-        float v[R];
-        if constexpr (MODE == M_LM) {
-            u64 acc[R];
-#pragma unroll
-            for (int r = 0; r < R; ++r) acc[r] = 0ull;
-            dot_bf16<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-                const float2 a = upk(acc[r]);
-                v[r] = a.x + a.y;
-            }
-        } else {
-#pragma unroll
-            for (int r = 0; r < R; ++r) v[r] = 0.f;
-            dot_i8<R, XC>(st, (int)p.ld, xd, p.nchunks, tid, v);
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
-        const float rs = row_reduce<R>(v, lane);
-        if (i >= NRB) mbar_wait(rempty0 + 8 * b, bph ^ 1, &abort_flag, p.err);
-        if ((lane & (32 / R - 1)) == 0) red[b][warp][lane / (32 / R)] = rs;
-        __syncwarp();
-        if (lane == 0) mbar_arrive(rfull0 + 8 * b);
-        if (++s == NS) {
-            s = 0;
-            sph ^= 1;
-        }
-        if (++b == NRB) {
-            b = 0;
-            bph ^= 1;
-        }
-    }
-}
+using namespace gemv;
 
 __global__ void set_pos_kernel(int* pos, int v) {
     if (threadIdx.x == 0) *pos = v;
 }
 
-__global__ void advance_kernel(int* pos) {
+struct AdvanceArgs {
+    int* pos[MAX_BATCH];
+    int n;
+};
+
+__global__ void advance_kernel(AdvanceArgs a) {
     pdl_wait();
     pdl_trigger();
-    if (threadIdx.x == 0) *pos += 1;
+    if (threadIdx.x < a.n) *a.pos[threadIdx.x] += 1;
 }
 
 // ---------------------------------------------------------------- host side
@@ -665,64 +57,58 @@ int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const
     return TASP_OK;
 }
 
-typedef void (*GemvFn)(const GemvParams);
-
-template <int MODE>
-GemvFn gemv_fn(int R, int XC) {
-    if (XC <= 1) {
-        if (R >= 8) return gemv_kernel<MODE, 8, 1>;
-        if (R >= 4) return gemv_kernel<MODE, 4, 1>;
-        return gemv_kernel<MODE, 2, 1>;
-    }
-    if (XC <= 2) {
-        if (R >= 4) return gemv_kernel<MODE, 4, 2>;
-        return gemv_kernel<MODE, 2, 2>;
-    }
-    if (XC <= 4) {
-        if (R >= 2) return gemv_kernel<MODE, 2, 4>;
-        if constexpr (MODE == M_QKV || MODE == M_GU)
-            return nullptr;  // rotary / SwiGLU pairs need two rows per stage
-        else
-            return gemv_kernel<MODE, 1, 4>;
-    }
-    return nullptr;
-}
-
-GemvFn pick(int mode, int R, int XC) {
-    switch (mode) {
-        case M_QKV: return gemv_fn<M_QKV>(R, XC);
-        case M_O: return gemv_fn<M_O>(R, XC);
-        case M_GU: return gemv_fn<M_GU>(R, XC);
-        case M_DOWN: return gemv_fn<M_DOWN>(R, XC);
-        default: return gemv_fn<M_LM>(R, XC);
+Fn pick_any(int nbk, int mode, int R, int XC) {
+    switch (nbk) {
+        case 1: return pick<1>(mode, R, XC);
+        case 2: return pick<2>(mode, R, XC);
+        default: return pick<4>(mode, R, XC);
     }
 }
 
-// Rows per stage: the largest power of two with R * row_bytes <= 32 KB (pairs need R >= 2).
-int rows_per_stage(int mode, int64_t ld) {
+// Kernel shape for a launch: NB (vectors per weight pass), XC (register chunks per
+// thread, NB * XC <= 4), the K pass length and R (rows per stage, <= 32 KB per stage,
+// pairs for the rotary / SwiGLU modes).
+struct Variant {
+    int nbk, XC, R, seg, passes;
+};
+
+Variant variant(int mode, int nb, int nchunks, int max_r) {
+    Variant v;
+    v.nbk = nb <= 1 ? 1 : (nb <= 2 ? 2 : 4);
+    const int xc_max = 4 / v.nbk;
+    v.XC = 1;
+    while (v.XC < xc_max && v.XC * CT < nchunks) v.XC <<= 1;
+    v.seg = std::min(nchunks, v.XC * CT);
+    v.passes = (nchunks + v.seg - 1) / v.seg;
     int R = 8;
-    while (R > 1 && (int64_t)R * ld > 32768) R >>= 1;
+    while (R > 1 && R * v.seg * 16 > 32768) R >>= 1;
     if ((mode == M_QKV || mode == M_GU) && R < 2) R = 2;
-    return R;
+    R = std::min(R, max_r);
+    if (v.XC == 2) R = std::min(R, 4);
+    if (v.XC == 4) R = std::min(R, 2);
+    if (v.nbk == 4) R = std::min(R, 4);
+    v.R = R;
+    return v;
 }
 
 std::mutex g_attr_mu;
 std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 
-int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
-    if (p.rows == 0) return TASP_OK;
+int launch_gemv(int mode, Params p, cudaStream_t s) {
+    if (p.rows == 0 || p.nb == 0) return TASP_OK;
+    if (p.nb > MAXNB) return fail(TASP_EINVAL, "more activation vectors than one GEMV pass takes");
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
-    int R = rows_per_stage(mode, p.ld);
-    int XC = 1;
-    while (XC * CT < p.nchunks) XC <<= 1;
-    if (XC > 4) return fail(TASP_EUNSUP, "row too long for the register-resident activation slice");
-    if (XC == 2 && R > 4) R = 4;
-    if (XC == 4 && R > 2) R = 2;
-    GemvFn fn = pick(mode, R, XC);
+    const Variant v = variant(mode, p.nb, p.nchunks, 8);
+    if (p.nx_w && (p.nx_bytes <= 0 || p.nx_bytes % 16 || p.nx_ld % 16 || p.nx_R < 1 || p.nx_grid < 1))
+        p.nx_w = nullptr;  // malformed prefetch description: skip the hint
+    if ((mode == M_QKV || mode == M_GU) && v.passes > 1)
+        return fail(TASP_EUNSUP, "hidden size too large for the register-resident activation slices of this batch");
+    Fn fn = pick_any(v.nbk, mode, v.R, v.XC);
     if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
-    p.err = err;
+    p.seg = v.seg;
+    p.passes = v.passes;
     {
         std::lock_guard<std::mutex> lk(g_attr_mu);
         auto it = g_attr.find((const void*)fn);
@@ -735,32 +121,121 @@ int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
         }
         p.smem_cap = it->second;
     }
-    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
-    if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
-    const int NG = (p.rows + R - 1) / R;
+    const Smem L = smem_plan(v.R, v.seg * 16, p.smem_cap);
+    if (L.nstages < 2) return fail(TASP_EUNSUP, "row too long for the shared-memory ring");
+    const int NG = (p.rows + v.R - 1) / v.R;
     const int grid = std::max(1, std::min(NG, di.sms));
-    return launch_pdl(fn, dim3(grid), dim3(GEMV_THREADS), (size_t)L.total, s, p);
+    return launch_pdl(fn, dim3(grid), dim3(THREADS), (size_t)L.total, s, p);
+}
+
+Params lm_params(const BatchView& bv, float* logits, int64_t logit_stride) {
+    const Plan& pl = *bv.ss[0]->plan;
+    const Shape& sh = pl.store->sh;
+    Params lm{};
+    lm.w = reinterpret_cast<const int8_t*>(pl.store->lm_head);
+    lm.ld = (int64_t)sh.d * 2;
+    lm.rows = sh.vocab;
+    lm.K = sh.d;
+    lm.nchunks = sh.d / 8;
+    lm.nb = bv.n;
+    lm.x_resid = bv.x;
+    lm.x_stride = bv.x_stride;
+    lm.gamma = pl.store->g_final;
+    lm.eps = sh.eps;
+    lm.logits = logits;
+    lm.logit_stride = logit_stride;
+    lm.err = bv.err;
+    return lm;
+}
+
+// One launch of a decode step.
+struct Op {
+    enum Type { GEMV, ATTN, COPY_HIDDEN, ADVANCE } type;
+    int kind;  // KernelKind reported to the profiling hook
+    int mode = 0;
+    Params p{};
+    AttnParams a{};
+    int m_kv = 0, S = 0;
+};
+
+// Point every GEMV at the next GEMV of the sequence for the L2 prefetch of its first
+// rows (the last one, the LM head or the final down projection, at the first QKV: the
+// next step replays the same sequence).
+void link_prefetch(std::vector<Op>& ops, int sms, bool wrap) {
+    std::vector<int> g;
+    for (int i = 0; i < (int)ops.size(); ++i)
+        if (ops[i].type == Op::GEMV && ops[i].p.rows > 0) g.push_back(i);
+    for (size_t k = 0; k < g.size(); ++k) {
+        if (k + 1 == g.size() && !wrap) break;
+        const Op& nx = ops[g[(k + 1) % g.size()]];
+        const Variant v = variant(nx.mode, nx.p.nb, nx.p.nchunks, 8);
+        Params& p = ops[g[k]].p;
+        p.nx_w = nx.p.w;
+        p.nx_map = nx.p.map;
+        p.nx_ld = nx.p.ld;
+        p.nx_rows = nx.p.rows;
+        p.nx_R = v.R;
+        p.nx_grid = std::max(1, std::min((nx.p.rows + v.R - 1) / v.R, sms));
+        p.nx_bytes = v.seg * 16;
+    }
 }
 
 }  // namespace
 
-int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
-                 int* launches) {
-    const Plan& pl = *se.plan;
+BatchView single_view(Session& se) {
+    const Shape& sh = se.plan->store->sh;
+    BatchView bv;
+    bv.n = 1;
+    bv.ss[0] = &se;
+    bv.x = se.x;
+    bv.q = se.q;
+    bv.o = se.o;
+    bv.h = se.h;
+    bv.x_stride = sh.d;
+    bv.q_stride = (int64_t)sh.Hq * sh.dh;
+    bv.h_stride = sh.df;
+    bv.part = se.part;
+    bv.ml = se.ml;
+    bv.cnt = se.cnt;
+    bv.err = se.err;
+    return bv;
+}
+
+int batch_attn_slots(const Plan& p, const Session* const* ss, int n, int sms) {
+    const Shape& sh = p.store->sh;
+    int smax = 1;
+    for (int b = 0; b < n; ++b)
+        for (const LayerPlan& lp : p.layers)
+            smax = std::max(smax, attn_splits(lp.m_kv, ss[b]->max_tokens, sms, sh.dh, sh.g()) /
+                                      attn_cluster(sh.dh, sh.g()));
+    return smax;
+}
+
+int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook,
+                  void* ctx, int* launches) {
+    if (bv.n < 1 || bv.n > MAX_BATCH) return fail(TASP_EINVAL, "a batch holds 1 to 4 sessions");
+    const Plan& pl = *bv.ss[0]->plan;
     const Shape& sh = pl.store->sh;
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
-    int nl = 0;
+    const int n = bv.n;
+    std::vector<Op> ops;
     const int l_begin = only_layer >= 0 ? only_layer : 0;
     const int l_end = only_layer >= 0 ? only_layer + 1 : sh.L;
-    auto pre = [&](int kind) { if (hook) hook(ctx, kind, true); };
-    auto post = [&](int kind) { if (hook) hook(ctx, kind, false); ++nl; };
+    auto gemv = [&](int kind, int mode, const Params& p) {
+        Op op;
+        op.type = Op::GEMV;
+        op.kind = kind;
+        op.mode = mode;
+        op.p = p;
+        ops.push_back(op);
+    };
     for (int l = l_begin; l < l_end; ++l) {
         const LayerPlan& lp = pl.layers[l];
         const bool first = (l == 0) && t.x_in != nullptr;
         // K1: RMSNorm + QKV GEMV + RoPE + KV append
-        GemvParams p{};
+        Params p{};
         p.w = lp.qkv_w;
         p.map = lp.qkv_map;
         p.scale = lp.qkv_s;
@@ -768,59 +243,79 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
         p.rows = lp.qkv_rows;
         p.K = sh.d;
         p.nchunks = sh.d / 16;
-        p.x_resid = se.x;
+        p.nb = n;
+        p.x_resid = bv.x;
+        p.x_stride = bv.x_stride;
         p.x_in = first ? t.x_in : nullptr;
-        p.x_resid_init = first ? se.x : nullptr;
+        p.xin_stride = sh.d;
+        p.x_resid_init = first ? bv.x : nullptr;
         p.gamma = lp.g_attn;
         p.eps = sh.eps;
-        p.q_out = se.q;
-        p.k_cache = se.K[l];
-        p.v_cache = se.V[l];
-        p.max_tokens = se.max_tokens;
-        p.rope = se.rope;
-        p.pos = se.d_pos;
+        p.q_out = bv.q;
+        p.q_stride = bv.q_stride;
+        for (int b = 0; b < n; ++b) {
+            const Session& se = *bv.ss[b];
+            p.k_cache[b] = se.K[l];
+            p.v_cache[b] = se.V[l];
+            p.max_tokens[b] = se.max_tokens;
+            p.rope[b] = se.rope;
+            p.pos[b] = se.d_pos;
+        }
         p.g = sh.g();
         p.dh = sh.dh;
-        pre(K_QKV);
-        if ((rc = launch_gemv(M_QKV, p, se.err, s))) return rc;
-        post(K_QKV);
-        // K2: split-KV attention over the retained KV heads
+        p.err = bv.err;
+        gemv(K_QKV, M_QKV, p);
+        // K2: split-KV attention over the retained KV heads of every session
         if (lp.m_kv > 0) {
             AttnParams a{};
-            a.q = se.q;
-            a.K = se.K[l];
-            a.V = se.V[l];
-            a.pos = se.d_pos;
-            a.max_tokens = se.max_tokens;
+            a.q = bv.q;
+            a.o = bv.o;
+            a.q_stride = bv.q_stride;
+            int S = 0;
+            for (int b = 0; b < n; ++b) {
+                const Session& se = *bv.ss[b];
+                a.K[b] = se.K[l];
+                a.V[b] = se.V[l];
+                a.pos[b] = se.d_pos;
+                a.max_tokens[b] = se.max_tokens;
+                S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
+            }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
-            a.part = t.att_part ? t.att_part : se.part;
-            a.ml = t.att_ml ? t.att_ml : se.ml;
-            a.cnt = t.att_cnt ? t.att_cnt : se.cnt;
-            a.o = se.o;
-            const int S = attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g());
-            pre(K_ATTN);
-            if ((rc = launch_attention(a, sh.dh, sh.g(), lp.m_kv, S, s))) return rc;
-            post(K_ATTN);
+            a.part = t.att_part ? t.att_part : bv.part;
+            a.ml = t.att_ml ? t.att_ml : bv.ml;
+            a.cnt = t.att_cnt ? t.att_cnt : bv.cnt;
+            a.part_stride = bv.part_stride;
+            a.ml_stride = bv.ml_stride;
+            a.cnt_stride = bv.cnt_stride;
+            Op op;
+            op.type = Op::ATTN;
+            op.kind = K_ATTN;
+            op.a = a;
+            op.m_kv = lp.m_kv;
+            op.S = S;
+            ops.push_back(op);
         }
         // K3: O-projection + residual
         if (lp.m_kv > 0) {
-            GemvParams o{};
+            Params o{};
             o.w = lp.o_w;
             o.scale = lp.o_s;
             o.ld = lp.o_ld;
             o.rows = sh.d;
             o.K = lp.o_K;
             o.nchunks = lp.o_ld / 16;
-            o.act = se.o;
-            o.resid_out = se.x;
-            pre(K_O);
-            if ((rc = launch_gemv(M_O, o, se.err, s))) return rc;
-            post(K_O);
+            o.nb = n;
+            o.act = bv.o;
+            o.act_stride = bv.q_stride;
+            o.resid_out = bv.x;
+            o.x_stride = bv.x_stride;
+            o.err = bv.err;
+            gemv(K_O, M_O, o);
         }
         // K4: RMSNorm + gate/up GEMV + SiLU(gate) * up
         const bool last = (l == sh.L - 1) && only_layer < 0;
         if (lp.c > 0) {
-            GemvParams gu{};
+            Params gu{};
             gu.w = lp.gu_w;
             gu.map = lp.gu_map;
             gu.scale = lp.gu_s;
@@ -828,71 +323,91 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
             gu.rows = lp.gu_rows;
             gu.K = sh.d;
             gu.nchunks = sh.d / 16;
-            gu.x_resid = se.x;
+            gu.nb = n;
+            gu.x_resid = bv.x;
+            gu.x_stride = bv.x_stride;
             gu.gamma = lp.g_mlp;
             gu.eps = sh.eps;
-            gu.h_out = se.h;
-            pre(K_GU);
-            if ((rc = launch_gemv(M_GU, gu, se.err, s))) return rc;
-            post(K_GU);
+            gu.h_out = bv.h;
+            gu.h_stride = bv.h_stride;
+            gu.err = bv.err;
+            gemv(K_GU, M_GU, gu);
             // K5: down projection + residual
-            GemvParams dn{};
+            Params dn{};
             dn.w = lp.dn_w;
             dn.scale = lp.dn_s;
             dn.ld = lp.dn_ld;
             dn.rows = sh.d;
             dn.K = lp.dn_K;
             dn.nchunks = lp.dn_ld / 16;
-            dn.act = se.h;
-            dn.resid_out = se.x;
+            dn.nb = n;
+            dn.act = bv.h;
+            dn.act_stride = bv.h_stride;
+            dn.resid_out = bv.x;
+            dn.x_stride = bv.x_stride;
             dn.hidden_out = last ? t.hidden_out : nullptr;
-            pre(K_DOWN);
-            if ((rc = launch_gemv(M_DOWN, dn, se.err, s))) return rc;
-            post(K_DOWN);
+            dn.hid_stride = sh.d;
+            dn.err = bv.err;
+            gemv(K_DOWN, M_DOWN, dn);
         } else if (last && t.hidden_out) {
-            TASP_CUDA(cudaMemcpyAsync(t.hidden_out, se.x, sizeof(float) * sh.d, cudaMemcpyDeviceToDevice, s));
+            Op op;
+            op.type = Op::COPY_HIDDEN;
+            op.kind = K_OTHER;
+            ops.push_back(op);
         }
     }
     if (only_layer < 0) {
-        if (t.logits) {
-            GemvParams lm{};
-            lm.w = reinterpret_cast<const int8_t*>(pl.store->lm_head);
-            lm.ld = (int64_t)sh.d * 2;
-            lm.rows = sh.vocab;
-            lm.K = sh.d;
-            lm.nchunks = sh.d / 8;
-            lm.x_resid = se.x;
-            lm.gamma = pl.store->g_final;
-            lm.eps = sh.eps;
-            lm.logits = t.logits;
-            pre(K_LM);
-            if ((rc = launch_gemv(M_LM, lm, se.err, s))) return rc;
-            post(K_LM);
-        }
+        if (t.logits) gemv(K_LM, M_LM, lm_params(bv, t.logits, sh.vocab));
         if (t.advance) {
-            pre(K_OTHER);
-            if ((rc = launch_pdl(advance_kernel, dim3(1), dim3(32), 0, s, se.d_pos))) return rc;
-            post(K_OTHER);
+            Op op;
+            op.type = Op::ADVANCE;
+            op.kind = K_OTHER;
+            ops.push_back(op);
         }
+    }
+    link_prefetch(ops, di.sms, only_layer < 0);
+
+    int nl = 0;
+    for (const Op& op : ops) {
+        if (hook) hook(ctx, op.kind, true);
+        switch (op.type) {
+            case Op::GEMV:
+                rc = launch_gemv(op.mode, op.p, s);
+                break;
+            case Op::ATTN:
+                rc = launch_attention(op.a, sh.dh, sh.g(), op.m_kv, op.S, n, s);
+                break;
+            case Op::COPY_HIDDEN: {
+                const cudaError_t e = cudaMemcpy2DAsync(t.hidden_out, (size_t)sh.d * 4, bv.x, (size_t)bv.x_stride * 4,
+                                                        (size_t)sh.d * 4, n, cudaMemcpyDeviceToDevice, s);
+                rc = e == cudaSuccess ? TASP_OK : cuda_fail(e, "hidden state copy");
+                break;
+            }
+            case Op::ADVANCE: {
+                AdvanceArgs aa{};
+                aa.n = n;
+                for (int b = 0; b < n; ++b) aa.pos[b] = bv.ss[b]->d_pos;
+                rc = launch_pdl(advance_kernel, dim3(1), dim3(32), 0, s, aa);
+                break;
+            }
+        }
+        if (rc) return rc;
+        if (hook) hook(ctx, op.kind, false);
+        if (op.type != Op::COPY_HIDDEN) ++nl;
     }
     if (launches) *launches = nl;
     return TASP_OK;
 }
 
+int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
+                 int* launches) {
+    return enqueue_batch(single_view(se), t, s, only_layer, hook, ctx, launches);
+}
+
 int enqueue_lm_head(Session& se, float* logits, cudaStream_t s) {
     const Shape& sh = se.plan->store->sh;
     if (sh.vocab == 0) return fail(TASP_EINVAL, "model has no LM head");
-    GemvParams lm{};
-    lm.w = reinterpret_cast<const int8_t*>(se.plan->store->lm_head);
-    lm.ld = (int64_t)sh.d * 2;
-    lm.rows = sh.vocab;
-    lm.K = sh.d;
-    lm.nchunks = sh.d / 8;
-    lm.x_resid = se.x;
-    lm.gamma = se.plan->store->g_final;
-    lm.eps = sh.eps;
-    lm.logits = logits;
-    return launch_gemv(M_LM, lm, se.err, s);
+    return launch_gemv(M_LM, lm_params(single_view(se), logits, sh.vocab), s);
 }
 
 int enqueue_set_pos(Session& se, int pos, cudaStream_t s) {

@@ -1,0 +1,13 @@
+// GEMV kernels for 1 activation vector per weight pass.
+#include "gemv.cuh"
+
+namespace tasp {
+namespace gemv {
+
+template <>
+Fn pick<1>(int mode, int R, int XC) {
+    return pick_nb<1>(mode, R, XC);
+}
+
+}  // namespace gemv
+}  // namespace tasp

@@ -4,6 +4,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <map>
 #include <memory>
 #include <mutex>
 #include <string>
@@ -366,9 +367,8 @@ static void session_free(Session* se) {
     delete se;
 }
 
-// Record (or re-record) the step graph of a session for a set of caller buffers.
-static int session_graph(Session& se, const StepTarget& t) {
-    StepGraph& g = se.graph;
+// Record (or re-record) the step graph of a batch view for a set of caller buffers.
+static int record_graph(StepGraph& g, const BatchView& bv, const StepTarget& t) {
     if (g.exec && g.x == t.x_in && g.hidden == t.hidden_out && g.logits == t.logits) return TASP_OK;
     if (g.exec) {
         cudaGraphExecDestroy(g.exec);
@@ -382,7 +382,7 @@ static int session_graph(Session& se, const StepTarget& t) {
         return cuda_fail(e, "cudaStreamBeginCapture");
     }
     int launches = 0;
-    int rc = enqueue_step(se, t, cs, -1, nullptr, nullptr, &launches);
+    int rc = enqueue_batch(bv, t, cs, -1, nullptr, nullptr, &launches);
     cudaGraph_t graph = nullptr;
     e = cudaStreamEndCapture(cs, &graph);
     cudaStreamDestroy(cs);
@@ -402,6 +402,127 @@ static int session_graph(Session& se, const StepTarget& t) {
     g.logits = t.logits;
     g.launches = launches;
     return TASP_OK;
+}
+
+static int session_graph(Session& se, const StepTarget& t) { return record_graph(se.graph, single_view(se), t); }
+
+// ---------------------------------------------------------------- batches
+// 2 to 4 sessions of one plan decoded together: every weight byte of a step is read
+// once for all of them (the decode step groups sessions per plan). A batch keeps the
+// step workspace for its sessions and its own CUDA graph; it is made on first use and
+// dropped when one of its sessions is released.
+struct Batch {
+    std::vector<Session*> ss;
+    Arena arena;
+    BatchView view;
+    uint16_t* x_stage = nullptr;  // BF16 [n][d] host-buffer staging
+    float* hidden_stage = nullptr;
+    float* logits_stage = nullptr;
+    StepGraph graph;
+};
+static std::map<std::vector<Session*>, Batch*> g_batches;  // guarded by g_mu
+
+static void batch_free(Batch* b) {
+    if (b->graph.exec) cudaGraphExecDestroy(b->graph.exec);
+    b->arena.release();
+    delete b;
+}
+
+static int batch_get(Session* const* ss, int n, Batch** out) {
+    std::vector<Session*> key(ss, ss + n);
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        auto it = g_batches.find(key);
+        if (it != g_batches.end()) {
+            *out = it->second;
+            return TASP_OK;
+        }
+    }
+    const Plan& p = *ss[0]->plan;
+    const Shape& sh = p.store->sh;
+    DevInfo di;
+    int rc = device_info(di);
+    if (rc) return rc;
+    const int smax = batch_attn_slots(p, ss, n, di.sms);
+    const int64_t xs = sh.d, qs = (int64_t)sh.Hq * sh.dh, hs = (sh.df + 3) & ~3;
+    const int64_t ps = (int64_t)sh.Hkv * smax * sh.g() * sh.dh, ms = (int64_t)sh.Hkv * smax * sh.g() * 2;
+    Layout lay;
+    lay.add((size_t)n * xs * 4);
+    lay.add((size_t)n * qs * 4);
+    lay.add((size_t)n * qs * 4);
+    lay.add((size_t)n * hs * 4);
+    lay.add((size_t)n * ps * 4);
+    lay.add((size_t)n * ms * 4);
+    lay.add((size_t)n * sh.Hkv * 4);
+    lay.add(sizeof(int));
+    lay.add((size_t)n * sh.d * 2);
+    lay.add((size_t)n * sh.d * 4);
+    lay.add((size_t)n * sh.vocab * 4);
+    auto b = std::make_unique<Batch>();
+    b->ss = key;
+    if ((rc = b->arena.reserve(lay.total))) return rc;
+    BatchView& v = b->view;
+    v.n = n;
+    for (int i = 0; i < n; ++i) v.ss[i] = ss[i];
+    v.x = (float*)b->arena.take((size_t)n * xs * 4);
+    v.q = (float*)b->arena.take((size_t)n * qs * 4);
+    v.o = (float*)b->arena.take((size_t)n * qs * 4);
+    v.h = (float*)b->arena.take((size_t)n * hs * 4);
+    v.part = (float*)b->arena.take((size_t)n * ps * 4);
+    v.ml = (float*)b->arena.take((size_t)n * ms * 4);
+    v.cnt = (int*)b->arena.take((size_t)n * sh.Hkv * 4);
+    v.err = (int*)b->arena.take(sizeof(int));
+    v.x_stride = xs;
+    v.q_stride = qs;
+    v.h_stride = hs;
+    v.part_stride = ps;
+    v.ml_stride = ms;
+    v.cnt_stride = sh.Hkv;
+    b->x_stage = (uint16_t*)b->arena.take((size_t)n * sh.d * 2);
+    b->hidden_stage = (float*)b->arena.take((size_t)n * sh.d * 4);
+    b->logits_stage = sh.vocab ? (float*)b->arena.take((size_t)n * sh.vocab * 4) : nullptr;
+    cudaError_t e = cudaMemset(b->arena.base, 0, b->arena.cap);  // tickets and the error word start at 0
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        b->arena.release();
+        return cuda_fail(e, "batch workspace");
+    }
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_batches.find(key);
+    if (it != g_batches.end()) {  // made meanwhile by another thread
+        b->arena.release();
+        *out = it->second;
+        return TASP_OK;
+    }
+    *out = b.get();
+    g_batches.emplace(key, b.release());
+    return TASP_OK;
+}
+
+// Drop every batch that holds session se (the device is idle).
+static void batches_drop(Session* se) {
+    std::vector<Batch*> gone;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        for (auto it = g_batches.begin(); it != g_batches.end();) {
+            if (std::find(it->first.begin(), it->first.end(), se) != it->first.end()) {
+                gone.push_back(it->second);
+                it = g_batches.erase(it);
+            } else {
+                ++it;
+            }
+        }
+    }
+    for (Batch* b : gone) batch_free(b);
+}
+
+// Device error words of the batches that hold session se.
+static std::vector<int*> batch_errors(Session* se) {
+    std::vector<int*> out;
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (auto& kv : g_batches)
+        if (std::find(kv.first.begin(), kv.first.end(), se) != kv.first.end()) out.push_back(kv.second->view.err);
+    return out;
 }
 
 static int check_sessions(tasp_session* const* ss, int n, Plan** plan) {
@@ -521,9 +642,15 @@ int tasp_session_status(tasp_session* s, int32_t clear, int32_t* device_error) {
     Session* se = as_session(s);
     if (!se || !device_error) return fail(TASP_EINVAL, "invalid session handle or NULL output");
     TASP_CUDA(cudaDeviceSynchronize());
+    std::vector<int*> words = batch_errors(se);
+    words.push_back(se->err);
     int v = 0;
-    TASP_CUDA(cudaMemcpy(&v, se->err, sizeof(int), cudaMemcpyDeviceToHost));
-    if (clear) TASP_CUDA(cudaMemset(se->err, 0, sizeof(int)));
+    for (int* w : words) {
+        int x = 0;
+        TASP_CUDA(cudaMemcpy(&x, w, sizeof(int), cudaMemcpyDeviceToHost));
+        if (clear) TASP_CUDA(cudaMemset(w, 0, sizeof(int)));
+        v |= x;
+    }
     *device_error = v;
     return TASP_OK;
 }
@@ -536,15 +663,26 @@ int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_b
     if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
     if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
-    for (int i = 0; i < n; ++i) {
-        Session* se = (Session*)sessions[i];
+    Session* const* ss = (Session* const*)sessions;
+    // groups of up to MAX_BATCH sessions share each weight pass
+    for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {
+        const int m = std::min(MAX_BATCH, n - i0);
         StepTarget t;
-        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i * sh.d;
-        t.hidden_out = d_hidden_out ? d_hidden_out + (size_t)i * sh.d : nullptr;
-        t.logits = d_logits ? d_logits + (size_t)i * sh.vocab : nullptr;
-        if ((rc = session_graph(*se, t))) return rc;
-        TASP_CUDA(cudaGraphLaunch(se->graph.exec, (cudaStream_t)stream));
-        se->pos += 1;
+        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i0 * sh.d;
+        t.hidden_out = d_hidden_out ? d_hidden_out + (size_t)i0 * sh.d : nullptr;
+        t.logits = d_logits ? d_logits + (size_t)i0 * sh.vocab : nullptr;
+        StepGraph* g = nullptr;
+        if (m == 1) {
+            if ((rc = session_graph(*ss[i0], t))) return rc;
+            g = &ss[i0]->graph;
+        } else {
+            Batch* b = nullptr;
+            if ((rc = batch_get(ss + i0, m, &b))) return rc;
+            if ((rc = record_graph(b->graph, b->view, t))) return rc;
+            g = &b->graph;
+        }
+        TASP_CUDA(cudaGraphLaunch(g->exec, (cudaStream_t)stream));
+        for (int i = i0; i < i0 + m; ++i) ss[i]->pos += 1;
     }
     return TASP_OK;
 }
@@ -558,22 +696,43 @@ int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* 
     const Shape& sh = p->store->sh;
     if (h_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
     cudaStream_t st = (cudaStream_t)stream;
-    for (int i = 0; i < n; ++i) {
-        Session* se = (Session*)sessions[i];
-        TASP_CUDA(cudaMemcpyAsync(se->x_stage, (const uint16_t*)h_x_bf16 + (size_t)i * sh.d, (size_t)sh.d * 2,
+    Session* const* ss = (Session* const*)sessions;
+    for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {
+        const int m = std::min(MAX_BATCH, n - i0);
+        uint16_t* xs;
+        float *hs, *ls;
+        StepGraph* g = nullptr;
+        Batch* b = nullptr;
+        if (m == 1) {
+            xs = ss[i0]->x_stage;
+            hs = ss[i0]->hidden_stage;
+            ls = ss[i0]->logits_stage;
+        } else {
+            if ((rc = batch_get(ss + i0, m, &b))) return rc;
+            xs = b->x_stage;
+            hs = b->hidden_stage;
+            ls = b->logits_stage;
+        }
+        TASP_CUDA(cudaMemcpyAsync(xs, (const uint16_t*)h_x_bf16 + (size_t)i0 * sh.d, (size_t)m * sh.d * 2,
                                   cudaMemcpyHostToDevice, st));
         StepTarget t;
-        t.x_in = se->x_stage;
-        t.hidden_out = h_hidden_out ? se->hidden_stage : nullptr;
-        t.logits = h_logits ? se->logits_stage : nullptr;
-        if ((rc = session_graph(*se, t))) return rc;
-        TASP_CUDA(cudaGraphLaunch(se->graph.exec, st));
-        se->pos += 1;
+        t.x_in = xs;
+        t.hidden_out = h_hidden_out ? hs : nullptr;
+        t.logits = h_logits ? ls : nullptr;
+        if (m == 1) {
+            if ((rc = session_graph(*ss[i0], t))) return rc;
+            g = &ss[i0]->graph;
+        } else {
+            if ((rc = record_graph(b->graph, b->view, t))) return rc;
+            g = &b->graph;
+        }
+        TASP_CUDA(cudaGraphLaunch(g->exec, st));
+        for (int i = i0; i < i0 + m; ++i) ss[i]->pos += 1;
         if (h_hidden_out)
-            TASP_CUDA(cudaMemcpyAsync(h_hidden_out + (size_t)i * sh.d, se->hidden_stage, (size_t)sh.d * 4,
+            TASP_CUDA(cudaMemcpyAsync(h_hidden_out + (size_t)i0 * sh.d, hs, (size_t)m * sh.d * 4,
                                       cudaMemcpyDeviceToHost, st));
         if (h_logits)
-            TASP_CUDA(cudaMemcpyAsync(h_logits + (size_t)i * sh.vocab, se->logits_stage, (size_t)sh.vocab * 4,
+            TASP_CUDA(cudaMemcpyAsync(h_logits + (size_t)i0 * sh.vocab, ls, (size_t)m * sh.vocab * 4,
                                       cudaMemcpyDeviceToHost, st));
     }
     TASP_CUDA(cudaStreamSynchronize(st));
@@ -649,6 +808,7 @@ int tasp_release(void* handle) {
     if (!handle) return TASP_OK;
     if (Session* se = as_session(handle)) {
         cudaError_t e = cudaDeviceSynchronize();
+        batches_drop(se);
         {
             std::lock_guard<std::mutex> lk(g_mu);
             se->plan->live_sessions--;
@@ -795,14 +955,23 @@ int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_
     if (!h_ms || !h_count || !d_x_bf16) return fail(TASP_EINVAL, "NULL buffers");
     const Shape& sh = p->store->sh;
     for (int k = 0; k < TASP_KERNEL_KINDS; ++k) { h_ms[k] = 0.f; h_count[k] = 0; }
-    for (int i = 0; i < n; ++i) {
-        Session* se = (Session*)sessions[i];
+    Session* const* ss = (Session* const*)sessions;
+    for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {
+        const int m = std::min(MAX_BATCH, n - i0);
+        BatchView bv;
+        if (m == 1) {
+            bv = single_view(*ss[i0]);
+        } else {
+            Batch* b = nullptr;
+            if ((rc = batch_get(ss + i0, m, &b))) return rc;
+            bv = b->view;
+        }
         ProfCtx pc;
         pc.s = (cudaStream_t)stream;
         StepTarget t;
-        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i * sh.d;
-        t.logits = d_logits ? d_logits + (size_t)i * sh.vocab : nullptr;
-        rc = enqueue_step(*se, t, pc.s, -1, prof_hook, &pc, nullptr);
+        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i0 * sh.d;
+        t.logits = d_logits ? d_logits + (size_t)i0 * sh.vocab : nullptr;
+        rc = enqueue_batch(bv, t, pc.s, -1, prof_hook, &pc, nullptr);
         cudaError_t e = cudaStreamSynchronize(pc.s);
         if (!rc && e == cudaSuccess && !pc.err) {
             for (size_t j = 0; j + 1 < pc.ev.size(); j += 2) {
@@ -812,7 +981,7 @@ int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_
                 h_ms[k] += ms;
                 h_count[k] += 1;
             }
-            se->pos += 1;
+            for (int i = i0; i < i0 + m; ++i) ss[i]->pos += 1;
         }
         for (cudaEvent_t ev : pc.ev) cudaEventDestroy(ev);
         if (rc) return rc;
@@ -830,7 +999,7 @@ int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_lo
     int per = 0;
     for (const LayerPlan& lp : p->layers) per += 1 + (lp.m_kv ? 2 : 0) + (lp.c ? 2 : 0);
     per += (with_logits && p->store->sh.vocab ? 1 : 0) + 1;
-    *out = per * n;
+    *out = per * ((n + MAX_BATCH - 1) / MAX_BATCH);  // one launch sequence per group of <= 4
     return TASP_OK;
 }
 

@@ -174,41 +174,66 @@ int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const in
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
 
 // attention.cu
+constexpr int MAX_BATCH = 4;  // sessions of one plan that share each weight pass
 struct AttnParams {
+    // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
     const float* q;      // FP32 rotated queries [m_q][dh] (kept heads, group-major)
-    const uint16_t* K;   // BF16 [m_kv][max_tokens][dh] of this layer
-    const uint16_t* V;
-    const int* pos;      // device position: the step attends to positions 0..pos
-    int max_tokens;
-    float qscale;        // log2(e) / sqrt(dh)
-    float* part;
-    float* ml;
-    int* cnt;            // zero between launches
     float* o;            // FP32 [m_q][dh]
+    int64_t q_stride;
+    const uint16_t* K[MAX_BATCH];  // BF16 [m_kv][max_tokens][dh] of this layer
+    const uint16_t* V[MAX_BATCH];
+    const int* pos[MAX_BATCH];     // device position: the step attends to positions 0..pos
+    int max_tokens[MAX_BATCH];
+    float qscale;        // log2(e) / sqrt(dh)
+    float* part;         // + b * part_stride
+    float* ml;           // + b * ml_stride
+    int* cnt;            // + b * cnt_stride; zero between launches
+    int64_t part_stride, ml_stride, cnt_stride;
 };
 int attn_supported(int dh, int g);
 int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
 int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g);
 int attn_splits_max();
-int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, cudaStream_t s);
+int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s);
 
 // decode.cu
 enum KernelKind { K_QKV = 0, K_ATTN = 1, K_O = 2, K_GU = 3, K_DOWN = 4, K_LM = 5, K_OTHER = 6 };
 
 struct StepTarget {
-    const uint16_t* x_in = nullptr;  // BF16 [d] step input (first layer) or nullptr (use residual)
-    float* hidden_out = nullptr;
-    float* logits = nullptr;
+    const uint16_t* x_in = nullptr;  // BF16 [n][d] step inputs (first layer) or nullptr (use residual)
+    float* hidden_out = nullptr;     // [n][d]
+    float* logits = nullptr;         // [n][vocab]
     bool advance = true;
-    // attention split scratch; nullptr = the session's own workspace
+    // attention split scratch; nullptr = the workspace of the batch view
     float* att_part = nullptr;
     float* att_ml = nullptr;
     int* att_cnt = nullptr;
 };
 
+// The n (<= MAX_BATCH) sessions of one plan that a decode step runs together, with the
+// step workspace they use: every weight byte is read once for all of them.
+struct BatchView {
+    int n = 0;
+    Session* ss[MAX_BATCH] = {};
+    float *x = nullptr, *q = nullptr, *o = nullptr, *h = nullptr;  // FP32 [n][...]
+    int64_t x_stride = 0, q_stride = 0, h_stride = 0;
+    float* part = nullptr;  // attention partials, session b at + b * part_stride
+    float* ml = nullptr;
+    int* cnt = nullptr;
+    int64_t part_stride = 0, ml_stride = 0, cnt_stride = 0;
+    int* err = nullptr;     // device error word of the step
+};
+// View of one session on its own workspace.
+BatchView single_view(Session& se);
+// Attention split slots (partials per kept group) a batch view must hold.
+int batch_attn_slots(const Plan& p, const Session* const* ss, int n, int sms);
+
 using KernelHook = void (*)(void* ctx, int kind, bool before);
 
-// Enqueue one decode step (or one isolated layer when only_layer >= 0) on `s`.
+// Enqueue one decode step of a batch (or one isolated layer when only_layer >= 0) on `s`.
+int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook,
+                  void* ctx, int* launches);
+// The same for one session on its own workspace.
 int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
                  int* launches);
 // Final RMSNorm + LM head on the session's residual (se.x) into logits [vocab].

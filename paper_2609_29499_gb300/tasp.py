@@ -287,8 +287,25 @@ def _handles(sessions):
     return ctypes.cast(arr, POINTER(c_void_p)), arr
 
 
+def _check_buffers(sessions, x, hidden, logits, device):
+    """Sizes, dtypes and placement of the caller buffers of an n-session step."""
+    import torch
+    if not sessions:
+        raise ValueError("need at least one session")
+    sh = sessions[0].plan.shape
+    n = len(sessions)
+    for t, want, dt in ((x, n * sh.d, torch.bfloat16), (hidden, n * sh.d, torch.float32),
+                        (logits, n * sh.vocab, torch.float32)):
+        if t is None:
+            continue
+        if t.dtype != dt or not t.is_contiguous() or t.numel() < want or t.is_cuda != device:
+            raise ValueError(f"buffer needs {want} contiguous {dt} elements on the {'GPU' if device else 'host'}")
+
+
 def decode_step(sessions, x_bf16, hidden=None, logits=None, stream=None):
-    """One decode step; x_bf16 is a CUDA bfloat16 tensor [n, d]; hidden / logits float32 CUDA tensors or None."""
+    """One decode step; x_bf16 is a CUDA bfloat16 tensor [n, d]; hidden / logits float32 CUDA tensors or None.
+    Sessions are grouped by up to 4 per weight pass."""
+    _check_buffers(sessions, x_bf16, hidden, logits, True)
     p, keep = _handles(sessions)
     _check(load().tasp_decode_step(p, len(sessions), x_bf16.data_ptr(),
                                    hidden.data_ptr() if hidden is not None else None,
@@ -304,6 +321,7 @@ def decode_step_static(session, x_bf16, hidden=None, logits=None, stream=None):
 
 def decode_step_host(sessions, x_bf16_host, hidden_host=None, logits_host=None, stream=None):
     """Decode step with host buffers (torch CPU tensors, ideally pinned); synchronizes the stream."""
+    _check_buffers(sessions, x_bf16_host, hidden_host, logits_host, False)
     p, keep = _handles(sessions)
     _check(load().tasp_decode_step_host(p, len(sessions), x_bf16_host.data_ptr(),
                                         hidden_host.data_ptr() if hidden_host is not None else None,

@@ -199,3 +199,18 @@ def test_planted_gqa_mistake_is_caught():
     right = fw.attend(q, K, V, 4)
     wrong = np.stack([fw.softmax(K[h % 2] @ q[h] / 4.0) @ V[h % 2] for h in range(8)])
     assert not np.allclose(right, wrong)
+
+
+def test_decode_sessions_is_per_session_decode():
+    # sessions sharing a mask are independent: each equals its own batch-1 decode (same
+    # arithmetic, so bit-identical), and sessions with different caches differ
+    sh = synth.tiny_shape(L=2)
+    m = _setup(sh)
+    x = np.stack([_steps(sh, 3) * (1 + i) for i in range(3)], axis=1)  # [S, n, d]
+    tps, seeds = [5, 9, 1], [7, 8, 7]
+    X = fw.decode_sessions(sh, m, x, tps, seeds, dtype=np.float64)
+    for i in range(3):
+        Xi = fw.decode(sh, m, x[:, i], tps[i], seeds[i], dtype=np.float64)
+        assert np.array_equal(X[:, i], Xi)
+    Y = fw.decode_sessions(sh, m, np.repeat(x[:, :1], 2, axis=1), [5, 5], [7, 8], dtype=np.float64)
+    assert not np.allclose(Y[:, 0], Y[:, 1])
