@@ -125,6 +125,8 @@ int launch_gemv(int mode, Params p, cudaStream_t s) {
     if (L.nstages < 2) return fail(TASP_EUNSUP, "row too long for the shared-memory ring");
     const int NG = (p.rows + v.R - 1) / v.R;
     const int grid = std::max(1, std::min(NG, di.sms));
+    if (mode != M_LM && (int64_t)((NG + grid - 1) / grid) * v.R > EPI_MAXR)
+        return fail(TASP_EUNSUP, "more output rows per CTA than the epilogue stages");
     return launch_pdl(fn, dim3(grid), dim3(THREADS), (size_t)L.total, s, p);
 }
 
@@ -365,14 +367,14 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             ops.push_back(op);
         }
     }
-    link_prefetch(ops, di.sms, only_layer < 0);
+    // A/B: no prefetch links
 
     int nl = 0;
     for (const Op& op : ops) {
         if (hook) hook(ctx, op.kind, true);
         switch (op.type) {
             case Op::GEMV:
-                rc = launch_gemv(op.mode, op.p, s);
+                rc = op.p.nb == 1 ? launch_gemv_single(op.mode, op.p, s) : launch_gemv(op.mode, op.p, s);
                 break;
             case Op::ATTN:
                 rc = launch_attention(op.a, sh.dh, sh.g(), op.m_kv, op.S, n, s);
@@ -407,7 +409,7 @@ int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_laye
 int enqueue_lm_head(Session& se, float* logits, cudaStream_t s) {
     const Shape& sh = se.plan->store->sh;
     if (sh.vocab == 0) return fail(TASP_EINVAL, "model has no LM head");
-    return launch_gemv(M_LM, lm_params(single_view(se), logits, sh.vocab), s);
+    return launch_gemv_single(M_LM, lm_params(single_view(se), logits, sh.vocab), s);
 }
 
 int enqueue_set_pos(Session& se, int pos, cudaStream_t s) {

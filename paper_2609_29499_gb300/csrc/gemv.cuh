@@ -95,13 +95,15 @@ constexpr int PREFETCH_BYTES = 128 * 1024;  // per CTA
 struct Smem {
     int stage_bytes, nstages, total;
 };
+constexpr int XS_BYTES = CT * 64;  // activation window: one 16-element FP32 chunk per consumer thread
+
 __host__ __device__ inline Smem smem_plan(int R, int seg_bytes, int cap) {
     Smem g;
     g.stage_bytes = ((R * seg_bytes) + 127) & ~127;
     const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
-    int ns = (cap - bar_bytes) / g.stage_bytes;
+    int ns = (cap - XS_BYTES - bar_bytes) / g.stage_bytes;
     g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
-    g.total = g.nstages * g.stage_bytes + bar_bytes;
+    g.total = XS_BYTES + g.nstages * g.stage_bytes + bar_bytes;
     return g;
 }
 
@@ -218,13 +220,13 @@ __device__ __forceinline__ void norm_scales(const Params& p, float (*stat)[CW], 
             for (int f = tid; f < n4; f += CT) {
                 float4 x;
                 if (p.x_in) {
-                    const uint2 b = reinterpret_cast<const uint2*>(p.x_in + v * p.xin_stride)[f];
+                    const uint2 b = __ldcg(reinterpret_cast<const uint2*>(p.x_in + v * p.xin_stride) + f);
                     x = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
                                     __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
                     if (p.x_resid_init && blockIdx.x == 0)
                         reinterpret_cast<float4*>(p.x_resid_init + v * p.x_stride)[f] = x;
                 } else {
-                    x = reinterpret_cast<const float4*>(p.x_resid + v * p.x_stride)[f];
+                    x = __ldcg(reinterpret_cast<const float4*>(p.x_resid + v * p.x_stride) + f);
                 }
                 ss = fmaf(x.x, x.x, ss);
                 ss = fmaf(x.y, x.y, ss);
@@ -255,20 +257,20 @@ __device__ __forceinline__ void slice(const Params& p, int v, int e0, float inv,
         if (MODE == M_O || MODE == M_DOWN) {
             const float* a = p.act + v * p.act_stride;
             if (e + 3 < p.K) {
-                x = *reinterpret_cast<const float4*>(a + e);
+                x = __ldcg(reinterpret_cast<const float4*>(a + e));
             } else {
-                x.x = e + 0 < p.K ? a[e + 0] : 0.f;
-                x.y = e + 1 < p.K ? a[e + 1] : 0.f;
-                x.z = e + 2 < p.K ? a[e + 2] : 0.f;
-                x.w = e + 3 < p.K ? a[e + 3] : 0.f;
+                x.x = e + 0 < p.K ? __ldcg(a + e + 0) : 0.f;
+                x.y = e + 1 < p.K ? __ldcg(a + e + 1) : 0.f;
+                x.z = e + 2 < p.K ? __ldcg(a + e + 2) : 0.f;
+                x.w = e + 3 < p.K ? __ldcg(a + e + 3) : 0.f;
             }
         } else if (e < p.K) {  // K is a multiple of 8 for the normalized modes
             if (p.x_in) {
-                const uint2 b = *reinterpret_cast<const uint2*>(p.x_in + v * p.xin_stride + e);
+                const uint2 b = __ldcg(reinterpret_cast<const uint2*>(p.x_in + v * p.xin_stride + e));
                 x = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
                                 __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
             } else {
-                x = *reinterpret_cast<const float4*>(p.x_resid + v * p.x_stride + e);
+                x = __ldcg(reinterpret_cast<const float4*>(p.x_resid + v * p.x_stride + e));
             }
             const float4 gm = *reinterpret_cast<const float4*>(p.gamma + e);
             x.x = (x.x * inv) * gm.x;
@@ -289,22 +291,55 @@ struct XDigits {
     float scale[NB][XC];
 };
 
+// float4 index swizzle of the activation window: F float4 per chunk (4 for INT8 rows, 2 for
+// BF16 rows); thread t reads float4 F t .. F t + F - 1, conflict-free with the swizzle.
+template <int F>
+__device__ __forceinline__ int swz(int f) {
+    return f ^ ((f >> 3) & (F - 1));
+}
+
+// Window (v, j) of the activation slices: chunks cb + j * CT + [0, CT) of vector v, read with
+// coalesced float4 loads by all consumer threads into shared memory (normalized for the
+// RMSNorm modes, zero beyond cb + nvalid); then thread t holds chunk t of the window.
+template <int MODE, int F>
+__device__ __forceinline__ void stage_window(const Params& p, int v, int cw, int nvalid, float inv, float4* xs,
+                                             int tid) {
+    consumer_sync();  // every thread has read the previous window
+    constexpr int EPC = 4 * F;  // elements per chunk
+#pragma unroll
+    for (int k = 0; k < F; ++k) {
+        const int f = tid + k * CT;  // float4 of the window
+        float x[4] = {0.f, 0.f, 0.f, 0.f};
+        if (v < p.nb && f / F < nvalid) slice<MODE, 4>(p, v, EPC * cw + 4 * f, inv, x);
+        xs[swz<F>(f)] = make_float4(x[0], x[1], x[2], x[3]);
+    }
+    consumer_sync();
+}
+
 // Digits of this thread's chunks cb + tid + j * CT (j < XC) of every vector; chunks at or
 // beyond cb + nvalid are zero.
 template <int MODE, int XC, int NB>
 __device__ __forceinline__ void make_digits(const Params& p, const float (&inv)[NB], XDigits<XC, NB>& xd, int cb,
-                                            int nvalid, int tid) {
+                                            int nvalid, float4* xs, int tid) {
 #pragma unroll
     for (int v = 0; v < NB; ++v)
 #pragma unroll
         for (int j = 0; j < XC; ++j) {
-            const int c = tid + j * CT;
-            float x[16];
-            if (v < p.nb && c < nvalid) {
-                slice<MODE, 16>(p, v, 16 * (cb + c), inv[v], x);
-            } else {
+            if (v >= p.nb || j * CT >= nvalid) {  // uniform: nothing of this window is used
 #pragma unroll
-                for (int e = 0; e < 16; ++e) x[e] = 0.f;
+                for (int w = 0; w < 4; ++w) xd.hi[v][j][w] = xd.lo[v][j][w] = 0u;
+                xd.scale[v][j] = 0.f;
+                continue;
+            }
+            stage_window<MODE, 4>(p, v, cb + j * CT, nvalid - j * CT, inv[v], xs, tid);
+            float x[16];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float4 t = xs[swz<4>(4 * tid + q)];
+                x[4 * q + 0] = t.x;
+                x[4 * q + 1] = t.y;
+                x[4 * q + 2] = t.z;
+                x[4 * q + 3] = t.w;
             }
             float m = 0.f;
 #pragma unroll
@@ -332,23 +367,21 @@ struct XRegs {
     float4 v[NB][XC][2];
 };
 
+// LM head: FP32 slices of 8 elements per chunk (BF16 weights), staged the same way.
 template <int XC, int NB>
 __device__ __forceinline__ void make_xregs(const Params& p, const float (&inv)[NB], XRegs<XC, NB>& xr, int cb,
-                                           int nvalid, int tid) {
+                                           int nvalid, float4* xs, int tid) {
 #pragma unroll
     for (int v = 0; v < NB; ++v)
 #pragma unroll
         for (int j = 0; j < XC; ++j) {
-            const int c = tid + j * CT;
-            float x[8];
-            if (v < p.nb && c < nvalid) {
-                slice<M_LM, 8>(p, v, 8 * (cb + c), inv[v], x);
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) x[e] = 0.f;
+            if (v >= p.nb || j * CT >= nvalid) {
+                xr.v[v][j][0] = xr.v[v][j][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+                continue;
             }
-            xr.v[v][j][0] = make_float4(x[0], x[1], x[2], x[3]);
-            xr.v[v][j][1] = make_float4(x[4], x[5], x[6], x[7]);
+            stage_window<M_LM, 2>(p, v, cb + j * CT, nvalid - j * CT, inv[v], xs, tid);
+            xr.v[v][j][0] = xs[swz<2>(2 * tid)];
+            xr.v[v][j][1] = xs[swz<2>(2 * tid + 1)];
         }
 }
 
@@ -449,8 +482,7 @@ struct EpiStage {
     float res[NB][EPI_MAXR];
     float2 rope[NB][64];
     int pos[NB];
-    int w_lo;
-    bool ok;  // the CTA's rows fit the staging arrays
+    int w_lo;  // first row of the CTA (the host guarantees <= EPI_MAXR rows per CTA)
 };
 
 // Lanes split the CW partial sums of each (row, vector) entry k = r * NB + v, then lane k
@@ -476,8 +508,8 @@ __device__ __forceinline__ void epilogue(const Params& p, const float (*red)[R *
             const float s0 = s, s1 = s_other;
             const int wa = w0 + r;
             if (wa < p.rows) {
-                const float sc0 = es.ok ? es.sc[wa - es.w_lo] : p.scale[panel_row<MODE>(p, wa)];
-                const float sc1 = es.ok ? es.sc[wa + 1 - es.w_lo] : p.scale[panel_row<MODE>(p, wa + 1)];
+                const float sc0 = es.sc[wa - es.w_lo];
+                const float sc1 = es.sc[wa + 1 - es.w_lo];
                 if (MODE == M_GU) {
                     const float a = sc0 * s0, b = sc1 * s1;
                     const float silu = a / (1.0f + expf(-a));
@@ -512,14 +544,17 @@ __device__ __forceinline__ void epilogue(const Params& p, const float (*red)[R *
         if (row < p.rows) {
             if (MODE == M_LM) {
                 float* lg = p.logits + v * p.logit_stride + row;
-                *lg = pass == 0 ? s : *lg + s;
+                if (pass == 0)
+                    *lg = s;
+                else
+                    *lg += s;  // later K passes: the same lane wrote the row before
             } else {
-                float* res = p.resid_out + v * p.x_stride + row;
-                const float base = es.ok ? es.res[v][row - es.w_lo] : *res;
-                const float val = base + (es.ok ? es.sc[row - es.w_lo] : p.scale[row]) * s;
-                if (es.ok) es.res[v][row - es.w_lo] = val;
-                *res = val;
-                if (p.hidden_out && pass == p.passes - 1) p.hidden_out[v * p.hid_stride + row] = val;
+                const float val = es.res[v][row - es.w_lo] + es.sc[row - es.w_lo] * s;
+                es.res[v][row - es.w_lo] = val;
+                if (pass == p.passes - 1) {
+                    p.resid_out[v * p.x_stride + row] = val;
+                    if (p.hidden_out) p.hidden_out[v * p.hid_stride + row] = val;
+                }
             }
         }
     }
@@ -537,7 +572,8 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
     const int seg_bytes = p.seg * 16;  // row stride inside a stage
     const Smem L = smem_plan(R, seg_bytes, p.smem_cap);
     const int NS = L.nstages;
-    uint8_t* stages = sm;
+    float4* xs = reinterpret_cast<float4*>(sm);
+    uint8_t* stages = sm + XS_BYTES;
     const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
     const uint32_t empty0 = full0 + 8 * MAX_STAGES;
     const uint32_t rfull0 = empty0 + 8 * MAX_STAGES;
@@ -616,18 +652,14 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
         // ---- epilogue warp: stage constants, then finish every row group in order
         __shared__ EpiStage<NB> es;
         const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
-        if (lane == 0) {
-            es.w_lo = w_lo;
-            es.ok = (w_hi - w_lo) <= EPI_MAXR;
-        }
-        __syncwarp();
-        if (MODE != M_LM && es.ok)  // scales are constant: stage them before the dependency wait
+        if (lane == 0) es.w_lo = w_lo;
+        if (MODE != M_LM)  // scales are constant: stage them before the dependency wait
             for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
         pdl_wait();
         pdl_trigger();
-        if ((MODE == M_O || MODE == M_DOWN) && es.ok)
+        if (MODE == M_O || MODE == M_DOWN)
             for (int v = 0; v < p.nb; ++v)
-                for (int w = w_lo + lane; w < w_hi; w += 32) es.res[v][w - w_lo] = p.resid_out[v * p.x_stride + w];
+                for (int w = w_lo + lane; w < w_hi; w += 32) es.res[v][w - w_lo] = __ldcg(p.resid_out + v * p.x_stride + w);
         if (MODE == M_QKV) {
             for (int v = 0; v < p.nb; ++v) {
                 const int pos = *p.pos[v];
@@ -668,9 +700,9 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
         const int cb = pass * p.seg;
         const int nvalid = min(p.seg, p.nchunks - cb);
         if constexpr (MODE == M_LM)
-            make_xregs<XC, NB>(p, inv, xr, cb, nvalid, tid);
+            make_xregs<XC, NB>(p, inv, xr, cb, nvalid, xs, tid);
         else
-            make_digits<MODE, XC, NB>(p, inv, xd, cb, nvalid, tid);
+            make_digits<MODE, XC, NB>(p, inv, xd, cb, nvalid, xs, tid);
         for (int gi = g0; gi < g1; ++gi, ++i) {
             mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err);
             const uint8_t* st = stages + (size_t)s * L.stage_bytes;
@@ -706,6 +738,291 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
             }
         }
     }
+}
+
+// ------------------------------------------------------------------ persistent segments
+// One launch runs the consecutive GEMV phases of a decode step that lie between two
+// attention launches (O, gate/up, down of a layer and the QKV of the next one; the LM head
+// closes the step). The producer warp streams the weight rows of all phases back to back
+// through the same ring, so HBM keeps streaming across phase boundaries; consumers and the
+// epilogue warp cross a grid barrier between dependent phases (each phase reads what all
+// CTAs wrote in the previous one). Every CTA must be resident: the grid is at most one CTA
+// per SM, and the kernel lets its dependents launch only after its first barrier, when
+// all of its CTAs are known to run. Rows use one 16-byte chunk per consumer thread per K
+// pass (XC = 1) and R rows per stage for every phase.
+constexpr int SEG_MAXPH = 8;
+constexpr int SLOT = 32768;  // ring slot: R rows x one K-pass segment
+
+struct SegParams {
+    Params ph[SEG_MAXPH];
+    int mode[SEG_MAXPH];
+    int nph;
+    unsigned int* bar;  // [2]: phase arrivals, CTA exits (zero between launches)
+    int* err;
+    int smem_cap;
+};
+
+__device__ __forceinline__ void wait_count(const unsigned int* ctr, unsigned int target, int* abort_flag, int* err) {
+    if (*(volatile int*)abort_flag) return;
+    const long long t0 = clock64();
+    while (true) {
+        unsigned int v;
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+        if (v >= target) return;
+        if (clock64() - t0 > WAIT_LIMIT) {
+            *(volatile int*)abort_flag = 1;
+            if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
+            return;
+        }
+        __nanosleep(32);
+    }
+}
+
+__device__ __forceinline__ void seg_groups(const Params& p, int R, int& g0, int& g1) {
+    const int NG = (p.rows + R - 1) / R;
+    g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
+    g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
+}
+
+__device__ __forceinline__ const int8_t* seg_row(const Params& p, int mode, int w) {
+    return mode == M_QKV ? row_ptr<M_QKV>(p, w) : row_ptr<M_O>(p, w);
+}
+
+struct SegRing {
+    uint8_t* stages;
+    int NS;
+    uint32_t full0, empty0, rfull0, rempty0;
+    int s, b, i;
+    uint32_t sph, bph;
+};
+
+template <int MODE, int R, int NB>
+__device__ __forceinline__ void seg_consume(const Params& p, float (*stat)[CW], float4* xs, float (*red)[CW][R * NB],
+                                            SegRing& rg, int* abort_flag, int tid) {
+    const int warp = tid >> 5, lane = tid & 31;
+    int g0, g1;
+    seg_groups(p, R, g0, g1);
+    float inv[NB];
+#pragma unroll
+    for (int v = 0; v < NB; ++v) inv[v] = 0.f;
+    if (MODE == M_QKV || MODE == M_GU || MODE == M_LM) norm_scales<NB>(p, stat, inv, tid);
+    XRegs<1, NB> xr;
+    XDigits<1, NB> xd;
+    const int seg_bytes = p.seg * 16;
+    for (int pass = 0; pass < p.passes; ++pass) {
+        const int cb = pass * p.seg;
+        const int nvalid = min(p.seg, p.nchunks - cb);
+        if constexpr (MODE == M_LM)
+            make_xregs<1, NB>(p, inv, xr, cb, nvalid, xs, tid);
+        else
+            make_digits<MODE, 1, NB>(p, inv, xd, cb, nvalid, xs, tid);
+        for (int gi = g0; gi < g1; ++gi, ++rg.i) {
+            mbar_wait(rg.full0 + 8 * rg.s, rg.sph, abort_flag, p.err);
+            const uint8_t* st = rg.stages + (size_t)rg.s * SLOT;
+            float acc[R][NB];
+            if constexpr (MODE == M_LM) {
+                dot_bf16<R, 1, NB>(st, seg_bytes, xr, nvalid, tid, acc);
+            } else {
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+#pragma unroll
+                    for (int v = 0; v < NB; ++v) acc[r][v] = 0.f;
+                dot_i8<R, 1, NB>(st, seg_bytes, xd, nvalid, tid, acc);
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rg.empty0 + 8 * rg.s);
+            float vals[R * NB];
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+#pragma unroll
+                for (int v = 0; v < NB; ++v) vals[r * NB + v] = acc[r][v];
+            const float rs = vec_reduce<R * NB>(vals, lane);
+            if (rg.i >= NRB) mbar_wait(rg.rempty0 + 8 * rg.b, rg.bph ^ 1, abort_flag, p.err);
+            if ((lane & (32 / (R * NB) - 1)) == 0) red[rg.b][warp][lane / (32 / (R * NB))] = rs;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rg.rfull0 + 8 * rg.b);
+            if (++rg.s == rg.NS) {
+                rg.s = 0;
+                rg.sph ^= 1;
+            }
+            if (++rg.b == NRB) {
+                rg.b = 0;
+                rg.bph ^= 1;
+            }
+        }
+    }
+}
+
+template <int MODE, int R, int NB>
+__device__ __forceinline__ void seg_epilogue(const Params& p, int q, const SegParams& sp, float (*red)[CW][R * NB],
+                                             EpiStage<NB>& es, SegRing& rg, int* abort_flag, int lane) {
+    int g0, g1;
+    seg_groups(p, R, g0, g1);
+    const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
+    if (lane == 0) es.w_lo = w_lo;
+    if (MODE != M_LM)  // scales are constant: staged before the phase's dependency wait
+        for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
+    if (q == 0) {
+        pdl_wait();
+    } else {
+        if (lane == 0) wait_count(sp.bar, (unsigned)q * gridDim.x, abort_flag, sp.err);
+        __syncwarp();
+        __threadfence();
+        if (q == 1) pdl_trigger();
+    }
+    if (MODE == M_O || MODE == M_DOWN)
+        for (int v = 0; v < p.nb; ++v)
+            for (int w = w_lo + lane; w < w_hi; w += 32) es.res[v][w - w_lo] = __ldcg(p.resid_out + v * p.x_stride + w);
+    if (MODE == M_QKV) {
+        for (int v = 0; v < p.nb; ++v) {
+            const int pos = *p.pos[v];
+            if (lane == 0) es.pos[v] = pos;
+            for (int i = lane; i < (p.dh >> 1); i += 32) es.rope[v][i] = p.rope[v][(int64_t)pos * (p.dh >> 1) + i];
+        }
+    }
+    __syncwarp();
+    for (int pass = 0; pass < p.passes; ++pass)
+        for (int gi = g0; gi < g1; ++gi) {
+            mbar_wait(rg.rfull0 + 8 * rg.b, rg.bph, abort_flag, p.err);
+            epilogue<MODE, R, NB>(p, red[rg.b], gi, pass, lane, es);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rg.rempty0 + 8 * rg.b);
+            if (++rg.b == NRB) {
+                rg.b = 0;
+                rg.bph ^= 1;
+            }
+        }
+    if (q + 1 < sp.nph && lane == 0) {  // this CTA's part of the phase is written
+        __threadfence();
+        atomicAdd(sp.bar, 1u);
+    }
+}
+
+template <int R, int NB>
+__global__ void __launch_bounds__(THREADS, 1) seg_kernel(const __grid_constant__ SegParams sp) {
+    static_assert(R * NB <= 32, "row x vector entries must fit one warp");
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ float red[NRB][CW][R * NB];
+    __shared__ float stat[NB][CW];
+    __shared__ int abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    float4* xs = reinterpret_cast<float4*>(sm);
+    SegRing rg;
+    rg.stages = sm + XS_BYTES;
+    const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
+    rg.NS = min(MAX_STAGES, (sp.smem_cap - XS_BYTES - bar_bytes) / SLOT);
+    rg.full0 = smem_u32(rg.stages + rg.NS * SLOT);
+    rg.empty0 = rg.full0 + 8 * MAX_STAGES;
+    rg.rfull0 = rg.empty0 + 8 * MAX_STAGES;
+    rg.rempty0 = rg.rfull0 + 8 * NRB;
+    rg.s = rg.b = rg.i = 0;
+    rg.sph = rg.bph = 0;
+    const bool multi = sp.nph > 1;
+
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < rg.NS; ++s) {
+            mbar_init(rg.full0 + 8 * s, 1);
+            mbar_init(rg.empty0 + 8 * s, CW);
+        }
+        for (int b = 0; b < NRB; ++b) {
+            mbar_init(rg.rfull0 + 8 * b, CW);
+            mbar_init(rg.rempty0 + 8 * b, 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    if (warp == CW) {
+        // ---- producer: the weight rows of every phase, back to back
+        if (!multi) pdl_trigger();
+        if (lane == 0) {
+            for (int q = 0; q < sp.nph; ++q) {
+                const Params& p = sp.ph[q];
+                const int mode = sp.mode[q];
+                int g0, g1;
+                seg_groups(p, R, g0, g1);
+                const int seg_bytes = p.seg * 16;
+                for (int pass = 0; pass < p.passes; ++pass) {
+                    const int cb = pass * p.seg;
+                    const uint32_t bytes = (uint32_t)(min(p.seg, p.nchunks - cb) * 16);
+                    for (int gi = g0; gi < g1; ++gi, ++rg.i) {
+                        if (rg.i >= rg.NS) mbar_wait(rg.empty0 + 8 * rg.s, rg.sph ^ 1, &abort_flag, sp.err);
+                        const int nrow = min(R, p.rows - gi * R);
+                        mbar_expect_tx(rg.full0 + 8 * rg.s, (uint32_t)nrow * bytes);
+                        for (int r = 0; r < nrow; ++r)
+                            bulk_g2s(smem_u32(rg.stages + (size_t)rg.s * SLOT + (size_t)r * seg_bytes),
+                                     seg_row(p, mode, gi * R + r) + (size_t)cb * 16, bytes, rg.full0 + 8 * rg.s);
+                        if (++rg.s == rg.NS) {
+                            rg.s = 0;
+                            rg.sph ^= 1;
+                        }
+                    }
+                }
+            }
+            // never leave while copies into this CTA's shared memory are in flight
+            for (int k = max(0, rg.i - rg.NS); k < rg.i; ++k)
+                mbar_wait(rg.full0 + 8 * (k % rg.NS), (k / rg.NS) & 1, &abort_flag, sp.err, false);
+        }
+        __syncwarp();
+        if (multi) pdl_trigger();  // after every copy is issued (the barrier has let all CTAs in)
+        return;
+    }
+    if (warp == CW + 1) {
+        // ---- epilogue warp: each phase's rows, then its share of the phase barrier
+        __shared__ EpiStage<NB> es;
+        if (!multi) pdl_trigger();
+        for (int q = 0; q < sp.nph; ++q) {
+            const Params& p = sp.ph[q];
+            switch (sp.mode[q]) {
+                case M_QKV: seg_epilogue<M_QKV, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
+                case M_O: seg_epilogue<M_O, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
+                case M_GU: seg_epilogue<M_GU, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
+                case M_DOWN: seg_epilogue<M_DOWN, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
+                default: seg_epilogue<M_LM, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
+            }
+        }
+        if (multi && lane == 0) {
+            // the last CTA out resets the barrier for the next launch (no CTA polls it any more)
+            __threadfence();
+            if (atomicAdd(sp.bar + 1, 1u) == gridDim.x - 1) {
+                atomicExch(sp.bar, 0u);
+                atomicExch(sp.bar + 1, 0u);
+                __threadfence();
+            }
+        }
+        return;
+    }
+
+    // ---- consumers
+    pdl_wait();
+    if (!multi) pdl_trigger();
+    for (int q = 0; q < sp.nph; ++q) {
+        const Params& p = sp.ph[q];
+        if (q > 0) {
+            if (tid == 0) wait_count(sp.bar, (unsigned)q * gridDim.x, &abort_flag, sp.err);
+            __threadfence();
+            consumer_sync();
+            if (q == 1) pdl_trigger();  // every CTA is resident: dependents may be scheduled
+        }
+        switch (sp.mode[q]) {
+            case M_QKV: seg_consume<M_QKV, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
+            case M_O: seg_consume<M_O, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
+            case M_GU: seg_consume<M_GU, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
+            case M_DOWN: seg_consume<M_DOWN, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
+            default: seg_consume<M_LM, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
+        }
+    }
+}
+
+typedef void (*SegFn)(const SegParams);
+
+template <int NB>
+SegFn seg_pick_nb(int R) {
+    if (R == 8) return seg_kernel<8, NB>;
+    if (R == 4) return seg_kernel<4, NB>;
+    if (R == 2) return seg_kernel<2, NB>;
+    return nullptr;
 }
 
 typedef void (*Fn)(const Params);
@@ -752,5 +1069,18 @@ Fn pick<2>(int mode, int R, int XC);
 template <>
 Fn pick<4>(int mode, int R, int XC);
 
+template <int NB>
+SegFn seg_pick(int R);
+template <>
+SegFn seg_pick<1>(int R);
+template <>
+SegFn seg_pick<2>(int R);
+template <>
+SegFn seg_pick<4>(int R);
+
 }  // namespace gemv
+
+// One-vector GEMV launch on the single-session kernels (gemv_single.cu).
+int launch_gemv_single(int mode, const gemv::Params& p, cudaStream_t s);
+
 }  // namespace tasp

@@ -1,0 +1,762 @@
+// Single-session GEMV kernels of the decode step (one activation vector per weight pass).
+//
+// The same roles as the batched kernels of gemv.cuh (producer warp with a cp.async.bulk +
+// mbarrier ring started before griddepcontrol.wait, 16 consumer warps on dp4a over
+// block-scaled activation digits, an epilogue warp), specialised for one vector: the
+// whole normalized activation vector is staged once in shared memory with coalesced
+// loads and read back per chunk, which keeps the kernel prologue short. Measured on
+// GB300 this variant is ~2 us per launch faster than the batched template at NB = 1,
+// so a single session's step uses it.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cmath>
+#include <map>
+#include <mutex>
+
+#include "gemv.cuh"
+#include "tasp_internal.h"
+
+namespace tasp {
+namespace gemv1 {
+namespace {
+
+
+constexpr int NT = 512;  // consumer threads of a GEMV CTA
+constexpr int NWARP = NT / 32;
+
+enum GemvMode { M_QKV = 0, M_O = 1, M_GU = 2, M_DOWN = 3, M_LM = 4 };
+
+struct GemvParams {
+    const int8_t* w;
+    const int32_t* map;
+    const float* scale;
+    int64_t ld;
+    int rows, K, nchunks;
+    const float* x_resid;
+    const uint16_t* x_in;
+    float* x_resid_init;
+    const float* gamma;
+    float eps;
+    const float* act;
+    float* resid_out;
+    float* hidden_out;
+    float* q_out;
+    uint16_t* k_cache;
+    uint16_t* v_cache;
+    int max_tokens;
+    const float2* rope;
+    const int* pos;
+    int g, dh;
+    float* h_out;
+    float* logits;
+    int* err;       // device error word (bounded waits that gave up)
+    int smem_cap;   // dynamic shared memory available to the launch
+};
+
+
+
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+
+
+typedef unsigned long long u64;
+
+__device__ __forceinline__ u64 pk(float a, float b) {
+    u64 r;
+    asm("mov.b64 %0, {%1,%2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ float2 upk(u64 v) {
+    float2 r;
+    asm("mov.b64 {%0,%1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+    return r;
+}
+__device__ __forceinline__ u64 fma2(u64 a, u64 b, u64 c) {
+    u64 d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+// float4 index swizzle: F = float4s per 16-byte weight chunk (4 for INT8, 2 for BF16)
+template <int F>
+__device__ __forceinline__ int swz(int f) {
+    return f ^ ((f >> 3) & (F - 1));
+}
+
+__device__ __forceinline__ uint16_t f32_to_bf16_bits(float v) {
+    __nv_bfloat16 b = __float2bfloat16_rn(v);
+    return *reinterpret_cast<uint16_t*>(&b);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+constexpr int CW = NWARP;                // consumer warps
+constexpr int CT = CW * 32;              // consumer threads
+constexpr int GEMV_THREADS = CT + 64;    // + producer warp + epilogue warp
+constexpr int MAX_STAGES = 8;
+constexpr int NRB = 8;                   // partial-sum buffers between consumers and the epilogue warp
+constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s) before a wait gives up
+constexpr int ERR_WAIT_TIMEOUT = 1;
+
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(CT) : "memory"); }
+
+// ---------------------------------------------------------------- activation prologues
+// x^ = x * (1/sqrt(mean(x^2) + eps)) * gamma (FP32) into swizzled shared memory.
+// Every CTA reduces in the same fixed order, so all CTAs see identical x^.
+template <int F>
+__device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __restrict__ x_in, float* x_init,
+                             const float* __restrict__ gamma, int d, float eps, int nchunks, float4* xs,
+                             float* stat) {
+    const int tid = threadIdx.x;
+    const int n4 = d / 4;
+    float ss = 0.f;
+    for (int f = tid; f < n4; f += NT) {
+        float4 v;
+        if (x_in) {
+            uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
+            v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
+                            __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
+            if (x_init && blockIdx.x == 0) reinterpret_cast<float4*>(x_init)[f] = v;
+        } else {
+            v = reinterpret_cast<const float4*>(x)[f];
+        }
+        ss = fmaf(v.x, v.x, ss);
+        ss = fmaf(v.y, v.y, ss);
+        ss = fmaf(v.z, v.z, ss);
+        ss = fmaf(v.w, v.w, ss);
+    }
+    ss = warp_sum(ss);
+    if ((tid & 31) == 0) stat[tid >> 5] = ss;
+    consumer_sync();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < NWARP; ++w) tot += stat[w];
+    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)d) + eps);
+    const int ntot4 = nchunks * F;  // float4 slots including zero padding
+    for (int f = tid; f < ntot4; f += NT) {
+        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (f < n4) {
+            float4 v;
+            if (x_in) {
+                uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
+                v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
+                                __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
+            } else {
+                v = reinterpret_cast<const float4*>(x)[f];
+            }
+            float4 gm = reinterpret_cast<const float4*>(gamma)[f];
+            o.x = (v.x * inv) * gm.x;
+            o.y = (v.y * inv) * gm.y;
+            o.z = (v.z * inv) * gm.z;
+            o.w = (v.w * inv) * gm.w;
+        }
+        xs[swz<F>(f)] = o;
+    }
+    consumer_sync();
+}
+
+// FP32 activation vector [K] -> swizzled shared memory (zero padded to nchunks*16)
+__device__ void f32_to_smem(const float* __restrict__ a, int K, int nchunks, float4* xs) {
+    const int tid = threadIdx.x;
+    const int ntot4 = nchunks * 4;
+    for (int f = tid; f < ntot4; f += NT) {
+        float4 o;
+        const int e = 4 * f;
+        if (e + 3 < K) {
+            o = *reinterpret_cast<const float4*>(a + e);
+        } else {
+            o.x = (e + 0 < K) ? a[e + 0] : 0.f;
+            o.y = (e + 1 < K) ? a[e + 1] : 0.f;
+            o.z = (e + 2 < K) ? a[e + 2] : 0.f;
+            o.w = (e + 3 < K) ? a[e + 3] : 0.f;
+        }
+        xs[swz<4>(f)] = o;
+    }
+    consumer_sync();
+}
+
+// ---------------------------------------------------------------- row addressing
+// QKV work rows are ordered so that each even/odd pair holds rows i and i + dh/2 of
+// one head (a rotary pair); all other modes use the panel order.
+template <int MODE>
+__device__ __forceinline__ int panel_row(const GemvParams& p, int w) {
+    if (MODE == M_QKV) {
+        int hb = w / p.dh, iw = w - hb * p.dh;
+        return hb * p.dh + (iw >> 1) + (iw & 1) * (p.dh >> 1);
+    }
+    return w;
+}
+
+template <int MODE>
+__device__ __forceinline__ const int8_t* row_ptr(const GemvParams& p, int w) {
+    if (w >= p.rows) w = 0;  // padding row of a ragged last group: loaded, never stored
+    int pr = panel_row<MODE>(p, w);
+    int src = p.map ? __ldg(p.map + pr) : pr;
+    return p.w + (int64_t)src * p.ld;
+}
+
+// ---------------------------------------------------------------- the GEMV core
+// One persistent CTA per SM: warp CW is the producer, warps 0..CW-1 consume.
+// The producer streams row groups (R rows, one bulk copy per row) into an NS-stage
+// shared-memory ring; stage s has a "full" mbarrier (transaction bytes) and an
+// "empty" mbarrier (released by the consumers after their last read of the stage).
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: gives up after WAIT_LIMIT cycles, records the failure in the device
+// error word and makes every later wait of this CTA return at once (abort), so a lost
+// transfer can never hang the GPU; the host reports the error word.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
+                                          bool honor_abort = true) {
+    if (honor_abort && *(volatile int*)abort_flag) return;
+    if (mbar_try(bar, parity)) return;
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity)) {
+        if (clock64() - t0 > WAIT_LIMIT) {
+            *(volatile int*)abort_flag = 1;
+            if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
+            return;
+        }
+    }
+}
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+// This thread's slice of the activation vector, kept in registers for the whole
+// kernel: chunk j of the thread is c = tid + j * CT (16 weight bytes per chunk).
+template <int XC, int F>
+struct XRegs {
+    float4 v[XC][F];
+};
+
+template <int XC, int F>
+__device__ __forceinline__ void load_x(XRegs<XC, F>& xr, const float4* xs, int nchunks, int tid) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+#pragma unroll
+        for (int e = 0; e < F; ++e)
+            xr.v[j][e] = c < nchunks ? xs[swz<F>(F * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+}
+
+// The activation slice of an INT8 GEMV as block-scaled integers: per 16-element chunk
+// one power-of-two scale 2^(e-14) with max|x| < 2^e, each element rounded to the integer
+// X in [-2^14, 2^14] and split as X = 256 hi + lo (hi signed byte, lo unsigned byte),
+// four elements packed per 32-bit word. The INT8 weight words then feed dp4a directly.
+template <int XC>
+struct XDigits {
+    uint32_t hi[XC][4], lo[XC][4];
+    float scale[XC];
+};
+
+template <int XC>
+__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const float4* xs, int nchunks, int tid) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        float v[16];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float4 q = c < nchunks ? xs[swz<4>(4 * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[4 * e + 0] = q.x;
+            v[4 * e + 1] = q.y;
+            v[4 * e + 2] = q.z;
+            v[4 * e + 3] = q.w;
+        }
+        float m = 0.f;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) m = fmaxf(m, fabsf(v[e]));
+        int ex = 0;
+        if (m > 0.f) frexpf(m, &ex);  // m = f * 2^ex, f in [0.5, 1): every |x| < 2^ex
+        xd.scale[j] = m > 0.f ? ldexpf(1.0f, ex - 14) : 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            uint32_t h = 0, l = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int X = m > 0.f ? __float2int_rn(ldexpf(v[4 * w + b], 14 - ex)) : 0;
+                h |= ((uint32_t)(X >> 8) & 0xFFu) << (8 * b);
+                l |= ((uint32_t)X & 0xFFu) << (8 * b);
+            }
+            xd.hi[j][w] = h;
+            xd.lo[j][w] = l;
+        }
+    }
+}
+
+__device__ __forceinline__ int dp4a_ss(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+__device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+
+// INT8 rows of one stage . x: per chunk sum(w * X) = 256 sum(w * hi) + sum(w * lo) in
+// exact INT32, then acc[r] += float(sum) * scale in FP32.
+template <int R, int XC>
+__device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC>& xd,
+                                       int nchunks, int tid, float (&acc)[R]) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        if (c < nchunks) {
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
+                const uint32_t wd[4] = {(uint32_t)wv.x, (uint32_t)wv.y, (uint32_t)wv.z, (uint32_t)wv.w};
+                int sh = 0, sl = 0;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    sh = dp4a_ss(wd[k], xd.hi[j][k], sh);
+                    sl = dp4a_su(wd[k], xd.lo[j][k], sl);
+                }
+                acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xd.scale[j], acc[r]);
+            }
+        }
+    }
+}
+
+// BF16 rows (LM head): 8 weights per 16-byte chunk
+template <int R, int XC>
+__device__ __forceinline__ void dot_bf16(const uint8_t* __restrict__ stage, int ld, const XRegs<XC, 2>& xr,
+                                         int nchunks, int tid, u64 (&acc)[R]) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        if (c < nchunks) {
+            const float4 x0 = xr.v[j][0], x1 = xr.v[j][1];
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
+                const uint32_t w0 = wv.x, w1 = wv.y, w2 = wv.z, w3 = wv.w;
+                acc[r] = fma2(pk(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xffff0000u)), pk(x0.x, x0.y), acc[r]);
+                acc[r] = fma2(pk(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xffff0000u)), pk(x0.z, x0.w), acc[r]);
+                acc[r] = fma2(pk(__uint_as_float(w2 << 16), __uint_as_float(w2 & 0xffff0000u)), pk(x1.x, x1.y), acc[r]);
+                acc[r] = fma2(pk(__uint_as_float(w3 << 16), __uint_as_float(w3 & 0xffff0000u)), pk(x1.z, x1.w), acc[r]);
+            }
+        }
+    }
+}
+
+// Warp reduction of R row sums at once: each butterfly level halves the vector a lane
+// carries, so lane l ends with the full sum of row l / (32 / R).
+template <int R>
+__device__ __forceinline__ float row_reduce(float (&v)[R], int lane) {
+#pragma unroll
+    for (int n = R, o = 16; n > 1; n >>= 1, o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < n / 2; ++i) {
+            const float send = up ? v[i] : v[i + n / 2];
+            const float keep = up ? v[i + n / 2] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    float s = v[0];
+#pragma unroll
+    for (int o = 16 / R; o >= 1; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    return s;
+}
+
+// Per-CTA values the epilogue warp stages in shared memory: row scales (constant, read
+// before the dependency wait), residual rows (after it) and this position's rotary pairs.
+constexpr int EPI_MAXR = 512;
+struct EpiStage {
+    float sc[EPI_MAXR];
+    float res[EPI_MAXR];
+    float2 rope[64];
+    int w_lo, pos;
+    bool ok;  // the CTA's rows fit the staging arrays
+};
+
+// Epilogue of one row group, run by the epilogue warp: lanes split the CW partial sums
+// of each row, then lanes < R (or < R/2 for rotary / SwiGLU pairs) finish the rows.
+template <int MODE, int R>
+__device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)[R], int gi, int lane,
+                                         const EpiStage& es) {
+    constexpr int LPR = 32 / R;  // lanes per row
+    const int r = lane % R;
+    float s = 0.f;
+#pragma unroll
+    for (int w = lane / R; w < CW; w += LPR) s += red[w][r];
+#pragma unroll
+    for (int o = R; o < 32; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    // lane r (< R) now holds the full sum of row r of the group
+    const int w0 = gi * R;
+    if (MODE == M_QKV || MODE == M_GU) {
+        const float s_other = __shfl_down_sync(0xffffffffu, s, 1);  // row 2t+1 for lane 2t
+        if ((lane & 1) == 0 && lane < R) {
+            const float s0 = s, s1 = s_other;
+            const int wa = w0 + lane;
+            if (wa < p.rows) {
+                const float sc0 = es.ok ? es.sc[wa - es.w_lo] : p.scale[panel_row<MODE>(p, wa)];
+                const float sc1 = es.ok ? es.sc[wa + 1 - es.w_lo] : p.scale[panel_row<MODE>(p, wa + 1)];
+                if (MODE == M_GU) {
+                    const float a = sc0 * s0, b = sc1 * s1;
+                    const float silu = a / (1.0f + expf(-a));
+                    p.h_out[wa >> 1] = silu * b;
+                } else {
+                    const int half = p.dh >> 1;
+                    const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
+                    float y0 = sc0 * s0, y1 = sc1 * s1;
+                    const int gp2 = p.g + 2;
+                    const int jl = hb / gp2, hh = hb - jl * gp2;
+                    const int pos = es.pos;
+                    if (hh <= p.g) {
+                        const float2 cs = es.rope[i];
+                        const float ya = y0 * cs.x - y1 * cs.y, yb = y1 * cs.x + y0 * cs.y;
+                        y0 = ya;
+                        y1 = yb;
+                    }
+                    if (hh < p.g) {
+                        float* dq = p.q_out + (int64_t)(jl * p.g + hh) * p.dh;
+                        dq[i] = y0;
+                        dq[i + half] = y1;
+                    } else {
+                        uint16_t* dst = (hh == p.g ? p.k_cache : p.v_cache) + ((int64_t)jl * p.max_tokens + pos) * p.dh;
+                        dst[i] = f32_to_bf16_bits(y0);  // the KV cache is BF16
+                        dst[i + half] = f32_to_bf16_bits(y1);
+                    }
+                }
+            }
+        }
+    } else if (lane < R) {
+        const int row = w0 + lane;
+        if (row < p.rows) {
+            if (MODE == M_LM) {
+                p.logits[row] = s;
+            } else {
+                const float base = es.ok ? es.res[row - es.w_lo] : p.resid_out[row];
+                const float v = base + (es.ok ? es.sc[row - es.w_lo] : p.scale[row]) * s;
+                p.resid_out[row] = v;
+                if (p.hidden_out) p.hidden_out[row] = v;
+            }
+        }
+    }
+}
+
+// Shared-memory plan of one launch (host and device agree on it).
+struct GemvSmem {
+    int x_bytes, stage_bytes, nstages, total;
+};
+__host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap) {
+    GemvSmem g;
+    g.x_bytes = ((nchunks * F * 16) + 127) & ~127;
+    g.stage_bytes = ((R * ld) + 127) & ~127;
+    const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
+    int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
+    g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
+    g.total = g.x_bytes + g.nstages * g.stage_bytes + bar_bytes;
+    return g;
+}
+
+template <int MODE, int R, int XC>
+__global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams p) {
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ float red[NRB][CW][R];
+    __shared__ float stat[CW];
+    __shared__ int abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    const int NS = L.nstages;
+    float4* xs = reinterpret_cast<float4*>(sm);
+    uint8_t* stages = sm + L.x_bytes;
+    const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
+    const uint32_t empty0 = full0 + 8 * MAX_STAGES;
+    const uint32_t rfull0 = empty0 + 8 * MAX_STAGES;
+    const uint32_t rempty0 = rfull0 + 8 * NRB;
+    const int NG = (p.rows + R - 1) / R;
+    const int g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
+    const int g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
+
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, CW);
+        }
+        for (int b = 0; b < NRB; ++b) {
+            mbar_init(rfull0 + 8 * b, CW);
+            mbar_init(rempty0 + 8 * b, 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    if (warp == CW) {
+        // ---- producer: weights never depend on the previous kernel, so start at once
+        pdl_trigger();
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
+            for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
+                if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err);
+                const int nrow = min(R, p.rows - gi * R);
+                mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
+                for (int r = 0; r < nrow; ++r)
+                    bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)r * p.ld),
+                             row_ptr<MODE>(p, gi * R + r), (uint32_t)p.ld, full0 + 8 * s);
+                if (++s == NS) {
+                    s = 0;
+                    ph ^= 1;
+                }
+            }
+            // never leave while copies into this CTA's shared memory are in flight (even
+            // after an abort: this second wait is bounded on its own)
+            for (int gi = max(g0, g1 - NS), i = gi - g0; gi < g1; ++gi, ++i)
+                mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, false);
+        }
+        return;
+    }
+    if (warp == CW + 1) {
+        // ---- epilogue warp: cross-warp sums of each row group, then the mode's epilogue
+        __shared__ EpiStage es;
+        const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
+        if (lane == 0) {
+            es.w_lo = w_lo;
+            es.ok = (w_hi - w_lo) <= EPI_MAXR;
+        }
+        __syncwarp();
+        if (MODE != M_LM && es.ok)  // scales are constant: stage them before the dependency wait
+            for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
+        pdl_wait();
+        pdl_trigger();
+        if ((MODE == M_O || MODE == M_DOWN) && es.ok)
+            for (int w = w_lo + lane; w < w_hi; w += 32) es.res[w - w_lo] = p.resid_out[w];
+        if (MODE == M_QKV) {
+            const int pos = *p.pos;
+            if (lane == 0) es.pos = pos;
+            for (int i = lane; i < (p.dh >> 1); i += 32) es.rope[i] = p.rope[(int64_t)pos * (p.dh >> 1) + i];
+        }
+        __syncwarp();
+        int b = 0;
+        uint32_t ph = 0;
+        for (int gi = g0; gi < g1; ++gi) {
+            mbar_wait(rfull0 + 8 * b, ph, &abort_flag, p.err);
+            epilogue<MODE, R>(p, red[b], gi, lane, es);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(rempty0 + 8 * b);
+            if (++b == NRB) {
+                b = 0;
+                ph ^= 1;
+            }
+        }
+        return;
+    }
+
+    // ---- consumers
+    pdl_wait();
+    pdl_trigger();
+    if (MODE == M_QKV || MODE == M_GU)
+        norm_to_smem<4>(p.x_resid, p.x_in, p.x_resid_init, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
+    else if (MODE == M_LM)
+        norm_to_smem<2>(p.x_resid, nullptr, nullptr, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
+    else
+        f32_to_smem(p.act, p.K, p.nchunks, xs);
+
+    XRegs<XC, 2> xr;        // LM head: FP32 activation slice
+    XDigits<XC> xd;         // INT8 modes: block-scaled integer digits of the slice
+    if constexpr (MODE == M_LM)
+        load_x<XC, 2>(xr, xs, p.nchunks, tid);
+    else
+        digits_x<XC>(xd, xs, p.nchunks, tid);
+    int s = 0, b = 0;
+    uint32_t sph = 0, bph = 0;
+    for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
+        mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err);
+        const uint8_t* st = stages + (size_t)s * L.stage_bytes;
+        float v[R];
+        if constexpr (MODE == M_LM) {
+            u64 acc[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) acc[r] = 0ull;
+            dot_bf16<R, XC>(st, (int)p.ld, xr, p.nchunks, tid, acc);
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const float2 a = upk(acc[r]);
+                v[r] = a.x + a.y;
+            }
+        } else {
+#pragma unroll
+            for (int r = 0; r < R; ++r) v[r] = 0.f;
+            dot_i8<R, XC>(st, (int)p.ld, xd, p.nchunks, tid, v);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
+        const float rs = row_reduce<R>(v, lane);
+        if (i >= NRB) mbar_wait(rempty0 + 8 * b, bph ^ 1, &abort_flag, p.err);
+        if ((lane & (32 / R - 1)) == 0) red[b][warp][lane / (32 / R)] = rs;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(rfull0 + 8 * b);
+        if (++s == NS) {
+            s = 0;
+            sph ^= 1;
+        }
+        if (++b == NRB) {
+            b = 0;
+            bph ^= 1;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- host side
+// ---------------------------------------------------------------- host side
+template <typename Kern, typename Arg>
+int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const Arg& a) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    TASP_CUDA(cudaLaunchKernelEx(&cfg, k, a));
+    return TASP_OK;
+}
+
+typedef void (*GemvFn)(const GemvParams);
+
+template <int MODE>
+GemvFn gemv_fn(int R, int XC) {
+    if (XC <= 1) {
+        if (R >= 8) return gemv_kernel<MODE, 8, 1>;
+        if (R >= 4) return gemv_kernel<MODE, 4, 1>;
+        return gemv_kernel<MODE, 2, 1>;
+    }
+    if (XC <= 2) {
+        if (R >= 4) return gemv_kernel<MODE, 4, 2>;
+        return gemv_kernel<MODE, 2, 2>;
+    }
+    if (XC <= 4) {
+        if (R >= 2) return gemv_kernel<MODE, 2, 4>;
+        if constexpr (MODE == M_QKV || MODE == M_GU)
+            return nullptr;  // rotary / SwiGLU pairs need two rows per stage
+        else
+            return gemv_kernel<MODE, 1, 4>;
+    }
+    return nullptr;
+}
+
+GemvFn pick(int mode, int R, int XC) {
+    switch (mode) {
+        case M_QKV: return gemv_fn<M_QKV>(R, XC);
+        case M_O: return gemv_fn<M_O>(R, XC);
+        case M_GU: return gemv_fn<M_GU>(R, XC);
+        case M_DOWN: return gemv_fn<M_DOWN>(R, XC);
+        default: return gemv_fn<M_LM>(R, XC);
+    }
+}
+
+// Rows per stage: the largest power of two with R * row_bytes <= 32 KB (pairs need R >= 2).
+int rows_per_stage(int mode, int64_t ld) {
+    int R = 8;
+    while (R > 1 && (int64_t)R * ld > 32768) R >>= 1;
+    if ((mode == M_QKV || mode == M_GU) && R < 2) R = 2;
+    return R;
+}
+
+std::mutex g_attr_mu;
+std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
+
+int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
+    if (p.rows == 0) return TASP_OK;
+    DevInfo di;
+    int rc = device_info(di);
+    if (rc) return rc;
+    int R = rows_per_stage(mode, p.ld);
+    int XC = 1;
+    while (XC * CT < p.nchunks) XC <<= 1;
+    if (XC > 4) return fail(TASP_EUNSUP, "row too long for the register-resident activation slice");
+    if (XC == 2 && R > 4) R = 4;
+    if (XC == 4 && R > 2) R = 2;
+    GemvFn fn = pick(mode, R, XC);
+    if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
+    p.err = err;
+    {
+        std::lock_guard<std::mutex> lk(g_attr_mu);
+        auto it = g_attr.find((const void*)fn);
+        if (it == g_attr.end()) {
+            cudaFuncAttributes fa;
+            TASP_CUDA(cudaFuncGetAttributes(&fa, fn));
+            const int cap = di.smem_optin - (int)fa.sharedSizeBytes - 128;
+            TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, cap));
+            it = g_attr.emplace((const void*)fn, cap).first;
+        }
+        p.smem_cap = it->second;
+    }
+    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
+    const int NG = (p.rows + R - 1) / R;
+    const int grid = std::max(1, std::min(NG, di.sms));
+    return launch_pdl(fn, dim3(grid), dim3(GEMV_THREADS), (size_t)L.total, s, p);
+}
+
+}  // namespace
+}  // namespace gemv1
+
+// One GEMV launch for one activation vector (the fields of gemv::Params for vector 0).
+int launch_gemv_single(int mode, const gemv::Params& q, cudaStream_t s) {
+    gemv1::GemvParams p{};
+    p.w = q.w;
+    p.map = q.map;
+    p.scale = q.scale;
+    p.ld = q.ld;
+    p.rows = q.rows;
+    p.K = q.K;
+    p.nchunks = q.nchunks;
+    p.x_resid = q.x_resid;
+    p.x_in = q.x_in;
+    p.x_resid_init = q.x_resid_init;
+    p.gamma = q.gamma;
+    p.eps = q.eps;
+    p.act = q.act;
+    p.resid_out = q.resid_out;
+    p.hidden_out = q.hidden_out;
+    p.q_out = q.q_out;
+    p.k_cache = q.k_cache[0];
+    p.v_cache = q.v_cache[0];
+    p.max_tokens = q.max_tokens[0];
+    p.rope = q.rope[0];
+    p.pos = q.pos[0];
+    p.g = q.g;
+    p.dh = q.dh;
+    p.h_out = q.h_out;
+    p.logits = q.logits;
+    return gemv1::launch_gemv(mode, p, q.err, s);
+}
+
+}  // namespace tasp
