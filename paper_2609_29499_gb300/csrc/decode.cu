@@ -101,8 +101,6 @@ int launch_gemv(int mode, Params p, cudaStream_t s) {
     int rc = device_info(di);
     if (rc) return rc;
     const Variant v = variant(mode, p.nb, p.nchunks, 8);
-    if (p.nx_w && (p.nx_bytes <= 0 || p.nx_bytes % 16 || p.nx_ld % 16 || p.nx_R < 1 || p.nx_grid < 1))
-        p.nx_w = nullptr;  // malformed prefetch description: skip the hint
     if ((mode == M_QKV || mode == M_GU) && v.passes > 1)
         return fail(TASP_EUNSUP, "hidden size too large for the register-resident activation slices of this batch");
     Fn fn = pick_any(v.nbk, mode, v.R, v.XC);
@@ -159,28 +157,6 @@ struct Op {
     AttnParams a{};
     int m_kv = 0, S = 0;
 };
-
-// Point every GEMV at the next GEMV of the sequence for the L2 prefetch of its first
-// rows (the last one, the LM head or the final down projection, at the first QKV: the
-// next step replays the same sequence).
-void link_prefetch(std::vector<Op>& ops, int sms, bool wrap) {
-    std::vector<int> g;
-    for (int i = 0; i < (int)ops.size(); ++i)
-        if (ops[i].type == Op::GEMV && ops[i].p.rows > 0) g.push_back(i);
-    for (size_t k = 0; k < g.size(); ++k) {
-        if (k + 1 == g.size() && !wrap) break;
-        const Op& nx = ops[g[(k + 1) % g.size()]];
-        const Variant v = variant(nx.mode, nx.p.nb, nx.p.nchunks, 8);
-        Params& p = ops[g[k]].p;
-        p.nx_w = nx.p.w;
-        p.nx_map = nx.p.map;
-        p.nx_ld = nx.p.ld;
-        p.nx_rows = nx.p.rows;
-        p.nx_R = v.R;
-        p.nx_grid = std::max(1, std::min((nx.p.rows + v.R - 1) / v.R, sms));
-        p.nx_bytes = v.seg * 16;
-    }
-}
 
 }  // namespace
 
@@ -367,8 +343,6 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             ops.push_back(op);
         }
     }
-    // A/B: no prefetch links
-
     int nl = 0;
     for (const Op& op : ops) {
         if (hook) hook(ctx, op.kind, true);

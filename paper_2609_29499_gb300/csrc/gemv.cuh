@@ -7,8 +7,9 @@
 //  * a producer warp streams row groups (R rows, one cp.async.bulk per row) into a
 //    shared-memory ring of up to 8 stages with full/empty mbarriers; weights never depend
 //    on the previous kernel, so it starts before griddepcontrol.wait;
-//  * 16 consumer warps: each thread reads its slice of every activation vector once
-//    (16 elements per 16-byte weight chunk) and turns it into block-scaled integers: per
+//  * 16 consumer warps: the activation vectors pass once through a 32 KB shared window
+//    (coalesced loads, RMSNorm applied on the way), from which each thread takes its
+//    slice (16 elements per 16-byte weight chunk) and turns it into block-scaled integers: per
 //    chunk one power-of-two scale 2^(e-14) with max|x| < 2^e, each element rounded to
 //    X in [-2^14, 2^14] and split X = 256 hi + lo (hi signed byte, lo unsigned byte). The
 //    raw INT8 weight words then feed dp4a directly (exact INT32 chunk sums, one FP32 FMA
@@ -21,7 +22,8 @@
 // row of the CTA, the digits are rebuilt for each pass, and the epilogue warp adds the
 // pass sums into the residual (or the logits) row by row.
 // Every wait is bounded: a timeout sets the device error word and aborts the CTA's later
-// waits instead of hanging.
+// waits instead of hanging. A step of one session uses the one-vector kernels of
+// gemv_single.cu instead (shorter prologue); these serve groups of 2-4 sessions.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -79,17 +81,8 @@ struct Params {
     int64_t logit_stride;
     int* err;              // device error word
     int smem_cap;          // dynamic shared memory available to the launch
-    // The next GEMV launch of the step: once its own copies are issued, the producer warp
-    // prefetches into L2 the first rows that the same CTA index streams there, so HBM
-    // stays busy through this launch's drain and the next one's ramp.
-    const int8_t* nx_w;    // nullptr: nothing to prefetch
-    const int32_t* nx_map;
-    int64_t nx_ld;
-    int nx_rows, nx_R, nx_grid;
-    int nx_bytes;          // bytes per row of its first K pass
 };
 
-constexpr int PREFETCH_BYTES = 128 * 1024;  // per CTA
 
 // Shared-memory plan of one launch (host and device agree on it).
 struct Smem {
@@ -169,9 +162,6 @@ __device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* ab
             return;
         }
     }
-}
-__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
@@ -476,6 +466,25 @@ __device__ __forceinline__ float vec_reduce(float (&v)[N], int lane) {
 }
 
 // ------------------------------------------------------------------ epilogue warp
+// Copy n floats src(i) -> dst[i] with one warp, eight independent loads in flight per lane
+// (a load followed by a shared store per element would wait out each load's latency).
+template <typename Src>
+__device__ __forceinline__ void warp_stage(float* dst, int n, Src src, int lane) {
+    for (int base = 0; base < n; base += 32 * 8) {
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + lane + 32 * k;
+            v[k] = i < n ? src(i) : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + lane + 32 * k;
+            if (i < n) dst[i] = v[k];
+        }
+    }
+}
+
 template <int NB>
 struct EpiStage {
     float sc[EPI_MAXR];
@@ -620,26 +629,6 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
                 }
             }
         }
-        __syncwarp();
-        if (p.nx_w && (int)blockIdx.x < p.nx_grid) {
-            // first rows of the same CTA index in the next launch (16-byte aligned rows)
-            const int NGn = (p.nx_rows + p.nx_R - 1) / p.nx_R;
-            const int r0 = (int)((int64_t)blockIdx.x * NGn / p.nx_grid) * p.nx_R;
-            const int r1 = min(p.nx_rows, (int)((int64_t)(blockIdx.x + 1) * NGn / p.nx_grid) * p.nx_R);
-            const int nrow = min(r1 - r0, max(1, PREFETCH_BYTES / p.nx_bytes));
-            if (!p.nx_map && (int64_t)p.nx_bytes == p.nx_ld) {
-                const int64_t total = (int64_t)nrow * p.nx_ld;
-                const int64_t piece = (total / 32 + 15) & ~int64_t(15);
-                const int64_t off = piece * lane;
-                if (nrow > 0 && off < total)
-                    prefetch_l2(p.nx_w + (int64_t)r0 * p.nx_ld + off, (uint32_t)min(piece, total - off));
-            } else {
-                for (int r = lane; r < nrow; r += 32) {
-                    const int src = p.nx_map ? __ldg(p.nx_map + r0 + r) : r0 + r;
-                    prefetch_l2(p.nx_w + (int64_t)src * p.nx_ld, (uint32_t)p.nx_bytes);
-                }
-            }
-        }
         if (lane == 0) {
             // never leave while copies into this CTA's shared memory are in flight (even
             // after an abort: this second wait is bounded on its own)
@@ -654,12 +643,12 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
         const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
         if (lane == 0) es.w_lo = w_lo;
         if (MODE != M_LM)  // scales are constant: stage them before the dependency wait
-            for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
+            warp_stage(es.sc, w_hi - w_lo, [&](int i) { return __ldg(p.scale + panel_row<MODE>(p, w_lo + i)); }, lane);
         pdl_wait();
         pdl_trigger();
         if (MODE == M_O || MODE == M_DOWN)
             for (int v = 0; v < p.nb; ++v)
-                for (int w = w_lo + lane; w < w_hi; w += 32) es.res[v][w - w_lo] = __ldcg(p.resid_out + v * p.x_stride + w);
+                warp_stage(es.res[v], w_hi - w_lo, [&](int i) { return __ldcg(p.resid_out + v * p.x_stride + w_lo + i); }, lane);
         if (MODE == M_QKV) {
             for (int v = 0; v < p.nb; ++v) {
                 const int pos = *p.pos[v];
@@ -740,291 +729,6 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
     }
 }
 
-// ------------------------------------------------------------------ persistent segments
-// One launch runs the consecutive GEMV phases of a decode step that lie between two
-// attention launches (O, gate/up, down of a layer and the QKV of the next one; the LM head
-// closes the step). The producer warp streams the weight rows of all phases back to back
-// through the same ring, so HBM keeps streaming across phase boundaries; consumers and the
-// epilogue warp cross a grid barrier between dependent phases (each phase reads what all
-// CTAs wrote in the previous one). Every CTA must be resident: the grid is at most one CTA
-// per SM, and the kernel lets its dependents launch only after its first barrier, when
-// all of its CTAs are known to run. Rows use one 16-byte chunk per consumer thread per K
-// pass (XC = 1) and R rows per stage for every phase.
-constexpr int SEG_MAXPH = 8;
-constexpr int SLOT = 32768;  // ring slot: R rows x one K-pass segment
-
-struct SegParams {
-    Params ph[SEG_MAXPH];
-    int mode[SEG_MAXPH];
-    int nph;
-    unsigned int* bar;  // [2]: phase arrivals, CTA exits (zero between launches)
-    int* err;
-    int smem_cap;
-};
-
-__device__ __forceinline__ void wait_count(const unsigned int* ctr, unsigned int target, int* abort_flag, int* err) {
-    if (*(volatile int*)abort_flag) return;
-    const long long t0 = clock64();
-    while (true) {
-        unsigned int v;
-        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
-        if (v >= target) return;
-        if (clock64() - t0 > WAIT_LIMIT) {
-            *(volatile int*)abort_flag = 1;
-            if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
-            return;
-        }
-        __nanosleep(32);
-    }
-}
-
-__device__ __forceinline__ void seg_groups(const Params& p, int R, int& g0, int& g1) {
-    const int NG = (p.rows + R - 1) / R;
-    g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
-    g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
-}
-
-__device__ __forceinline__ const int8_t* seg_row(const Params& p, int mode, int w) {
-    return mode == M_QKV ? row_ptr<M_QKV>(p, w) : row_ptr<M_O>(p, w);
-}
-
-struct SegRing {
-    uint8_t* stages;
-    int NS;
-    uint32_t full0, empty0, rfull0, rempty0;
-    int s, b, i;
-    uint32_t sph, bph;
-};
-
-template <int MODE, int R, int NB>
-__device__ __forceinline__ void seg_consume(const Params& p, float (*stat)[CW], float4* xs, float (*red)[CW][R * NB],
-                                            SegRing& rg, int* abort_flag, int tid) {
-    const int warp = tid >> 5, lane = tid & 31;
-    int g0, g1;
-    seg_groups(p, R, g0, g1);
-    float inv[NB];
-#pragma unroll
-    for (int v = 0; v < NB; ++v) inv[v] = 0.f;
-    if (MODE == M_QKV || MODE == M_GU || MODE == M_LM) norm_scales<NB>(p, stat, inv, tid);
-    XRegs<1, NB> xr;
-    XDigits<1, NB> xd;
-    const int seg_bytes = p.seg * 16;
-    for (int pass = 0; pass < p.passes; ++pass) {
-        const int cb = pass * p.seg;
-        const int nvalid = min(p.seg, p.nchunks - cb);
-        if constexpr (MODE == M_LM)
-            make_xregs<1, NB>(p, inv, xr, cb, nvalid, xs, tid);
-        else
-            make_digits<MODE, 1, NB>(p, inv, xd, cb, nvalid, xs, tid);
-        for (int gi = g0; gi < g1; ++gi, ++rg.i) {
-            mbar_wait(rg.full0 + 8 * rg.s, rg.sph, abort_flag, p.err);
-            const uint8_t* st = rg.stages + (size_t)rg.s * SLOT;
-            float acc[R][NB];
-            if constexpr (MODE == M_LM) {
-                dot_bf16<R, 1, NB>(st, seg_bytes, xr, nvalid, tid, acc);
-            } else {
-#pragma unroll
-                for (int r = 0; r < R; ++r)
-#pragma unroll
-                    for (int v = 0; v < NB; ++v) acc[r][v] = 0.f;
-                dot_i8<R, 1, NB>(st, seg_bytes, xd, nvalid, tid, acc);
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(rg.empty0 + 8 * rg.s);
-            float vals[R * NB];
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-#pragma unroll
-                for (int v = 0; v < NB; ++v) vals[r * NB + v] = acc[r][v];
-            const float rs = vec_reduce<R * NB>(vals, lane);
-            if (rg.i >= NRB) mbar_wait(rg.rempty0 + 8 * rg.b, rg.bph ^ 1, abort_flag, p.err);
-            if ((lane & (32 / (R * NB) - 1)) == 0) red[rg.b][warp][lane / (32 / (R * NB))] = rs;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(rg.rfull0 + 8 * rg.b);
-            if (++rg.s == rg.NS) {
-                rg.s = 0;
-                rg.sph ^= 1;
-            }
-            if (++rg.b == NRB) {
-                rg.b = 0;
-                rg.bph ^= 1;
-            }
-        }
-    }
-}
-
-template <int MODE, int R, int NB>
-__device__ __forceinline__ void seg_epilogue(const Params& p, int q, const SegParams& sp, float (*red)[CW][R * NB],
-                                             EpiStage<NB>& es, SegRing& rg, int* abort_flag, int lane) {
-    int g0, g1;
-    seg_groups(p, R, g0, g1);
-    const int w_lo = g0 * R, w_hi = min(g1 * R, p.rows);
-    if (lane == 0) es.w_lo = w_lo;
-    if (MODE != M_LM)  // scales are constant: staged before the phase's dependency wait
-        for (int w = w_lo + lane; w < w_hi; w += 32) es.sc[w - w_lo] = p.scale[panel_row<MODE>(p, w)];
-    if (q == 0) {
-        pdl_wait();
-    } else {
-        if (lane == 0) wait_count(sp.bar, (unsigned)q * gridDim.x, abort_flag, sp.err);
-        __syncwarp();
-        __threadfence();
-        if (q == 1) pdl_trigger();
-    }
-    if (MODE == M_O || MODE == M_DOWN)
-        for (int v = 0; v < p.nb; ++v)
-            for (int w = w_lo + lane; w < w_hi; w += 32) es.res[v][w - w_lo] = __ldcg(p.resid_out + v * p.x_stride + w);
-    if (MODE == M_QKV) {
-        for (int v = 0; v < p.nb; ++v) {
-            const int pos = *p.pos[v];
-            if (lane == 0) es.pos[v] = pos;
-            for (int i = lane; i < (p.dh >> 1); i += 32) es.rope[v][i] = p.rope[v][(int64_t)pos * (p.dh >> 1) + i];
-        }
-    }
-    __syncwarp();
-    for (int pass = 0; pass < p.passes; ++pass)
-        for (int gi = g0; gi < g1; ++gi) {
-            mbar_wait(rg.rfull0 + 8 * rg.b, rg.bph, abort_flag, p.err);
-            epilogue<MODE, R, NB>(p, red[rg.b], gi, pass, lane, es);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(rg.rempty0 + 8 * rg.b);
-            if (++rg.b == NRB) {
-                rg.b = 0;
-                rg.bph ^= 1;
-            }
-        }
-    if (q + 1 < sp.nph && lane == 0) {  // this CTA's part of the phase is written
-        __threadfence();
-        atomicAdd(sp.bar, 1u);
-    }
-}
-
-template <int R, int NB>
-__global__ void __launch_bounds__(THREADS, 1) seg_kernel(const __grid_constant__ SegParams sp) {
-    static_assert(R * NB <= 32, "row x vector entries must fit one warp");
-    extern __shared__ __align__(128) uint8_t sm[];
-    __shared__ float red[NRB][CW][R * NB];
-    __shared__ float stat[NB][CW];
-    __shared__ int abort_flag;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    float4* xs = reinterpret_cast<float4*>(sm);
-    SegRing rg;
-    rg.stages = sm + XS_BYTES;
-    const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
-    rg.NS = min(MAX_STAGES, (sp.smem_cap - XS_BYTES - bar_bytes) / SLOT);
-    rg.full0 = smem_u32(rg.stages + rg.NS * SLOT);
-    rg.empty0 = rg.full0 + 8 * MAX_STAGES;
-    rg.rfull0 = rg.empty0 + 8 * MAX_STAGES;
-    rg.rempty0 = rg.rfull0 + 8 * NRB;
-    rg.s = rg.b = rg.i = 0;
-    rg.sph = rg.bph = 0;
-    const bool multi = sp.nph > 1;
-
-    if (tid == 0) {
-        abort_flag = 0;
-        for (int s = 0; s < rg.NS; ++s) {
-            mbar_init(rg.full0 + 8 * s, 1);
-            mbar_init(rg.empty0 + 8 * s, CW);
-        }
-        for (int b = 0; b < NRB; ++b) {
-            mbar_init(rg.rfull0 + 8 * b, CW);
-            mbar_init(rg.rempty0 + 8 * b, 1);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-
-    if (warp == CW) {
-        // ---- producer: the weight rows of every phase, back to back
-        if (!multi) pdl_trigger();
-        if (lane == 0) {
-            for (int q = 0; q < sp.nph; ++q) {
-                const Params& p = sp.ph[q];
-                const int mode = sp.mode[q];
-                int g0, g1;
-                seg_groups(p, R, g0, g1);
-                const int seg_bytes = p.seg * 16;
-                for (int pass = 0; pass < p.passes; ++pass) {
-                    const int cb = pass * p.seg;
-                    const uint32_t bytes = (uint32_t)(min(p.seg, p.nchunks - cb) * 16);
-                    for (int gi = g0; gi < g1; ++gi, ++rg.i) {
-                        if (rg.i >= rg.NS) mbar_wait(rg.empty0 + 8 * rg.s, rg.sph ^ 1, &abort_flag, sp.err);
-                        const int nrow = min(R, p.rows - gi * R);
-                        mbar_expect_tx(rg.full0 + 8 * rg.s, (uint32_t)nrow * bytes);
-                        for (int r = 0; r < nrow; ++r)
-                            bulk_g2s(smem_u32(rg.stages + (size_t)rg.s * SLOT + (size_t)r * seg_bytes),
-                                     seg_row(p, mode, gi * R + r) + (size_t)cb * 16, bytes, rg.full0 + 8 * rg.s);
-                        if (++rg.s == rg.NS) {
-                            rg.s = 0;
-                            rg.sph ^= 1;
-                        }
-                    }
-                }
-            }
-            // never leave while copies into this CTA's shared memory are in flight
-            for (int k = max(0, rg.i - rg.NS); k < rg.i; ++k)
-                mbar_wait(rg.full0 + 8 * (k % rg.NS), (k / rg.NS) & 1, &abort_flag, sp.err, false);
-        }
-        __syncwarp();
-        if (multi) pdl_trigger();  // after every copy is issued (the barrier has let all CTAs in)
-        return;
-    }
-    if (warp == CW + 1) {
-        // ---- epilogue warp: each phase's rows, then its share of the phase barrier
-        __shared__ EpiStage<NB> es;
-        if (!multi) pdl_trigger();
-        for (int q = 0; q < sp.nph; ++q) {
-            const Params& p = sp.ph[q];
-            switch (sp.mode[q]) {
-                case M_QKV: seg_epilogue<M_QKV, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
-                case M_O: seg_epilogue<M_O, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
-                case M_GU: seg_epilogue<M_GU, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
-                case M_DOWN: seg_epilogue<M_DOWN, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
-                default: seg_epilogue<M_LM, R, NB>(p, q, sp, red, es, rg, &abort_flag, lane); break;
-            }
-        }
-        if (multi && lane == 0) {
-            // the last CTA out resets the barrier for the next launch (no CTA polls it any more)
-            __threadfence();
-            if (atomicAdd(sp.bar + 1, 1u) == gridDim.x - 1) {
-                atomicExch(sp.bar, 0u);
-                atomicExch(sp.bar + 1, 0u);
-                __threadfence();
-            }
-        }
-        return;
-    }
-
-    // ---- consumers
-    pdl_wait();
-    if (!multi) pdl_trigger();
-    for (int q = 0; q < sp.nph; ++q) {
-        const Params& p = sp.ph[q];
-        if (q > 0) {
-            if (tid == 0) wait_count(sp.bar, (unsigned)q * gridDim.x, &abort_flag, sp.err);
-            __threadfence();
-            consumer_sync();
-            if (q == 1) pdl_trigger();  // every CTA is resident: dependents may be scheduled
-        }
-        switch (sp.mode[q]) {
-            case M_QKV: seg_consume<M_QKV, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
-            case M_O: seg_consume<M_O, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
-            case M_GU: seg_consume<M_GU, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
-            case M_DOWN: seg_consume<M_DOWN, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
-            default: seg_consume<M_LM, R, NB>(p, stat, xs, red, rg, &abort_flag, tid); break;
-        }
-    }
-}
-
-typedef void (*SegFn)(const SegParams);
-
-template <int NB>
-SegFn seg_pick_nb(int R) {
-    if (R == 8) return seg_kernel<8, NB>;
-    if (R == 4) return seg_kernel<4, NB>;
-    if (R == 2) return seg_kernel<2, NB>;
-    return nullptr;
-}
-
 typedef void (*Fn)(const Params);
 
 // The instantiated variants: NB * XC <= 4 keeps the digit registers of the tuned
@@ -1068,15 +772,6 @@ template <>
 Fn pick<2>(int mode, int R, int XC);
 template <>
 Fn pick<4>(int mode, int R, int XC);
-
-template <int NB>
-SegFn seg_pick(int R);
-template <>
-SegFn seg_pick<1>(int R);
-template <>
-SegFn seg_pick<2>(int R);
-template <>
-SegFn seg_pick<4>(int R);
 
 }  // namespace gemv
 

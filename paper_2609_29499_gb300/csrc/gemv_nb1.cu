@@ -9,10 +9,5 @@ Fn pick<1>(int mode, int R, int XC) {
     return pick_nb<1>(mode, R, XC);
 }
 
-template <>
-SegFn seg_pick<1>(int R) {
-    return seg_pick_nb<1>(R);
-}
-
 }  // namespace gemv
 }  // namespace tasp

@@ -9,10 +9,5 @@ Fn pick<2>(int mode, int R, int XC) {
     return pick_nb<2>(mode, R, XC);
 }
 
-template <>
-SegFn seg_pick<2>(int R) {
-    return seg_pick_nb<2>(R);
-}
-
 }  // namespace gemv
 }  // namespace tasp

@@ -9,10 +9,5 @@ Fn pick<4>(int mode, int R, int XC) {
     return pick_nb<4>(mode, R, XC);
 }
 
-template <>
-SegFn seg_pick<4>(int R) {
-    return seg_pick_nb<4>(R);
-}
-
 }  // namespace gemv
 }  // namespace tasp
