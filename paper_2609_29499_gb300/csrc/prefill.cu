@@ -87,14 +87,21 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
 }
 
 // ------------------------------------------------------------------ GEMM
+// A CTA computes an (MT x 128) x 256 output tile: MT = 2 sub-tiles of 128 rows share every
+// 256 x 64 weight tile (two M = 128 accumulators fill the 512 TMEM columns), which halves
+// the operand bytes per FLOP of a single 128 x 256 tile; MT = 1 is kept for GEMMs with too
+// few tiles to fill the GPU. CTAs run M-fastest, so the CTAs in flight share weight tiles.
 constexpr int BM = 128, BN = 256, BK = 64;
-constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int GEMM_THREADS = 192;
-constexpr int GEMM_SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
-constexpr uint32_t TMEM_COLS = 256;
+template <int MT>
+struct GemmCfg {
+    static constexpr int STAGES = MT == 2 ? 3 : 4;
+    static constexpr int STAGE_BYTES = MT * A_BYTES + B_BYTES;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+    static constexpr uint32_t TMEM_COLS = 256 * MT;
+};
 constexpr uint32_t IDESC = idesc_f16(BM, BN);
 
 enum EpiMode { EP_STORE = 0, EP_RESID = 1, EP_SWIGLU = 2 };
@@ -107,18 +114,93 @@ struct GemmArgs {
     __half* hout;        // SWIGLU: hout[m][n/2] = SiLU(s_g gate) * (s_u up), n even = gate
     int ldh;
     int mode;
+    int vec;             // rows of out / hout are 16-byte aligned (vector stores)
     int* err;
 };
 
+// Epilogue of 32 accumulator columns [nb, nb + 32) of one output row.
+__device__ __forceinline__ void gemm_epi32(const GemmArgs& g, int row, int nb, const uint32_t (&r)[32]) {
+    if (g.vec && nb + 32 <= g.N) {
+        float sc[32];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const float4 t = __ldg(reinterpret_cast<const float4*>(g.scale + nb) + k);
+            sc[4 * k] = t.x;
+            sc[4 * k + 1] = t.y;
+            sc[4 * k + 2] = t.z;
+            sc[4 * k + 3] = t.w;
+        }
+        if (g.mode == EP_SWIGLU) {
+            uint32_t hw[8];
+#pragma unroll
+            for (int j = 0; j < 16; j += 2) {
+                const float a0 = __uint_as_float(r[2 * j]) * sc[2 * j];
+                const float b0 = __uint_as_float(r[2 * j + 1]) * sc[2 * j + 1];
+                const float a1 = __uint_as_float(r[2 * j + 2]) * sc[2 * j + 2];
+                const float b1 = __uint_as_float(r[2 * j + 3]) * sc[2 * j + 3];
+                const __half2 h = __floats2half2_rn(a0 / (1.0f + expf(-a0)) * b0, a1 / (1.0f + expf(-a1)) * b1);
+                hw[j >> 1] = *reinterpret_cast<const uint32_t*>(&h);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(g.hout + (int64_t)row * g.ldh + (nb >> 1));
+            dst[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            dst[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        } else {
+            float4* o4 = reinterpret_cast<float4*>(g.out + (int64_t)row * g.ldo + nb);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                float4 v = make_float4(__uint_as_float(r[4 * k]) * sc[4 * k], __uint_as_float(r[4 * k + 1]) * sc[4 * k + 1],
+                                       __uint_as_float(r[4 * k + 2]) * sc[4 * k + 2],
+                                       __uint_as_float(r[4 * k + 3]) * sc[4 * k + 3]);
+                if (g.mode == EP_RESID) {
+                    const float4 t = o4[k];
+                    v.x += t.x;
+                    v.y += t.y;
+                    v.z += t.z;
+                    v.w += t.w;
+                }
+                o4[k] = v;
+            }
+        }
+        return;
+    }
+    if (g.mode == EP_SWIGLU) {
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            const int n = nb + j;
+            if (n + 1 < g.N) {
+                const float a = __uint_as_float(r[j]) * g.scale[n];
+                const float b = __uint_as_float(r[j + 1]) * g.scale[n + 1];
+                g.hout[(int64_t)row * g.ldh + (n >> 1)] = __float2half_rn(a / (1.0f + expf(-a)) * b);
+            }
+        }
+    } else {
+        float* o = g.out + (int64_t)row * g.ldo;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const int n = nb + j;
+            if (n < g.N) {
+                const float v = __uint_as_float(r[j]) * g.scale[n];
+                if (g.mode == EP_RESID)
+                    o[n] += v;
+                else
+                    o[n] = v;
+            }
+        }
+    }
+}
+
+template <int MT>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmArgs g) {
+    using C = GemmCfg<MT>;
+    constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_acc;
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+    const int m0 = blockIdx.x * (BM * MT), n0 = blockIdx.y * BN;
     const int nk = (g.K + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
@@ -132,7 +214,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
-                     "r"(TMEM_COLS)
+                     "r"(C::TMEM_COLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -147,10 +229,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 const int s = kb % STAGES;
                 if (kb >= STAGES) mbar_wait(smem_u32(&bar_empty[s]), ((kb / STAGES) - 1) & 1, &abort_flag, g.err);
                 const uint32_t fb = smem_u32(&bar_full[s]);
-                mbar_expect_tx(fb, STAGE_BYTES);
-                const uint32_t a = smem_u32(sm + s * STAGE_BYTES);
-                tma_load_2d(a, &tmA, kb * BK, m0, fb);
-                tma_load_2d(a + A_BYTES, &tmB, kb * BK, n0, fb);
+                mbar_expect_tx(fb, C::STAGE_BYTES);
+                const uint32_t a = smem_u32(sm + s * C::STAGE_BYTES);
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) tma_load_2d(a + mt * A_BYTES, &tmA, kb * BK, m0 + BM * mt, fb);
+                tma_load_2d(a + MT * A_BYTES, &tmB, kb * BK, n0, fb);
             }
             for (int kb = max(0, nk - STAGES); kb < nk; ++kb)  // no copy may outlive the CTA
                 mbar_wait(smem_u32(&bar_full[kb % STAGES]), (kb / STAGES) & 1, &abort_flag, g.err, false);
@@ -161,16 +244,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 const int s = kb % STAGES;
                 mbar_wait(smem_u32(&bar_full[s]), (kb / STAGES) & 1, &abort_flag, g.err);
                 tc_fence_after();
-                const uint32_t a = smem_u32(sm + s * STAGE_BYTES), b = a + A_BYTES;
+                const uint32_t a = smem_u32(sm + s * C::STAGE_BYTES), b = a + MT * A_BYTES;
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk) {
-                    const uint64_t ad = sw128_desc(a + kk * 32), bd = sw128_desc(b + kk * 32);
+                    const uint64_t bd = sw128_desc(b + kk * 32);
                     const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
-                    asm volatile(
-                        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
-                        "l"(ad), "l"(bd), "r"(IDESC), "r"(accum)
-                        : "memory");
+#pragma unroll
+                    for (int mt = 0; mt < MT; ++mt) {
+                        const uint64_t ad = sw128_desc(a + mt * A_BYTES + kk * 32);
+                        asm volatile(
+                            "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256u * mt),
+                            "l"(ad), "l"(bd), "r"(IDESC), "r"(accum)
+                            : "memory");
+                    }
                 }
                 asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                                  smem_u32(&bar_empty[s]))
@@ -184,45 +271,23 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         mbar_wait(smem_u32(&bar_acc), 0, &abort_flag, g.err);
         tc_fence_after();
         const int q = warp & 3;
-        const int row = m0 + 32 * q + lane;
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 32) {
-            uint32_t r[32];
-            asm volatile(
-                "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-                "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-                  "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-                  "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
-                  "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
-                  "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-                : "r"(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0));
-            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            if (row >= g.M) continue;
-            const int nb = n0 + c0;
-            if (g.mode == EP_SWIGLU) {
-#pragma unroll
-                for (int j = 0; j < 32; j += 2) {
-                    const int n = nb + j;
-                    if (n + 1 < g.N) {
-                        const float a = __uint_as_float(r[j]) * g.scale[n];
-                        const float b = __uint_as_float(r[j + 1]) * g.scale[n + 1];
-                        g.hout[(int64_t)row * g.ldh + (n >> 1)] = __float2half_rn(a / (1.0f + expf(-a)) * b);
-                    }
-                }
-            } else {
-                float* o = g.out + (int64_t)row * g.ldo;
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int n = nb + j;
-                    if (n < g.N) {
-                        const float v = __uint_as_float(r[j]) * g.scale[n];
-                        if (g.mode == EP_RESID)
-                            o[n] += v;
-                        else
-                            o[n] = v;
-                    }
-                }
+        for (int mt = 0; mt < MT; ++mt) {
+            const int row = m0 + BM * mt + 32 * q + lane;
+#pragma unroll 1
+            for (int c0 = 0; c0 < BN; c0 += 32) {
+                uint32_t r[32];
+                asm volatile(
+                    "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+                    "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                    : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+                      "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+                      "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+                      "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+                      "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+                    : "r"(tmem + ((uint32_t)(32 * q) << 16) + 256u * mt + (uint32_t)c0));
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                if (row < g.M) gemm_epi32(g, row, n0 + c0, r);
             }
         }
     }
@@ -230,7 +295,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     if (warp == 1)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TMEM_COLS) : "memory");
 }
 
 // ------------------------------------------------------------------ elementwise kernels
@@ -305,8 +370,12 @@ __global__ void i8_to_f16_kernel(const int8_t* __restrict__ src, const int32_t* 
 }
 
 // ------------------------------------------------------------------ causal attention
+// Flash attention on mma.sync m16n8k16 with FP16 operands: the BF16 K/V tiles are widened to
+// FP16 in shared memory after they land (exact: 8 significant bits fit in 11, for values in
+// FP16's normal range), queries and probabilities enter as FP16 (11 significant bits, like
+// the GEMM operands of the prefill), accumulation and the online softmax stay FP32.
 constexpr int PA_WARPS = 8;
-constexpr int PA_QB = PA_WARPS * 8;  // queries per CTA (8 per warp)
+constexpr int PA_QB = PA_WARPS * 16;  // queries per CTA (16 per warp)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
@@ -321,23 +390,20 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t a, uint32_t& r0, uint32_t& r1
                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                  : "r"(a));
 }
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+__device__ __forceinline__ void mma16816_f16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
     asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
         "{%0,%1,%2,%3};"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t& hi, uint32_t& lo) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
-    const float2 hf = __bfloat1622float2(h);
-    const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
-    hi = *reinterpret_cast<const uint32_t*>(&h);
-    lo = *reinterpret_cast<const uint32_t*>(&l);
+__device__ __forceinline__ uint32_t pack_h2(float x0, float x1) {
+    const __half2 h = __floats2half2_rn(x0, x1);
+    return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// One CTA: one kept query head, 64 consecutive queries (8 per warp). The A operand rows
-// 0-7 hold the warp's 8 queries (BF16 high part), rows 8-15 the low parts.
+// One CTA: one kept query head, 128 consecutive queries (16 per warp: fragment rows r and
+// r + 8 of lane l are queries l / 4 and l / 4 + 8 of the warp).
 template <int DH>
 __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float* __restrict__ Qf, const uint16_t* K,
                                                                      const uint16_t* V, int T, int max_tokens, int g,
@@ -347,8 +413,8 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
     const int h = blockIdx.y, jl = h / g;
     const int q0 = (gridDim.x - 1 - blockIdx.x) * PA_QB;  // the longest blocks start first
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int qw = q0 + warp * 8;                 // this warp's first query
-    const int row_q = qw + (lane >> 2);           // query of this lane's fragment rows
+    const int qw = q0 + warp * 16;                // this warp's first query
+    const int rq[2] = {qw + (lane >> 2), qw + 8 + (lane >> 2)};  // queries of this lane's fragment rows
     const int qc = (lane & 3) * 2;
     const uint16_t* Kg = K + (int64_t)jl * max_tokens * DH;
     const uint16_t* Vg = V + (int64_t)jl * max_tokens * DH;
@@ -359,20 +425,21 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
 #pragma unroll
     for (int ks = 0; ks < KS; ++ks)
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-            const int col = ks * 16 + hf * 8 + qc;
+        for (int i = 0; i < 4; ++i) {  // a0: row r, k 0-7; a1: row r+8; a2: row r, k 8-15; a3: row r+8
+            const int rr = rq[i & 1];
+            const int col = ks * 16 + (i >> 1) * 8 + qc;
             float x0 = 0.f, x1 = 0.f;
-            if (row_q < T) {
-                const float* qp = Qf + ((int64_t)h * T + row_q) * DH + col;
+            if (rr < T) {
+                const float* qp = Qf + ((int64_t)h * T + rr) * DH + col;
                 x0 = qp[0] * qscale;
                 x1 = qp[1] * qscale;
             }
-            split_pack(x0, x1, qa[ks][2 * hf], qa[ks][2 * hf + 1]);
+            qa[ks][i] = pack_h2(x0, x1);
         }
     float acc[NT][4];
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
-    float m_run = -INFINITY, l_run = 0.f;
+    float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
 
     auto issue = [&](int kt, int st) {
         uint8_t* kt_s = &tiles[st][0][0];
@@ -387,6 +454,20 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
         }
         asm volatile("cp.async.commit_group;" ::: "memory");
     };
+    // BF16 -> FP16 in place, 8 elements per 16-byte chunk
+    auto widen = [&](int st) {
+        for (int c = tid; c < 2 * 16 * CPR; c += PA_WARPS * 32) {
+            const int kv = c / (16 * CPR), rc = c - kv * 16 * CPR;
+            const int r = rc / CPR, cc = rc - r * CPR;
+            uint4* p = reinterpret_cast<uint4*>(&tiles[st][kv][r * ROWB + cc * 16]);
+            uint4 w = *p;
+            uint32_t* u = reinterpret_cast<uint32_t*>(&w);
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                u[k] = pack_h2(__uint_as_float(u[k] << 16), __uint_as_float(u[k] & 0xffff0000u));
+            *p = w;
+        }
+    };
     if (ntile > 0) issue(0, 0);
     for (int kt = 0; kt < ntile; ++kt) {
         const int st = kt & 1;
@@ -397,8 +478,10 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
             asm volatile("cp.async.wait_group 0;" ::: "memory");
         }
         __syncthreads();
+        widen(st);
+        __syncthreads();
         const int base = kt * 16;
-        if (base <= qw + 7) {  // some key of the tile is visible to this warp's queries
+        if (base <= qw + 15) {  // some key of the tile is visible to this warp's queries
             const uint8_t* kt_s = &tiles[st][0][0];
             const uint8_t* vt_s = &tiles[st][1][0];
             float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
@@ -408,58 +491,64 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
             for (int ks = 0; ks < KS; ++ks) {
                 uint32_t b00, b01, b10, b11;
                 ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
-                mma16816(s0, qa[ks], b00, b01);
-                mma16816(s1, qa[ks], b10, b11);
+                mma16816_f16(s0, qa[ks], b00, b01);
+                mma16816_f16(s1, qa[ks], b10, b11);
             }
-            float sc[4] = {s0[0] + s0[2], s0[1] + s0[3], s1[0] + s1[2], s1[1] + s1[3]};
+            // sc[i][e]: row r / r+8 (i), keys base + qc, +1, +8, +9 (e)
+            float sc[2][4] = {{s0[0], s0[1], s1[0], s1[1]}, {s0[2], s0[3], s1[2], s1[3]}};
             const int kp[4] = {base + qc, base + qc + 1, base + 8 + qc, base + 9 + qc};
+            float pv[2][4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-                if (kp[e] > row_q || kp[e] >= kend) sc[e] = -INFINITY;  // causal
-            float mt = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
-            mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
-            mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
-            const float m_new = fmaxf(m_run, mt);
-            if (m_new != -INFINITY) {  // key 0 is visible to every query: finite from the first tile on
-                const float corr = exp2f(m_run - m_new);
-                float pv[4];
+            for (int i = 0; i < 2; ++i) {
 #pragma unroll
-                for (int e = 0; e < 4; ++e) pv[e] = exp2f(sc[e] - m_new);
-                l_run = l_run * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
-                m_run = m_new;
+                for (int e = 0; e < 4; ++e)
+                    if (kp[e] > rq[i] || kp[e] >= kend) sc[i][e] = -INFINITY;  // causal
+                float mt = fmaxf(fmaxf(sc[i][0], sc[i][1]), fmaxf(sc[i][2], sc[i][3]));
+                mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
+                mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
+                const float m_new = fmaxf(m_run[i], mt);
+                // key 0 is visible to every query, so m_new is finite from the first tile on
+                // (rows past T are computed like the others and never stored)
+                const float corr = m_new == -INFINITY ? 1.f : exp2f(m_run[i] - m_new);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) pv[i][e] = m_new == -INFINITY ? 0.f : exp2f(sc[i][e] - m_new);
+                l_run[i] = l_run[i] * corr + ((pv[i][0] + pv[i][1]) + (pv[i][2] + pv[i][3]));
+                m_run[i] = m_new;
 #pragma unroll
                 for (int nt = 0; nt < NT; ++nt) {
-                    acc[nt][0] *= corr;
-                    acc[nt][1] *= corr;
-                    acc[nt][2] *= corr;
-                    acc[nt][3] *= corr;
+                    acc[nt][2 * i] *= corr;
+                    acc[nt][2 * i + 1] *= corr;
                 }
-                uint32_t pa[4];
-                split_pack(pv[0], pv[1], pa[0], pa[1]);
-                split_pack(pv[2], pv[3], pa[2], pa[3]);
-                const uint32_t vrow =
-                    smem_u32(vt_s + (8 * ((lane >> 3) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 4) & 1));
+            }
+            uint32_t pa[4];
+            pa[0] = pack_h2(pv[0][0], pv[0][1]);  // row r, keys qc, qc+1
+            pa[1] = pack_h2(pv[1][0], pv[1][1]);  // row r+8
+            pa[2] = pack_h2(pv[0][2], pv[0][3]);  // row r, keys 8+qc, 9+qc
+            pa[3] = pack_h2(pv[1][2], pv[1][3]);  // row r+8
+            const uint32_t vrow =
+                smem_u32(vt_s + (8 * ((lane >> 3) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 4) & 1));
 #pragma unroll
-                for (int nt = 0; nt < NT; nt += 2) {
-                    uint32_t v0, v1, v2, v3;
-                    ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
-                    mma16816(acc[nt], pa, v0, v1);
-                    mma16816(acc[nt + 1], pa, v2, v3);
-                }
+            for (int nt = 0; nt < NT; nt += 2) {
+                uint32_t v0, v1, v2, v3;
+                ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
+                mma16816_f16(acc[nt], pa, v0, v1);
+                mma16816_f16(acc[nt + 1], pa, v2, v3);
             }
         }
         __syncthreads();  // the stage is refilled two tiles later
     }
-    l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
-    l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
-    if (row_q < T) {
-        const float inv = 1.0f / l_run;
-        __half* o = O + (int64_t)row_q * ldo + h * DH;
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-            const int dim = nt * 8 + qc;
-            o[dim] = __float2half_rn((acc[nt][0] + acc[nt][2]) * inv);
-            o[dim + 1] = __float2half_rn((acc[nt][1] + acc[nt][3]) * inv);
+    for (int i = 0; i < 2; ++i) {
+        l_run[i] += __shfl_xor_sync(0xffffffffu, l_run[i], 1);
+        l_run[i] += __shfl_xor_sync(0xffffffffu, l_run[i], 2);
+        if (rq[i] < T) {
+            const float inv = 1.0f / l_run[i];
+            __half* o = O + (int64_t)rq[i] * ldo + h * DH;
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int dim = nt * 8 + qc;
+                *reinterpret_cast<__half2*>(o + dim) = __floats2half2_rn(acc[nt][2 * i] * inv, acc[nt][2 * i + 1] * inv);
+            }
         }
     }
 }
@@ -500,20 +589,37 @@ int make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int b
     return TASP_OK;
 }
 
-int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, const GemmArgs& ga,
-                cudaStream_t s) {
+int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, GemmArgs ga, cudaStream_t s) {
     if (M == 0 || N == 0) return TASP_OK;
-    CUtensorMap ta, tb;
-    int rc = make_map(&ta, A, M, K, lda, BM);
+    DevInfo di;
+    int rc = device_info(di);
     if (rc) return rc;
+    // two row sub-tiles per CTA when that still gives every SM a tile
+    const int tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * ((N + BN - 1) / BN);
+    const int MT = tiles2 >= di.sms ? 2 : 1;
+    CUtensorMap ta, tb;
+    if ((rc = make_map(&ta, A, M, K, lda, BM))) return rc;
     if ((rc = make_map(&tb, B, N, K, ldb, BN))) return rc;
-    static bool attr = false;
-    if (!attr) {
-        TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMM_SMEM));
-        attr = true;
+    ga.vec = ga.mode == EP_SWIGLU ? ((reinterpret_cast<uintptr_t>(ga.hout) & 15) == 0 && ga.ldh % 8 == 0)
+                                  : ((reinterpret_cast<uintptr_t>(ga.out) & 15) == 0 && ga.ldo % 4 == 0);
+    ga.vec = ga.vec && (reinterpret_cast<uintptr_t>(ga.scale) & 15) == 0;
+    static bool attr[2] = {false, false};
+    const dim3 grid((M + BM * MT - 1) / (BM * MT), (N + BN - 1) / BN);
+    if (MT == 2) {
+        if (!attr[1]) {
+            TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           GemmCfg<2>::SMEM));
+            attr[1] = true;
+        }
+        gemm_tc_kernel<2><<<grid, GEMM_THREADS, GemmCfg<2>::SMEM, s>>>(ta, tb, ga);
+    } else {
+        if (!attr[0]) {
+            TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           GemmCfg<1>::SMEM));
+            attr[0] = true;
+        }
+        gemm_tc_kernel<1><<<grid, GEMM_THREADS, GemmCfg<1>::SMEM, s>>>(ta, tb, ga);
     }
-    dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM);
-    gemm_tc_kernel<<<grid, GEMM_THREADS, GEMM_SMEM, s>>>(ta, tb, ga);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }
