@@ -403,13 +403,26 @@ __device__ __forceinline__ uint32_t pack_h2(float x0, float x1) {
 }
 
 // One CTA: one kept query head, 128 consecutive queries (16 per warp: fragment rows r and
-// r + 8 of lane l are queries l / 4 and l / 4 + 8 of the warp).
+// r + 8 of lane l are queries l / 4 and l / 4 + 8 of the warp). Keys stream in tiles of
+// PA_KT = 64 through a double-buffered cp.async ring in dynamic shared memory; the online
+// softmax is updated once per tile.
+constexpr int PA_KT = 64;
 template <int DH>
-__global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float* __restrict__ Qf, const uint16_t* K,
+struct PaCfg {
+    static constexpr int ROWB = DH * 2 + 16;  // padded row: conflict-free ldmatrix
+    static constexpr int TILEB = PA_KT * ROWB;
+    static constexpr int SMEM = 2 * 2 * TILEB;  // [stage][K, V]
+};
+
+template <int DH>
+__global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const float* __restrict__ Qf, const uint16_t* K,
                                                                      const uint16_t* V, int T, int max_tokens, int g,
                                                                      float qscale, __half* O, int ldo) {
-    constexpr int ROWB = DH * 2 + 16, TILEB = 16 * ROWB, KS = DH / 16, NT = DH / 8, CPR = DH * 2 / 16;
-    __shared__ __align__(128) uint8_t tiles[2][2][TILEB];
+    using C = PaCfg<DH>;
+    constexpr int ROWB = C::ROWB, TILEB = C::TILEB, KS = DH / 16, NT = DH / 8, CPR = DH * 2 / 16;
+    constexpr int SUB = PA_KT / 16;  // 16-key sub-tiles per tile
+    extern __shared__ __align__(128) uint8_t pa_sm[];
+    auto tile = [&](int st, int kv) { return pa_sm + (2 * st + kv) * TILEB; };
     const int h = blockIdx.y, jl = h / g;
     const int q0 = (gridDim.x - 1 - blockIdx.x) * PA_QB;  // the longest blocks start first
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -419,7 +432,7 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
     const uint16_t* Kg = K + (int64_t)jl * max_tokens * DH;
     const uint16_t* Vg = V + (int64_t)jl * max_tokens * DH;
     const int kend = min(T, q0 + PA_QB);  // keys needed by this CTA: 0 .. kend-1
-    const int ntile = (kend + 15) / 16;
+    const int ntile = (kend + PA_KT - 1) / PA_KT;
 
     uint32_t qa[KS][4];
 #pragma unroll
@@ -442,11 +455,11 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
 
     auto issue = [&](int kt, int st) {
-        uint8_t* kt_s = &tiles[st][0][0];
-        uint8_t* vt_s = &tiles[st][1][0];
-        for (int c = tid; c < 16 * CPR; c += PA_WARPS * 32) {
+        uint8_t* kt_s = tile(st, 0);
+        uint8_t* vt_s = tile(st, 1);
+        for (int c = tid; c < PA_KT * CPR; c += PA_WARPS * 32) {
             const int r = c / CPR, cc = c - r * CPR;
-            const int pos = kt * 16 + r;
+            const int pos = kt * PA_KT + r;
             const bool ok = pos < kend;
             const int64_t off = (int64_t)(ok ? pos : 0) * DH + cc * 8;
             cp_async16(smem_u32(kt_s + r * ROWB + cc * 16), Kg + off, ok ? 16 : 0);
@@ -456,10 +469,10 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
     };
     // BF16 -> FP16 in place, 8 elements per 16-byte chunk
     auto widen = [&](int st) {
-        for (int c = tid; c < 2 * 16 * CPR; c += PA_WARPS * 32) {
-            const int kv = c / (16 * CPR), rc = c - kv * 16 * CPR;
+        for (int c = tid; c < 2 * PA_KT * CPR; c += PA_WARPS * 32) {
+            const int kv = c / (PA_KT * CPR), rc = c - kv * PA_KT * CPR;
             const int r = rc / CPR, cc = rc - r * CPR;
-            uint4* p = reinterpret_cast<uint4*>(&tiles[st][kv][r * ROWB + cc * 16]);
+            uint4* p = reinterpret_cast<uint4*>(tile(st, kv) + r * ROWB + cc * 16);
             uint4 w = *p;
             uint32_t* u = reinterpret_cast<uint32_t*>(&w);
 #pragma unroll
@@ -480,39 +493,62 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
         __syncthreads();
         widen(st);
         __syncthreads();
-        const int base = kt * 16;
+        const int base = kt * PA_KT;
         if (base <= qw + 15) {  // some key of the tile is visible to this warp's queries
-            const uint8_t* kt_s = &tiles[st][0][0];
-            const uint8_t* vt_s = &tiles[st][1][0];
-            float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
-            const uint32_t krow =
-                smem_u32(kt_s + (8 * ((lane >> 4) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 3) & 1));
+            const uint8_t* kt_s = tile(st, 0);
+            const uint8_t* vt_s = tile(st, 1);
+            // scores of the tile: sub-tile u, keys base + 16u + {qc, qc+1} (s[u][0][.]) and
+            // + 8 + {qc, qc+1} (s[u][1][.]); element [2i + e]: row r (i = 0) / r + 8, key +e
+            float sc[SUB][2][4];
 #pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                uint32_t b00, b01, b10, b11;
-                ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
-                mma16816_f16(s0, qa[ks], b00, b01);
-                mma16816_f16(s1, qa[ks], b10, b11);
+            for (int u = 0; u < SUB; ++u) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) sc[u][0][e] = sc[u][1][e] = 0.f;
+                if (base + 16 * u <= qw + 15) {
+                    const uint32_t krow = smem_u32(kt_s + (16 * u + 8 * ((lane >> 4) & 1) + (lane & 7)) * ROWB +
+                                                   16 * ((lane >> 3) & 1));
+#pragma unroll
+                    for (int ks = 0; ks < KS; ++ks) {
+                        uint32_t b00, b01, b10, b11;
+                        ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
+                        mma16816_f16(sc[u][0], qa[ks], b00, b01);
+                        mma16816_f16(sc[u][1], qa[ks], b10, b11);
+                    }
+                }
             }
-            // sc[i][e]: row r / r+8 (i), keys base + qc, +1, +8, +9 (e)
-            float sc[2][4] = {{s0[0], s0[1], s1[0], s1[1]}, {s0[2], s0[3], s1[2], s1[3]}};
-            const int kp[4] = {base + qc, base + qc + 1, base + 8 + qc, base + 9 + qc};
-            float pv[2][4];
+            float (&pv)[SUB][2][4] = sc;  // probabilities overwrite the scores in place
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
+                float mt = -INFINITY;
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if (kp[e] > rq[i] || kp[e] >= kend) sc[i][e] = -INFINITY;  // causal
-                float mt = fmaxf(fmaxf(sc[i][0], sc[i][1]), fmaxf(sc[i][2], sc[i][3]));
+                for (int u = 0; u < SUB; ++u)
+#pragma unroll
+                    for (int hlf = 0; hlf < 2; ++hlf)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int kp = base + 16 * u + 8 * hlf + qc + e;
+                            float& v = sc[u][hlf][2 * i + e];
+                            if (kp > rq[i] || kp >= kend) v = -INFINITY;  // causal
+                            mt = fmaxf(mt, v);
+                        }
                 mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
                 mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
                 const float m_new = fmaxf(m_run[i], mt);
                 // key 0 is visible to every query, so m_new is finite from the first tile on
                 // (rows past T are computed like the others and never stored)
                 const float corr = m_new == -INFINITY ? 1.f : exp2f(m_run[i] - m_new);
+                float ls = 0.f;
 #pragma unroll
-                for (int e = 0; e < 4; ++e) pv[i][e] = m_new == -INFINITY ? 0.f : exp2f(sc[i][e] - m_new);
-                l_run[i] = l_run[i] * corr + ((pv[i][0] + pv[i][1]) + (pv[i][2] + pv[i][3]));
+                for (int u = 0; u < SUB; ++u)
+#pragma unroll
+                    for (int hlf = 0; hlf < 2; ++hlf)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const float p = m_new == -INFINITY ? 0.f : exp2f(sc[u][hlf][2 * i + e] - m_new);
+                            pv[u][hlf][2 * i + e] = p;
+                            ls += p;
+                        }
+                l_run[i] = l_run[i] * corr + ls;
                 m_run[i] = m_new;
 #pragma unroll
                 for (int nt = 0; nt < NT; ++nt) {
@@ -520,19 +556,23 @@ __global__ void __launch_bounds__(PA_WARPS * 32) attn_prefill_kernel(const float
                     acc[nt][2 * i + 1] *= corr;
                 }
             }
-            uint32_t pa[4];
-            pa[0] = pack_h2(pv[0][0], pv[0][1]);  // row r, keys qc, qc+1
-            pa[1] = pack_h2(pv[1][0], pv[1][1]);  // row r+8
-            pa[2] = pack_h2(pv[0][2], pv[0][3]);  // row r, keys 8+qc, 9+qc
-            pa[3] = pack_h2(pv[1][2], pv[1][3]);  // row r+8
-            const uint32_t vrow =
-                smem_u32(vt_s + (8 * ((lane >> 3) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 4) & 1));
 #pragma unroll
-            for (int nt = 0; nt < NT; nt += 2) {
-                uint32_t v0, v1, v2, v3;
-                ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
-                mma16816_f16(acc[nt], pa, v0, v1);
-                mma16816_f16(acc[nt + 1], pa, v2, v3);
+            for (int u = 0; u < SUB; ++u) {
+                if (base + 16 * u > qw + 15) continue;  // no visible key in this sub-tile
+                uint32_t pa[4];
+                pa[0] = pack_h2(pv[u][0][0], pv[u][0][1]);  // row r, keys qc, qc+1
+                pa[1] = pack_h2(pv[u][0][2], pv[u][0][3]);  // row r+8
+                pa[2] = pack_h2(pv[u][1][0], pv[u][1][1]);  // row r, keys 8+qc, 9+qc
+                pa[3] = pack_h2(pv[u][1][2], pv[u][1][3]);  // row r+8
+                const uint32_t vrow = smem_u32(vt_s + (16 * u + 8 * ((lane >> 3) & 1) + (lane & 7)) * ROWB +
+                                               16 * ((lane >> 4) & 1));
+#pragma unroll
+                for (int nt = 0; nt < NT; nt += 2) {
+                    uint32_t v0, v1, v2, v3;
+                    ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
+                    mma16816_f16(acc[nt], pa, v0, v1);
+                    mma16816_f16(acc[nt + 1], pa, v2, v3);
+                }
             }
         }
         __syncthreads();  // the stage is refilled two tiles later
@@ -686,6 +726,16 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
     TASP_CUDA(cudaMemsetAsync(O, 0, (size_t)T * ld_o * 2, s));
     TASP_CUDA(cudaMemsetAsync(H, 0, (size_t)T * ld_h * 2, s));
     const float qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
+    {
+        static bool attr = false;  // the key/value ring exceeds the default 48 KB of shared memory
+        if (!attr) {
+            TASP_CUDA(cudaFuncSetAttribute(attn_prefill_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           PaCfg<128>::SMEM));
+            TASP_CUDA(cudaFuncSetAttribute(attn_prefill_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           PaCfg<64>::SMEM));
+            attr = true;
+        }
+    }
     for (int l = 0; l < sh.L && !rc; ++l) {
         const LayerPlan& lp = pl.layers[l];
         const F16Panels& f = pl.f16[l];
@@ -700,10 +750,10 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
                                                             se.max_tokens);
             const int qb = (T + PA_QB - 1) / PA_QB;
             if (sh.dh == 128)
-                attn_prefill_kernel<128><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, 0, s>>>(
+                attn_prefill_kernel<128><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, PaCfg<128>::SMEM, s>>>(
                     Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
             else
-                attn_prefill_kernel<64><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, 0, s>>>(
+                attn_prefill_kernel<64><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, PaCfg<64>::SMEM, s>>>(
                     Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
             TASP_CUDA(cudaGetLastError());
             GemmArgs go{};
