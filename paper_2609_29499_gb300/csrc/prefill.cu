@@ -423,8 +423,10 @@ __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const fl
     constexpr int SUB = PA_KT / 16;  // 16-key sub-tiles per tile
     extern __shared__ __align__(128) uint8_t pa_sm[];
     auto tile = [&](int st, int kv) { return pa_sm + (2 * st + kv) * TILEB; };
-    const int h = blockIdx.y, jl = h / g;
-    const int q0 = (gridDim.x - 1 - blockIdx.x) * PA_QB;  // the longest blocks start first
+    // grid (heads, query blocks): blocks are scheduled x-fastest, so the longest query blocks
+    // of every head run first and the short ones fill the tail
+    const int h = blockIdx.x, jl = h / g;
+    const int q0 = (gridDim.y - 1 - blockIdx.y) * PA_QB;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int qw = q0 + warp * 16;                // this warp's first query
     const int rq[2] = {qw + (lane >> 2), qw + 8 + (lane >> 2)};  // queries of this lane's fragment rows
@@ -501,21 +503,22 @@ __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const fl
             // + 8 + {qc, qc+1} (s[u][1][.]); element [2i + e]: row r (i = 0) / r + 8, key +e
             float sc[SUB][2][4];
 #pragma unroll
-            for (int u = 0; u < SUB; ++u) {
+            for (int u = 0; u < SUB; ++u)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) sc[u][0][e] = sc[u][1][e] = 0.f;
-                if (base + 16 * u <= qw + 15) {
-                    const uint32_t krow = smem_u32(kt_s + (16 * u + 8 * ((lane >> 4) & 1) + (lane & 7)) * ROWB +
-                                                   16 * ((lane >> 3) & 1));
+            // k-steps outer, sub-tiles inner: 2 SUB independent accumulation chains in flight
+            // (sub-tiles past the warp's last query are computed and masked below)
+            const uint32_t krow0 =
+                smem_u32(kt_s + (8 * ((lane >> 4) & 1) + (lane & 7)) * ROWB + 16 * ((lane >> 3) & 1));
 #pragma unroll
-                    for (int ks = 0; ks < KS; ++ks) {
-                        uint32_t b00, b01, b10, b11;
-                        ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
-                        mma16816_f16(sc[u][0], qa[ks], b00, b01);
-                        mma16816_f16(sc[u][1], qa[ks], b10, b11);
-                    }
+            for (int ks = 0; ks < KS; ++ks)
+#pragma unroll
+                for (int u = 0; u < SUB; ++u) {
+                    uint32_t b00, b01, b10, b11;
+                    ldsm_x4(krow0 + 16 * u * ROWB + ks * 32, b00, b01, b10, b11);
+                    mma16816_f16(sc[u][0], qa[ks], b00, b01);
+                    mma16816_f16(sc[u][1], qa[ks], b10, b11);
                 }
-            }
             float (&pv)[SUB][2][4] = sc;  // probabilities overwrite the scores in place
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
@@ -750,10 +753,10 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
                                                             se.max_tokens);
             const int qb = (T + PA_QB - 1) / PA_QB;
             if (sh.dh == 128)
-                attn_prefill_kernel<128><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, PaCfg<128>::SMEM, s>>>(
+                attn_prefill_kernel<128><<<dim3(lp.m_kv * sh.g(), qb), PA_WARPS * 32, PaCfg<128>::SMEM, s>>>(
                     Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
             else
-                attn_prefill_kernel<64><<<dim3(qb, lp.m_kv * sh.g()), PA_WARPS * 32, PaCfg<64>::SMEM, s>>>(
+                attn_prefill_kernel<64><<<dim3(lp.m_kv * sh.g(), qb), PA_WARPS * 32, PaCfg<64>::SMEM, s>>>(
                     Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
             TASP_CUDA(cudaGetLastError());
             GemmArgs go{};
