@@ -637,9 +637,13 @@ int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
-    // two row sub-tiles per CTA when that still gives every SM a tile
-    const int tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * ((N + BN - 1) / BN);
-    const int MT = tiles2 >= di.sms ? 2 : 1;
+    // two row sub-tiles per CTA unless wave quantization eats their gain: cost = waves x
+    // tile time, a one-sub-tile CTA taking half the time of a two-sub-tile CTA but ~1.25x
+    // the time per FLOP (87 against 131 FLOP per operand byte)
+    const int nt = (N + BN - 1) / BN;
+    const int tiles1 = ((M + BM - 1) / BM) * nt, tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * nt;
+    const double cost1 = 1.25 * ((tiles1 + di.sms - 1) / di.sms), cost2 = 2.0 * ((tiles2 + di.sms - 1) / di.sms);
+    const int MT = cost2 <= cost1 ? 2 : 1;
     CUtensorMap ta, tb;
     if ((rc = make_map(&ta, A, M, K, lda, BM))) return rc;
     if ((rc = make_map(&tb, B, N, K, ldb, BN))) return rc;

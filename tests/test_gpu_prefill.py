@@ -82,3 +82,10 @@ def test_prefill_8b_two_layers_all_masks(tasp):
 def test_prefill_8b_full_depth_512(tasp):
     sh = synth.LLAMA3_8B
     _prefill_case(tasp, sh, synth.CFG4.masks[0], 512, 2, [0, 15, 31], logits_rows=np.arange(0, sh.vocab, 997))
+
+
+def test_prefill_8b_two_layers_bench_length(tasp):
+    # the benchmark's prompt length (2,048 tokens: two-row-tile GEMMs, 16 query blocks per
+    # head in the attention schedule) on a two-layer cut of the 8B widths
+    sh = dataclasses.replace(synth.LLAMA3_8B, L=2)
+    _prefill_case(tasp, sh, synth.CFG4.masks[0], 2048, 2, [0, 1], logits_rows=np.arange(0, sh.vocab, 499))
