@@ -127,9 +127,10 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
  * step groups the turns that share a mask). A group of 2-4 sessions keeps a step
  * workspace (~ n x (d + 2 H_q d_h + d_f + vocab) x 4 bytes plus attention
  * partials) until one of its sessions is released. Results per session do not
- * depend on the group (up to FP32 summation order). The step is replayed from a
- * CUDA graph captured on first use for this (sessions, buffers) combination;
- * call it outside any stream capture. async on `stream`.
+ * depend on the group (up to FP32 summation order). The inputs are copied on
+ * `stream` into the session's (or group's) own staging buffer, and the step is
+ * replayed from a CUDA graph captured on first use for this (sessions, output
+ * buffers) combination; call it outside any stream capture. async on `stream`.
  * Errors: EMASK (sessions on different plans), ECAP (a session is full),
  * EINVAL, ENOMEM, ECUDA. */
 int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,

@@ -415,7 +415,7 @@ struct Batch {
     std::vector<Session*> ss;
     Arena arena;
     BatchView view;
-    uint16_t* x_stage = nullptr;  // BF16 [n][d] host-buffer staging
+    uint16_t* x_stage = nullptr;  // BF16 [n][d] step-input staging (device and host-buffer steps)
     float* hidden_stage = nullptr;
     float* logits_stage = nullptr;
     StepGraph graph;
@@ -664,11 +664,19 @@ int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_b
     const Shape& sh = p->store->sh;
     if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
     Session* const* ss = (Session* const*)sessions;
+    cudaStream_t st = (cudaStream_t)stream;
     // groups of up to MAX_BATCH sessions share each weight pass
     for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {
         const int m = std::min(MAX_BATCH, n - i0);
+        Batch* b = nullptr;
+        if (m > 1 && (rc = batch_get(ss + i0, m, &b))) return rc;
+        // the inputs go through the group's fixed staging buffer, so the recorded step graph
+        // depends only on the output buffers and stays valid while callers vary the inputs
+        uint16_t* xs = m == 1 ? ss[i0]->x_stage : b->x_stage;
+        TASP_CUDA(cudaMemcpyAsync(xs, (const uint16_t*)d_x_bf16 + (size_t)i0 * sh.d, (size_t)m * sh.d * 2,
+                                  cudaMemcpyDeviceToDevice, st));
         StepTarget t;
-        t.x_in = (const uint16_t*)d_x_bf16 + (size_t)i0 * sh.d;
+        t.x_in = xs;
         t.hidden_out = d_hidden_out ? d_hidden_out + (size_t)i0 * sh.d : nullptr;
         t.logits = d_logits ? d_logits + (size_t)i0 * sh.vocab : nullptr;
         StepGraph* g = nullptr;
@@ -676,12 +684,10 @@ int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_b
             if ((rc = session_graph(*ss[i0], t))) return rc;
             g = &ss[i0]->graph;
         } else {
-            Batch* b = nullptr;
-            if ((rc = batch_get(ss + i0, m, &b))) return rc;
             if ((rc = record_graph(b->graph, b->view, t))) return rc;
             g = &b->graph;
         }
-        TASP_CUDA(cudaGraphLaunch(g->exec, (cudaStream_t)stream));
+        TASP_CUDA(cudaGraphLaunch(g->exec, st));
         for (int i = i0; i < i0 + m; ++i) ss[i]->pos += 1;
     }
     return TASP_OK;

@@ -151,7 +151,7 @@ struct Session {
     int* cnt = nullptr;     // attention split tickets [Hkv]
     int* err = nullptr;     // device error word (0 = no kernel reported a failure)
     int att_splits_max = 0;
-    uint16_t* x_stage = nullptr;  // BF16 [d] host-buffer staging
+    uint16_t* x_stage = nullptr;  // BF16 [d] step-input staging (device and host-buffer steps)
     float* logits_stage = nullptr;
     float* hidden_stage = nullptr;
     StepGraph graph;
