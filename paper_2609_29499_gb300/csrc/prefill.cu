@@ -332,9 +332,12 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const float* __restri
 
 // Projected rows Y [T][qkv rows] (group-major panel order, scaled) -> rotated queries (FP32,
 // [m_q][T][dh]) and the plan-bound KV cache (BF16 keys rotated, values as is) at 0..T-1.
+// Rotary embedding on q and k, KV-cache write (BF16); optionally also the tensor-core
+// attention's operands: Qh = FP16(q * qscale) [head][T][dh], Kh = FP16 of the cached BF16
+// keys [group][T][dh], VT = FP16 of the cached BF16 values transposed, [group][dh][Tp].
 __global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int g, int dh,
                                const float2* __restrict__ rope, float* Qf, uint16_t* Kc, uint16_t* Vc,
-                               int max_tokens) {
+                               int max_tokens, __half* Qh, float qscale, __half* Kh, __half* VT, int Tp) {
     const int t = blockIdx.x, jl = blockIdx.y;
     const int half = dh >> 1;
     for (int w = threadIdx.x; w < (g + 2) * half; w += blockDim.x) {
@@ -348,14 +351,30 @@ __global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int 
             y1 = b;
         }
         if (hh < g) {
-            float* q = Qf + ((int64_t)(jl * g + hh) * T + t) * dh;
-            q[i] = y0;
-            q[i + half] = y1;
+            const int64_t qrow = (int64_t)(jl * g + hh) * T + t;
+            if (Qf) {
+                float* q = Qf + qrow * dh;
+                q[i] = y0;
+                q[i + half] = y1;
+            }
+            if (Qh) {
+                Qh[qrow * dh + i] = __float2half_rn(y0 * qscale);
+                Qh[qrow * dh + i + half] = __float2half_rn(y1 * qscale);
+            }
         } else {
             uint16_t* dst = (hh == g ? Kc : Vc) + ((int64_t)jl * max_tokens + t) * dh;
             __nv_bfloat16 b0 = __float2bfloat16_rn(y0), b1 = __float2bfloat16_rn(y1);
             dst[i] = *reinterpret_cast<uint16_t*>(&b0);
             dst[i + half] = *reinterpret_cast<uint16_t*>(&b1);
+            const __half h0 = __float2half_rn(__bfloat162float(b0)), h1 = __float2half_rn(__bfloat162float(b1));
+            if (hh == g && Kh) {
+                Kh[((int64_t)jl * T + t) * dh + i] = h0;
+                Kh[((int64_t)jl * T + t) * dh + i + half] = h1;
+            }
+            if (hh == g + 1 && VT) {
+                VT[((int64_t)jl * dh + i) * Tp + t] = h0;
+                VT[((int64_t)jl * dh + i + half) * Tp + t] = h1;
+            }
         }
     }
 }
@@ -596,6 +615,260 @@ __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const fl
     }
 }
 
+// ------------------------------------------------------------------ causal attention on tcgen05
+// One CTA: 128 queries of one kept head, head dim 128. Keys stream in tiles of 64:
+//  * warp 0 loads Q once and, per tile, the FP16 key tile and the transposed FP16 value tile
+//    (TMA, 128-byte swizzle) into a 2-stage ring;
+//  * warp 1 issues S_j = Q K_j^T (M 128, N 64) into one of two TMEM score buffers, and
+//    O += P_{j-1} V_{j-1} (M 128, N 128) into the TMEM output;
+//  * warps 2-5 own one query row per thread: they read S_j from TMEM, apply the causal mask,
+//    keep a running maximum that may lag the true one by up to 8 (log2 units; O in TMEM is
+//    rescaled only when it would lag more), write P_j = 2^(S - m) as FP16 into shared memory
+//    in the swizzled operand layout, and finally divide O by the running sum.
+// Every wait is bounded and reports to the device error word.
+constexpr int AT_KT = 64;
+constexpr int AT_Q_BYTES = 128 * 128 * 2;
+constexpr int AT_K_BYTES = AT_KT * 128 * 2;
+constexpr int AT_VT_BYTES = 128 * AT_KT * 2;
+constexpr int AT_STAGE_BYTES = AT_K_BYTES + AT_VT_BYTES;
+constexpr int AT_P_BYTES = 128 * AT_KT * 2;
+constexpr int AT_SMEM = AT_Q_BYTES + 2 * AT_STAGE_BYTES + 2 * AT_P_BYTES + 1024;
+constexpr uint32_t AT_TMEM_COLS = 256;  // S0 [0, 64), S1 [64, 128), O [128, 256)
+constexpr uint32_t IDESC_S = idesc_f16(128, AT_KT), IDESC_O = idesc_f16(128, 128);
+constexpr float AT_LAZY = 8.0f;
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]),
+        "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
+        "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t tmem, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+        "l"(ad), "l"(bd), "r"(idesc), "r"(accum)
+        : "memory");
+}
+__device__ __forceinline__ void mbar_arrive1(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__global__ void __launch_bounds__(192, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmVT, int T, int g, __half* O, int ldo, int* err) {
+    extern __shared__ uint8_t smraw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sq = sm;
+    uint8_t* sst = sm + AT_Q_BYTES;                     // stage s: K at +0 (two 8 KB halves), VT at +AT_K_BYTES
+    uint8_t* sp = sm + AT_Q_BYTES + 2 * AT_STAGE_BYTES;  // P buffer b at + b * AT_P_BYTES
+    __shared__ __align__(8) uint64_t bar_q, kv_full[2], kv_empty[2], s_full[2], s_empty[2], p_full[2], p_empty[2],
+        o_done;
+    __shared__ uint32_t tmem_base;
+    __shared__ int abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.x, jl = h / g;
+    const int q0 = (gridDim.y - 1 - blockIdx.y) * 128;  // the longest query blocks of every head first
+    const int kend = min(T, q0 + 128);
+    const int ntile = (kend + AT_KT - 1) / AT_KT;
+    auto B = [](uint64_t& b) { return smem_u32(&b); };
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        mbar_init(B(bar_q), 1);
+        mbar_init(B(o_done), 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(B(kv_full[i]), 1);
+            mbar_init(B(kv_empty[i]), 1);
+            mbar_init(B(s_full[i]), 1);
+            mbar_init(B(s_empty[i]), 4);
+            mbar_init(B(p_full[i]), 4);
+            mbar_init(B(p_empty[i]), 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
+                     "r"(AT_TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {  // ---- TMA producer
+            mbar_expect_tx(B(bar_q), AT_Q_BYTES);
+            tma_load_2d(smem_u32(sq), &tmQ, 0, h * T + q0, B(bar_q));
+            tma_load_2d(smem_u32(sq + AT_Q_BYTES / 2), &tmQ, 64, h * T + q0, B(bar_q));
+            for (int j = 0; j < ntile; ++j) {
+                const int s = j & 1;
+                if (j >= 2) mbar_wait(B(kv_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
+                const uint32_t fb = B(kv_full[s]);
+                mbar_expect_tx(fb, AT_STAGE_BYTES);
+                uint8_t* st = sst + s * AT_STAGE_BYTES;
+                tma_load_2d(smem_u32(st), &tmK, 0, jl * T + j * AT_KT, fb);
+                tma_load_2d(smem_u32(st + AT_K_BYTES / 2), &tmK, 64, jl * T + j * AT_KT, fb);
+                tma_load_2d(smem_u32(st + AT_K_BYTES), &tmVT, j * AT_KT, jl * 128, fb);
+            }
+            // no copy may outlive the CTA
+            mbar_wait(B(bar_q), 0, &abort_flag, err, false);
+            for (int j = max(0, ntile - 2); j < ntile; ++j)
+                mbar_wait(B(kv_full[j & 1]), (j >> 1) & 1, &abort_flag, err, false);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // ---- MMA issuer
+            mbar_wait(B(bar_q), 0, &abort_flag, err);
+            tc_fence_after();
+            const uint32_t qa = smem_u32(sq);
+            for (int j = 0; j <= ntile; ++j) {
+                if (j < ntile) {  // S_j = Q K_j^T into score buffer j % 2
+                    const int s = j & 1;
+                    mbar_wait(B(kv_full[s]), (j >> 1) & 1, &abort_flag, err);
+                    if (j >= 2) mbar_wait(B(s_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
+                    tc_fence_after();
+                    const uint32_t kb = smem_u32(sst + s * AT_STAGE_BYTES);
+#pragma unroll
+                    for (int blk = 0; blk < 2; ++blk)
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc_mma(tmem + 64u * s, sw128_desc(qa + blk * (AT_Q_BYTES / 2) + kk * 32),
+                                   sw128_desc(kb + blk * (AT_K_BYTES / 2) + kk * 32), IDESC_S, (blk | kk) ? 1u : 0u);
+                    tc_commit(B(s_full[s]));
+                }
+                if (j >= 1) {  // O += P_{j-1} V_{j-1}
+                    const int jp = j - 1, s = jp & 1;
+                    mbar_wait(B(p_full[s]), (jp >> 1) & 1, &abort_flag, err);
+                    tc_fence_after();
+                    const uint32_t pa = smem_u32(sp + s * AT_P_BYTES);
+                    const uint32_t vb = smem_u32(sst + s * AT_STAGE_BYTES + AT_K_BYTES);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        tc_mma(tmem + 128u, sw128_desc(pa + kk * 32), sw128_desc(vb + kk * 32), IDESC_O,
+                               (jp > 0 || kk > 0) ? 1u : 0u);
+                    tc_commit(B(p_empty[s]));
+                    tc_commit(B(kv_empty[s]));
+                }
+            }
+            tc_commit(B(o_done));
+        }
+    } else {  // ---- softmax warps 2..5: TMEM lanes 32 (warp % 4) ..
+        const int qw = warp & 3;
+        const int row = 32 * qw + lane, qi = q0 + row;
+        const uint32_t trow = tmem + ((uint32_t)(32 * qw) << 16);
+        float m_run = -INFINITY, l_run = 0.f;
+        for (int j = 0; j < ntile; ++j) {
+            const int s = j & 1;
+            mbar_wait(B(s_full[s]), (j >> 1) & 1, &abort_flag, err);
+            tc_fence_after();
+            uint32_t v0[32], v1[32];
+            tmem_ld32(trow + 64u * s, v0);
+            tmem_ld32(trow + 64u * s + 32u, v1);
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive1(B(s_empty[s]));
+            float x[64];
+            const int k0 = j * AT_KT;
+            float mt = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                const float v = __uint_as_float(c < 32 ? v0[c] : v1[c - 32]);
+                const int k = k0 + c;
+                x[c] = (k > qi || k >= kend) ? -INFINITY : v;  // causal
+                mt = fmaxf(mt, x[c]);
+            }
+            if (j == 0) {
+                m_run = mt;  // key 0 is visible to every row
+            } else {
+                const bool need = mt > m_run + AT_LAZY;
+                if (__any_sync(0xffffffffu, need)) {
+                    // O must hold P_{j-1} V_{j-1} before it is rescaled
+                    mbar_wait(B(p_empty[(j - 1) & 1]), ((j - 1) >> 1) & 1, &abort_flag, err);
+                    tc_fence_after();
+                    const float corr = need ? exp2f(m_run - mt) : 1.0f;
+#pragma unroll 1
+                    for (int c0 = 0; c0 < 128; c0 += 32) {
+                        uint32_t o[32];
+                        tmem_ld32(trow + 128u + c0, o);
+                        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
+                        tmem_st32(trow + 128u + c0, o);
+                    }
+                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    if (need) {
+                        l_run *= corr;
+                        m_run = mt;
+                    }
+                }
+            }
+            // P_j = 2^(S - m) in FP16 (<= 2^8 by the lag bound), row-sum in FP32
+            uint32_t pw[32];
+            float ls = 0.f;
+#pragma unroll
+            for (int c = 0; c < 64; c += 2) {
+                const float p0 = exp2f(x[c] - m_run), p1 = exp2f(x[c + 1] - m_run);
+                ls += p0 + p1;
+                pw[c >> 1] = pack_h2(p0, p1);
+            }
+            l_run += ls;
+            if (j >= 2) mbar_wait(B(p_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);  // P buffer free
+            uint8_t* prow = sp + s * AT_P_BYTES + row * 128;
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) =
+                    make_uint4(pw[4 * c], pw[4 * c + 1], pw[4 * c + 2], pw[4 * c + 3]);
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive1(B(p_full[s]));
+        }
+        mbar_wait(B(o_done), 0, &abort_flag, err);
+        tc_fence_after();
+        const float inv = 1.0f / l_run;
+#pragma unroll 1
+        for (int c0 = 0; c0 < 128; c0 += 32) {
+            uint32_t o[32];
+            tmem_ld32(trow + 128u + c0, o);
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            if (qi < T) {
+                uint32_t hw[16];
+#pragma unroll
+                for (int c = 0; c < 32; c += 2)
+                    hw[c >> 1] = pack_h2(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv);
+                uint4* dst = reinterpret_cast<uint4*>(O + (int64_t)qi * ldo + h * 128 + c0);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) dst[k] = make_uint4(hw[4 * k], hw[4 * k + 1], hw[4 * k + 2], hw[4 * k + 3]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(AT_TMEM_COLS) : "memory");
+}
+
 // ------------------------------------------------------------------ host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::mutex g_enc_mu;
@@ -732,6 +1005,22 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
     TASP_CUDA(cudaMallocAsync((void**)&H, (size_t)T * ld_h * 2, s));
     TASP_CUDA(cudaMemsetAsync(O, 0, (size_t)T * ld_o * 2, s));
     TASP_CUDA(cudaMemsetAsync(H, 0, (size_t)T * ld_h * 2, s));
+    // tensor-core attention operands (head dim 128): scaled FP16 queries, FP16 keys and
+    // transposed FP16 values (rows padded to Tp keys, padding zero)
+    const bool tc_attn = sh.dh == 128;
+    const int Tp = (T + 7) & ~7;
+    __half *Qh = nullptr, *Kh = nullptr, *VT = nullptr;
+    if (tc_attn) {
+        TASP_CUDA(cudaMallocAsync((void**)&Qh, (size_t)sh.Hq * T * 128 * 2, s));
+        TASP_CUDA(cudaMallocAsync((void**)&Kh, (size_t)sh.Hkv * T * 128 * 2, s));
+        TASP_CUDA(cudaMallocAsync((void**)&VT, (size_t)sh.Hkv * 128 * Tp * 2, s));
+        TASP_CUDA(cudaMemsetAsync(VT, 0, (size_t)sh.Hkv * 128 * Tp * 2, s));
+        static bool attr = false;
+        if (!attr) {
+            TASP_CUDA(cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM));
+            attr = true;
+        }
+    }
     const float qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
     {
         static bool attr = false;  // the key/value ring exceeds the default 48 KB of shared memory
@@ -753,15 +1042,21 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
             ga.M = T; ga.N = lp.qkv_rows; ga.K = sh.d; ga.scale = lp.qkv_s; ga.out = Y; ga.ldo = ld_y;
             ga.mode = EP_STORE; ga.err = se.err;
             if ((rc = launch_gemm(Xh, ld_x, T, f.qkv, f.ld_d, lp.qkv_rows, sh.d, ga, s))) break;
-            rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, Qf, se.K[l], se.V[l],
-                                                            se.max_tokens);
-            const int qb = (T + PA_QB - 1) / PA_QB;
-            if (sh.dh == 128)
-                attn_prefill_kernel<128><<<dim3(lp.m_kv * sh.g(), qb), PA_WARPS * 32, PaCfg<128>::SMEM, s>>>(
-                    Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
-            else
+            rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, tc_attn ? nullptr : Qf,
+                                                            se.K[l], se.V[l], se.max_tokens, Qh, qscale, Kh, VT, Tp);
+            if (tc_attn) {
+                CUtensorMap mq, mk, mv;
+                const int mq_rows = lp.m_kv * sh.g() * T;
+                if ((rc = make_map(&mq, Qh, mq_rows, 128, 128, 128))) break;
+                if ((rc = make_map(&mk, Kh, lp.m_kv * T, 128, 128, AT_KT))) break;
+                if ((rc = make_map(&mv, VT, lp.m_kv * 128, Tp, Tp, 128))) break;
+                attn_tc_kernel<<<dim3(lp.m_kv * sh.g(), (T + 127) / 128), 192, AT_SMEM, s>>>(mq, mk, mv, T, sh.g(), O,
+                                                                                           ld_o, se.err);
+            } else {
+                const int qb = (T + PA_QB - 1) / PA_QB;
                 attn_prefill_kernel<64><<<dim3(lp.m_kv * sh.g(), qb), PA_WARPS * 32, PaCfg<64>::SMEM, s>>>(
                     Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
+            }
             TASP_CUDA(cudaGetLastError());
             GemmArgs go{};
             go.M = T; go.N = sh.d; go.K = lp.o_K; go.scale = lp.o_s; go.out = X; go.ldo = sh.d;
@@ -792,6 +1087,9 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
     cudaFreeAsync(Qf, s);
     cudaFreeAsync(O, s);
     cudaFreeAsync(H, s);
+    if (Qh) cudaFreeAsync(Qh, s);
+    if (Kh) cudaFreeAsync(Kh, s);
+    if (VT) cudaFreeAsync(VT, s);
     return rc;
 }
 
