@@ -87,21 +87,13 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
 }
 
 // ------------------------------------------------------------------ GEMM
-// A CTA computes an (MT x 128) x 256 output tile: MT = 2 sub-tiles of 128 rows share every
-// 256 x 64 weight tile (two M = 128 accumulators fill the 512 TMEM columns), which halves
-// the operand bytes per FLOP of a single 128 x 256 tile; MT = 1 is kept for GEMMs with too
-// few tiles to fill the GPU. CTAs run M-fastest, so the CTAs in flight share weight tiles.
+// Persistent GEMM on the 5th-generation tensor cores: one CTA per SM walks 128 x 256 output
+// tiles (M fastest, so the CTAs in flight share weight tiles in L2), with two 256-column
+// TMEM accumulators: the MMA warp fills one while the epilogue warps drain the other.
 constexpr int BM = 128, BN = 256, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int GEMM_THREADS = 192;
-template <int MT>
-struct GemmCfg {
-    static constexpr int STAGES = MT == 2 ? 3 : 4;
-    static constexpr int STAGE_BYTES = MT * A_BYTES + B_BYTES;
-    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;  // + alignment slack
-    static constexpr uint32_t TMEM_COLS = 256 * MT;
-};
 constexpr uint32_t IDESC = idesc_f16(BM, BN);
 
 enum EpiMode { EP_STORE = 0, EP_RESID = 1, EP_SWIGLU = 2 };
@@ -189,32 +181,41 @@ __device__ __forceinline__ void gemm_epi32(const GemmArgs& g, int row, int nb, c
     }
 }
 
-template <int MT>
+// Warp 0 streams the A (activation) and B (weight) k-blocks of all the CTA's tiles through a
+// 4-stage TMA ring that runs on across tile boundaries; warp 1 issues tcgen05.mma; warps 2-5
+// read an accumulator with tcgen05.ld and run the epilogue.
+constexpr int PG_STAGES = 4;
+constexpr int PG_STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int PG_SMEM = PG_STAGES * PG_STAGE_BYTES + 1024;
+
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmArgs g) {
-    using C = GemmCfg<MT>;
-    constexpr int STAGES = C::STAGES;
+    gemm_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const GemmArgs g) {
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_acc;
+    __shared__ __align__(8) uint64_t bar_full[PG_STAGES], bar_empty[PG_STAGES], acc_full[2], acc_empty[2];
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * (BM * MT), n0 = blockIdx.y * BN;
+    const int mt = (g.M + BM - 1) / BM, ntl = (g.N + BN - 1) / BN;
+    const int ntiles = mt * ntl;
     const int nk = (g.K + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
-        for (int s = 0; s < STAGES; ++s) {
+        for (int s = 0; s < PG_STAGES; ++s) {
             mbar_init(smem_u32(&bar_full[s]), 1);
             mbar_init(smem_u32(&bar_empty[s]), 1);
         }
-        mbar_init(smem_u32(&bar_acc), 1);
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_u32(&acc_full[a]), 1);
+            mbar_init(smem_u32(&acc_empty[a]), 4);
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
-                     "r"(C::TMEM_COLS)
+                     "r"(512)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -224,56 +225,63 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const uint32_t tmem = tmem_base;
 
     if (warp == 0) {
-        if (lane == 0) {  // ---- TMA producer
-            for (int kb = 0; kb < nk; ++kb) {
-                const int s = kb % STAGES;
-                if (kb >= STAGES) mbar_wait(smem_u32(&bar_empty[s]), ((kb / STAGES) - 1) & 1, &abort_flag, g.err);
-                const uint32_t fb = smem_u32(&bar_full[s]);
-                mbar_expect_tx(fb, C::STAGE_BYTES);
-                const uint32_t a = smem_u32(sm + s * C::STAGE_BYTES);
-#pragma unroll
-                for (int mt = 0; mt < MT; ++mt) tma_load_2d(a + mt * A_BYTES, &tmA, kb * BK, m0 + BM * mt, fb);
-                tma_load_2d(a + MT * A_BYTES, &tmB, kb * BK, n0, fb);
+        if (lane == 0) {  // ---- TMA producer: k-blocks of all this CTA's tiles, back to back
+            int kbg = 0;  // k-blocks issued so far
+            for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+                const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
+                for (int kb = 0; kb < nk; ++kb, ++kbg) {
+                    const int s = kbg % PG_STAGES;
+                    if (kbg >= PG_STAGES)
+                        mbar_wait(smem_u32(&bar_empty[s]), ((kbg / PG_STAGES) - 1) & 1, &abort_flag, g.err);
+                    const uint32_t fb = smem_u32(&bar_full[s]);
+                    mbar_expect_tx(fb, PG_STAGE_BYTES);
+                    const uint32_t a = smem_u32(sm + s * PG_STAGE_BYTES);
+                    tma_load_2d(a, &tmA, kb * BK, m0, fb);
+                    tma_load_2d(a + A_BYTES, &tmB, kb * BK, n0, fb);
+                }
             }
-            for (int kb = max(0, nk - STAGES); kb < nk; ++kb)  // no copy may outlive the CTA
-                mbar_wait(smem_u32(&bar_full[kb % STAGES]), (kb / STAGES) & 1, &abort_flag, g.err, false);
+            for (int k = max(0, kbg - PG_STAGES); k < kbg; ++k)  // no copy may outlive the CTA
+                mbar_wait(smem_u32(&bar_full[k % PG_STAGES]), (k / PG_STAGES) & 1, &abort_flag, g.err, false);
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---- MMA issuer
-            for (int kb = 0; kb < nk; ++kb) {
-                const int s = kb % STAGES;
-                mbar_wait(smem_u32(&bar_full[s]), (kb / STAGES) & 1, &abort_flag, g.err);
+            int kbg = 0, it = 0;
+            for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
+                const int a = it & 1;
+                if (it >= 2) mbar_wait(smem_u32(&acc_empty[a]), ((it >> 1) - 1) & 1, &abort_flag, g.err);
                 tc_fence_after();
-                const uint32_t a = smem_u32(sm + s * C::STAGE_BYTES), b = a + MT * A_BYTES;
+                for (int kb = 0; kb < nk; ++kb, ++kbg) {
+                    const int s = kbg % PG_STAGES;
+                    mbar_wait(smem_u32(&bar_full[s]), (kbg / PG_STAGES) & 1, &abort_flag, g.err);
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(sm + s * PG_STAGE_BYTES), sb = sa + A_BYTES;
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk) {
-                    const uint64_t bd = sw128_desc(b + kk * 32);
-                    const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
-#pragma unroll
-                    for (int mt = 0; mt < MT; ++mt) {
-                        const uint64_t ad = sw128_desc(a + mt * A_BYTES + kk * 32);
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
                         asm volatile(
                             "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256u * mt),
-                            "l"(ad), "l"(bd), "r"(IDESC), "r"(accum)
+                            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256u * a),
+                            "l"(sw128_desc(sa + kk * 32)), "l"(sw128_desc(sb + kk * 32)), "r"(IDESC), "r"(accum)
                             : "memory");
                     }
+                    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                                     smem_u32(&bar_empty[s]))
+                                 : "memory");
                 }
                 asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                                 smem_u32(&bar_empty[s]))
+                                 smem_u32(&acc_full[a]))
                              : "memory");
             }
-            asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                             smem_u32(&bar_acc))
-                         : "memory");
         }
-    } else {  // ---- epilogue: warps 2..5, warp w reads TMEM lanes 32 (w % 4) ..
-        mbar_wait(smem_u32(&bar_acc), 0, &abort_flag, g.err);
-        tc_fence_after();
+    } else {  // ---- epilogue warps 2..5: TMEM lanes 32 (warp % 4) ..
         const int q = warp & 3;
-#pragma unroll 1
-        for (int mt = 0; mt < MT; ++mt) {
-            const int row = m0 + BM * mt + 32 * q + lane;
+        int it = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
+            const int a = it & 1;
+            const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
+            mbar_wait(smem_u32(&acc_full[a]), (it >> 1) & 1, &abort_flag, g.err);
+            tc_fence_after();
+            const int row = m0 + 32 * q + lane;
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 32) {
                 uint32_t r[32];
@@ -285,17 +293,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                       "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
                       "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
                       "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-                    : "r"(tmem + ((uint32_t)(32 * q) << 16) + 256u * mt + (uint32_t)c0));
+                    : "r"(tmem + ((uint32_t)(32 * q) << 16) + 256u * a + (uint32_t)c0));
                 asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
                 if (row < g.M) gemm_epi32(g, row, n0 + c0, r);
             }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
         }
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TMEM_COLS) : "memory");
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
 }
 
 // ------------------------------------------------------------------ elementwise kernels
@@ -910,36 +921,19 @@ int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
-    // two row sub-tiles per CTA unless wave quantization eats their gain: cost = waves x
-    // tile time, a one-sub-tile CTA taking half the time of a two-sub-tile CTA but ~1.25x
-    // the time per FLOP (87 against 131 FLOP per operand byte)
-    const int nt = (N + BN - 1) / BN;
-    const int tiles1 = ((M + BM - 1) / BM) * nt, tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * nt;
-    const double cost1 = 1.25 * ((tiles1 + di.sms - 1) / di.sms), cost2 = 2.0 * ((tiles2 + di.sms - 1) / di.sms);
-    const int MT = cost2 <= cost1 ? 2 : 1;
     CUtensorMap ta, tb;
     if ((rc = make_map(&ta, A, M, K, lda, BM))) return rc;
     if ((rc = make_map(&tb, B, N, K, ldb, BN))) return rc;
     ga.vec = ga.mode == EP_SWIGLU ? ((reinterpret_cast<uintptr_t>(ga.hout) & 15) == 0 && ga.ldh % 8 == 0)
                                   : ((reinterpret_cast<uintptr_t>(ga.out) & 15) == 0 && ga.ldo % 4 == 0);
     ga.vec = ga.vec && (reinterpret_cast<uintptr_t>(ga.scale) & 15) == 0;
-    static bool attr[2] = {false, false};
-    const dim3 grid((M + BM * MT - 1) / (BM * MT), (N + BN - 1) / BN);
-    if (MT == 2) {
-        if (!attr[1]) {
-            TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           GemmCfg<2>::SMEM));
-            attr[1] = true;
-        }
-        gemm_tc_kernel<2><<<grid, GEMM_THREADS, GemmCfg<2>::SMEM, s>>>(ta, tb, ga);
-    } else {
-        if (!attr[0]) {
-            TASP_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           GemmCfg<1>::SMEM));
-            attr[0] = true;
-        }
-        gemm_tc_kernel<1><<<grid, GEMM_THREADS, GemmCfg<1>::SMEM, s>>>(ta, tb, ga);
+    static bool attr = false;
+    if (!attr) {
+        TASP_CUDA(cudaFuncSetAttribute(gemm_persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, PG_SMEM));
+        attr = true;
     }
+    const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+    gemm_persist_kernel<<<std::min(tiles, di.sms), GEMM_THREADS, PG_SMEM, s>>>(ta, tb, ga);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }
