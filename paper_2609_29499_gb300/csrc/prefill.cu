@@ -341,14 +341,48 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const float* __restri
     }
 }
 
+// The same with 16-byte loads and 8-byte stores (d % 4 == 0, FP32 rows; 16-byte aligned X and
+// gamma, 8-byte aligned out rows).
+__global__ void __launch_bounds__(256) rmsnorm_rows_vec_kernel(const float* __restrict__ X, int d,
+                                                                const float* __restrict__ gamma, float eps,
+                                                                __half* out, int ldo) {
+    __shared__ float red[8];
+    const int t = blockIdx.x, tid = threadIdx.x;
+    const float4* xr = reinterpret_cast<const float4*>(X + (int64_t)t * d);
+    const int n4 = d >> 2;
+    float ss = 0.f;
+    for (int f = tid; f < n4; f += 256) {
+        const float4 v = xr[f];
+        ss = fmaf(v.x, v.x, ss);
+        ss = fmaf(v.y, v.y, ss);
+        ss = fmaf(v.z, v.z, ss);
+        ss = fmaf(v.w, v.w, ss);
+    }
+    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if ((tid & 31) == 0) red[tid >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)d) + eps);
+    const float4* g4 = reinterpret_cast<const float4*>(gamma);
+    uint2* o2 = reinterpret_cast<uint2*>(out + (int64_t)t * ldo);
+    for (int f = tid; f < n4; f += 256) {
+        const float4 v = xr[f], gm = g4[f];
+        const __half2 a = __floats2half2_rn((v.x * inv) * gm.x, (v.y * inv) * gm.y);
+        const __half2 b = __floats2half2_rn((v.z * inv) * gm.z, (v.w * inv) * gm.w);
+        o2[f] = make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&b));
+    }
+}
+
 // Projected rows Y [T][qkv rows] (group-major panel order, scaled) -> rotated queries (FP32,
 // [m_q][T][dh]) and the plan-bound KV cache (BF16 keys rotated, values as is) at 0..T-1.
 // Rotary embedding on q and k, KV-cache write (BF16); optionally also the tensor-core
-// attention's operands: Qh = FP16(q * qscale) [head][T][dh], Kh = FP16 of the cached BF16
-// keys [group][T][dh], VT = FP16 of the cached BF16 values transposed, [group][dh][Tp].
+// attention's operands Qh = FP16(q * qscale) [head][T][dh] and Kh = FP16 of the cached BF16
+// keys [group][T][dh] (the transposed values come from v_transpose_kernel).
 __global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int g, int dh,
                                const float2* __restrict__ rope, float* Qf, uint16_t* Kc, uint16_t* Vc,
-                               int max_tokens, __half* Qh, float qscale, __half* Kh, __half* VT, int Tp) {
+                               int max_tokens, __half* Qh, float qscale, __half* Kh) {
     const int t = blockIdx.x, jl = blockIdx.y;
     const int half = dh >> 1;
     for (int w = threadIdx.x; w < (g + 2) * half; w += blockDim.x) {
@@ -382,11 +416,34 @@ __global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int 
                 Kh[((int64_t)jl * T + t) * dh + i] = h0;
                 Kh[((int64_t)jl * T + t) * dh + i + half] = h1;
             }
-            if (hh == g + 1 && VT) {
-                VT[((int64_t)jl * dh + i) * Tp + t] = h0;
-                VT[((int64_t)jl * dh + i + half) * Tp + t] = h1;
-            }
         }
+    }
+}
+
+// FP16 of the cached BF16 values of one KV group, transposed: VT [group][128][Tp] from
+// V [group][max_tokens][128]; 64 tokens per CTA through a shared tile (coalesced both ways).
+__global__ void __launch_bounds__(256) v_transpose_kernel(const uint16_t* __restrict__ V, int max_tokens, int T,
+                                                           __half* VT, int Tp) {
+    __shared__ __half tile[128][64 + 8];
+    const int t0 = blockIdx.x * 64, jl = blockIdx.y, tid = threadIdx.x;
+    const uint16_t* src = V + ((int64_t)jl * max_tokens + t0) * 128;
+    for (int c = tid; c < 64 * 16; c += 256) {  // 64 tokens x 16 chunks of 8 dims
+        const int tt = c >> 4, dc = (c & 15) * 8;
+        uint4 w = make_uint4(0, 0, 0, 0);
+        if (t0 + tt < T) w = *reinterpret_cast<const uint4*>(src + (int64_t)tt * 128 + dc);
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            tile[dc + 2 * k][tt] = __float2half_rn(__uint_as_float(u[k] << 16));
+            tile[dc + 2 * k + 1][tt] = __float2half_rn(__uint_as_float(u[k] & 0xffff0000u));
+        }
+    }
+    __syncthreads();
+    for (int c = tid; c < 128 * 8; c += 256) {  // 128 dims x 8 chunks of 8 tokens
+        const int dd = c >> 3, tc = (c & 7) * 8;
+        if (t0 + tc + 8 <= Tp)
+            *reinterpret_cast<uint4*>(VT + ((int64_t)jl * 128 + dd) * Tp + t0 + tc) =
+                *reinterpret_cast<const uint4*>(&tile[dd][tc]);
     }
 }
 
@@ -1016,6 +1073,10 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
         }
     }
     const float qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
+    bool vec_norm = sh.d % 4 == 0 && ld_x % 4 == 0;
+    for (const LayerPlan& lp : pl.layers)
+        vec_norm = vec_norm && (reinterpret_cast<uintptr_t>(lp.g_attn) & 15) == 0 &&
+                   (reinterpret_cast<uintptr_t>(lp.g_mlp) & 15) == 0;
     {
         static bool attr = false;  // the key/value ring exceeds the default 48 KB of shared memory
         if (!attr) {
@@ -1029,7 +1090,10 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
     for (int l = 0; l < sh.L && !rc; ++l) {
         const LayerPlan& lp = pl.layers[l];
         const F16Panels& f = pl.f16[l];
-        rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, l == 0 ? d_embeds : nullptr, X, sh.d, lp.g_attn, sh.eps, Xh, ld_x);
+        if (l == 0 || !vec_norm)  // the first layer also widens the BF16 embeddings into X
+            rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, l == 0 ? d_embeds : nullptr, X, sh.d, lp.g_attn, sh.eps, Xh, ld_x);
+        else
+            rmsnorm_rows_vec_kernel<<<T, 256, 0, s>>>(X, sh.d, lp.g_attn, sh.eps, Xh, ld_x);
         TASP_CUDA(cudaGetLastError());
         if (lp.m_kv > 0) {
             GemmArgs ga{};
@@ -1037,8 +1101,9 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
             ga.mode = EP_STORE; ga.err = se.err;
             if ((rc = launch_gemm(Xh, ld_x, T, f.qkv, f.ld_d, lp.qkv_rows, sh.d, ga, s))) break;
             rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, tc_attn ? nullptr : Qf,
-                                                            se.K[l], se.V[l], se.max_tokens, Qh, qscale, Kh, VT, Tp);
+                                                            se.K[l], se.V[l], se.max_tokens, Qh, qscale, Kh);
             if (tc_attn) {
+                v_transpose_kernel<<<dim3((T + 63) / 64, lp.m_kv), 256, 0, s>>>(se.V[l], se.max_tokens, T, VT, Tp);
                 CUtensorMap mq, mk, mv;
                 const int mq_rows = lp.m_kv * sh.g() * T;
                 if ((rc = make_map(&mq, Qh, mq_rows, 128, 128, 128))) break;
@@ -1058,7 +1123,10 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
             if ((rc = launch_gemm(O, ld_o, T, f.o, f.ld_o, sh.d, lp.o_K, go, s))) break;
         }
         if (lp.c > 0) {
-            rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, nullptr, nullptr, sh.d, lp.g_mlp, sh.eps, Xh, ld_x);
+            if (vec_norm)
+                rmsnorm_rows_vec_kernel<<<T, 256, 0, s>>>(X, sh.d, lp.g_mlp, sh.eps, Xh, ld_x);
+            else
+                rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, nullptr, nullptr, sh.d, lp.g_mlp, sh.eps, Xh, ld_x);
             TASP_CUDA(cudaGetLastError());
             GemmArgs gg{};
             gg.M = T; gg.N = lp.gu_rows; gg.K = sh.d; gg.scale = lp.gu_s; gg.hout = H; gg.ldh = ld_h;
