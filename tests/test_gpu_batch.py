@@ -249,3 +249,28 @@ def test_70b_batch_of_five_full_depth(tasp):
         s.release()
     assert np.isfinite(got).all() and np.isfinite(logits).all()
     plan.release()
+
+
+def test_70b_width_row_indexed_batch_is_bit_identical(tasp):
+    # the mixed-turn bench's configuration: a group of four sessions on a plan whose Q/K/V and
+    # gate/up panels are row maps into the shared store reads the same bytes as materialized
+    # panels, so every output bit agrees (the paper's one-store check, at 70B widths)
+    wl = synth.CFG5
+    sh = _cut(wl.shape, 2)
+    recipe = wl.masks[2]
+    n, steps = 4, 2
+    t_priors = [1500, 700, 256, 2000]
+    kv_seeds = [wl.kv_seed + i for i in range(n)]
+    xb = synth.step_inputs_bf16(wl.x_seed, steps, n, sh.d)
+    outs = []
+    for mode in (tasp.PANELS_COMPACT, tasp.PANELS_ROW_INDEXED):
+        plan = lib_plan(tasp, sh, recipe, panel_mode=mode)
+        ss = _sessions(tasp, plan, t_priors, kv_seeds, steps)
+        outs.append(_run(tasp, ss, xb, sh.vocab))
+        for s in ss:
+            assert s.device_error() == 0
+            s.release()
+        plan.release()
+    (h0, l0), (h1, l1) = outs
+    assert np.array_equal(h0.view(np.uint32), h1.view(np.uint32))
+    assert np.array_equal(l0.view(np.uint32), l1.view(np.uint32))
