@@ -89,12 +89,14 @@ __device__ __forceinline__ uint32_t cluster_rank() {
 }
 __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
     uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
+// (volatile: kept after the cluster barrier that orders it after the remote writes; no
+// memory clobber, so independent loads still issue back to back)
 __device__ __forceinline__ float ld_cluster(uint32_t addr) {
     float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
     return v;
 }
 
@@ -107,6 +109,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     __shared__ float cm[8], cl[8];              // this CTA's merged (max, sum) per head
     __shared__ __align__(16) float cacc[8][DH];  // this CTA's merged unnormalized output
     __shared__ float Mh[8], Lh[8], wts[CLUSTERS_MAX][8];
+    __shared__ float we[AT_WARPS][8];        // per-warp weights of each head in the CTA merge
+    __shared__ float rw[CS][8], rl[CS][8];   // per-rank weights and sums in the cluster merge
+    __shared__ float Mt[8], Lt[8];           // cluster-wide (max, sum) per head
     __shared__ int is_last;
     const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x, bz = blockIdx.z;
     const int NC = S / CS, cid = split / CS;
@@ -241,72 +246,102 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
 
     // ---- merge the warps of this CTA (the tile memory is reused)
+    constexpr int WS = DH + 4;  // padded row of a warp's partial outputs: conflict-free float2 stores
     __syncthreads();
-    float* wacc = reinterpret_cast<float*>(sm);  // [AT_WARPS][8][DH]
+    float* wacc = reinterpret_cast<float*>(sm);  // [AT_WARPS][8][WS]
 #pragma unroll
     for (int nt = 0; nt < C::NT; ++nt) {
         const int dim = nt * 8 + qc;
-        float* dst = wacc + (warp * 8 + h) * DH + dim;
-        dst[0] = any ? acc[nt][0] + acc[nt][2] : 0.f;
-        dst[1] = any ? acc[nt][1] + acc[nt][3] : 0.f;
+        *reinterpret_cast<float2*>(wacc + (warp * 8 + h) * WS + dim) =
+            any ? make_float2(acc[nt][0] + acc[nt][2], acc[nt][1] + acc[nt][3]) : make_float2(0.f, 0.f);
     }
     if ((lane & 3) == 0) {
         red_m[warp][h] = any ? m_run : -INFINITY;
         red_l[warp][h] = any ? l_run : 0.f;
     }
     __syncthreads();
+    // per head: the maximum over warps, each warp's weight 2^(m_w - M) and the weighted sum
     if (tid < 8) {
         float M = -INFINITY;
 #pragma unroll
         for (int w = 0; w < AT_WARPS; ++w) M = fmaxf(M, red_m[w][tid]);
         float Ls = 0.f;
 #pragma unroll
-        for (int w = 0; w < AT_WARPS; ++w)
-            if (red_m[w][tid] != -INFINITY) Ls = fmaf(red_l[w][tid], exp2f(red_m[w][tid] - M), Ls);
+        for (int w = 0; w < AT_WARPS; ++w) {
+            const float e = red_m[w][tid] == -INFINITY ? 0.f : exp2f(red_m[w][tid] - M);
+            we[w][tid] = e;
+            Ls = fmaf(red_l[w][tid], e, Ls);
+        }
         cm[tid] = M;
         cl[tid] = Ls;
     }
-    for (int it = tid; it < G * DH; it += AT_THREADS) {
-        const int hh = it / DH, dim = it - hh * DH;
-        float M = -INFINITY;
+    __syncthreads();
+    for (int it = tid; it < G * DH / 4; it += AT_THREADS) {
+        const int hh = it / (DH / 4), d4 = it - hh * (DH / 4);
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int w = 0; w < AT_WARPS; ++w) M = fmaxf(M, red_m[w][hh]);
-        float As = 0.f;
-#pragma unroll
-        for (int w = 0; w < AT_WARPS; ++w)
-            if (red_m[w][hh] != -INFINITY) As = fmaf(wacc[(w * 8 + hh) * DH + dim], exp2f(red_m[w][hh] - M), As);
-        cacc[hh][dim] = As;
+        for (int w = 0; w < AT_WARPS; ++w) {
+            const float e = we[w][hh];
+            const float4 v = *reinterpret_cast<const float4*>(wacc + (w * 8 + hh) * WS + d4 * 4);
+            a.x = fmaf(v.x, e, a.x);
+            a.y = fmaf(v.y, e, a.y);
+            a.z = fmaf(v.z, e, a.z);
+            a.w = fmaf(v.w, e, a.w);
+        }
+        *reinterpret_cast<float4*>(&cacc[hh][d4 * 4]) = a;
     }
 
     // ---- merge the CTAs of the cluster through distributed shared memory
     cluster_sync();
-    constexpr int ITEMS = G * DH / CS;  // (head, dim) outputs merged by each CTA of the cluster
     const uint32_t cm_a = smem_u32(cm), cl_a = smem_u32(cl), ca_a = smem_u32(&cacc[0][0]);
-    for (int it = tid; it < ITEMS; it += AT_THREADS) {
-        const int item = (int)rank * ITEMS + it;
+    // per head: every rank's (max, sum), the cluster maximum (CS consecutive lanes per head)
+    // and each rank's weight 2^(m_r - M)
+    if (tid < 8 * CS) {
+        const int hh = tid / CS, r = tid - hh * CS;
+        const float m = ld_cluster(map_to_rank(cm_a + 4 * hh, r));
+        const float l = ld_cluster(map_to_rank(cl_a + 4 * hh, r));
+        float M = m;
+#pragma unroll
+        for (int o = CS / 2; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        rw[r][hh] = m == -INFINITY ? 0.f : exp2f(m - M);
+        rl[r][hh] = l;
+        if (r == 0) Mt[hh] = M;
+    }
+    __syncthreads();
+    if (tid < 8) {
+        float Ls = 0.f;
+#pragma unroll
+        for (int r = 0; r < CS; ++r) Ls = fmaf(rl[r][tid], rw[r][tid], Ls);
+        Lt[tid] = Ls;
+    }
+    __syncthreads();
+    // (head, dim) outputs of this CTA's slice: 4 lanes per output, each summing a quarter of the ranks
+    constexpr int ITEMS = G * DH / CS;
+    constexpr int RQ = CS / 4;
+    for (int base = 0; base < ITEMS * 4; base += AT_THREADS) {
+        const int it = base + tid;
+        const bool act = it < ITEMS * 4;
+        const int item = (int)rank * ITEMS + (act ? it >> 2 : 0), q4 = it & 3;
         const int hh = item / DH, dim = item - hh * DH;
-        float mr[CS];
-        float M = -INFINITY;
+        float As = 0.f;
+        if (act) {
 #pragma unroll
-        for (int r = 0; r < CS; ++r) {
-            mr[r] = ld_cluster(map_to_rank(cm_a + 4 * hh, r));
-            M = fmaxf(M, mr[r]);
+            for (int k = 0; k < RQ; ++k) {
+                const int r = q4 * RQ + k;
+                As = fmaf(ld_cluster(map_to_rank(ca_a + 4 * (hh * DH + dim), r)), rw[r][hh], As);
+            }
         }
-        float Ls = 0.f, As = 0.f;
-#pragma unroll
-        for (int r = 0; r < CS; ++r) {
-            if (mr[r] == -INFINITY) continue;
-            const float e = exp2f(mr[r] - M);
-            Ls = fmaf(ld_cluster(map_to_rank(cl_a + 4 * hh, r)), e, Ls);
-            As = fmaf(ld_cluster(map_to_rank(ca_a + 4 * (hh * DH + dim), r)), e, As);
-        }
-        if (NC == 1) {
-            o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Ls;
-        } else {
-            part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
-            if (dim == 0) {
-                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = M;
-                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Ls;
+        As += __shfl_xor_sync(0xffffffffu, As, 1);
+        As += __shfl_xor_sync(0xffffffffu, As, 2);
+        if (act && q4 == 0) {
+            if (NC == 1) {
+                o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Lt[hh];
+            } else {
+                part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
+                if (dim == 0) {
+                    ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = Mt[hh];
+                    ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Lt[hh];
+                }
             }
         }
     }
