@@ -4,9 +4,8 @@
 // the group); its CTAs split the cached positions. Within a CTA:
 //  * every 16-position K/V tile of the CTA's range is requested at once with cp.async
 //    (16-byte chunks, zero-filled past the last position) into a padded shared-memory
-//    layout read conflict-free by ldmatrix; tiles of earlier positions are requested
-//    before the programmatic-dependency wait, only the tile holding the token written
-//    by this step's QKV kernel waits for it;
+//    layout read conflict-free by ldmatrix before the programmatic-dependency wait;
+//    only the row of the token written by this step's QKV kernel waits for it;
 //  * S = q K^T and O += P V run on the tensor cores (mma.sync m16n8k16, BF16 in, FP32
 //    accumulate). The 16 rows of the A operand hold the g query heads twice: rows r
 //    carry bf16(x) and rows r + 8 carry bf16(x - bf16(x)), so the two halves summed in
@@ -14,9 +13,11 @@
 //    are used exactly (the cache is BF16);
 //  * online softmax in the log2 domain (scores pre-scaled by log2(e)/sqrt(d_h)); warps
 //    merge through shared memory.
-// The CTAs of a cluster then merge through distributed shared memory (each CTA merges a
-// slice of the (head, dim) outputs from all CTAs' partials) between two cluster
-// barriers. Contexts longer than one cluster holds use several clusters per group;
+// The CTAs of a cluster then merge through distributed shared memory: each CTA stores
+// its (max, sum) per head into every CTA and each partial output into the CTA that
+// finalizes that (head, dim) slice, one cluster barrier makes the stores visible, and
+// each CTA merges its slice from its own shared memory. Contexts longer than one
+// cluster holds use several clusters per group;
 // their partials go through global scratch and the last cluster (atomic ticket, no
 // waiting) merges them.
 #include <cuda_bf16.h>
@@ -82,6 +83,18 @@ __device__ __forceinline__ void split_pack(float x0, float x1, uint32_t& hi, uin
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+__device__ __forceinline__ void st_cluster(uint32_t addr, float2 v) {
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(v.x), "f"(v.y) : "memory");
+}
+__device__ __forceinline__ void st_cluster(uint32_t addr, float4 v) {
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z),
+                 "f"(v.w)
+                 : "memory");
+}
 __device__ __forceinline__ uint32_t cluster_rank() {
     uint32_t r;
     asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -92,13 +105,6 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
     asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
-// (volatile: kept after the cluster barrier that orders it after the remote writes; no
-// memory clobber, so independent loads still issue back to back)
-__device__ __forceinline__ float ld_cluster(uint32_t addr) {
-    float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
-    return v;
-}
 
 template <int DH, int G, int CS>
 __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p) {
@@ -107,11 +113,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     extern __shared__ __align__(128) uint8_t sm[];
     __shared__ float red_m[AT_WARPS][8], red_l[AT_WARPS][8];
     __shared__ float cm[8], cl[8];              // this CTA's merged (max, sum) per head
-    __shared__ __align__(16) float cacc[8][DH];  // this CTA's merged unnormalized output
+    constexpr int ITEMS = G * DH / CS;          // (head, dim) outputs each CTA of the cluster finalizes
+    __shared__ __align__(16) float inbox[CS][ITEMS];  // every rank's partial outputs of this CTA's slice
+    __shared__ float2 inml[CS][8];                  // every rank's (max, sum) per head
     __shared__ float Mh[8], Lh[8], wts[CLUSTERS_MAX][8];
-    __shared__ float we[AT_WARPS][8];        // per-warp weights of each head in the CTA merge
-    __shared__ float rw[CS][8], rl[CS][8];   // per-rank weights and sums in the cluster merge
-    __shared__ float Mt[8], Lt[8];           // cluster-wide (max, sum) per head
+    __shared__ float we[AT_WARPS][8];  // per-warp weights of each head in the CTA merge
+    __shared__ float rw[CS][8];        // per-rank weights of each head in the cluster merge
+    __shared__ float Mt[8], Lt[8];     // cluster-wide (max, sum) per head
     __shared__ int is_last;
     const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x, bz = blockIdx.z;
     const int NC = S / CS, cid = split / CS;
@@ -124,6 +132,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     const int max_tokens = p.max_tokens[bz];
     const uint32_t rank = cluster_rank();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // first half of a cluster barrier: waited on before the first remote store, so every
+    // CTA of the cluster is known to be running by then
+    cluster_arrive_relaxed();
 
     const int T = *p.pos[bz] + 1;  // written by the previous step, which has completed
     const int chunk = (((T + S - 1) / S) + TILE - 1) / TILE * TILE;
@@ -133,7 +144,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     const int ntiles = (p1 - p0 + TILE - 1) / TILE;
     const int dep_tile = (p1 == T && ntiles > 0) ? ntiles - 1 : -1;  // holds this step's new token
 
-    auto issue = [&](int ti, int slot) {
+    // rows of tile ti into slot `slot`, except position `skip` (zero-filled past p1)
+    auto issue = [&](int ti, int slot, int skip) {
         const int base = p0 + ti * TILE;
         uint8_t* kt = sm + slot * 2 * C::TILEB;
         uint8_t* vt = kt + C::TILEB;
@@ -141,6 +153,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
         for (int c = lane; c < TILE * C::CPR; c += 32) {
             const int r = c / C::CPR, cc = c - r * C::CPR;
             const int pos = base + r;
+            if (pos == skip) continue;
             const bool ok = pos < p1;
             const int64_t off = (int64_t)(ok ? pos : p0) * DH + cc * 8;
             cp_async16(smem_u32(kt + r * C::ROWB + cc * 16), Kg + off, ok ? 16 : 0);
@@ -148,14 +161,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
         }
     };
 
-    // first batch of tiles, except the one that depends on this step's QKV kernel
+    // first batch of tiles; the row of this step's token (written by the QKV kernel) waits
     const int nb0 = min(C::MAXT, ntiles);
-    for (int t = warp; t < nb0; t += AT_WARPS)
-        if (t != dep_tile) issue(t, t);
+    for (int t = warp; t < nb0; t += AT_WARPS) issue(t, t, t == dep_tile ? T - 1 : -1);
     cp_commit();
     pdl_wait();
     pdl_trigger();
-    if (dep_tile >= 0 && dep_tile < nb0 && dep_tile % AT_WARPS == warp) issue(dep_tile, dep_tile);
+    if (dep_tile >= 0 && dep_tile < nb0 && dep_tile % AT_WARPS == warp && lane < C::CPR) {
+        const int r = T - 1 - (p0 + dep_tile * TILE);
+        const int64_t off = (int64_t)(T - 1) * DH + lane * 8;
+        uint8_t* kt = sm + dep_tile * 2 * C::TILEB;
+        cp_async16(smem_u32(kt + r * C::ROWB + lane * 16), Kg + off, 16);
+        cp_async16(smem_u32(kt + C::TILEB + r * C::ROWB + lane * 16), Vg + off, 16);
+    }
     cp_commit();
 
     const int h = lane >> 2;        // head row of this lane's fragments
@@ -184,7 +202,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     for (int b0 = 0; b0 < ntiles; b0 += C::MAXT) {
         const int nb = min(C::MAXT, ntiles - b0);
         if (b0 > 0) {  // later batches (very long contexts): reuse this warp's slots
-            for (int t = warp; t < nb; t += AT_WARPS) issue(b0 + t, t);
+            for (int t = warp; t < nb; t += AT_WARPS) issue(b0 + t, t, -1);
             cp_commit();
         }
         cp_wait_all();
@@ -276,6 +294,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
         cl[tid] = Ls;
     }
     __syncthreads();
+    // ---- merge the CTAs of the cluster: push each (head, dim) output of this CTA to the
+    // rank that finalizes it, and this CTA's (max, sum) of each head to every rank
+    cluster_wait();  // every CTA of the cluster is running (first barrier half)
+    const uint32_t inbox_a = smem_u32(&inbox[rank][0]), inml_a = smem_u32(&inml[rank][0]);
+    if (tid < 8 * CS) {
+        const int r = tid >> 3, hh = tid & 7;
+        st_cluster(map_to_rank(inml_a + 8 * hh, r), make_float2(cm[hh], cl[hh]));
+    }
     for (int it = tid; it < G * DH / 4; it += AT_THREADS) {
         const int hh = it / (DH / 4), d4 = it - hh * (DH / 4);
         float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -288,66 +314,45 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             a.z = fmaf(v.z, e, a.z);
             a.w = fmaf(v.w, e, a.w);
         }
-        *reinterpret_cast<float4*>(&cacc[hh][d4 * 4]) = a;
+        const int item = it * 4, k = item / ITEMS;  // ITEMS is a multiple of 4: one owner per float4
+        st_cluster(map_to_rank(inbox_a + 4 * (item - k * ITEMS), k), a);
     }
-
-    // ---- merge the CTAs of the cluster through distributed shared memory
-    cluster_sync();
-    const uint32_t cm_a = smem_u32(cm), cl_a = smem_u32(cl), ca_a = smem_u32(&cacc[0][0]);
-    // per head: every rank's (max, sum), the cluster maximum (CS consecutive lanes per head)
-    // and each rank's weight 2^(m_r - M)
-    if (tid < 8 * CS) {
-        const int hh = tid / CS, r = tid - hh * CS;
-        const float m = ld_cluster(map_to_rank(cm_a + 4 * hh, r));
-        const float l = ld_cluster(map_to_rank(cl_a + 4 * hh, r));
-        float M = m;
-#pragma unroll
-        for (int o = CS / 2; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-        rw[r][hh] = m == -INFINITY ? 0.f : exp2f(m - M);
-        rl[r][hh] = l;
-        if (r == 0) Mt[hh] = M;
-    }
-    __syncthreads();
+    cluster_sync();  // the pushed values are visible to their owners; nothing is read remotely after this
+    // finalize this CTA's slice from its own shared memory
     if (tid < 8) {
+        float M = -INFINITY;
+#pragma unroll
+        for (int r = 0; r < CS; ++r) M = fmaxf(M, inml[r][tid].x);
         float Ls = 0.f;
 #pragma unroll
-        for (int r = 0; r < CS; ++r) Ls = fmaf(rl[r][tid], rw[r][tid], Ls);
+        for (int r = 0; r < CS; ++r) {
+            const float e = inml[r][tid].x == -INFINITY ? 0.f : exp2f(inml[r][tid].x - M);
+            rw[r][tid] = e;
+            Ls = fmaf(inml[r][tid].y, e, Ls);
+        }
+        Mt[tid] = M;
         Lt[tid] = Ls;
     }
     __syncthreads();
-    // (head, dim) outputs of this CTA's slice: 4 lanes per output, each summing a quarter of the ranks
-    constexpr int ITEMS = G * DH / CS;
-    constexpr int RQ = CS / 4;
-    for (int base = 0; base < ITEMS * 4; base += AT_THREADS) {
-        const int it = base + tid;
-        const bool act = it < ITEMS * 4;
-        const int item = (int)rank * ITEMS + (act ? it >> 2 : 0), q4 = it & 3;
+    for (int it = tid; it < ITEMS; it += AT_THREADS) {
+        const int item = (int)rank * ITEMS + it;
         const int hh = item / DH, dim = item - hh * DH;
         float As = 0.f;
-        if (act) {
 #pragma unroll
-            for (int k = 0; k < RQ; ++k) {
-                const int r = q4 * RQ + k;
-                As = fmaf(ld_cluster(map_to_rank(ca_a + 4 * (hh * DH + dim), r)), rw[r][hh], As);
-            }
-        }
-        As += __shfl_xor_sync(0xffffffffu, As, 1);
-        As += __shfl_xor_sync(0xffffffffu, As, 2);
-        if (act && q4 == 0) {
-            if (NC == 1) {
-                o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Lt[hh];
-            } else {
-                part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
-                if (dim == 0) {
-                    ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = Mt[hh];
-                    ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Lt[hh];
-                }
+        for (int r = 0; r < CS; ++r) As = fmaf(inbox[r][it], rw[r][hh], As);
+        if (NC == 1) {
+            o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Lt[hh];
+        } else {
+            part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
+            if (dim == 0) {
+                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 0] = Mt[hh];
+                ml[((int64_t)(jl * NC + cid) * G + hh) * 2 + 1] = Lt[hh];
             }
         }
     }
-    if (NC > 1) __threadfence();
-    cluster_sync();  // no CTA leaves while others may still read its shared memory
     if (NC == 1) return;
+    __threadfence();
+    cluster_sync();  // every slice of this cluster is written before its ticket is taken
 
     // ---- several clusters per group: the last one (ticket) merges their partials
     if (rank != 0) return;
