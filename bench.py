@@ -56,6 +56,9 @@ def parse():
     ap.add_argument("--workload", choices=["decode", "prefill", "mixed"], default="decode",
                     help="decode (the headline metric), the prefill of one prompt on the 8B shape, or "
                          "mixed-turn serving (70B shape, 16 turns over the dense plan and five masks)")
+    ap.add_argument("--union", action="store_true",
+                    help="mixed workload: one union-of-masks step for all turns (every weight row read once "
+                         "for all plans) instead of one weight pass per plan group")
     ap.add_argument("--panels", choices=["row-indexed", "compact"], default="row-indexed",
                     help="mixed workload: Q/K/V and gate/up panels as row maps into the shared store "
                          "(zero copy) or materialized copies")
@@ -548,6 +551,8 @@ def run_mixed(args):
     lg = {pi: torch.empty((len(idx), sh.vocab), dtype=torch.float32, device="cuda") for pi, idx in groups.items()}
     gs = {pi: [sessions[i] for i in idx] for pi, idx in groups.items()}
     stream = torch.cuda.current_stream()
+    if args.union:
+        return run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s)
 
     def step(t):
         for pi in groups:
@@ -646,6 +651,83 @@ def run_mixed(args):
            "step_roofline": {"bytes_per_step": int(step_bytes), "achieved": round(step_gbs, 1), "peak": peak,
                              "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
            "e2e": e2e, "gpu_launches": launches * K, "clocks": clocks, "cpu_baseline": cpu,
+           "device_error": errs, "setup_s": round(setup_s, 1)}
+    print(json.dumps(out), flush=True)
+
+
+def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s):
+    """The mixed-turn step as one union-of-masks step over all turns: each layer's dense
+    panels are read once for every session (tensor-core skinny GEMMs), each session's mask
+    applied where its units meet it; the LM head runs per group of four sessions."""
+    import torch
+    K, Wm = args.steps, args.warmup
+    n = len(turns)
+    x = torch.from_numpy(np.ascontiguousarray(xb).view(np.int16)).view(torch.bfloat16).cuda()
+    lg = torch.empty((n, sh.vocab), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    for t in range(Wm):
+        tasp.decode_step_union(sessions, x[t], None, lg)
+    torch.cuda.synchronize()
+    ctx0 = [s.position for s in sessions]
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for t in range(K):
+        tasp.decode_step_union(sessions, x[Wm + t], None, lg)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1) / K
+    tok_s = n / (ms * 1e-3)
+    err, launches = tasp.union_status(sessions)
+    errs = err + sum(s.device_error() for s in sessions)
+    # bytes of one step: every dense panel byte (and row scale) once, the LM head once per
+    # group of four, every turn's KV cache
+    d, qd, df = sh.d, sh.Hq * sh.dh, sh.df
+    qkv_rows = (sh.Hq + 2 * sh.Hkv) * sh.dh
+    layer_w = qkv_rows * d + d * qd + 2 * df * d + d * df + 4 * (qkv_rows + d + 2 * df + d)
+    lm = sh.vocab * d * 2 * ((n + 3) // 4)
+    kvb = 0
+    for i, (pi, _) in enumerate(turns):
+        dims = [plans[pi].layer_dims(l) for l in range(sh.L)]
+        kvb += kv_bytes(dims, sh.dh, ctx0[i] + K // 2 + 1)
+    step_bytes = sh.L * layer_w + lm + kvb
+    peak, peak_kind = measured_peak()
+    step_gbs = step_bytes / (ms * 1e-3) / 1e9
+    e2e = None
+    if not args.no_e2e:
+        xh = torch.from_numpy(np.ascontiguousarray(xb).view(np.int16)).view(torch.bfloat16).pin_memory()
+        lh = torch.empty((n, sh.vocab), dtype=torch.float32).pin_memory()
+        xd = torch.empty((n, sh.d), dtype=torch.bfloat16, device="cuda")
+        te = time.perf_counter()
+        for t in range(K):
+            xd.copy_(xh[t], non_blocking=True)
+            tasp.decode_step_union(sessions, xd, None, lg)
+            lh.copy_(lg, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+        e2e_ms = (time.perf_counter() - te) * 1e3 / K
+        e2e = {"value": round(n / (e2e_ms * 1e-3), 2), "unit": "tokens/s", "h2d_bytes_per_step": n * sh.d * 2,
+               "d2h_bytes_per_step": n * sh.vocab * 4}
+    for s in sessions:
+        s.release()
+    for p in plans.values():
+        p.release()
+    groups = {}
+    for pi, _ in turns:
+        groups[pi] = groups.get(pi, 0) + 1
+    out = {"metric": "mixed-turn decode tokens/s (70B-shape, 16 turns over dense + 5 masks, union-of-masks step)",
+           "value": round(tok_s, 2), "unit": "tokens/s", "n_gpus": 1, "steps": K, "warmup": Wm,
+           "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "int8w-f16", "data": "synthetic",
+           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else "") + "_union", "turns": n,
+                      "plans": {("dense" if pi == len(wl.masks) else f"mask{pi}"): c for pi, c in groups.items()},
+                      "prompt_tokens": [T for _, T in turns],
+                      "l2": "inputs larger than L2 (each step streams the dense panels)"},
+           "roofline": None,
+           "step_roofline": {"bytes_per_step": int(step_bytes), "achieved": round(step_gbs, 1), "peak": peak,
+                             "unit": "GB/s", "frac": round(step_gbs / peak, 4), "peak_source": peak_kind},
+           "e2e": e2e, "gpu_launches": launches * K, "clocks": clocks, "cpu_baseline": None,
            "device_error": errs, "setup_s": round(setup_s, 1)}
     print(json.dumps(out), flush=True)
 

@@ -266,6 +266,36 @@ int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_lo
 int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, float* d_hidden_out, float* d_logits,
                             void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Union-of-masks batched decode (the next step after per-plan grouping).
+ * ------------------------------------------------------------------------- */
+
+/* One decode step for 1 <= n <= 16 sessions whose plans may differ (each turn keeps
+ * the mask it was started with: its KV cache stays plan-shaped). Every weight row
+ * of the shared store is read once for all n sessions: the projections run dense
+ * for all of them on the tensor cores (INT8 rows converted to FP16 in shared
+ * memory, activations in FP16 with a per-session power-of-two scale, FP32
+ * accumulation), and each session's mask is applied where a unit meets it: Q/K/V of
+ * a dropped group are not written, attention runs over the session's own kept
+ * groups, dropped heads enter the O projection as zeros and dropped channel units
+ * leave SiLU(gate) * up at zero. This equals the session's compacted plan up to
+ * FP32 summation order and FP16 rounding of the activations (the mask-as-zero
+ * reading of a plan, Sec. 3). d_x_bf16 is device BF16 [n][d]; d_hidden_out FP32
+ * [n][d] and d_logits FP32 [n][vocab] are optional (NULL skips). The sessions must
+ * share one weight store; d, H_q d_h and d_f must be multiples of 128. The set of
+ * sessions keeps a workspace (~ 16 x (2 d + 2 H_q d_h + d_f) x 4 bytes, partial
+ * sums of ~ 16 x 4 x (rows of the largest projection) bytes, attention partials)
+ * and a CUDA graph captured on first use for these output buffers; inputs are
+ * copied on `stream` into its staging buffer. Call it outside any stream capture.
+ * async on `stream`. Errors: EMASK (sessions on different stores), ECAP (a session
+ * is full), EUNSUP (shape), EINVAL, ENOMEM, ECUDA. */
+int tasp_decode_step_union(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,
+                           float* d_logits, void* stream);
+
+/* Device error word (bit 0: a bounded wait gave up) and graph launch count of the
+ * union workspace of these sessions (created if absent). sync. */
+int tasp_union_status(tasp_session* const* sessions, int32_t n, int32_t* device_error, int32_t* launches);
+
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char* tasp_last_error(void);
 

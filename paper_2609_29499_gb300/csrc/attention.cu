@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     __shared__ float Mt[8], Lt[8];     // cluster-wide (max, sum) per head
     __shared__ int is_last;
     const int split = blockIdx.x, jl = blockIdx.y, S = gridDim.x, bz = blockIdx.z;
+    if (jl >= p.m_kv[bz]) return;  // the session's plan keeps fewer groups (whole cluster exits)
     const int NC = S / CS, cid = split / CS;
     // session bz of the batch
     const float* const q_in = p.q + bz * p.q_stride;
@@ -471,7 +472,7 @@ int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, i
     }
     if (splits % cs) return fail(TASP_EINVAL, "attention splits must be a multiple of the cluster size");
     cudaLaunchConfig_t cfg = {};
-    if (nb < 1 || nb > MAX_BATCH) return fail(TASP_EINVAL, "attention batch of 1 to 4 sessions");
+    if (nb < 1 || nb > UNION_MAX) return fail(TASP_EINVAL, "attention batch of 1 to 16 sessions");
     cfg.gridDim = dim3(splits, m_kv, nb);
     cfg.blockDim = dim3(AT_THREADS);
     cfg.dynamicSmemBytes = smem_of(dh);

@@ -256,6 +256,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 a.V[b] = se.V[l];
                 a.pos[b] = se.d_pos;
                 a.max_tokens[b] = se.max_tokens;
+                a.m_kv[b] = lp.m_kv;
                 S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
@@ -378,6 +379,13 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
 int enqueue_step(Session& se, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook, void* ctx,
                  int* launches) {
     return enqueue_batch(single_view(se), t, s, only_layer, hook, ctx, launches);
+}
+
+int enqueue_lm_heads(const BatchView& bv, float* logits, cudaStream_t s) {
+    const Shape& sh = bv.ss[0]->plan->store->sh;
+    if (sh.vocab == 0) return fail(TASP_EINVAL, "model has no LM head");
+    const Params p = lm_params(bv, logits, sh.vocab);
+    return bv.n == 1 ? launch_gemv_single(M_LM, p, s) : launch_gemv(M_LM, p, s);
 }
 
 int enqueue_lm_head(Session& se, float* logits, cudaStream_t s) {

@@ -815,6 +815,7 @@ int tasp_release(void* handle) {
     if (Session* se = as_session(handle)) {
         cudaError_t e = cudaDeviceSynchronize();
         batches_drop(se);
+        union_drop(se);
         {
             std::lock_guard<std::mutex> lk(g_mu);
             se->plan->live_sessions--;

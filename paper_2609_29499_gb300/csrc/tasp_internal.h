@@ -174,16 +174,18 @@ int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const in
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
 
 // attention.cu
-constexpr int MAX_BATCH = 4;  // sessions of one plan that share each weight pass
+constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pass
+constexpr int UNION_MAX = 16;  // sessions (of any plans) in one union-of-masks step
 struct AttnParams {
     // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
     const float* q;      // FP32 rotated queries [m_q][dh] (kept heads, group-major)
     float* o;            // FP32 [m_q][dh]
     int64_t q_stride;
-    const uint16_t* K[MAX_BATCH];  // BF16 [m_kv][max_tokens][dh] of this layer
-    const uint16_t* V[MAX_BATCH];
-    const int* pos[MAX_BATCH];     // device position: the step attends to positions 0..pos
-    int max_tokens[MAX_BATCH];
+    const uint16_t* K[UNION_MAX];  // BF16 [m_kv][max_tokens][dh] of this layer
+    const uint16_t* V[UNION_MAX];
+    const int* pos[UNION_MAX];     // device position: the step attends to positions 0..pos
+    int max_tokens[UNION_MAX];
+    int m_kv[UNION_MAX];           // kept groups of the session's plan (grid y covers the largest)
     float qscale;        // log2(e) / sqrt(dh)
     float* part;         // + b * part_stride
     float* ml;           // + b * ml_stride
@@ -230,6 +232,10 @@ int batch_attn_slots(const Plan& p, const Session* const* ss, int n, int sms);
 
 using KernelHook = void (*)(void* ctx, int kind, bool before);
 
+// union.cu: free the union-step workspaces (and graphs) that include this session.
+void union_drop(Session* se);
+// Final RMSNorm + LM head of a batch view's residuals into logits [n][vocab].
+int enqueue_lm_heads(const BatchView& bv, float* logits, cudaStream_t s);
 // Enqueue one decode step of a batch (or one isolated layer when only_layer >= 0) on `s`.
 int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int only_layer, KernelHook hook,
                   void* ctx, int* launches);

@@ -30,7 +30,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
-            "tasp_session_prefill",
+            "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
             "tasp_last_error",
             "tasp_version")
 
@@ -96,6 +96,8 @@ def load(path: str = LIB_PATH):
         "tasp_decode_step_static": (c_int32, [P, P, P, P, P]),
         "tasp_session_kv_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
         "tasp_session_prefill": (c_int32, [P, P, c_int32, P, P]),
+        "tasp_decode_step_union": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
+        "tasp_union_status": (c_int32, [POINTER(P), c_int32, POINTER(c_int32), POINTER(c_int32)]),
         "tasp_last_error": (ctypes.c_char_p, []),
         "tasp_version": (ctypes.c_char_p, []),
     }
@@ -310,6 +312,24 @@ def decode_step(sessions, x_bf16, hidden=None, logits=None, stream=None):
     _check(load().tasp_decode_step(p, len(sessions), x_bf16.data_ptr(),
                                    hidden.data_ptr() if hidden is not None else None,
                                    logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
+
+
+def decode_step_union(sessions, x_bf16, hidden=None, logits=None, stream=None):
+    """Union-of-masks decode step: up to 16 sessions whose plans may differ (one shared store), every
+    weight row read once for all of them; buffers as in decode_step."""
+    _check_buffers(sessions, x_bf16, hidden, logits, True)
+    p, keep = _handles(sessions)
+    _check(load().tasp_decode_step_union(p, len(sessions), x_bf16.data_ptr(),
+                                         hidden.data_ptr() if hidden is not None else None,
+                                         logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
+
+
+def union_status(sessions):
+    """(device error word, graph launches) of the union workspace of these sessions."""
+    p, keep = _handles(sessions)
+    err, nl = c_int32(0), c_int32(0)
+    _check(load().tasp_union_status(p, len(sessions), ctypes.byref(err), ctypes.byref(nl)))
+    return err.value, nl.value
 
 
 def decode_step_static(session, x_bf16, hidden=None, logits=None, stream=None):
