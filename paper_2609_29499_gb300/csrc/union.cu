@@ -18,7 +18,7 @@
 // FP16 (each session scaled by a power of two so its largest entry is below 2^14; exact
 // rescaling). A persistent CTA per SM walks (128-row tile, K slice) units:
 //  * warp 0 streams 128 x 128 INT8 weight tiles and the 16 x 128 FP16 activation tile of
-//    the same K range with TMA (128-byte swizzle) into a 4-stage ring;
+//    the same K range with TMA (128-byte swizzle) into an 8-stage ring;
 //  * warps 2-5 convert each INT8 tile to FP16 (exact: v + 1152 is built in the FP16 bit
 //    pattern 0x6400 | (v ^ 0x80) and 1152 subtracted) into the MMA operand layout;
 //  * warp 1 issues tcgen05.mma (M = 128, N = 16, K = 16) into one of two 16-column TMEM
@@ -49,7 +49,7 @@ using namespace tc;
 constexpr int US = UNION_MAX;  // sessions per union step = MMA N
 constexpr int SK_BM = 128;     // weight rows per tile (MMA M)
 constexpr int SK_BK = 128;     // K (INT8 bytes) per stage
-constexpr int SK_NST = 4;
+constexpr int SK_NST = 8;
 constexpr int SK_W_BYTES = SK_BM * SK_BK;      // INT8 tile
 constexpr int SK_X_BYTES = US * SK_BK * 2;     // FP16 activation tile (two 64-column boxes)
 constexpr int SK_A_HALF = SK_BM * 64 * 2;      // FP16 operand tile of 64 columns
@@ -247,66 +247,113 @@ struct PrepArgs {
     float* xinv;               // [US]: 2^-e of the session's scale
 };
 
-__device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
-    for (int o = 16; o; o >>= 1) {
-        const float w = __shfl_xor_sync(0xffffffffu, v, o);
-        v = is_max ? fmaxf(v, w) : v + w;
-    }
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    float t = is_max ? 0.f : 0.f;
-    for (int w = 0; w < nw; ++w) t = is_max ? fmaxf(t, red[w]) : t + red[w];
-    return t;
+constexpr int PREP_CS = 8;  // CTAs (one cluster) per session in prep_kernel
+
+__device__ __forceinline__ float warp_sum(float v) {
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float2 ld_cluster2(const float2* p, uint32_t rank) {
+    uint32_t a = smem_u32(p), r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+    float2 v;
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(r) : "memory");
+    return v;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-// One CTA per session: the projection input (RMSNorm x gamma, a copy, or the plan's heads
-// scattered to dense order), scaled by 2^e so that its largest magnitude is below 2^14.
-__global__ void __launch_bounds__(256) prep_kernel(const PrepArgs p) {
-    __shared__ float red[8];
-    const int b = blockIdx.x;
-    const float* src = p.src + b * p.src_ld;
-    auto value = [&](int k) -> float {
-        if (p.mode == PR_HEADS) {
-            const int hd = k / p.dh, j = hd / p.g;
-            const int lj = p.gmap[b * p.Hkv + j];
-            return lj < 0 ? 0.f : src[(int64_t)(lj * p.g + (hd - j * p.g)) * p.dh + (k - hd * p.dh)];
-        }
-        return src[k];
-    };
-    float rs = 1.f;
+// Four consecutive entries k..k+3 of the projection input of session b (before the
+// RMSNorm factor): x * gamma, a copy, or the plan's heads in dense order.
+__device__ __forceinline__ float4 prep_in(const PrepArgs& p, const float* src, int b, int k) {
+    if (p.mode == PR_HEADS) {
+        const int hd = k / p.dh, j = hd / p.g;
+        const int lj = p.gmap[b * p.Hkv + j];
+        if (lj < 0) return make_float4(0.f, 0.f, 0.f, 0.f);
+        return *reinterpret_cast<const float4*>(src + (int64_t)(lj * p.g + (hd - j * p.g)) * p.dh + (k - hd * p.dh));
+    }
+    float4 v = *reinterpret_cast<const float4*>(src + k);
     if (p.mode == PR_NORM) {
-        if (p.in_bf16) {  // first layer: the residual starts as the step input
-            float* x = const_cast<float*>(src);
-            for (int k = threadIdx.x; k < p.K; k += blockDim.x)
-                x[k] = __uint_as_float((uint32_t)p.in_bf16[(int64_t)b * p.K + k] << 16);
-            __syncthreads();
+        const float4 g = *reinterpret_cast<const float4*>(p.gamma + k);
+        v.x *= g.x;
+        v.y *= g.y;
+        v.z *= g.z;
+        v.w *= g.w;
+    }
+    return v;
+}
+
+// One 8-CTA cluster per session: the projection input (RMSNorm(x) * gamma, a copy, or the
+// plan's heads scattered to dense order), scaled by 2^e so that its largest magnitude is
+// below 2^14, as FP16. Each CTA takes K/8 entries; the cluster combines the sum of squares
+// and the largest magnitude through distributed shared memory.
+__global__ void __launch_bounds__(256) prep_kernel(const PrepArgs p) {
+    __shared__ float2 red[8];
+    __shared__ float2 tot;  // this CTA's (sum of squares, max |in|)
+    const int b = blockIdx.y, rank = blockIdx.x;  // cluster = the session's 8 CTAs along x
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int chunk = (p.K / PREP_CS + 3) & ~3;
+    const int k0 = rank * chunk, k1 = min(p.K, k0 + chunk);
+    float* x = const_cast<float*>(p.src) + b * p.src_ld;
+    if (p.in_bf16) {  // first layer: the residual starts as the step input (this CTA's entries)
+        for (int k = k0 + threadIdx.x; k < k1; k += blockDim.x)
+            x[k] = __uint_as_float((uint32_t)p.in_bf16[(int64_t)b * p.K + k] << 16);
+        __syncthreads();
+    }
+    float ss = 0.f, mx = 0.f;
+    for (int k = k0 + 4 * threadIdx.x; k < k1; k += 4 * blockDim.x) {
+        if (p.mode == PR_NORM) {
+            const float4 v = *reinterpret_cast<const float4*>(x + k);
+            ss = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, ss))));
         }
-        float ss = 0.f;
-        for (int k = threadIdx.x; k < p.K; k += blockDim.x) ss = fmaf(src[k], src[k], ss);
-        ss = block_reduce(ss, false, red);
-        rs = rsqrtf(ss / (float)p.K + p.eps);
+        const float4 v = prep_in(p, x, b, k);
+        mx = fmaxf(mx, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
     }
-    float mx = 0.f;
-    for (int k = threadIdx.x; k < p.K; k += blockDim.x) {
-        const float v = p.mode == PR_NORM ? src[k] * rs * p.gamma[k] : value(k);
-        mx = fmaxf(mx, fabsf(v));
+    ss = warp_sum(ss);
+    mx = warp_max(mx);
+    if (lane == 0) red[warp] = make_float2(ss, mx);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float2 t = make_float2(0.f, 0.f);
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+            t.x += red[w].x;
+            t.y = fmaxf(t.y, red[w].y);
+        }
+        tot = t;
     }
-    mx = block_reduce(mx, true, red);
+    cluster_sync_all();
+    float2 all = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int r = 0; r < PREP_CS; ++r) {  // same order in every CTA
+        const float2 t = ld_cluster2(&tot, r);
+        all.x += t.x;
+        all.y = fmaxf(all.y, t.y);
+    }
+    const float rs = p.mode == PR_NORM ? rsqrtf(all.x / (float)p.K + p.eps) : 1.f;
+    const float amax = all.y * rs;
     int e = 0;
-    if (mx > 0.f) {
+    if (amax > 0.f) {
         int ex;
-        frexpf(mx, &ex);  // mx < 2^ex
+        frexpf(amax, &ex);  // amax < 2^ex
         e = 14 - ex;
     }
-    const float sc = ldexpf(1.f, e);
+    const float sc = ldexpf(rs, e);
     __half* dst = p.x16 + b * p.ld16;
-    for (int k = threadIdx.x; k < p.K; k += blockDim.x) {
-        const float v = p.mode == PR_NORM ? src[k] * rs * p.gamma[k] : value(k);
-        dst[k] = __float2half_rn(v * sc);
+    for (int k = k0 + 4 * threadIdx.x; k < k1; k += 4 * blockDim.x) {
+        const float4 v = prep_in(p, x, b, k);
+        const __half2 h0 = __floats2half2_rn(v.x * sc, v.y * sc), h1 = __floats2half2_rn(v.z * sc, v.w * sc);
+        uint2 o;
+        o.x = *reinterpret_cast<const uint32_t*>(&h0);
+        o.y = *reinterpret_cast<const uint32_t*>(&h1);
+        *reinterpret_cast<uint2*>(dst + k) = o;
     }
-    if (threadIdx.x == 0) p.xinv[b] = ldexpf(1.f, -e);
+    if (rank == 0 && threadIdx.x == 0) p.xinv[b] = ldexpf(1.f, -e);
+    cluster_sync_all();  // no CTA leaves while others may read its total
 }
 
 // ------------------------------------------------------------------ finish kernels
@@ -596,7 +643,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
     const int g = sh.g(), qd = sh.Hq * sh.dh, nu = sh.n_units();
     int rc = 0, nl = 0;
     auto prep = [&](int mode, const float* src, int64_t src_ld, const uint16_t* in_bf16, const float* gamma, int K,
-                    const int* gmap) {
+                    const int* gmap) -> int {
         PrepArgs p{};
         p.mode = mode;
         p.K = K;
@@ -613,7 +660,19 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         p.ld16 = w.ld16;
         p.xinv = w.xinv;
         ++nl;
-        return launch(prep_kernel, dim3(n), dim3(256), s, p);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(PREP_CS, n);
+        cfg.blockDim = dim3(256);
+        cfg.stream = s;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = PREP_CS;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        TASP_CUDA(cudaLaunchKernelEx(&cfg, prep_kernel, p));
+        return TASP_OK;
     };
     auto fin = [&](int S, int rows, const float* scale) {
         FinArgs f{};
