@@ -447,10 +447,10 @@ int attn_cluster(int dh, int g) { return cluster_size(pick(dh, g, 16), dh); }
 
 // Splits (CTAs) per kept group: one cluster, or several when the context exceeds what
 // one cluster keeps resident.
-int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g) {
+int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap) {
     (void)m_kv;
     (void)sms;
-    const int cs = attn_cluster(dh, g);
+    const int cs = std::min(attn_cluster(dh, g), cs_cap);
     const int tiles = (max_tokens + TILE - 1) / TILE;
     int nc = (tiles + cs * maxt_of(dh) - 1) / (cs * maxt_of(dh));
     nc = std::max(1, std::min(nc, CLUSTERS_MAX));
@@ -459,8 +459,9 @@ int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g) {
 
 int attn_splits_max() { return CLUSTERS_MAX * 16; }
 
-int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s) {
-    const int cs = attn_cluster(dh, g);
+int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s,
+                     int cs_cap) {
+    const int cs = std::min(attn_cluster(dh, g), cs_cap);
     AttnFn fn = pick(dh, g, cs);
     if (!fn) return fail(TASP_EUNSUP, "attention kernel not built for this (head_dim, query heads per group)");
     static bool attr[2][9][2] = {};

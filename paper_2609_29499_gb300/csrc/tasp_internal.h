@@ -194,9 +194,11 @@ struct AttnParams {
 };
 int attn_supported(int dh, int g);
 int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
-int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g);
+int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap = 16);
 int attn_splits_max();
-int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s);
+// cs_cap: largest cluster size to use (16 or 8; many short sessions run better on 8)
+int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s,
+                     int cs_cap = 16);
 
 // decode.cu
 enum KernelKind { K_QKV = 0, K_ATTN = 1, K_O = 2, K_GU = 3, K_DOWN = 4, K_LM = 5, K_OTHER = 6 };

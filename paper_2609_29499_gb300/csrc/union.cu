@@ -18,9 +18,10 @@
 // FP16 (each session scaled by a power of two so its largest entry is below 2^14; exact
 // rescaling). A persistent CTA per SM walks (128-row tile, K slice) units:
 //  * warp 0 streams 128 x 128 INT8 weight tiles and the 16 x 128 FP16 activation tile of
-//    the same K range with TMA (128-byte swizzle) into an 8-stage ring;
+//    the same K range with TMA (128-byte swizzle) into a 4-stage ring;
 //  * warps 2-5 convert each INT8 tile to FP16 (exact: v + 1152 is built in the FP16 bit
-//    pattern 0x6400 | (v ^ 0x80) and 1152 subtracted) into the MMA operand layout;
+//    pattern 0x6400 | (v ^ 0x80) and 1152 subtracted) into one of four MMA operand
+//    buffers, so the conversion runs ahead of the MMAs' completion;
 //  * warp 1 issues tcgen05.mma (M = 128, N = 16, K = 16) into one of two 16-column TMEM
 //    accumulators;
 //  * warps 6-9 read the accumulator (tcgen05.ld) and store the unit's FP32 partial sums.
@@ -49,16 +50,18 @@ using namespace tc;
 constexpr int US = UNION_MAX;  // sessions per union step = MMA N
 constexpr int SK_BM = 128;     // weight rows per tile (MMA M)
 constexpr int SK_BK = 128;     // K (INT8 bytes) per stage
-constexpr int SK_NST = 8;
+constexpr int SK_NST = 4;   // INT8 + activation stages
+constexpr int SK_NA = 4;    // FP16 operand buffers (the converters run up to SK_NA - 1 blocks ahead of the MMAs)
 constexpr int SK_W_BYTES = SK_BM * SK_BK;      // INT8 tile
 constexpr int SK_X_BYTES = US * SK_BK * 2;     // FP16 activation tile (two 64-column boxes)
 constexpr int SK_A_HALF = SK_BM * 64 * 2;      // FP16 operand tile of 64 columns
 constexpr int SK_A_BYTES = 2 * SK_A_HALF;
 constexpr int SK_STAGE = SK_W_BYTES + SK_X_BYTES;
-constexpr int SK_SMEM = SK_NST * SK_STAGE + 2 * SK_A_BYTES + 1024;
+constexpr int SK_SMEM = SK_NST * SK_STAGE + SK_NA * SK_A_BYTES + 1024;
 constexpr int SK_THREADS = 320;
 constexpr uint32_t SK_IDESC = idesc_f16(SK_BM, US);
 constexpr int SK_UNITS_PER_CTA = 3;  // target units per CTA when choosing K slices
+constexpr int UN_ATT_CS = 8;         // attention cluster size: 16 sessions fill the GPU with 8-CTA clusters
 
 struct SkArgs {
     int rows, K;  // weight panel rows; reduction length (multiple of 128)
@@ -84,8 +87,8 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
     uint8_t* ring = sm;                      // stage s: INT8 tile, then the activation tile
-    uint8_t* abuf = sm + SK_NST * SK_STAGE;  // two FP16 operand buffers
-    __shared__ __align__(8) uint64_t full[SK_NST], empty[SK_NST], afull[2], aempty[2], accf[2], acce[2];
+    uint8_t* abuf = sm + SK_NST * SK_STAGE;  // SK_NA FP16 operand buffers
+    __shared__ __align__(8) uint64_t full[SK_NST], empty[SK_NST], afull[SK_NA], aempty[SK_NA], accf[2], acce[2];
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -99,9 +102,11 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
             mbar_init(smem_u32(&full[s]), 1);
             mbar_init(smem_u32(&empty[s]), 4 + 1);  // 4 converter warps + the MMAs that read the activations
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < SK_NA; ++b) {
             mbar_init(smem_u32(&afull[b]), 4);
             mbar_init(smem_u32(&aempty[b]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&accf[b]), 1);
             mbar_init(smem_u32(&acce[b]), 4);
         }
@@ -148,8 +153,8 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
                 if (it >= 2) mbar_wait(smem_u32(&acce[acc]), ((it >> 1) - 1) & 1, &abort_flag, a.err);
                 fence_after();
                 for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                    const int s = g % SK_NST, ab = g & 1;
-                    mbar_wait(smem_u32(&afull[ab]), (g >> 1) & 1, &abort_flag, a.err);
+                    const int s = g % SK_NST, ab = g % SK_NA;
+                    mbar_wait(smem_u32(&afull[ab]), (g / SK_NA) & 1, &abort_flag, a.err);
                     mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
                     fence_after();
                     const uint32_t sa = smem_u32(abuf + ab * SK_A_BYTES);
@@ -175,9 +180,9 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
             const int kb0 = ks * a.kbs, kb1 = min(nkb, kb0 + a.kbs);
             (void)tile;
             for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                const int s = g % SK_NST, ab = g & 1;
+                const int s = g % SK_NST, ab = g % SK_NA;
                 mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
-                if (g >= 2) mbar_wait(smem_u32(&aempty[ab]), ((g >> 1) - 1) & 1, &abort_flag, a.err);
+                if (g >= SK_NA) mbar_wait(smem_u32(&aempty[ab]), ((g / SK_NA) - 1) & 1, &abort_flag, a.err);
                 const uint8_t* wrow = ring + s * SK_STAGE + r * 128;
                 uint8_t* arow = abuf + ab * SK_A_BYTES + r * 128;
                 const int sw = r & 7;  // 128-byte swizzle: 16-byte chunk c of row r sits at c ^ (r % 8)
@@ -738,8 +743,8 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
             if ((rc = device_info(di))) return rc;
             int S_att = 0;
             for (int b = 0; b < n; ++b)
-                S_att = std::max(S_att, attn_splits(a.m_kv[b] > 0 ? a.m_kv[b] : 1, w.ss[b]->max_tokens, di.sms, sh.dh, g));
-            if ((rc = launch_attention(a, sh.dh, g, mkv, S_att, n, s))) return rc;
+                S_att = std::max(S_att, attn_splits(a.m_kv[b], w.ss[b]->max_tokens, di.sms, sh.dh, g, UN_ATT_CS));
+            if ((rc = launch_attention(a, sh.dh, g, mkv, S_att, n, s, UN_ATT_CS))) return rc;
             ++nl;
         }
         // O projection + residual (the dropped heads are zero in the scattered input)
