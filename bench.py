@@ -658,7 +658,7 @@ def run_mixed(args):
 def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s):
     """The mixed-turn step as one union-of-masks step over all turns: each layer's dense
     panels are read once for every session (tensor-core skinny GEMMs), each session's mask
-    applied where its units meet it; the LM head runs per group of four sessions."""
+    applied where its units meet it; the LM head (BF16) is one more skinny GEMM for all turns."""
     import torch
     K, Wm = args.steps, args.warmup
     n = len(turns)
@@ -682,12 +682,12 @@ def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s):
     tok_s = n / (ms * 1e-3)
     err, launches = tasp.union_status(sessions)
     errs = err + sum(s.device_error() for s in sessions)
-    # bytes of one step: every dense panel byte (and row scale) once, the LM head once per
-    # group of four, every turn's KV cache
+    # bytes of one step: every dense panel byte (and row scale) once, the LM head once, every
+    # turn's KV cache
     d, qd, df = sh.d, sh.Hq * sh.dh, sh.df
     qkv_rows = (sh.Hq + 2 * sh.Hkv) * sh.dh
     layer_w = qkv_rows * d + d * qd + 2 * df * d + d * df + 4 * (qkv_rows + d + 2 * df + d)
-    lm = sh.vocab * d * 2 * ((n + 3) // 4)
+    lm = sh.vocab * d * 2
     kvb = 0
     for i, (pi, _) in enumerate(turns):
         dims = [plans[pi].layer_dims(l) for l in range(sh.L)]

@@ -60,6 +60,10 @@ constexpr int SK_STAGE = SK_W_BYTES + SK_X_BYTES;
 constexpr int SK_SMEM = SK_NST * SK_STAGE + SK_NA * SK_A_BYTES + 1024;
 constexpr int SK_THREADS = 320;
 constexpr uint32_t SK_IDESC = idesc_f16(SK_BM, US);
+// BF16 weights (the LM head): both operands BF16 (instruction-descriptor A/B format 1)
+constexpr uint32_t SK_IDESC_BF16 = SK_IDESC | (1u << 7) | (1u << 10);
+constexpr int SK_WB_BF16 = 2 * SK_A_HALF;  // BF16 weight tile 128 x 128 (two 64-column boxes)
+constexpr int SK_SMEM_BF16 = SK_NST * (SK_WB_BF16 + SK_X_BYTES) + 1024;
 constexpr int SK_UNITS_PER_CTA = 3;  // target units per CTA when choosing K slices
 constexpr int UN_ATT_CS = 8;         // attention cluster size: 16 sessions fill the GPU with 8-CTA clusters
 
@@ -82,11 +86,15 @@ __device__ __forceinline__ void i8x4_to_h(uint32_t w, uint32_t& lo, uint32_t& hi
     hi = *reinterpret_cast<const uint32_t*>(&hb);
 }
 
+// BW: BF16 weights (the LM head), read by the MMAs straight from the stage (no conversion).
+template <bool BW>
 __global__ void __launch_bounds__(SK_THREADS, 1)
     skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const SkArgs a) {
+    constexpr int WBYTES = BW ? SK_WB_BF16 : SK_W_BYTES;
+    constexpr int STAGE = WBYTES + SK_X_BYTES;
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-    uint8_t* ring = sm;                      // stage s: INT8 tile, then the activation tile
+    uint8_t* ring = sm;                      // stage s: weight tile, then the activation tile
     uint8_t* abuf = sm + SK_NST * SK_STAGE;  // SK_NA FP16 operand buffers
     __shared__ __align__(8) uint64_t full[SK_NST], empty[SK_NST], afull[SK_NA], aempty[SK_NA], accf[2], acce[2];
     __shared__ uint32_t tmem_base;
@@ -100,7 +108,7 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
         abort_flag = 0;
         for (int s = 0; s < SK_NST; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&empty[s]), 4 + 1);  // 4 converter warps + the MMAs that read the activations
+            mbar_init(smem_u32(&empty[s]), BW ? 1 : 4 + 1);  // converter warps (INT8) + the MMAs
         }
         for (int b = 0; b < SK_NA; ++b) {
             mbar_init(smem_u32(&afull[b]), 4);
@@ -133,11 +141,16 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
                     const int s = g % SK_NST;
                     if (g >= SK_NST) mbar_wait(smem_u32(&empty[s]), ((g / SK_NST) - 1) & 1, &abort_flag, a.err);
                     const uint32_t fb = smem_u32(&full[s]);
-                    mbar_expect_tx(fb, SK_STAGE);
-                    const uint32_t st = smem_u32(ring + s * SK_STAGE);
-                    tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
-                    tma_load_2d(st + SK_W_BYTES, &tmX, kb * SK_BK, 0, fb);
-                    tma_load_2d(st + SK_W_BYTES + SK_X_BYTES / 2, &tmX, kb * SK_BK + 64, 0, fb);
+                    mbar_expect_tx(fb, STAGE);
+                    const uint32_t st = smem_u32(ring + s * STAGE);
+                    if (BW) {
+                        tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
+                        tma_load_2d(st + SK_A_HALF, &tmW, kb * SK_BK + 64, tile * SK_BM, fb);
+                    } else {
+                        tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
+                    }
+                    tma_load_2d(st + WBYTES, &tmX, kb * SK_BK, 0, fb);
+                    tma_load_2d(st + WBYTES + SK_X_BYTES / 2, &tmX, kb * SK_BK + 64, 0, fb);
                 }
             }
             for (int k = max(0, g - SK_NST); k < g; ++k)  // no copy may outlive the CTA
@@ -154,25 +167,26 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
                 fence_after();
                 for (int kb = kb0; kb < kb1; ++kb, ++g) {
                     const int s = g % SK_NST, ab = g % SK_NA;
-                    mbar_wait(smem_u32(&afull[ab]), (g / SK_NA) & 1, &abort_flag, a.err);
+                    if (!BW) mbar_wait(smem_u32(&afull[ab]), (g / SK_NA) & 1, &abort_flag, a.err);
                     mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
                     fence_after();
-                    const uint32_t sa = smem_u32(abuf + ab * SK_A_BYTES);
-                    const uint32_t sx = smem_u32(ring + s * SK_STAGE + SK_W_BYTES);
+                    const uint32_t sa = BW ? smem_u32(ring + s * STAGE) : smem_u32(abuf + ab * SK_A_BYTES);
+                    const uint32_t sx = smem_u32(ring + s * STAGE + WBYTES);
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
                             mma_f16(tmem + 16u * acc, sw128_desc(sa + h * SK_A_HALF + kk * 32),
-                                    sw128_desc(sx + h * (SK_X_BYTES / 2) + kk * 32), SK_IDESC,
+                                    sw128_desc(sx + h * (SK_X_BYTES / 2) + kk * 32), BW ? SK_IDESC_BF16 : SK_IDESC,
                                     (kb > kb0 || h > 0 || kk > 0) ? 1u : 0u);
-                    commit(smem_u32(&aempty[ab]));
+                    if (!BW) commit(smem_u32(&aempty[ab]));
                     commit(smem_u32(&empty[s]));
                 }
                 commit(smem_u32(&accf[acc]));
             }
         }
-    } else if (warp < 6) {  // ---- converters: thread = weight row of the tile
+    } else if (warp < 6) {  // ---- converters (INT8 weights): thread = weight row of the tile
+      if constexpr (!BW) {
         const int r = (warp - 2) * 32 + lane;
         int g = 0;
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
@@ -183,7 +197,7 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
                 const int s = g % SK_NST, ab = g % SK_NA;
                 mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
                 if (g >= SK_NA) mbar_wait(smem_u32(&aempty[ab]), ((g / SK_NA) - 1) & 1, &abort_flag, a.err);
-                const uint8_t* wrow = ring + s * SK_STAGE + r * 128;
+                const uint8_t* wrow = ring + s * STAGE + r * 128;
                 uint8_t* arow = abuf + ab * SK_A_BYTES + r * 128;
                 const int sw = r & 7;  // 128-byte swizzle: 16-byte chunk c of row r sits at c ^ (r % 8)
 #pragma unroll
@@ -207,6 +221,7 @@ __global__ void __launch_bounds__(SK_THREADS, 1)
                 }
             }
         }
+      }
     } else {  // ---- epilogue warps 6-9: TMEM lanes 32 (warp % 4) ..
         const int q = warp & 3;
         int it = 0;
@@ -247,9 +262,10 @@ struct PrepArgs {
     float eps;
     const int* gmap;           // PR_HEADS: [US][Hkv] dense group -> plan group (-1: dropped)
     int g, dh, Hkv;
-    __half* x16;               // [US][ld16]
+    __half* x16;               // [US][ld16] (BF16 bits when bf16)
     int64_t ld16;
     float* xinv;               // [US]: 2^-e of the session's scale
+    int bf16;                  // write BF16 (for BF16 weights) instead of FP16
 };
 
 constexpr int PREP_CS = 8;  // CTAs (one cluster) per session in prep_kernel
@@ -351,10 +367,16 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepArgs p) {
     __half* dst = p.x16 + b * p.ld16;
     for (int k = k0 + 4 * threadIdx.x; k < k1; k += 4 * blockDim.x) {
         const float4 v = prep_in(p, x, b, k);
-        const __half2 h0 = __floats2half2_rn(v.x * sc, v.y * sc), h1 = __floats2half2_rn(v.z * sc, v.w * sc);
         uint2 o;
-        o.x = *reinterpret_cast<const uint32_t*>(&h0);
-        o.y = *reinterpret_cast<const uint32_t*>(&h1);
+        if (p.bf16) {
+            const __nv_bfloat162 h0 = __floats2bfloat162_rn(v.x * sc, v.y * sc), h1 = __floats2bfloat162_rn(v.z * sc, v.w * sc);
+            o.x = *reinterpret_cast<const uint32_t*>(&h0);
+            o.y = *reinterpret_cast<const uint32_t*>(&h1);
+        } else {
+            const __half2 h0 = __floats2half2_rn(v.x * sc, v.y * sc), h1 = __floats2half2_rn(v.z * sc, v.w * sc);
+            o.x = *reinterpret_cast<const uint32_t*>(&h0);
+            o.y = *reinterpret_cast<const uint32_t*>(&h1);
+        }
         *reinterpret_cast<uint2*>(dst + k) = o;
     }
     if (rank == 0 && threadIdx.x == 0) p.xinv[b] = ldexpf(1.f, -e);
@@ -451,6 +473,20 @@ __global__ void finish_gu_kernel(const GuFin p) {
     p.h[b * p.ld + c] = v;
 }
 
+// LM head: logits_b[row] = sum (no row scale: the head is BF16 as stored).
+struct LogitFin {
+    FinArgs f;
+    float* logits;  // [n][rows]
+};
+__global__ void finish_logits_kernel(const LogitFin p) {
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int row = (int)(t / US), b = (int)(t % US);
+    if (row >= p.f.rows || b >= p.f.n) return;
+    float acc = 0.f;
+    for (int s = 0; s < p.f.S; ++s) acc += p.f.part[((int64_t)s * p.f.rows + row) * US + b];
+    p.logits[(int64_t)b * p.f.rows + row] = acc * p.f.xinv[b];
+}
+
 struct UnAdvance {
     int* pos[US];
     int n;
@@ -504,15 +540,21 @@ void slices(int rows, int K, int sms, int& S, int& kbs) {
     S = (nkb + kbs - 1) / kbs;
 }
 
-int launch_skinny(const int8_t* W, int rows, int K, const __half* x16, int64_t ld16, float* part, int* err,
+// W: INT8 [rows][K], or BF16 [rows][K] when bw (the LM head)
+int launch_skinny(const void* W, bool bw, int rows, int K, const __half* x16, int64_t ld16, float* part, int* err,
                   int& S_out, cudaStream_t s) {
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
     if (K % SK_BK) return fail(TASP_EUNSUP, "union decode needs reduction lengths that are multiples of 128");
     CUtensorMap tw, tx;
-    if ((rc = map2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, W, rows, K, K, SK_BK, SK_BM))) return rc;
-    if ((rc = map2d(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, x16, US, K, ld16 * 2, 64, US))) return rc;
+    if (bw) {
+        if ((rc = map2d(&tw, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, rows, K, (int64_t)K * 2, 64, SK_BM))) return rc;
+        if ((rc = map2d(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x16, US, K, ld16 * 2, 64, US))) return rc;
+    } else {
+        if ((rc = map2d(&tw, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, W, rows, K, K, SK_BK, SK_BM))) return rc;
+        if ((rc = map2d(&tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, x16, US, K, ld16 * 2, 64, US))) return rc;
+    }
     SkArgs a{};
     a.rows = rows;
     a.K = K;
@@ -520,7 +562,10 @@ int launch_skinny(const int8_t* W, int rows, int K, const __half* x16, int64_t l
     a.part = part;
     a.err = err;
     const int units = ((rows + SK_BM - 1) / SK_BM) * a.S;
-    skinny_kernel<<<std::min(units, di.sms), SK_THREADS, SK_SMEM, s>>>(tw, tx, a);
+    if (bw)
+        skinny_kernel<true><<<std::min(units, di.sms), SK_THREADS, SK_SMEM_BF16, s>>>(tw, tx, a);
+    else
+        skinny_kernel<false><<<std::min(units, di.sms), SK_THREADS, SK_SMEM, s>>>(tw, tx, a);
     TASP_CUDA(cudaGetLastError());
     S_out = a.S;
     return TASP_OK;
@@ -559,6 +604,7 @@ size_t part_floats(const Shape& sh, int sms) {
     need(sh.d, sh.Hq * sh.dh);
     need(2 * sh.df, sh.d);
     need(sh.d, sh.df);
+    if (sh.vocab) need(sh.vocab, sh.d);
     return mx;
 }
 
@@ -625,7 +671,9 @@ int union_get(Session* const* ss, int n, UnionWs** out) {
     TASP_CUDA(cudaMemcpy(w->gmap, gm.data(), gm.size() * 4, cudaMemcpyHostToDevice));
     TASP_CUDA(cudaMemcpy(w->keep, kp.data(), kp.size(), cudaMemcpyHostToDevice));
     if (!g_skinny_attr) {  // before any stream capture
-        TASP_CUDA(cudaFuncSetAttribute(skinny_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SK_SMEM));
+        TASP_CUDA(cudaFuncSetAttribute(skinny_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SK_SMEM));
+        TASP_CUDA(cudaFuncSetAttribute(skinny_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       SK_SMEM_BF16));
         g_skinny_attr = true;
     }
     *out = w.get();
@@ -648,7 +696,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
     const int g = sh.g(), qd = sh.Hq * sh.dh, nu = sh.n_units();
     int rc = 0, nl = 0;
     auto prep = [&](int mode, const float* src, int64_t src_ld, const uint16_t* in_bf16, const float* gamma, int K,
-                    const int* gmap) -> int {
+                    const int* gmap, int bf16 = 0) -> int {
         PrepArgs p{};
         p.mode = mode;
         p.K = K;
@@ -664,6 +712,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         p.x16 = w.x16;
         p.ld16 = w.ld16;
         p.xinv = w.xinv;
+        p.bf16 = bf16;
         ++nl;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(PREP_CS, n);
@@ -696,7 +745,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         int S = 0;
         // Q/K/V for every session's kept groups
         if ((rc = prep(PR_NORM, w.x, sh.d, l == 0 ? w.x_stage : nullptr, ls.g_attn, sh.d, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.qkv, sh.qkv_rows_dense(), sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.qkv, false, sh.qkv_rows_dense(), sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
         ++nl;
         {
             QkvFin p{};
@@ -749,7 +798,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         }
         // O projection + residual (the dropped heads are zero in the scattered input)
         if ((rc = prep(PR_HEADS, w.o, qd, nullptr, nullptr, qd, gmap))) return rc;
-        if ((rc = launch_skinny(ls.o, sh.d, qd, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.o, false, sh.d, qd, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
         ++nl;
         {
             ResFin p{};
@@ -762,7 +811,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         }
         // gate/up + SiLU(gate) * up, zero for the dropped channel units
         if ((rc = prep(PR_NORM, w.x, sh.d, nullptr, ls.g_mlp, sh.d, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.gu, 2 * sh.df, sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.gu, false, 2 * sh.df, sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
         ++nl;
         {
             GuFin p{};
@@ -777,7 +826,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         }
         // down projection + residual
         if ((rc = prep(PR_COPY, w.h, sh.df, nullptr, nullptr, sh.df, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.down, sh.d, sh.df, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.down, false, sh.d, sh.df, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
         ++nl;
         {
             ResFin p{};
@@ -789,18 +838,18 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
             ++nl;
         }
     }
-    // final RMSNorm + LM head, up to four sessions per launch
+    // final RMSNorm + LM head (BF16) for all sessions in one weight pass
     if (logits) {
-        for (int b0 = 0; b0 < n; b0 += MAX_BATCH) {
-            BatchView bv;
-            bv.n = std::min(MAX_BATCH, n - b0);
-            for (int b = 0; b < bv.n; ++b) bv.ss[b] = w.ss[b0 + b];
-            bv.x = w.x + (size_t)b0 * sh.d;
-            bv.x_stride = sh.d;
-            bv.err = w.err;
-            if ((rc = enqueue_lm_heads(bv, logits + (size_t)b0 * sh.vocab, s))) return rc;
-            ++nl;
-        }
+        int S = 0;
+        if ((rc = prep(PR_NORM, w.x, sh.d, nullptr, st.g_final, sh.d, nullptr, 1))) return rc;
+        if ((rc = launch_skinny(st.lm_head, true, sh.vocab, sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        ++nl;
+        LogitFin p{};
+        p.f = fin(S, sh.vocab, nullptr);
+        p.logits = logits;
+        if ((rc = launch(finish_logits_kernel, dim3((unsigned)(((int64_t)sh.vocab * US + 255) / 256)), dim3(256), s, p)))
+            return rc;
+        ++nl;
     }
     UnAdvance ad{};
     ad.n = n;
