@@ -6,13 +6,15 @@
 // plan's compacted panels on the 5th-generation tensor cores:
 //  * operands FP16 (INT8 weights are exact in FP16; activations keep 11 significant
 //    bits), FP32 accumulators in tensor memory, per-weight-row scales in the epilogue;
-//  * a CTA computes a 128 x 256 output tile: warp 0 streams 128 x 64 and 256 x 64 operand
-//    tiles with TMA (128-byte swizzle) into a 4-stage ring, warp 1 allocates 256 TMEM
-//    columns and issues tcgen05.mma (M = 128, N = 256, K = 16 per instruction), warps 2-5
-//    read the accumulator back with tcgen05.ld and apply the epilogue;
+//  * one persistent CTA per SM walks 128 x 256 output tiles: warp 0 streams 128 x 64 and
+//    256 x 64 operand tiles with TMA (128-byte swizzle) into a 4-stage ring, warp 1
+//    allocates 512 TMEM columns (two accumulators) and issues tcgen05.mma (M = 128,
+//    N = 256, K = 16 per instruction), warps 2-5 read one accumulator back with tcgen05.ld
+//    and apply the epilogue while the MMAs fill the other;
 //  * every mbarrier wait is bounded and reports to the session's device error word.
-// Attention is a causal flash-attention on mma.sync (BF16 K/V from the cache, queries
-// and probabilities split into BF16 high/low halves as in the decode kernel).
+// Attention is a causal flash-attention over the kept heads: for head dim 128 on tcgen05
+// (S = Q K^T and O += P V in tensor memory, FP16 operands, softmax warps owning one query
+// row each), for head dim 64 on mma.sync with FP16 operands.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -22,69 +24,14 @@
 #include <mutex>
 
 #include "tasp_internal.h"
+#include "tc_ptx.cuh"
 
 namespace tasp {
 
 namespace {
 
-// ------------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-constexpr long long WAIT_LIMIT = 4000000000ll;  // clock cycles (~2 s)
-// Bounded wait: after WAIT_LIMIT cycles it records the failure and makes the CTA's later
-// waits return at once, so a lost transfer can never hang the GPU.
-__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
-                                          bool honor_abort = true) {
-    if (honor_abort && *(volatile int*)abort_flag) return;
-    if (mbar_try(bar, parity)) return;
-    const long long t0 = clock64();
-    while (!mbar_try(bar, parity)) {
-        if (clock64() - t0 > WAIT_LIMIT) {
-            *(volatile int*)abort_flag = 1;
-            if (err) atomicOr(err, 1);
-            return;
-        }
-    }
-}
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
-        "[%4];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
-        : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// UMMA shared-memory descriptor of a K-major operand tile written by TMA with 128-byte
-// swizzle: 8-row x 128-byte swizzle atoms stacked along the rows (stride 1024 bytes).
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address / 16
-    d |= (uint64_t)1 << 16;                     // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(1024 >> 4) << 32;           // stride byte offset: 8 rows x 128 bytes
-    d |= (uint64_t)1 << 46;                     // descriptor version of the 5th-generation tensor core
-    d |= (uint64_t)2 << 61;                     // swizzle: 128 bytes
-    return d;
-}
-// Instruction descriptor of kind::f16: D FP32, A and B FP16, both K-major, M x N.
-__host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
-    return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
+// ------------------------------------------------------------------ PTX helpers (tc_ptx.cuh)
+using namespace tc;
 
 // ------------------------------------------------------------------ GEMM
 // Persistent GEMM on the 5th-generation tensor cores: one CTA per SM walks 128 x 256 output
@@ -219,9 +166,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    tc_fence_before();
+    fence_before();
     __syncthreads();
-    tc_fence_after();
+    fence_after();
     const uint32_t tmem = tmem_base;
 
     if (warp == 0) {
@@ -249,11 +196,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
                 const int a = it & 1;
                 if (it >= 2) mbar_wait(smem_u32(&acc_empty[a]), ((it >> 1) - 1) & 1, &abort_flag, g.err);
-                tc_fence_after();
+                fence_after();
                 for (int kb = 0; kb < nk; ++kb, ++kbg) {
                     const int s = kbg % PG_STAGES;
                     mbar_wait(smem_u32(&bar_full[s]), (kbg / PG_STAGES) & 1, &abort_flag, g.err);
-                    tc_fence_after();
+                    fence_after();
                     const uint32_t sa = smem_u32(sm + s * PG_STAGE_BYTES), sb = sa + A_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
@@ -280,7 +227,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             const int a = it & 1;
             const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
             mbar_wait(smem_u32(&acc_full[a]), (it >> 1) & 1, &abort_flag, g.err);
-            tc_fence_after();
+            fence_after();
             const int row = m0 + 32 * q + lane;
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 32) {
@@ -297,15 +244,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
                 if (row < g.M) gemm_epi32(g, row, n0 + c0, r);
             }
-            tc_fence_before();
+            fence_before();
             __syncwarp();
             if (lane == 0)
                 asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[a])) : "memory");
         }
     }
-    tc_fence_before();
+    fence_before();
     __syncthreads();
-    tc_fence_after();
+    fence_after();
     if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
 }
 
@@ -725,19 +672,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
         "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
         : "memory");
 }
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void tc_mma(uint32_t tmem, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t accum) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
-        "l"(ad), "l"(bd), "r"(idesc), "r"(accum)
-        : "memory");
-}
-__device__ __forceinline__ void mbar_arrive1(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 
 __global__ void __launch_bounds__(192, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -778,9 +712,9 @@ __global__ void __launch_bounds__(192, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    tc_fence_before();
+    fence_before();
     __syncthreads();
-    tc_fence_after();
+    fence_after();
     const uint32_t tmem = tmem_base;
 
     if (warp == 0) {
@@ -806,38 +740,38 @@ __global__ void __launch_bounds__(192, 1)
     } else if (warp == 1) {
         if (lane == 0) {  // ---- MMA issuer
             mbar_wait(B(bar_q), 0, &abort_flag, err);
-            tc_fence_after();
+            fence_after();
             const uint32_t qa = smem_u32(sq);
             for (int j = 0; j <= ntile; ++j) {
                 if (j < ntile) {  // S_j = Q K_j^T into score buffer j % 2
                     const int s = j & 1;
                     mbar_wait(B(kv_full[s]), (j >> 1) & 1, &abort_flag, err);
                     if (j >= 2) mbar_wait(B(s_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
-                    tc_fence_after();
+                    fence_after();
                     const uint32_t kb = smem_u32(sst + s * AT_STAGE_BYTES);
 #pragma unroll
                     for (int blk = 0; blk < 2; ++blk)
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            tc_mma(tmem + 64u * s, sw128_desc(qa + blk * (AT_Q_BYTES / 2) + kk * 32),
+                            mma_f16(tmem + 64u * s, sw128_desc(qa + blk * (AT_Q_BYTES / 2) + kk * 32),
                                    sw128_desc(kb + blk * (AT_K_BYTES / 2) + kk * 32), IDESC_S, (blk | kk) ? 1u : 0u);
-                    tc_commit(B(s_full[s]));
+                    commit(B(s_full[s]));
                 }
                 if (j >= 1) {  // O += P_{j-1} V_{j-1}
                     const int jp = j - 1, s = jp & 1;
                     mbar_wait(B(p_full[s]), (jp >> 1) & 1, &abort_flag, err);
-                    tc_fence_after();
+                    fence_after();
                     const uint32_t pa = smem_u32(sp + s * AT_P_BYTES);
                     const uint32_t vb = smem_u32(sst + s * AT_STAGE_BYTES + AT_K_BYTES);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        tc_mma(tmem + 128u, sw128_desc(pa + kk * 32), sw128_desc(vb + kk * 32), IDESC_O,
+                        mma_f16(tmem + 128u, sw128_desc(pa + kk * 32), sw128_desc(vb + kk * 32), IDESC_O,
                                (jp > 0 || kk > 0) ? 1u : 0u);
-                    tc_commit(B(p_empty[s]));
-                    tc_commit(B(kv_empty[s]));
+                    commit(B(p_empty[s]));
+                    commit(B(kv_empty[s]));
                 }
             }
-            tc_commit(B(o_done));
+            commit(B(o_done));
         }
     } else {  // ---- softmax warps 2..5: TMEM lanes 32 (warp % 4) ..
         const int qw = warp & 3;
@@ -847,14 +781,14 @@ __global__ void __launch_bounds__(192, 1)
         for (int j = 0; j < ntile; ++j) {
             const int s = j & 1;
             mbar_wait(B(s_full[s]), (j >> 1) & 1, &abort_flag, err);
-            tc_fence_after();
+            fence_after();
             uint32_t v0[32], v1[32];
             tmem_ld32(trow + 64u * s, v0);
             tmem_ld32(trow + 64u * s + 32u, v1);
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            tc_fence_before();
+            fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive1(B(s_empty[s]));
+            if (lane == 0) mbar_arrive(B(s_empty[s]));
             float x[64];
             const int k0 = j * AT_KT;
             float mt = -INFINITY;
@@ -872,7 +806,7 @@ __global__ void __launch_bounds__(192, 1)
                 if (__any_sync(0xffffffffu, need)) {
                     // O must hold P_{j-1} V_{j-1} before it is rescaled
                     mbar_wait(B(p_empty[(j - 1) & 1]), ((j - 1) >> 1) & 1, &abort_flag, err);
-                    tc_fence_after();
+                    fence_after();
                     const float corr = need ? exp2f(m_run - mt) : 1.0f;
 #pragma unroll 1
                     for (int c0 = 0; c0 < 128; c0 += 32) {
@@ -907,12 +841,12 @@ __global__ void __launch_bounds__(192, 1)
                 *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) =
                     make_uint4(pw[4 * c], pw[4 * c + 1], pw[4 * c + 2], pw[4 * c + 3]);
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
-            tc_fence_before();
+            fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive1(B(p_full[s]));
+            if (lane == 0) mbar_arrive(B(p_full[s]));
         }
         mbar_wait(B(o_done), 0, &abort_flag, err);
-        tc_fence_after();
+        fence_after();
         const float inv = 1.0f / l_run;
 #pragma unroll 1
         for (int c0 = 0; c0 < 128; c0 += 32) {
@@ -930,9 +864,9 @@ __global__ void __launch_bounds__(192, 1)
             }
         }
     }
-    tc_fence_before();
+    fence_before();
     __syncthreads();
-    tc_fence_after();
+    fence_after();
     if (warp == 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(AT_TMEM_COLS) : "memory");
 }
