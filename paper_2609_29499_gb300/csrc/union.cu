@@ -24,6 +24,8 @@
 //  * warp 1 issues tcgen05.mma (M = 128, N = 16, K = 16) into one of two 16-column TMEM
 //    accumulators;
 //  * warps 6-9 read the accumulator (tcgen05.ld) and store the unit's FP32 partial sums.
+// The BF16 LM head runs through the same kernel: TMA writes its weight tiles straight into the
+// MMA operand layout (no conversion) and the activations are BF16.
 // Small finish kernels then sum the K slices in a fixed order, apply the row scales and
 // each session's mask, and run the projection's epilogue.
 #include <cuda.h>

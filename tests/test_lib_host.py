@@ -95,3 +95,18 @@ def test_invalid_requests_are_rejected(lib):
         lib.mask_select(bad, lib.all_keep_mask())
     assert e.value.code == lib.EINVAL
     assert "multiples of 16" in str(e.value)
+
+
+def test_union_step_argument_checks_need_no_gpu(lib):
+    # the union entry rejects a null session list, a null input and a session count outside
+    # 1..16 before it touches a session or the device
+    so = lib.load()
+    P = ctypes.c_void_p
+    arr = (P * 17)()
+    x = ctypes.c_void_p(16)  # never dereferenced: the count is rejected first
+    assert so.tasp_decode_step_union(None, 1, x, None, None, None) == lib.EINVAL
+    assert so.tasp_decode_step_union(arr, 1, None, None, None, None) == lib.EINVAL
+    for n in (0, 17, -1):
+        assert so.tasp_decode_step_union(arr, n, x, None, None, None) == lib.EINVAL
+    assert "16 sessions" in so.tasp_last_error().decode()
+    assert so.tasp_union_status(None, 1, None, None) == lib.EINVAL
