@@ -72,6 +72,12 @@ constexpr int SK_SMEM_BF16 = SK_NST * (SK_WB_BF16 + SK_X_BYTES) + 1024;
 constexpr int SK_UNITS_PER_CTA = 3;  // target units per CTA when choosing K slices
 constexpr int UN_ATT_CS = 8;         // attention cluster size: 16 sessions fill the GPU with 8-CTA clusters
 
+// Programmatic dependent launch: every union kernel lets the next one launch early and waits
+// for the previous one (all of whose writes it may read, and whose reads it may overwrite)
+// only where it first touches dependent data.
+__device__ __forceinline__ void grid_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 struct SkArgs {
     int rows, K;  // weight panel rows; reduction length (multiple of 128)
     int S, kbs;   // K slices and 128-column blocks per slice
@@ -135,10 +141,20 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
     __syncthreads();
     fence_after();
     const uint32_t tmem = tmem_base;
+    grid_trigger();
 
     if (warp == 0) {
         if (lane == 0) {  // ---- TMA producer
-            int g = 0;
+            // the first stages' weight tiles go out before the dependency wait (weights are
+            // constant); activations, written by the previous kernel, after it
+            int g = 0, xs = 0;  // stages issued, stages whose activation tile is issued
+            auto issue_x = [&](int gx, int kb) {
+                const uint32_t st = smem_u32(ring + (gx % SK_NST) * STAGE);
+                const uint32_t fb = smem_u32(&full[gx % SK_NST]);
+                tma_load_2d(st + WBYTES, &tmX, kb * SK_BK, 0, fb);
+                tma_load_2d(st + WBYTES + SK_X_BYTES / 2, &tmX, kb * SK_BK + 64, 0, fb);
+            };
+            int pre_kb[SK_NST];
             for (int u = blockIdx.x; u < units; u += gridDim.x) {
                 const int tile = u / a.S, ks = u - tile * a.S;
                 const int kb0 = ks * a.kbs, kb1 = min(nkb, kb0 + a.kbs);
@@ -148,15 +164,23 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
                     const uint32_t fb = smem_u32(&full[s]);
                     mbar_expect_tx(fb, STAGE);
                     const uint32_t st = smem_u32(ring + s * STAGE);
-                    if (BW) {
-                        tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
-                        tma_load_2d(st + SK_A_HALF, &tmW, kb * SK_BK + 64, tile * SK_BM, fb);
+                    tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
+                    if (BW) tma_load_2d(st + SK_A_HALF, &tmW, kb * SK_BK + 64, tile * SK_BM, fb);
+                    if (g < SK_NST) {
+                        pre_kb[g] = kb;
+                        if (g == SK_NST - 1) {
+                            grid_wait();
+                            for (; xs <= g; ++xs) issue_x(xs, pre_kb[xs]);
+                        }
                     } else {
-                        tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
+                        issue_x(g, kb);
+                        xs = g + 1;
                     }
-                    tma_load_2d(st + WBYTES, &tmX, kb * SK_BK, 0, fb);
-                    tma_load_2d(st + WBYTES + SK_X_BYTES / 2, &tmX, kb * SK_BK + 64, 0, fb);
                 }
+            }
+            if (xs < g || g == 0) {  // fewer k-blocks than stages: their activations are still due
+                grid_wait();
+                for (; xs < g; ++xs) issue_x(xs, pre_kb[xs]);
             }
             for (int k = max(0, g - SK_NST); k < g; ++k)  // no copy may outlive the CTA
                 mbar_wait(smem_u32(&full[k % SK_NST]), (k / SK_NST) & 1, &abort_flag, a.err, false);
@@ -319,6 +343,8 @@ __device__ __forceinline__ float4 prep_in(const PrepArgs& p, const float* src, i
 // below 2^14, as FP16. Each CTA takes K/8 entries; the cluster combines the sum of squares
 // and the largest magnitude through distributed shared memory.
 __global__ void __launch_bounds__(256) prep_kernel(const PrepArgs p) {
+    grid_wait();
+    grid_trigger();
     __shared__ float2 red[8];
     __shared__ float2 tot;  // this CTA's (sum of squares, max |in|)
     const int b = blockIdx.y, rank = blockIdx.x;  // cluster = the session's 8 CTAs along x
@@ -415,6 +441,8 @@ struct QkvFin {
     int max_tokens[US];
 };
 __global__ void finish_qkv_kernel(const QkvFin p) {
+    grid_wait();
+    grid_trigger();
     const int hb = blockIdx.x, half = p.dh >> 1;
     const int b = threadIdx.x % US, i = threadIdx.x / US;
     if (b >= p.f.n || i >= half) return;
@@ -450,6 +478,8 @@ struct ResFin {
     float* hidden;  // [n][ld] or nullptr
 };
 __global__ void finish_resid_kernel(const ResFin p) {
+    grid_wait();
+    grid_trigger();
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int row = (int)(t / US), b = (int)(t % US);
     if (row >= p.f.rows || b >= p.f.n) return;
@@ -467,6 +497,8 @@ struct GuFin {
     int n_units, cu;
 };
 __global__ void finish_gu_kernel(const GuFin p) {
+    grid_wait();
+    grid_trigger();
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int c = (int)(t / US), b = (int)(t % US);
     if (2 * c >= p.f.rows || b >= p.f.n) return;
@@ -484,6 +516,8 @@ struct LogitFin {
     float* logits;  // [n][rows]
 };
 __global__ void finish_logits_kernel(const LogitFin p) {
+    grid_wait();
+    grid_trigger();
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int row = (int)(t / US), b = (int)(t % US);
     if (row >= p.f.rows || b >= p.f.n) return;
@@ -497,6 +531,7 @@ struct UnAdvance {
     int n;
 };
 __global__ void union_advance_kernel(const UnAdvance a) {
+    grid_wait();
     if (threadIdx.x < a.n) *a.pos[threadIdx.x] += 1;
 }
 
@@ -545,6 +580,32 @@ void slices(int rows, int K, int sms, int& S, int& kbs) {
     S = (nkb + kbs - 1) / kbs;
 }
 
+// Launch with programmatic stream serialization (the kernel waits with griddepcontrol.wait);
+// cluster_x > 1 adds a cluster dimension.
+template <typename K, typename... A>
+int launch_pdl(K kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, int cluster_x, const A&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = cluster_x;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = cluster_x > 1 ? 2 : 1;
+    TASP_CUDA(cudaLaunchKernelEx(&cfg, kern, args...));
+    return TASP_OK;
+}
+template <typename K, typename A>
+int launch(K kern, dim3 grid, dim3 block, cudaStream_t s, const A& a) {
+    return launch_pdl(kern, grid, block, 0, s, 1, a);
+}
+
 // W: INT8 [rows][K], or BF16 [rows][K] when bw (the LM head)
 int launch_skinny(const void* W, bool bw, int rows, int K, const __half* x16, int64_t ld16, float* part, int* err,
                   int& S_out, cudaStream_t s) {
@@ -568,11 +629,11 @@ int launch_skinny(const void* W, bool bw, int rows, int K, const __half* x16, in
     a.err = err;
     const int units = ((rows + SK_BM - 1) / SK_BM) * a.S;
     const int grid = std::min(units, SK_CTAS_PER_SM * di.sms);
-    if (bw)
-        skinny_kernel<true><<<grid, SK_THREADS, SK_SMEM_BF16, s>>>(tw, tx, a);
-    else
-        skinny_kernel<false><<<grid, SK_THREADS, SK_SMEM, s>>>(tw, tx, a);
-    TASP_CUDA(cudaGetLastError());
+    if (bw) {
+        if ((rc = launch_pdl(skinny_kernel<true>, dim3(grid), dim3(SK_THREADS), SK_SMEM_BF16, s, 1, tw, tx, a))) return rc;
+    } else {
+        if ((rc = launch_pdl(skinny_kernel<false>, dim3(grid), dim3(SK_THREADS), SK_SMEM, s, 1, tw, tx, a))) return rc;
+    }
     S_out = a.S;
     return TASP_OK;
 }
@@ -687,12 +748,6 @@ int union_get(Session* const* ss, int n, UnionWs** out) {
     return TASP_OK;
 }
 
-template <typename K, typename A>
-int launch(K kern, dim3 grid, dim3 block, cudaStream_t s, const A& a) {
-    kern<<<grid, block, 0, s>>>(a);
-    TASP_CUDA(cudaGetLastError());
-    return TASP_OK;
-}
 
 // One union step on `s` (inputs in w.x_stage).
 int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int* launches) {
@@ -720,19 +775,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         p.xinv = w.xinv;
         p.bf16 = bf16;
         ++nl;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(PREP_CS, n);
-        cfg.blockDim = dim3(256);
-        cfg.stream = s;
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeClusterDimension;
-        at[0].val.clusterDim.x = PREP_CS;
-        at[0].val.clusterDim.y = 1;
-        at[0].val.clusterDim.z = 1;
-        cfg.attrs = at;
-        cfg.numAttrs = 1;
-        TASP_CUDA(cudaLaunchKernelEx(&cfg, prep_kernel, p));
-        return TASP_OK;
+        return launch_pdl(prep_kernel, dim3(PREP_CS, n), dim3(256), 0, s, PREP_CS, p);
     };
     auto fin = [&](int S, int rows, const float* scale) {
         FinArgs f{};
