@@ -427,7 +427,8 @@ __device__ __forceinline__ float fin_sum(const FinArgs& f, int row, int b) {
     return acc * f.scale[row] * f.xinv[b];
 }
 
-// Q/K/V: block = one dense head row block (group j, head hh of g + 2); thread = (pair i, session b).
+// Q/K/V: blockIdx.x = one dense head row block (group j, head hh of g + 2), blockIdx.y = a
+// quarter of its rotary pairs; thread = (pair i, session b).
 struct QkvFin {
     FinArgs f;
     int g, dh, Hkv;
@@ -444,7 +445,7 @@ __global__ void finish_qkv_kernel(const QkvFin p) {
     grid_wait();
     grid_trigger();
     const int hb = blockIdx.x, half = p.dh >> 1;
-    const int b = threadIdx.x % US, i = threadIdx.x / US;
+    const int b = threadIdx.x % US, i = blockIdx.y * (blockDim.x / US) + threadIdx.x / US;
     if (b >= p.f.n || i >= half) return;
     const int j = hb / (p.g + 2), hh = hb - j * (p.g + 2);
     const int lj = p.gmap[b * p.Hkv + j];
@@ -812,7 +813,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
                 p.pos[b] = w.ss[b]->d_pos;
                 p.max_tokens[b] = w.ss[b]->max_tokens;
             }
-            if ((rc = launch(finish_qkv_kernel, dim3(sh.Hkv * (g + 2)), dim3(US * (sh.dh / 2)), s, p))) return rc;
+            if ((rc = launch(finish_qkv_kernel, dim3(sh.Hkv * (g + 2), 4), dim3(US * (sh.dh / 8)), s, p))) return rc;
             ++nl;
         }
         // attention of each session over its own kept groups
