@@ -5,7 +5,8 @@ Each session must match the oracle's decode of that session alone under its own 
 (the mask-as-zero forward of Sec. 3), and agree with the per-plan decode path. Covered:
 three kinds of plan (a greedy mask, the dense fallback, an explicit ragged mask), the
 largest step (16 sessions), ragged contexts, the 8B widths with all five masks plus the
-dense plan, logits, and the argument errors.
+dense plan, logits, the 70B widths with 16 sessions, bit-identical repeats and panel
+layouts, and the argument errors.
 """
 import dataclasses
 
@@ -213,5 +214,56 @@ def test_8b_two_layers_union_all_masks(tasp):
         assert rel_l2(lg[:, i], lg_pp[:, i]) <= TOL_UNION
     for s in ss:
         s.release()
+    for p in plans:
+        p.release()
+
+
+def test_union_is_deterministic_and_ignores_panel_layout(tasp, layer1_plans):
+    # the union step sums in a fixed order (no atomics), and it reads the shared store
+    # whatever a plan's panel layout: compacted and row-indexed plans give the same bits
+    wl, plans, _ = layer1_plans
+    sh = wl.shape
+    steps, n = 3, 5
+    pick = [0, 1, 2, 0, 1]
+    t_priors, kv_seeds = [128, 9, 64, 33, 100], [3, 4, 5, 6, 7]
+    xb = synth.step_inputs_bf16(91, steps, n, sh.d)
+    outs = []
+    for _ in range(2):
+        ss = _make(tasp, [plans[k] for k in pick], t_priors, kv_seeds, steps)
+        outs.append(_run_union(tasp, ss, xb)[0])
+        for s in ss:
+            s.release()
+    assert np.array_equal(outs[0].view(np.uint32), outs[1].view(np.uint32))
+    row = lib_plan(tasp, sh, wl.masks[0], panel_mode=tasp.PANELS_ROW_INDEXED)
+    ss = _make(tasp, [row if k == 0 else plans[k] for k in pick], t_priors, kv_seeds, steps)
+    got = _run_union(tasp, ss, xb)[0]
+    for s in ss:
+        s.release()
+    row.release()
+    assert np.array_equal(got.view(np.uint32), outs[0].view(np.uint32))
+
+
+def test_70b_width_sixteen_sessions_agree_with_per_plan(tasp):
+    # the 70B widths (two-layer cut): 16 sessions over the five masks and the dense plan, the
+    # down projection's 28,672-long reduction split in K slices; agreement with the per-plan path
+    sh = dataclasses.replace(synth.LLAMA3_70B, L=2)
+    recipes = list(synth.CFG5.masks)
+    plans = [lib_plan(tasp, sh, r) for r in recipes] + [tasp.Plan(sh, tasp.all_keep_mask())]
+    n, steps = 16, 2
+    pick = [(i * 7) % 6 for i in range(n)]
+    t_priors = [64 + 37 * i for i in range(n)]
+    kv_seeds = [500 + i for i in range(n)]
+    xb = synth.step_inputs_bf16(707, steps, n, sh.d)
+    ss = _make(tasp, [plans[k] for k in pick], t_priors, kv_seeds, steps)
+    got, _ = _run_union(tasp, ss, xb)
+    assert tasp.union_status(ss)[0] == 0
+    for s in ss:
+        s.release()
+    ss = _make(tasp, [plans[k] for k in pick], t_priors, kv_seeds, steps)
+    ref, _ = _run_per_plan(tasp, ss, xb)
+    for s in ss:
+        s.release()
+    for i in range(n):
+        assert rel_l2(got[:, i], ref[:, i]) <= TOL_UNION, (i, pick[i], rel_l2(got[:, i], ref[:, i]))
     for p in plans:
         p.release()
