@@ -912,9 +912,10 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
 
 int union_check(Session* const* ss, int n, bool step) {
     if (n < 1 || n > US) return fail(TASP_EINVAL, "a union step holds 1 to 16 sessions");
+    for (int b = 0; b < n; ++b)
+        if (!ss[b] || ss[b]->magic != SESSION_MAGIC) return fail(TASP_EINVAL, "invalid session handle");
     const Store* st = ss[0]->plan->store;
     for (int b = 0; b < n; ++b) {
-        if (!ss[b] || ss[b]->magic != SESSION_MAGIC) return fail(TASP_EINVAL, "invalid session handle");
         if (ss[b]->plan->store != st) return fail(TASP_EMASK, "union step sessions must share one weight store");
         if (step && ss[b]->pos >= ss[b]->max_tokens) return fail(TASP_ECAP, "KV capacity exhausted");
         for (int c = 0; c < b; ++c)
