@@ -58,9 +58,11 @@ typedef struct tasp_model_desc {
 } tasp_model_desc;
 
 enum tasp_mask_kind {
-    TASP_MASK_ALL_KEEP = 0, /* dense fallback: every unit retained; panels are the store itself */
-    TASP_MASK_GREEDY = 1,   /* budgeted greedy by score per active FLOP with closure (Sec. 3.3) */
-    TASP_MASK_EXPLICIT = 2  /* caller-given retained groups / channel units per layer */
+    TASP_MASK_ALL_KEEP = 0,       /* dense fallback: every unit retained; panels are the store itself */
+    TASP_MASK_GREEDY = 1,         /* budgeted greedy by score per active FLOP with closure (Sec. 3.3) */
+    TASP_MASK_EXPLICIT = 2,       /* caller-given retained groups / channel units per layer */
+    TASP_MASK_GREEDY_QHEADS = 3,  /* the greedy over query-head candidates (Sec. 3.3, Table 1) */
+    TASP_MASK_EXPLICIT_QHEADS = 4 /* caller-given retained query heads / channel units per layer */
 };
 
 enum tasp_panel_mode {
@@ -76,6 +78,13 @@ enum tasp_panel_mode {
  * [r_lo, r_hi] the per-layer retention range. For kind EXPLICIT:
  * keep_groups / keep_units are host int32 lists concatenated over layers with
  * n_groups / n_units [L] giving each layer's count (indices ascending).
+ * Query-head kinds (Sec. 3.3: a KV head stays whenever one of its query heads
+ * does; query heads never move across groups): GREEDY_QHEADS takes `scores`
+ * [L][Hq + df/chan_unit] (query heads first, then channel units) with the
+ * same budget fields, and charges a head its Q rows and O columns plus, for
+ * the first head of a group, the group's K and V rows; EXPLICIT_QHEADS takes
+ * keep_qheads / n_qheads (ascending heads, concatenated over layers) with
+ * keep_units / n_units, and keeps the KV head of every listed head.
  * Unused fields may be NULL / 0. */
 typedef struct tasp_mask_desc {
     int32_t kind;
@@ -87,6 +96,8 @@ typedef struct tasp_mask_desc {
     const int32_t* n_groups;
     const int32_t* keep_units;
     const int32_t* n_units;
+    const int32_t* keep_qheads;
+    const int32_t* n_qheads;
 } tasp_mask_desc;
 
 typedef struct tasp_plan tasp_plan;
@@ -103,6 +114,8 @@ typedef struct tasp_session tasp_session;
  * identical model_desc share it), runs the host mask compiler, packs the
  * panels on the device. sync. *out receives the plan.
  * Errors: EINVAL (bad desc, mask violates closure/budget, empty layer),
+ * EUNSUP (a query-head mask that keeps part of a group: the device kernels
+ * take whole GQA groups; query-head masks whose groups are whole compile),
  * ENOMEM, ECUDA. */
 int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out);
 
@@ -182,6 +195,14 @@ int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* 
  * flop-mlp), the total, the global budget B and the dense total. */
 int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
                      int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops);
+
+/* tasp_mask_select plus the retained query heads: keep_qheads [L*Hq] with
+ * n_qheads [L] (ascending per layer). For the group kinds these are all g heads
+ * of every kept group; for the query-head kinds keep_groups holds the KV heads
+ * that the closure keeps. Host only; any output may be NULL. */
+int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
+                            int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
+                            int32_t* n_units, int64_t* flops);
 
 /* ---------------------------------------------------------------------------
  * Introspection and measurement (tests and benchmark).

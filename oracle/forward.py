@@ -34,7 +34,7 @@ import numpy as np
 
 import synth
 from . import weights as wts
-from .pack import pack_layer
+from .pack import kept_qheads, pack_layer
 from .quant import dequantize_rows
 
 
@@ -71,13 +71,14 @@ def softmax(s, axis=-1):
     return e / np.sum(e, axis=axis, keepdims=True)
 
 
-def attend(q, K, V, g):
-    """q [Hq, d_h], K/V [Hkv, T, d_h] -> o [Hq, d_h] (GQA: head h reads group h // g)."""
+def attend(q, K, V, g, gmap=None):
+    """q [Hq, d_h], K/V [Hkv, T, d_h] -> o [Hq, d_h] (GQA: head h reads group h // g, or
+    the KV row ``gmap[h]`` when given)."""
     Hq, dh = q.shape
     o = np.empty_like(q)
     scale = q.dtype.type(1.0 / np.sqrt(dh))
     for h in range(Hq):
-        j = h // g
+        j = h // g if gmap is None else gmap[h]
         p = softmax((K[j] @ q[h]) * scale)
         o[h] = p @ V[j]
     return o
@@ -106,14 +107,28 @@ def layer_step(shape, W, x, Kc, Vc, pos):
     return x2.astype(dt), k, v
 
 
-def compact_weights(shape, lq, keep_groups, keep_chans, dtype=np.float32):
-    P = pack_layer(shape, lq, keep_groups, keep_chans)
+def compact_weights(shape, lq, keep_groups, keep_chans, dtype=np.float32, keep_qheads=None):
+    """Dequantized packed panels plus the row roles of the qkv panel: per kept group its
+    kept query heads' row blocks, then K, then V (``oracle.pack``); ``gmap`` gives each
+    kept query head the position of its KV head among the kept groups."""
+    P = pack_layer(shape, lq, keep_groups, keep_chans, keep_qheads)
+    qh = set(kept_qheads(shape, keep_groups, keep_qheads))
+    blocks, q_blk, k_blk, v_blk, gmap = 0, [], [], [], []
+    for i, j in enumerate(keep_groups):
+        for h in range(j * shape.g, (j + 1) * shape.g):
+            if h in qh:
+                q_blk.append(blocks)
+                gmap.append(i)
+                blocks += 1
+        k_blk.append(blocks)
+        v_blk.append(blocks + 1)
+        blocks += 2
     return dict(qkv=dequantize_rows(P["qkv_w"], P["qkv_s"], dtype),
                 o=dequantize_rows(P["o_w"], P["o_s"], dtype),
                 gu=dequantize_rows(P["gu_w"], P["gu_s"], dtype),
                 down=dequantize_rows(P["down_w"], P["down_s"], dtype),
                 g_attn=lq.g_attn.astype(dtype), g_mlp=lq.g_mlp.astype(dtype),
-                m_kv=len(keep_groups))
+                m_kv=len(keep_groups), q_blk=q_blk, k_blk=k_blk, v_blk=v_blk, gmap=gmap)
 
 
 def layer_step_compact(shape, P, x, Kc, Vc, pos):
@@ -121,14 +136,14 @@ def layer_step_compact(shape, P, x, Kc, Vc, pos):
     dt = x.dtype
     g, dh, m = shape.g, shape.dh, P["m_kv"]
     xn = rmsnorm(x, P["g_attn"], shape.eps)
-    y = (P["qkv"] @ xn).reshape(m, g + 2, dh)
+    y = (P["qkv"] @ xn).reshape(-1, dh)
     c, s = rope_cos_sin([pos], dh, shape.rope_theta)
-    q = apply_rope(y[:, :g, :].reshape(m * g, dh), c, s)
-    k = apply_rope(y[:, g, :], c, s)
-    v = y[:, g + 1, :]
+    q = apply_rope(y[P["q_blk"]], c, s)
+    k = apply_rope(y[P["k_blk"]], c, s)
+    v = y[P["v_blk"]]
     K = np.concatenate([Kc, k[:, None, :]], axis=1)
     V = np.concatenate([Vc, v[:, None, :]], axis=1)
-    o = attend(q, K, V, g).reshape(-1) if m else np.zeros(0, dt)
+    o = attend(q, K, V, g, P["gmap"]).reshape(-1) if len(P["gmap"]) else np.zeros(0, dt)
     x1 = x + P["o"] @ o
     xn2 = rmsnorm(x1, P["g_mlp"], shape.eps)
     z = P["gu"] @ xn2
@@ -163,15 +178,15 @@ def decode(shape, mask, x_steps, t_prior, kv_seed, compact=False, dtype=np.float
     S = X.shape[0]
     for layer in (range(shape.L) if layers is None else layers):
         lq = wts.gen_layer(shape, layer)
-        kg, kc = mask.keep_groups[layer], mask.keep_chans[layer]
+        kg, kc, qh = mask.keep_groups[layer], mask.keep_chans[layer], mask.qheads(shape, layer)
         if prior is not None:
             Kd, Vd = prior(layer)
             Kd, Vd = np.asarray(Kd, dtype), np.asarray(Vd, dtype)
         if compact:
-            W = compact_weights(shape, lq, kg, kc, dtype)
+            W = compact_weights(shape, lq, kg, kc, dtype, qh)
             Kc, Vc = (Kd[kg], Vd[kg]) if prior is not None else prior_cache(shape, layer, kv_seed, t_prior, kg, dtype)
         else:
-            W = wts.dense_zeroed(shape, lq, kg, kc, dtype)
+            W = wts.dense_zeroed(shape, lq, kg, kc, dtype, qh)
             Kc, Vc = (Kd, Vd) if prior is not None else prior_cache(shape, layer, kv_seed, t_prior, None, dtype)
         nkv = Kc.shape[0]
         Kall = np.zeros((nkv, t_prior + S, shape.dh), dtype)
@@ -199,7 +214,8 @@ def decode_sessions(shape, mask, x_steps, t_priors, kv_seeds, dtype=np.float32):
     S, n = X.shape[0], X.shape[1]
     for layer in range(shape.L):
         lq = wts.gen_layer(shape, layer)
-        W = wts.dense_zeroed(shape, lq, mask.keep_groups[layer], mask.keep_chans[layer], dtype)
+        W = wts.dense_zeroed(shape, lq, mask.keep_groups[layer], mask.keep_chans[layer], dtype,
+                             mask.qheads(shape, layer))
         for i in range(n):
             tp = int(t_priors[i])
             Kc, Vc = prior_cache(shape, layer, kv_seeds[i], tp, None, dtype)
@@ -265,7 +281,8 @@ def prefill(shape, mask, X, dtype=np.float32, layers=None):
     kv = []
     for layer in (range(shape.L) if layers is None else layers):
         lq = wts.gen_layer(shape, layer)
-        W = wts.dense_zeroed(shape, lq, mask.keep_groups[layer], mask.keep_chans[layer], dtype)
+        W = wts.dense_zeroed(shape, lq, mask.keep_groups[layer], mask.keep_chans[layer], dtype,
+                             mask.qheads(shape, layer))
         X, K, V = layer_prefill(shape, W, X)
         kv.append((K, V))
     return X, kv

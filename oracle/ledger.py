@@ -9,7 +9,8 @@ retained SwiGLU channels:
 The active-FLOP ratio is sum over layers of the retained FLOPs divided by the
 same sum at full width; embeddings, final norm and LM head are excluded from
 the budget (the paper states they are dense and enter both sides unchanged).
-A KV head is charged once per retained group.
+A KV head is charged once per retained group; with query-head candidates a
+query head costs 2 d d_h (Q) + 2 d_h d (O) and a KV head 4 d d_h (K and V).
 
 Pins: the closed forms of the three shapes (single layer 5,636,096 FLOP/layer,
 8B 436,207,616, 70B 1,711,276,032), the 70B candidate count 80 x (64 + 28) =
@@ -36,6 +37,16 @@ def group_cost(shape) -> int:
     return layer_flops(shape, shape.g, 1, 0)
 
 
+def qhead_cost(shape) -> int:
+    """FLOPs of one query head alone (its Q rows and O columns; Sec. 3.3 query-head candidates)."""
+    return layer_flops(shape, 1, 0, 0)
+
+
+def kv_cost(shape) -> int:
+    """FLOPs of one KV head (its K and V rows), charged by the closure with its first query head."""
+    return layer_flops(shape, 0, 1, 0)
+
+
 def chan_unit_cost(shape) -> int:
     """Marginal FLOPs of one SwiGLU channel unit (chan_unit coupled channels)."""
     return layer_flops(shape, 0, 0, shape.chan_unit)
@@ -51,13 +62,17 @@ def paper_candidate_count(shape) -> int:
     return shape.L * (shape.Hq + shape.df // 1024)
 
 
-def mask_flops(shape, keep_groups, keep_chans) -> int:
-    return sum(layer_flops(shape, shape.g * len(kg), len(kg), len(kc))
-               for kg, kc in zip(keep_groups, keep_chans))
+def mask_flops(shape, keep_groups, keep_chans, keep_qheads=None) -> int:
+    """Retained layer FLOPs of a mask; ``keep_qheads`` (per layer) overrides the g query
+    heads per kept group of a group-granular mask."""
+    if keep_qheads is None:
+        keep_qheads = [[0] * (shape.g * len(kg)) for kg in keep_groups]
+    return sum(layer_flops(shape, len(qh), len(kg), len(kc))
+               for kg, kc, qh in zip(keep_groups, keep_chans, keep_qheads))
 
 
-def mask_ratio(shape, keep_groups, keep_chans) -> float:
-    return mask_flops(shape, keep_groups, keep_chans) / (shape.L * dense_layer_flops(shape))
+def mask_ratio(shape, keep_groups, keep_chans, keep_qheads=None) -> float:
+    return mask_flops(shape, keep_groups, keep_chans, keep_qheads) / (shape.L * dense_layer_flops(shape))
 
 
 def launched_flops(panels_per_layer) -> int:

@@ -25,10 +25,20 @@ Readings used here (the paper leaves them open; all are listed in the design doc):
   unit while the total stays within B = floor(T sum F / 2**24) and its layer
   within floor(HI F_l / 2**24).
 
+Query-head candidates (``compile_mask_qheads``; Table 1 counts 64 per 70B
+layer): a query head is charged its Q rows and O columns, and the closure
+charges the K and V rows of its KV head to the first head of the group that is
+accepted, so the ratio of a head is taken over its marginal cost at the moment
+of the pick.
+
 Pins: the single-layer closed form (1 of 2 groups and top-832 channels, ratio
 0.569767...), agreement with a library sort (np.argsort) on the single-layer
 case, the budget window, per-layer range, maximality of the result and
-closure on every compiled mask.
+closure on every compiled mask. For query heads: hand-derived single-layer
+cases (one where the closure cost reverses the order of two heads, one where a
+second group does not fit, a ratio tie), two single-layer closed forms, the
+reduction to the group compiler at g = 1, closure minimality and maximality
+on the 8B/70B shapes.
 """
 from __future__ import annotations
 
@@ -51,10 +61,16 @@ def to_fixed(r: float) -> int:
 
 @dataclass
 class Mask:
-    keep_groups: list  # per layer, sorted kept group indices
+    keep_groups: list  # per layer, sorted kept group (KV head) indices
     keep_units: list   # per layer, sorted kept channel-unit indices
     keep_chans: list   # per layer, sorted kept channel indices
     info: dict = field(default_factory=dict)
+    keep_qheads: list | None = None  # per layer, sorted kept query heads; None = all g heads of each kept group
+
+    def qheads(self, shape, layer: int) -> list:
+        if self.keep_qheads is not None:
+            return self.keep_qheads[layer]
+        return [j * shape.g + i for j in self.keep_groups[layer] for i in range(shape.g)]
 
 
 def all_keep(shape) -> Mask:
@@ -157,6 +173,104 @@ def compile_mask(shape, scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85) -
 
 
 # --------------------------------------------------------------------------
+# Query-head candidates with the GQA closure (Sec. 3.3; Table 1: 64 query-head
+# candidates and 28 channel groups per 70B layer).
+# --------------------------------------------------------------------------
+
+def explicit_qheads(shape, qheads, units) -> Mask:
+    """Mask from kept query heads and channel units; the kept KV heads are the closure
+    (exactly the groups of the kept query heads)."""
+    kq = [sorted(int(h) for h in hs) for hs in qheads]
+    m = explicit(shape, [sorted({h // shape.g for h in hs}) for hs in kq], units)
+    m.keep_qheads = kq
+    return m
+
+
+def compile_mask_qheads(shape, scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85) -> Mask:
+    """Greedy dependency-closed mask over query heads and channel units.
+
+    ``scores`` [L, H_q + n_chan_units] (uint32): query heads first, then channel units.
+    The candidate's cost is its marginal active FLOPs with the closure applied first
+    (Sec. 3.3): a query head costs its Q rows and O columns, plus its KV head's K and
+    V rows when no query head of its group is kept yet; a channel unit costs its
+    gate/up rows and down columns. The greedy repeatedly accepts the candidate of
+    highest score per marginal cost among those that still fit; costs change as KV
+    heads come on, so the ratios are taken afresh at every pick. The phases, budgets
+    and tie order are those of ``compile_mask`` (query head before channel unit, then
+    lower index; globally lower layer first). With g = 1 a query head's marginal cost
+    is always a whole group's and the result equals ``compile_mask``'s.
+    """
+    L, Hq, g, U = shape.L, shape.Hq, shape.g, shape.n_chan_units
+    scores = np.asarray(scores, dtype=np.uint64)
+    assert scores.shape == (L, Hq + U)
+    c_q, c_kv, c_u = ledger.qhead_cost(shape), ledger.kv_cost(shape), ledger.chan_unit_cost(shape)
+    b, cap, B, tt = _layer_budgets(shape, target_u24, budget, r_lo, r_hi)
+
+    kept = [[False] * (Hq + U) for _ in range(L)]
+    kv_on = [[False] * shape.Hkv for _ in range(L)]
+    lcost = [0] * L
+
+    def marginal(layer, u):
+        if u < Hq:
+            return c_q + (0 if kv_on[layer][u // g] else c_kv)
+        return c_u
+
+    def accept(layer, u):
+        c = marginal(layer, u)
+        kept[layer][u] = True
+        if u < Hq:
+            kv_on[layer][u // g] = True
+        lcost[layer] += c
+        return c
+
+    def precedes(a, c, layer_first):
+        # a, c = (layer, unit, marginal cost): higher score/cost first, then the tie order
+        sa, sc = int(scores[a[0], a[1]]), int(scores[c[0], c[1]])
+        lhs, rhs = sa * c[2], sc * a[2]
+        if lhs != rhs:
+            return lhs > rhs
+        ka = (a[0], a[1] >= Hq, a[1]) if layer_first else (a[1] >= Hq, a[1], a[0])
+        kc = (c[0], c[1] >= Hq, c[1]) if layer_first else (c[1] >= Hq, c[1], c[0])
+        return ka < kc
+
+    def best_fitting(layers, fits, layer_first):
+        best = None
+        for layer in layers:
+            for u in range(Hq + U):
+                if kept[layer][u]:
+                    continue
+                cand = (layer, u, marginal(layer, u))
+                if fits(cand) and (best is None or precedes(cand, best, layer_first)):
+                    best = cand
+        return best
+
+    for layer in range(L):
+        # (1) forced minimum: best query head (with its KV head) and best channel unit
+        for lo_u, hi_u in ((0, Hq), (Hq, Hq + U)):
+            accept(layer, max(range(lo_u, hi_u), key=lambda u: (int(scores[layer, u]), -u)))
+        # (2) per-layer greedy within the layer budget
+        while True:
+            cand = best_fitting([layer], lambda c: lcost[c[0]] + c[2] <= b[c[0]], False)
+            if cand is None:
+                break
+            accept(layer, cand[1])
+    # (3) global top-up within B and the per-layer cap
+    total = sum(lcost)
+    while True:
+        cand = best_fitting(range(L), lambda c: total + c[2] <= B and lcost[c[0]] + c[2] <= cap[c[0]], True)
+        if cand is None:
+            break
+        total += accept(cand[0], cand[1])
+    qheads = [[u for u in range(Hq) if kept[layer][u]] for layer in range(L)]
+    units = [[u - Hq for u in range(Hq, Hq + U) if kept[layer][u]] for layer in range(L)]
+    m = explicit_qheads(shape, qheads, units)
+    dense = ledger.dense_layer_flops(shape) * L
+    m.info = dict(budget_flops=B, total_flops=total, dense_flops=dense, ratio=total / dense,
+                  layer_budget=b, layer_cap=cap, layer_flops=lcost, layer_target_fixed=tt)
+    return m
+
+
+# --------------------------------------------------------------------------
 # Dependency closure at the level of individual matrices (Sec. 3.3).
 # --------------------------------------------------------------------------
 
@@ -165,7 +279,7 @@ def expand(shape, mask: Mask) -> list[dict]:
     out = []
     for layer in range(shape.L):
         kg, kc = mask.keep_groups[layer], mask.keep_chans[layer]
-        qh = [j * shape.g + i for j in kg for i in range(shape.g)]
+        qh = mask.qheads(shape, layer)
         out.append(dict(q_heads=set(qh), kv_heads=set(kg), o_heads=set(qh),
                         gate=set(kc), up=set(kc), down=set(kc)))
     return out

@@ -6,8 +6,9 @@ tensors over one shared INT8 store. The panel layout the build uses (and
 which the library's panels must match byte for byte) is:
 
 * ``qkv``  [(m_q + 2 m_kv) d_h, d]: for each kept group j in ascending order,
-  the d_h rows of each of its g query heads (heads j g .. j g + g - 1), then
-  the d_h rows of K head j, then the d_h rows of V head j.
+  the d_h rows of each of its kept query heads (of heads j g .. j g + g - 1, all g
+  of them for a group-granular mask, ascending), then the d_h rows of K head j,
+  then the d_h rows of V head j.
 * ``o``    [d, m_q d_h]: the O-projection columns of the kept query heads in
   ascending head order; scales are the dense per-row scales [d].
 * ``gu``   [2 c, d]: for each kept channel c_i in ascending order, the gate
@@ -26,24 +27,33 @@ from __future__ import annotations
 import numpy as np
 
 
-def qkv_rows(shape, keep_groups):
+def kept_qheads(shape, keep_groups, keep_qheads=None):
+    """Kept query heads in ascending order (all g heads of each kept group by default)."""
+    if keep_qheads is None:
+        return [h for j in keep_groups for h in range(j * shape.g, (j + 1) * shape.g)]
+    return sorted(keep_qheads)
+
+
+def qkv_rows(shape, keep_groups, keep_qheads=None):
     """Dense-matrix row sources of the qkv panel: list of (proj, row)."""
     rows = []
     g, dh = shape.g, shape.dh
+    qh = set(kept_qheads(shape, keep_groups, keep_qheads))
     for j in keep_groups:
         for h in range(j * g, (j + 1) * g):
-            rows += [("q", h * dh + i) for i in range(dh)]
+            if h in qh:
+                rows += [("q", h * dh + i) for i in range(dh)]
         rows += [("k", j * dh + i) for i in range(dh)]
         rows += [("v", j * dh + i) for i in range(dh)]
     return rows
 
 
-def pack_layer(shape, lq, keep_groups, keep_chans) -> dict:
-    g, dh = shape.g, shape.dh
-    src = qkv_rows(shape, keep_groups)
+def pack_layer(shape, lq, keep_groups, keep_chans, keep_qheads=None) -> dict:
+    dh = shape.dh
+    src = qkv_rows(shape, keep_groups, keep_qheads)
     qkv_w = np.stack([lq.q[p][r] for p, r in src]) if src else np.zeros((0, shape.d), np.int8)
     qkv_s = np.array([lq.s[p][r] for p, r in src], dtype=np.float32)
-    ocols = [h * dh + i for j in keep_groups for h in range(j * g, (j + 1) * g) for i in range(dh)]
+    ocols = [h * dh + i for h in kept_qheads(shape, keep_groups, keep_qheads) for i in range(dh)]
     o_w = np.ascontiguousarray(lq.q["o"][:, ocols])
     kc = np.asarray(keep_chans, dtype=np.int64)
     gu_w = np.empty((2 * len(kc), shape.d), dtype=np.int8)

@@ -75,16 +75,26 @@ def lm_head_f32(shape, row0: int = 0, nrows: int | None = None) -> np.ndarray:
     return synth.bf16_to_f32(synth.lm_head_bf16(shape.seed, shape.vocab, shape.d, row0, nrows))
 
 
-def dense_zeroed(shape, lq: LayerQ, keep_groups, keep_chans, dtype=np.float32) -> dict:
-    """Dequantized dense matrices with the pruned units set to zero (mask-as-zero)."""
+def dense_zeroed(shape, lq: LayerQ, keep_groups, keep_chans, dtype=np.float32, keep_qheads=None) -> dict:
+    """Dequantized dense matrices with the pruned units set to zero (mask-as-zero).
+
+    ``keep_qheads`` (sorted query heads) prunes single query heads: their Q rows and O
+    columns are zeroed; K/V rows are zeroed for the groups not in ``keep_groups``. The
+    default keeps all g query heads of every kept group.
+    """
     g, dh = shape.g, shape.dh
     W = {name: dequantize_rows(lq.q[name], lq.s[name], dtype) for name in PROJ_NAMES}
-    drop_g = [j for j in range(shape.Hkv) if j not in set(keep_groups)]
-    for j in drop_g:
-        W["q"][j * g * dh:(j + 1) * g * dh, :] = 0
-        W["k"][j * dh:(j + 1) * dh, :] = 0
-        W["v"][j * dh:(j + 1) * dh, :] = 0
-        W["o"][:, j * g * dh:(j + 1) * g * dh] = 0
+    kg = set(keep_groups)
+    qh = set(keep_qheads) if keep_qheads is not None else {j * g + i for j in kg for i in range(g)}
+    assert all(h // g in kg for h in qh), "a kept query head needs its KV head (GQA closure)"
+    for h in range(shape.Hq):
+        if h not in qh:
+            W["q"][h * dh:(h + 1) * dh, :] = 0
+            W["o"][:, h * dh:(h + 1) * dh] = 0
+    for j in range(shape.Hkv):
+        if j not in kg:
+            W["k"][j * dh:(j + 1) * dh, :] = 0
+            W["v"][j * dh:(j + 1) * dh, :] = 0
     keep_c = np.zeros(shape.df, dtype=bool)
     keep_c[np.asarray(keep_chans, dtype=np.int64)] = True
     W["gate"][~keep_c, :] = 0

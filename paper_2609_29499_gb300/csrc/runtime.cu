@@ -552,20 +552,23 @@ extern "C" {
 const char* tasp_last_error(void) { return g_err.c_str(); }
 const char* tasp_version(void) { return "tasp-gb300 0.1 (sm_103a)"; }
 
-int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
-                     int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops) {
+int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
+                            int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
+                            int32_t* n_units, int64_t* flops) {
     Shape sh;
     int rc = validate_shape(model, sh, false);
     if (rc) return rc;
     if (!mask) return fail(TASP_EINVAL, "mask_desc is NULL");
     MaskSel sel;
     if ((rc = select_mask(sh, *mask, sel))) return rc;
-    size_t og = 0, ou = 0;
+    size_t og = 0, ou = 0, oq = 0;
     for (int l = 0; l < sh.L; ++l) {
         if (n_groups) n_groups[l] = (int32_t)sel.groups[l].size();
         if (n_units) n_units[l] = (int32_t)sel.units[l].size();
+        if (n_qheads) n_qheads[l] = (int32_t)sel.qheads[l].size();
         for (int j : sel.groups[l]) if (keep_groups) keep_groups[og++] = j;
         for (int u : sel.units[l]) if (keep_units) keep_units[ou++] = u;
+        for (int h : sel.qheads[l]) if (keep_qheads) keep_qheads[oq++] = h;
         if (flops) flops[l] = sel.layer_flops[l];
     }
     if (flops) {
@@ -574,6 +577,11 @@ int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, i
         flops[sh.L + 2] = sel.dense;
     }
     return TASP_OK;
+}
+
+int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
+                     int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops) {
+    return tasp_mask_select_qheads(model, mask, nullptr, nullptr, keep_groups, n_groups, keep_units, n_units, flops);
 }
 
 int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out) {
@@ -587,9 +595,13 @@ int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, 
         return fail(TASP_EINVAL, "unknown panel mode");
     MaskSel sel;
     if ((rc = select_mask(sh, *mask, sel))) return rc;
-    for (int l = 0; l < sh.L; ++l)
+    for (int l = 0; l < sh.L; ++l) {
         if (sel.groups[l].empty() && sel.units[l].empty())
             return fail(TASP_EINVAL, "mask leaves a layer empty (layer " + std::to_string(l) + ")");
+        if (sel.qheads[l].size() != sel.groups[l].size() * (size_t)sh.g())
+            return fail(TASP_EUNSUP, "query-head mask keeps part of a GQA group (layer " + std::to_string(l) +
+                                         "); the device kernels take whole groups");
+    }
     Store* st = nullptr;
     if ((rc = store_acquire(sh, &st))) return rc;
     auto p = std::make_unique<Plan>();

@@ -38,9 +38,10 @@ struct Shape {
 int64_t layer_flops(const Shape& s, int64_t m_q, int64_t m_kv, int64_t c);
 inline int64_t dense_layer_flops(const Shape& s) { return layer_flops(s, s.Hq, s.Hkv, s.df); }
 
-// Host mask compiler result: per layer kept groups and channel units (ascending).
+// Host mask compiler result: per layer kept groups (KV heads), query heads and channel
+// units (ascending). For the group-granular kinds `qheads` holds every head of each kept group.
 struct MaskSel {
-    std::vector<std::vector<int>> groups, units;
+    std::vector<std::vector<int>> groups, qheads, units;
     std::vector<int64_t> layer_flops;
     int64_t total = 0, budget = 0, dense = 0;
 };

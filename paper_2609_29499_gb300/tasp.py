@@ -18,7 +18,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libtasp.so")
 
 OK, EINVAL, EMASK, ECAP, ENOMEM, EBUSY, ECUDA, EUNSUP = 0, -1, -2, -3, -4, -5, -6, -7
-MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT = 0, 1, 2
+MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT, MASK_GREEDY_QHEADS, MASK_EXPLICIT_QHEADS = 0, 1, 2, 3, 4
 PANELS_COMPACT, PANELS_ROW_INDEXED = 0, 1
 (EXPORT_KEEP_GROUPS, EXPORT_KEEP_CHANS, EXPORT_QKV_W, EXPORT_QKV_S, EXPORT_O_W, EXPORT_O_S, EXPORT_GU_W,
  EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S) = range(10)
@@ -28,6 +28,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 # Symbols declared in include/tasp.h (the CPU test checks they are all exported).
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
+            "tasp_mask_select_qheads",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -45,7 +46,8 @@ class MaskDesc(ctypes.Structure):
     _fields_ = [("kind", c_int32), ("panel_mode", c_int32), ("flop_budget", c_double), ("r_lo", c_double),
                 ("r_hi", c_double), ("scores", POINTER(c_uint32)), ("target_u24", POINTER(c_uint32)),
                 ("keep_groups", POINTER(c_int32)), ("n_groups", POINTER(c_int32)),
-                ("keep_units", POINTER(c_int32)), ("n_units", POINTER(c_int32))]
+                ("keep_units", POINTER(c_int32)), ("n_units", POINTER(c_int32)),
+                ("keep_qheads", POINTER(c_int32)), ("n_qheads", POINTER(c_int32))]
 
 
 class PlanInfo(ctypes.Structure):
@@ -87,6 +89,7 @@ def load(path: str = LIB_PATH):
         "tasp_session_status": (c_int32, [P, c_int32, POINTER(c_int32)]),
         "tasp_decode_step_host": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
         "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
+        "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
         "tasp_plan_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
@@ -124,7 +127,7 @@ class _MaskArgs:
     """Owns the numpy buffers a MaskDesc points to."""
 
     def __init__(self, kind, panel_mode=PANELS_COMPACT, budget=0.57, r_lo=0.35, r_hi=0.85, scores=None,
-                 target_u24=None, groups=None, units=None):
+                 target_u24=None, groups=None, units=None, qheads=None):
         self.keep = []
         d = MaskDesc()
         d.kind, d.panel_mode, d.flop_budget, d.r_lo, d.r_hi = kind, panel_mode, budget, r_lo, r_hi
@@ -144,6 +147,12 @@ class _MaskArgs:
             d.n_groups = ng.ctypes.data_as(POINTER(c_int32))
             d.keep_units = ku.ctypes.data_as(POINTER(c_int32))
             d.n_units = nu.ctypes.data_as(POINTER(c_int32))
+        if qheads is not None:
+            kq = np.ascontiguousarray(np.concatenate([np.asarray(h, np.int32) for h in qheads] + [np.zeros(0, np.int32)]))
+            nq = np.ascontiguousarray([len(h) for h in qheads], dtype=np.int32)
+            self.keep += [kq, nq]
+            d.keep_qheads = kq.ctypes.data_as(POINTER(c_int32))
+            d.n_qheads = nq.ctypes.data_as(POINTER(c_int32))
         self.desc = d
 
 
@@ -153,6 +162,22 @@ def greedy_mask(scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85, panel_mod
 
 def explicit_mask(groups, units, panel_mode=PANELS_COMPACT):
     return _MaskArgs(MASK_EXPLICIT, panel_mode, groups=groups, units=units)
+
+
+def greedy_qhead_mask(scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85, panel_mode=PANELS_COMPACT):
+    """Greedy over query-head candidates; ``scores`` [L, Hq + df/chan_unit] (heads first)."""
+    return _MaskArgs(MASK_GREEDY_QHEADS, panel_mode, budget, r_lo, r_hi, scores=scores, target_u24=target_u24)
+
+
+def explicit_qhead_mask(qheads, units, panel_mode=PANELS_COMPACT):
+    """Retained query heads and channel units per layer; the closure adds their KV heads."""
+    m = _MaskArgs(MASK_EXPLICIT_QHEADS, panel_mode, qheads=qheads)
+    ku = np.ascontiguousarray(np.concatenate([np.asarray(u, np.int32) for u in units] + [np.zeros(0, np.int32)]))
+    nu = np.ascontiguousarray([len(u) for u in units], dtype=np.int32)
+    m.keep += [ku, nu]
+    m.desc.keep_units = ku.ctypes.data_as(POINTER(c_int32))
+    m.desc.n_units = nu.ctypes.data_as(POINTER(c_int32))
+    return m
 
 
 def all_keep_mask():
@@ -178,6 +203,32 @@ def mask_select(shape, mask: _MaskArgs):
         og += ng[layer]
         ou += nu[layer]
     return groups, units, fl
+
+
+def mask_select_qheads(shape, mask: _MaskArgs):
+    """Host-only mask compilation with the retained query heads:
+    (query heads per layer, KV heads per layer, channel units per layer, flops array)."""
+    lib = load()
+    L, U = shape.L, shape.df // shape.chan_unit
+    kq = np.zeros(L * shape.Hq, np.int32)
+    nq = np.zeros(L, np.int32)
+    kg = np.zeros(L * shape.Hkv, np.int32)
+    ng = np.zeros(L, np.int32)
+    ku = np.zeros(L * U, np.int32)
+    nu = np.zeros(L, np.int32)
+    fl = np.zeros(L + 3, np.int64)
+    md = model_desc(shape)
+    _check(lib.tasp_mask_select_qheads(ctypes.byref(md), ctypes.byref(mask.desc), kq.ctypes.data, nq.ctypes.data,
+                                       kg.ctypes.data, ng.ctypes.data, ku.ctypes.data, nu.ctypes.data,
+                                       fl.ctypes.data))
+    out = []
+    for flat, counts in ((kq, nq), (kg, ng), (ku, nu)):
+        lists, o = [], 0
+        for layer in range(L):
+            lists.append(flat[o:o + counts[layer]].tolist())
+            o += counts[layer]
+        out.append(lists)
+    return out[0], out[1], out[2], fl
 
 
 def _stream_ptr(stream):

@@ -110,3 +110,73 @@ def test_union_step_argument_checks_need_no_gpu(lib):
         assert so.tasp_decode_step_union(arr, n, x, None, None, None) == lib.EINVAL
     assert "16 sessions" in so.tasp_last_error().decode()
     assert so.tasp_union_status(None, 1, None, None) == lib.EINVAL
+
+
+# ---------------------------------------------------------------------------
+# Query-head candidates (Sec. 3.3, Table 1): the library's heap-based greedy against the
+# oracle's plain rescans, bit for bit.
+# ---------------------------------------------------------------------------
+
+QHEAD_CASES = [(synth.LAYER1, (1000, 1001)), (synth.LLAMA3_8B, synth.MASK_SEEDS), (synth.LLAMA3_70B, (1000, 1004)),
+               (synth.tiny_shape(L=7), (3, 4, 5)),
+               (synth.ModelShape(L=5, d=128, Hq=8, Hkv=2, dh=32, df=256, vocab=0, chan_unit=16), (21, 22))]
+
+
+@pytest.mark.parametrize("shape,seeds", QHEAD_CASES)
+def test_host_qhead_compiler_matches_oracle(lib, shape, seeds):
+    for seed in seeds:
+        for budget, lo, hi in ((0.57, 0.35, 0.85), (0.3, 0.2, 0.5)):
+            sc = synth.mask_scores_u32(seed, shape.L, shape.Hq + shape.n_chan_units)
+            tg = synth.layer_target_u24(seed, shape.L)
+            want = maskc.compile_mask_qheads(shape, sc, tg, budget, lo, hi)
+            qh, groups, units, fl = lib.mask_select_qheads(shape, lib.greedy_qhead_mask(sc, tg, budget, lo, hi))
+            assert qh == want.keep_qheads
+            assert groups == want.keep_groups
+            assert units == want.keep_units
+            assert fl[:shape.L].tolist() == want.info["layer_flops"]
+            assert fl[shape.L] == want.info["total_flops"]
+            assert fl[shape.L + 1] == want.info["budget_flops"]
+
+
+def test_host_qhead_hand_cases_match_oracle(lib):
+    # single-layer cases shaped like the oracle's hand-derived pins (4 channel units of 4
+    # channels, as the library wants df a multiple of 16), with ratio and score ties
+    sh = synth.ModelShape(L=1, d=64, Hq=4, Hkv=2, dh=16, df=16, vocab=0, chan_unit=4)
+    for q, ch, r in (([100, 60, 95, 0], [1, 0, 0, 0], 0.75), ([10**6, 4096, 0, 0], [10**5, 1536, 0, 0], 0.49),
+                     ([7, 7, 7, 7], [7, 7, 7, 7], 0.6), ([0, 0, 0, 0], [0, 0, 0, 0], 0.9)):
+        sc = np.array([q + ch], dtype=np.uint32)
+        want = maskc.compile_mask_qheads(sh, sc, [0], r, r, r)
+        qh, groups, units, fl = lib.mask_select_qheads(sh, lib.greedy_qhead_mask(sc, [0], r, r, r))
+        assert (qh, groups, units) == (want.keep_qheads, want.keep_groups, want.keep_units)
+        assert fl[sh.L] == want.info["total_flops"]
+
+
+def test_explicit_qhead_masks_and_group_kinds(lib):
+    sh = synth.tiny_shape(L=3)
+    q, u = [[1, 2, 3], [3], [0, 2]], [[0, 3], [2], [1, 4]]
+    qh, groups, units, fl = lib.mask_select_qheads(sh, lib.explicit_qhead_mask(q, u))
+    want = maskc.explicit_qheads(sh, q, u)
+    assert qh == q and groups == want.keep_groups == [[0, 1], [1], [0, 1]] and units == u
+    assert fl[sh.L] == ledger.mask_flops(sh, want.keep_groups, want.keep_chans, want.keep_qheads)
+    # group kinds report every head of each kept group
+    qh, groups, _, _ = lib.mask_select_qheads(sh, lib.explicit_mask([[1], [0, 1], [0]], [[0], [0], [0]]))
+    assert groups == [[1], [0, 1], [0]] and qh == [[2, 3], [0, 1, 2, 3], [0, 1]]
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select_qheads(sh, lib.explicit_qhead_mask([[2, 1], [0], [0]], u))  # not ascending
+    assert e.value.code == lib.EINVAL
+    with pytest.raises(lib.TaspError) as e:
+        lib.mask_select_qheads(sh, lib.explicit_qhead_mask([[4], [0], [0]], u))  # head out of range
+    assert e.value.code == lib.EINVAL
+
+
+def test_partial_group_plans_are_refused_before_device_work(lib):
+    # the device kernels take whole GQA groups: a query-head mask that keeps part of a group
+    # is refused by the host compiler before any store or panel is made
+    sh = synth.LAYER1
+    so = lib.load()
+    md = lib.model_desc(sh)
+    m = lib.explicit_qhead_mask([[0, 1, 4, 5, 6, 7]], [[0, 9]])
+    out = ctypes.c_void_p()
+    assert so.tasp_compile_mask(ctypes.byref(md), ctypes.byref(m.desc), ctypes.byref(out)) == lib.EUNSUP
+    assert "whole groups" in so.tasp_last_error().decode()
+    assert not out.value
