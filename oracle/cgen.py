@@ -43,6 +43,13 @@ def _load():
         lib.og_weight_int8.restype = ctypes.c_int
         lib.og_weight_int8.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                        ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int]
+        lib.og_quant_row_grouped.restype = None
+        lib.og_quant_row_grouped.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+                                             ctypes.c_void_p]
+        lib.og_weight_int8_grouped.restype = ctypes.c_int
+        lib.og_weight_int8_grouped.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                               ctypes.c_int64, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
+                                               ctypes.c_int]
         _lib = lib
     return _lib
 
@@ -83,4 +90,22 @@ def weight_int8(key: int, row0: int, nrows: int, cols: int, sigma: float):
     rc = _load().og_weight_int8(key, row0, nrows, cols, sigma, q.ctypes.data, s.ctypes.data, n_threads())
     if rc != 0:
         raise RuntimeError(f"og_weight_int8 failed with {rc}")
+    return q, s
+
+
+def quant_row_grouped(w: np.ndarray, group: int):
+    w = np.ascontiguousarray(w, dtype=np.float32)
+    q = np.empty(w.shape[0], dtype=np.int8)
+    s = np.empty(w.shape[0] // group, dtype=np.float32)
+    _load().og_quant_row_grouped(w.ctypes.data, w.shape[0], group, q.ctypes.data, s.ctypes.data)
+    return q, s
+
+
+def weight_int8_grouped(key: int, row0: int, nrows: int, cols: int, group: int, sigma: float):
+    q = np.empty((nrows, cols), dtype=np.int8)
+    s = np.empty((nrows, cols // group), dtype=np.float32)
+    rc = _load().og_weight_int8_grouped(key, row0, nrows, cols, group, sigma, q.ctypes.data, s.ctypes.data,
+                                        n_threads())
+    if rc != 0:
+        raise RuntimeError(f"og_weight_int8_grouped failed with {rc}")
     return q, s

@@ -9,6 +9,9 @@
  * Quantizer (the paper's "symmetric INT8 weights", Table 1, read per output
  * channel with FP32 scales): for a dense row w, a = max|w|, s = fl32(a / 127),
  * q = clamp(rint(fl32(w / s)), -127, 127); a zero row has s = 0 and q = 0.
+ * The groupwise variant (Table 1: group size 128, BF16 scales) applies the same
+ * rule to each run of `group` consecutive columns with the scale rounded to
+ * BF16 (nearest, ties to even on the FP32 bit pattern) before it divides.
  *
  * Build: gcc -O2 -ffp-contract=off -fno-fast-math -fPIC -shared -pthread.
  */
@@ -76,10 +79,45 @@ void og_quant_row(const float* w, int64_t n, int8_t* q, float* s_out) {
     }
 }
 
+/* FP32 -> nearest BF16 value (ties to even), as FP32; finite inputs. */
+static float og_bf16(float x) {
+    uint32_t u;
+    memcpy(&u, &x, 4);
+    u = (uint32_t)(((uint64_t)u + 0x7FFFu + ((u >> 16) & 1u)) >> 16) << 16;
+    float r;
+    memcpy(&r, &u, 4);
+    return r;
+}
+
+/* Quantize one dense FP32 row of n values in groups of `group` columns (n a multiple of
+ * group): q [n], s_out [n / group] (BF16 values held in FP32). */
+void og_quant_row_grouped(const float* w, int64_t n, int64_t group, int8_t* q, float* s_out) {
+    for (int64_t g0 = 0, gi = 0; g0 < n; g0 += group, ++gi) {
+        float a = 0.0f;
+        for (int64_t j = g0; j < g0 + group; ++j) {
+            float v = fabsf(w[j]);
+            if (v > a) a = v;
+        }
+        float sc = og_bf16(a / 127.0f);
+        s_out[gi] = sc;
+        if (sc == 0.0f) {
+            memset(q + g0, 0, (size_t)group);
+            continue;
+        }
+        for (int64_t j = g0; j < g0 + group; ++j) {
+            float r = rintf(w[j] / sc);
+            if (r > 127.0f) r = 127.0f;
+            if (r < -127.0f) r = -127.0f;
+            q[j] = (int8_t)r;
+        }
+    }
+}
+
 typedef struct {
     uint64_t key;
     int64_t abs0; /* absolute index of local row 0 */
     int64_t row0, row1, cols;
+    int64_t group; /* 0: one scale per row; else columns per scale group */
     float sigma;
     int8_t* q;
     float* s;
@@ -91,16 +129,35 @@ static void* og_worker(void* p) {
     if (!buf) return (void*)1;
     for (int64_t r = j->row0; r < j->row1; ++r) {
         og_normal(j->key, (uint64_t)(j->abs0 + r) * (uint64_t)j->cols, j->cols, j->sigma, buf);
-        og_quant_row(buf, j->cols, j->q + r * j->cols, j->s + r);
+        if (j->group)
+            og_quant_row_grouped(buf, j->cols, j->group, j->q + r * j->cols, j->s + r * (j->cols / j->group));
+        else
+            og_quant_row(buf, j->cols, j->q + r * j->cols, j->s + r);
     }
     free(buf);
     return 0;
 }
 
+static int og_run(uint64_t key, int64_t row0, int64_t nrows, int64_t cols, int64_t group, float sigma, int8_t* q,
+                  float* s, int nthreads);
+
 /* Regenerate rows [row0, row0+nrows) of a [rows, cols] N(0, sigma) matrix and quantize
  * each row; q is [nrows, cols], s is [nrows]. Returns 0 on success. */
 int og_weight_int8(uint64_t key, int64_t row0, int64_t nrows, int64_t cols, float sigma, int8_t* q,
                    float* s, int nthreads) {
+    return og_run(key, row0, nrows, cols, 0, sigma, q, s, nthreads);
+}
+
+/* As og_weight_int8 with groupwise scales: s is [nrows, cols / group]. Returns 3 when cols
+ * is not a positive multiple of group. */
+int og_weight_int8_grouped(uint64_t key, int64_t row0, int64_t nrows, int64_t cols, int64_t group, float sigma,
+                           int8_t* q, float* s, int nthreads) {
+    if (group < 1 || cols % group) return 3;
+    return og_run(key, row0, nrows, cols, group, sigma, q, s, nthreads);
+}
+
+static int og_run(uint64_t key, int64_t row0, int64_t nrows, int64_t cols, int64_t group, float sigma, int8_t* q,
+                  float* s, int nthreads) {
     if (nthreads < 1) nthreads = 1;
     if (nthreads > 256) nthreads = 256;
     if (nthreads > nrows) nthreads = (int)(nrows > 0 ? nrows : 1);
@@ -117,6 +174,7 @@ int og_weight_int8(uint64_t key, int64_t row0, int64_t nrows, int64_t cols, floa
         jobs[t].row0 = a;
         jobs[t].row1 = b;
         jobs[t].cols = cols;
+        jobs[t].group = group;
         jobs[t].sigma = sigma;
         jobs[t].q = q;
         jobs[t].s = s;

@@ -35,7 +35,7 @@ import numpy as np
 import synth
 from . import weights as wts
 from .pack import kept_qheads, pack_layer
-from .quant import dequantize_rows
+from .quant import dequantize
 
 
 def rmsnorm(x, gamma, eps):
@@ -123,10 +123,10 @@ def compact_weights(shape, lq, keep_groups, keep_chans, dtype=np.float32, keep_q
         k_blk.append(blocks)
         v_blk.append(blocks + 1)
         blocks += 2
-    return dict(qkv=dequantize_rows(P["qkv_w"], P["qkv_s"], dtype),
-                o=dequantize_rows(P["o_w"], P["o_s"], dtype),
-                gu=dequantize_rows(P["gu_w"], P["gu_s"], dtype),
-                down=dequantize_rows(P["down_w"], P["down_s"], dtype),
+    return dict(qkv=dequantize(P["qkv_w"], P["qkv_s"], dtype),
+                o=dequantize(P["o_w"], P["o_s"], dtype),
+                gu=dequantize(P["gu_w"], P["gu_s"], dtype),
+                down=dequantize(P["down_w"], P["down_s"], dtype),
                 g_attn=lq.g_attn.astype(dtype), g_mlp=lq.g_mlp.astype(dtype),
                 m_kv=len(keep_groups), q_blk=q_blk, k_blk=k_blk, v_blk=v_blk, gmap=gmap)
 

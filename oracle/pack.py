@@ -16,7 +16,10 @@ which the library's panels must match byte for byte) is:
 * ``down`` [d, c]: the down-projection columns of the kept channels; scales
   are the dense per-row scales [d].
 
-The all-keep mask packs to the shared store itself.
+The all-keep mask packs to the shared store itself. In a groupwise store the
+qkv / gu scale rows travel with their weight rows, and O / down keep the
+scale columns of the kept column groups (kept heads and channel units must
+then be whole scale groups: d_h and the channel unit multiples of the group).
 
 Pin: the compacted forward (oracle.forward, ``compact=True``) consumes these
 panels and must equal the mask-as-zero forward; a permuted or misaligned
@@ -48,20 +51,35 @@ def qkv_rows(shape, keep_groups, keep_qheads=None):
     return rows
 
 
+def _column_groups(cols, group):
+    """Scale groups of kept columns that come in whole runs of ``group``; else ValueError."""
+    cols = np.asarray(cols, dtype=np.int64)
+    if len(cols) % group or np.any(cols.reshape(-1, group) != cols[::group, None] + np.arange(group)) \
+            or np.any(cols[::group] % group):
+        raise ValueError("a groupwise store packs kept columns in whole scale groups only")
+    return cols[::group] // group
+
+
 def pack_layer(shape, lq, keep_groups, keep_chans, keep_qheads=None) -> dict:
-    dh = shape.dh
+    dh, grp = shape.dh, shape.quant_group
+    srow = (shape.d // grp,) if grp else ()  # trailing scale dims of a row of the qkv / gu panels
     src = qkv_rows(shape, keep_groups, keep_qheads)
     qkv_w = np.stack([lq.q[p][r] for p, r in src]) if src else np.zeros((0, shape.d), np.int8)
-    qkv_s = np.array([lq.s[p][r] for p, r in src], dtype=np.float32)
+    qkv_s = np.array([lq.s[p][r] for p, r in src], dtype=np.float32).reshape((len(src),) + srow)
     ocols = [h * dh + i for h in kept_qheads(shape, keep_groups, keep_qheads) for i in range(dh)]
     o_w = np.ascontiguousarray(lq.q["o"][:, ocols])
     kc = np.asarray(keep_chans, dtype=np.int64)
     gu_w = np.empty((2 * len(kc), shape.d), dtype=np.int8)
     gu_w[0::2] = lq.q["gate"][kc]
     gu_w[1::2] = lq.q["up"][kc]
-    gu_s = np.empty(2 * len(kc), dtype=np.float32)
+    gu_s = np.empty((2 * len(kc),) + srow, dtype=np.float32)
     gu_s[0::2] = lq.s["gate"][kc]
     gu_s[1::2] = lq.s["up"][kc]
     down_w = np.ascontiguousarray(lq.q["down"][:, kc])
-    return dict(qkv_w=qkv_w, qkv_s=qkv_s, o_w=o_w, o_s=lq.s["o"].copy(), gu_w=gu_w, gu_s=gu_s,
-                down_w=down_w, down_s=lq.s["down"].copy())
+    if grp:  # O / down keep the scales of the kept column groups
+        o_s = np.ascontiguousarray(lq.s["o"][:, _column_groups(ocols, grp)])
+        down_s = np.ascontiguousarray(lq.s["down"][:, _column_groups(kc, grp)])
+    else:
+        o_s, down_s = lq.s["o"].copy(), lq.s["down"].copy()
+    return dict(qkv_w=qkv_w, qkv_s=qkv_s, o_w=o_w, o_s=o_s, gu_w=gu_w, gu_s=gu_s,
+                down_w=down_w, down_s=down_s)

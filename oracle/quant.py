@@ -81,3 +81,13 @@ def dequantize_groupwise(q: np.ndarray, s: np.ndarray, group: int = 128, dtype=n
     rows, cols = q.shape
     qg = q.reshape(rows, cols // group, group).astype(dtype)
     return (qg * np.asarray(s, dtype=dtype)[:, :, None]).reshape(rows, cols).astype(dtype)
+
+
+def dequantize(q: np.ndarray, s: np.ndarray, dtype=np.float32) -> np.ndarray:
+    """Per-row (s [rows]) or groupwise (s [rows, cols / group]) dequantization."""
+    s = np.asarray(s)
+    if s.ndim == 1:
+        return dequantize_rows(q, s, dtype)
+    if q.shape[1] == 0:
+        return np.zeros(q.shape, dtype)
+    return dequantize_groupwise(q, s, q.shape[1] // s.shape[1], dtype)

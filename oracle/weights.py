@@ -3,7 +3,8 @@
 Every dense projection is generated in PyTorch [out, in] layout from the
 seeded recipe of ``synth`` (N(0, 0.02), FP32) and quantized per output row with
 ``oracle.quant`` (or, bit-identically, the oracle's C regenerator for large
-layers). The result is the shared INT8 store of the paper's backing-store
+layers); a shape with ``quant_group`` > 0 takes the groupwise format instead
+(one BF16 scale per output row and run of ``quant_group`` input columns). The result is the shared INT8 store of the paper's backing-store
 semantics (Appendix, "Backing-store semantics"): one copy of every projection,
 independent of any mask.
 """
@@ -15,7 +16,7 @@ import numpy as np
 
 import synth
 from . import cgen
-from .quant import dequantize_rows, quantize_rows
+from .quant import dequantize, quantize_groupwise, quantize_rows
 
 # (tensor id, rows, cols) of each projection as functions of the shape
 _PROJ = {
@@ -32,7 +33,8 @@ PROJ_NAMES = tuple(_PROJ)
 
 @dataclass
 class LayerQ:
-    """Quantized dense layer: q[name] int8 [out, in], s[name] float32 [out], norm gains."""
+    """Quantized dense layer: q[name] int8 [out, in], s[name] float32 [out] (or
+    [out, in / group] for a groupwise store), norm gains."""
     q: dict
     s: dict
     g_attn: np.ndarray
@@ -53,10 +55,13 @@ def gen_proj_q(shape, layer: int, name: str, row0: int = 0, nrows: int | None = 
     if use_c is None:
         use_c = nrows * cols > (1 << 20) and cgen.available()
     key = synth.stream_key(shape.seed, tid, layer, 0)
+    group = shape.quant_group
     if use_c:
+        if group:
+            return cgen.weight_int8_grouped(key, row0, nrows, cols, group, synth.WEIGHT_SIGMA)
         return cgen.weight_int8(key, row0, nrows, cols, synth.WEIGHT_SIGMA)
     w = synth.weight_f32(shape.seed, tid, layer, rows, cols, row0, nrows)
-    return quantize_rows(w)
+    return quantize_groupwise(w, group) if group else quantize_rows(w)
 
 
 def gen_layer(shape, layer: int, use_c: bool | None = None) -> LayerQ:
@@ -83,7 +88,7 @@ def dense_zeroed(shape, lq: LayerQ, keep_groups, keep_chans, dtype=np.float32, k
     default keeps all g query heads of every kept group.
     """
     g, dh = shape.g, shape.dh
-    W = {name: dequantize_rows(lq.q[name], lq.s[name], dtype) for name in PROJ_NAMES}
+    W = {name: dequantize(lq.q[name], lq.s[name], dtype) for name in PROJ_NAMES}
     kg = set(keep_groups)
     qh = set(keep_qheads) if keep_qheads is not None else {j * g + i for j in kg for i in range(g)}
     assert all(h // g in kg for h in qh), "a kept query head needs its KV head (GQA closure)"

@@ -119,6 +119,9 @@ def _check(rc):
 
 def model_desc(shape) -> ModelDesc:
     """ModelDesc from any object with L, d, Hq, Hkv, dh, df, vocab, chan_unit, eps, rope_theta, seed."""
+    if getattr(shape, "quant_group", 0):
+        raise TaspError(EUNSUP, "the device store holds one INT8 scale per output row; groupwise scales are "
+                                "not built there")
     return ModelDesc(shape.L, shape.d, shape.Hq, shape.Hkv, shape.dh, shape.df, shape.vocab, shape.chan_unit,
                      shape.eps, shape.rope_theta, shape.seed)
 

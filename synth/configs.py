@@ -24,6 +24,7 @@ class ModelShape:
     eps: float = 1e-5
     rope_theta: float = 500000.0
     seed: int = 0
+    quant_group: int = 0  # INT8 scale granularity: 0 = one scale per output row, else columns per scale
 
     @property
     def g(self) -> int:
@@ -80,6 +81,7 @@ CFG5 = Workload("llama3_70b_mixed_turns", LLAMA3_70B, masks=tuple(MaskRecipe(s) 
 CONFIGS = {1: CFG1, 2: CFG2, 3: CFG3, 4: CFG4, 5: CFG5}
 
 
-def tiny_shape(L=2, d=128, Hq=4, Hkv=2, dh=32, df=192, vocab=64, chan_unit=16, seed=3) -> ModelShape:
+def tiny_shape(L=2, d=128, Hq=4, Hkv=2, dh=32, df=192, vocab=64, chan_unit=16, seed=3, quant_group=0) -> ModelShape:
     """A small shape for fast oracle pins."""
-    return ModelShape(L=L, d=d, Hq=Hq, Hkv=Hkv, dh=dh, df=df, vocab=vocab, chan_unit=chan_unit, seed=seed)
+    return ModelShape(L=L, d=d, Hq=Hq, Hkv=Hkv, dh=dh, df=df, vocab=vocab, chan_unit=chan_unit, seed=seed,
+                      quant_group=quant_group)

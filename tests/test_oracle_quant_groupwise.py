@@ -91,3 +91,89 @@ def test_groupwise_is_more_accurate_than_per_row_on_the_synthetic_weights():
     r_row = np.linalg.norm(wr.astype(np.float64) @ x - y) / np.linalg.norm(y)
     r_grp = np.linalg.norm(wg.astype(np.float64) @ x - y) / np.linalg.norm(y)
     assert r_grp < r_row
+
+
+# ---------------------------------------------------------------------------
+# Groupwise stores through the rest of the oracle: C regenerator, packing, forward.
+# ---------------------------------------------------------------------------
+
+def test_c_groupwise_quantizer_is_bit_identical():
+    from oracle import cgen
+    if not cgen.available():
+        pytest.skip("no C compiler")
+    rng = np.random.default_rng(3)
+    w = (rng.standard_normal((40, 512)) * 0.02).astype(np.float32)
+    w[5, 128:256] = 0  # a zero group
+    w[7, :128] = np.float32(2.0 ** -10) * np.arange(-64, 64, dtype=np.float32) / np.float32(2)  # ties
+    q, s = quant.quantize_groupwise(w)
+    for r in range(w.shape[0]):
+        qc, sc = cgen.quant_row_grouped(w[r], 128)
+        assert np.array_equal(qc, q[r]) and np.array_equal(sc.view(np.uint32), s[r].view(np.uint32))
+    # and the threaded regenerator against the numpy generator + quantizer
+    sh = synth.LLAMA3_8B
+    key = synth.stream_key(sh.seed, synth.T_WDOWN, 3, 0)
+    qc, sc = cgen.weight_int8_grouped(key, 17, 9, sh.df, 128, synth.WEIGHT_SIGMA)
+    qn, sn = quant.quantize_groupwise(synth.weight_f32(sh.seed, synth.T_WDOWN, 3, sh.d, sh.df, 17, 9))
+    assert np.array_equal(qc, qn) and np.array_equal(sc.view(np.uint32), sn.view(np.uint32))
+
+
+GSHAPE = synth.tiny_shape(L=3, dh=32, chan_unit=32, quant_group=32)
+
+
+def _steps(sh, n):
+    return synth.bf16_to_f32(synth.step_inputs_bf16(11, n, 1, sh.d)[:, 0])
+
+
+@pytest.mark.parametrize("kind", ["groups", "qheads"])
+def test_groupwise_mask_as_zero_equals_compacted(kind):
+    from oracle import forward as fw
+    from oracle import maskc
+    sh = GSHAPE
+    u = [[0, 3, 5], [2], [1, 4]]
+    m = maskc.explicit(sh, [[0, 1], [1], [0]], u) if kind == "groups" else \
+        maskc.explicit_qheads(sh, [[1, 2, 3], [3], [0, 2]], u)
+    x = _steps(sh, 4).astype(np.float64)
+    Xz = fw.decode(sh, m, x, 7, 7, dtype=np.float64)
+    Xc = fw.decode(sh, m, x, 7, 7, compact=True, dtype=np.float64)
+    assert np.linalg.norm(Xz - Xc) <= 1e-12 * np.linalg.norm(Xz)
+
+
+def test_groupwise_panels_keep_the_scales_of_kept_groups():
+    from oracle import pack, weights
+    sh = GSHAPE
+    lq = weights.gen_layer(sh, 1)
+    assert lq.s["q"].shape == (sh.Hq * sh.dh, sh.d // 32) and lq.s["down"].shape == (sh.d, sh.df // 32)
+    kc = list(range(64, 96)) + list(range(160, 192))  # channel units 2 and 5
+    P = pack.pack_layer(sh, lq, [1], kc, [3])
+    assert P["qkv_s"].shape == (3 * sh.dh, sh.d // 32)
+    assert np.array_equal(P["o_s"], lq.s["o"][:, [3]])          # head 3 = column group 3
+    assert np.array_equal(P["down_s"], lq.s["down"][:, [2, 5]])
+    assert np.array_equal(P["gu_s"][0::2], lq.s["gate"][kc]) and np.array_equal(P["gu_s"][1::2], lq.s["up"][kc])
+    # kept channels that split a scale group cannot be packed as whole groups
+    with pytest.raises(ValueError):
+        pack.pack_layer(sh, lq, [1], list(range(16, 48)), [3])
+
+
+def test_groupwise_layer_is_closer_to_the_unquantized_layer():
+    # one decode step of a layer on the unquantized FP32 weights against the same step on
+    # per-row and on groupwise INT8 weights: the groupwise step is the closer one
+    from oracle import forward as fw
+    from oracle import weights
+    row, grp = synth.tiny_shape(L=1, d=256, dh=64, df=512, chan_unit=64), \
+        synth.tiny_shape(L=1, d=256, dh=64, df=512, chan_unit=64, quant_group=64)
+    W0 = {}
+    for name in weights.PROJ_NAMES:
+        tid, r, c = weights.proj_dims(row, name)
+        W0[name] = synth.weight_f32(row.seed, tid, 0, r, c).astype(np.float64)
+    lq = weights.gen_layer(row, 0)
+    W0["g_attn"], W0["g_mlp"] = lq.g_attn.astype(np.float64), lq.g_mlp.astype(np.float64)
+    allg, allc = list(range(row.Hkv)), list(range(row.df))
+    x = _steps(row, 1)[0].astype(np.float64)
+    K, V = fw.prior_cache(row, 0, 7, 16, None, np.float64)
+    y0, _, _ = fw.layer_step(row, W0, x, K, V, 16)
+    errs = []
+    for sh in (row, grp):
+        W = weights.dense_zeroed(sh, weights.gen_layer(sh, 0), allg, allc, np.float64)
+        y, _, _ = fw.layer_step(sh, W, x, K, V, 16)
+        errs.append(np.linalg.norm(y - x - (y0 - x)) / np.linalg.norm(y0 - x))
+    assert 0 < errs[1] < errs[0] < 5e-2
