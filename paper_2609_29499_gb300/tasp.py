@@ -304,6 +304,7 @@ class Session:
     @classmethod
     def prefill(cls, plan: "Plan", embeds_bf16, max_new_tokens: int, logits=None, stream=None) -> "Session":
         """Prefill a prompt (CUDA bfloat16 tensor [T, d]) into a new session bound to `plan`."""
+        _check_prompt(plan.shape, embeds_bf16, logits)
         h = c_void_p()
         _check(load().tasp_prefill(plan.handle, embeds_bf16.data_ptr(), int(embeds_bf16.shape[0]), max_new_tokens,
                                    _stream_ptr(stream), ctypes.byref(h),
@@ -312,6 +313,7 @@ class Session:
 
     def prefill_into(self, embeds_bf16, logits=None, stream=None):
         """Prefill a prompt into this (existing) session from position 0."""
+        _check_prompt(self.plan.shape, embeds_bf16, logits)
         _check(load().tasp_session_prefill(self.handle, embeds_bf16.data_ptr(), int(embeds_bf16.shape[0]),
                                            _stream_ptr(stream), logits.data_ptr() if logits is not None else None))
 
@@ -330,6 +332,9 @@ class Session:
         return v.value
 
     def layer_step(self, layer, x_in, x_out, stream=None):
+        import torch
+        for t in (x_in, x_out):
+            _need(t, self.plan.shape.d, torch.float32, True, "layer residual")
         _check(load().tasp_layer_step(self.handle, layer, x_in.data_ptr(), x_out.data_ptr(), _stream_ptr(stream)))
 
     def release(self):
@@ -343,6 +348,13 @@ def _handles(sessions):
     return ctypes.cast(arr, POINTER(c_void_p)), arr
 
 
+def _need(t, want, dt, device, what="buffer"):
+    """Raise unless t holds at least `want` contiguous elements of dtype dt on the GPU (device=True)
+    or the host; the library takes raw pointers and cannot check them itself."""
+    if t.dtype != dt or not t.is_contiguous() or t.numel() < want or t.is_cuda != device:
+        raise ValueError(f"{what} needs {want} contiguous {dt} elements on the {'GPU' if device else 'host'}")
+
+
 def _check_buffers(sessions, x, hidden, logits, device):
     """Sizes, dtypes and placement of the caller buffers of an n-session step."""
     import torch
@@ -352,10 +364,17 @@ def _check_buffers(sessions, x, hidden, logits, device):
     n = len(sessions)
     for t, want, dt in ((x, n * sh.d, torch.bfloat16), (hidden, n * sh.d, torch.float32),
                         (logits, n * sh.vocab, torch.float32)):
-        if t is None:
-            continue
-        if t.dtype != dt or not t.is_contiguous() or t.numel() < want or t.is_cuda != device:
-            raise ValueError(f"buffer needs {want} contiguous {dt} elements on the {'GPU' if device else 'host'}")
+        if t is not None:
+            _need(t, want, dt, device)
+
+
+def _check_prompt(shape, embeds, logits):
+    import torch
+    if embeds.dim() != 2 or embeds.shape[1] != shape.d or embeds.shape[0] < 1:
+        raise ValueError(f"prompt embeddings must be [T >= 1, {shape.d}]")
+    _need(embeds, embeds.shape[0] * shape.d, torch.bfloat16, True, "prompt")
+    if logits is not None:
+        _need(logits, shape.vocab, torch.float32, True, "logits")
 
 
 def decode_step(sessions, x_bf16, hidden=None, logits=None, stream=None):
@@ -388,6 +407,7 @@ def union_status(sessions):
 
 def decode_step_static(session, x_bf16, hidden=None, logits=None, stream=None):
     """Allocation-free decode step of one session (static attention scratch, no CUDA graph)."""
+    _check_buffers([session], x_bf16, hidden, logits, True)
     _check(load().tasp_decode_step_static(session.handle, x_bf16.data_ptr(),
                                           hidden.data_ptr() if hidden is not None else None,
                                           logits.data_ptr() if logits is not None else None, _stream_ptr(stream)))
@@ -405,6 +425,7 @@ def decode_step_host(sessions, x_bf16_host, hidden_host=None, logits_host=None, 
 
 def profile_step(sessions, x_bf16, logits=None, stream=None):
     """Eager step with CUDA events around each kernel: {kind: (ms, launches)}."""
+    _check_buffers(sessions, x_bf16, None, logits, True)
     p, keep = _handles(sessions)
     ms = np.zeros(KERNEL_KINDS, np.float32)
     cnt = np.zeros(KERNEL_KINDS, np.int32)

@@ -180,3 +180,36 @@ def test_partial_group_plans_are_refused_before_device_work(lib):
     assert so.tasp_compile_mask(ctypes.byref(md), ctypes.byref(m.desc), ctypes.byref(out)) == lib.EUNSUP
     assert "whole groups" in so.tasp_last_error().decode()
     assert not out.value
+
+
+def test_binding_rejects_host_or_mistyped_buffers_before_any_call(lib):
+    # the library takes raw device pointers it cannot check: every wrapper refuses host
+    # tensors, wrong dtypes and short buffers before anything reaches the library
+    import torch
+    sh = synth.tiny_shape(L=1)
+
+    class FakePlan:
+        shape = sh
+        handle = ctypes.c_void_p(16)
+
+    sess = lib.Session(FakePlan(), 0, handle=ctypes.c_void_p(16))  # never dereferenced
+    x_host = torch.zeros((1, sh.d), dtype=torch.bfloat16)
+    f_host = torch.zeros(sh.d, dtype=torch.float32)
+    with pytest.raises(ValueError, match="GPU"):
+        lib.decode_step([sess], x_host)
+    with pytest.raises(ValueError, match="GPU"):
+        lib.decode_step_static(sess, x_host)
+    with pytest.raises(ValueError, match="GPU"):
+        lib.decode_step_union([sess], x_host)
+    with pytest.raises(ValueError, match="GPU"):
+        lib.profile_step([sess], x_host)
+    with pytest.raises(ValueError, match="layer residual"):
+        sess.layer_step(0, f_host, f_host)
+    with pytest.raises(ValueError, match="prompt"):
+        lib.Session.prefill(FakePlan(), torch.zeros((4, sh.d), dtype=torch.bfloat16), 8)
+    with pytest.raises(ValueError, match="prompt"):
+        sess.prefill_into(torch.zeros((4, sh.d + 1), dtype=torch.bfloat16))
+    with pytest.raises(ValueError, match="host"):  # the host-buffer entry wants host tensors of the right type
+        lib.decode_step_host([sess], torch.zeros((1, sh.d), dtype=torch.float32))
+    with pytest.raises(ValueError):
+        lib.decode_step_host([sess], torch.zeros((1, sh.d - 1), dtype=torch.bfloat16))
