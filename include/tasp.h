@@ -20,7 +20,10 @@
  *    synchronizing; their device outputs are valid once the stream reaches
  *    that point. Functions marked "sync" synchronize the device before return.
  *  - BF16 buffers hold IEEE bfloat16 bit patterns (uint16); FP32 buffers hold
- *    float. Matrices are row-major.
+ *    float. Matrices are row-major. A d_* buffer must be aligned to its
+ *    element size (2 bytes for BF16, 4 for FP32); a misaligned one is refused
+ *    with TASP_EINVAL before any work. The library cannot tell a device
+ *    pointer from a host one: passing a host pointer as d_* is undefined.
  *  - All sizes are element counts unless the name says bytes.
  */
 #ifndef TASP_H

@@ -60,6 +60,7 @@ using namespace tasp;
 
 extern "C" int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, float* d_hidden_out, float* d_logits,
                                        void* stream) {
+    if (int rc = check_aligned({{d_x_bf16, 2}, {d_hidden_out, 4}, {d_logits, 4}})) return rc;
     Session* se = (Session*)s;
     if (!se || se->magic != SESSION_MAGIC) return fail(TASP_EINVAL, "invalid session handle");
     if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");

@@ -669,8 +669,10 @@ int tasp_session_status(tasp_session* s, int32_t clear, int32_t* device_error) {
 
 int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_hidden_out,
                      float* d_logits, void* stream) {
+    int rc = check_aligned({{d_x_bf16, 2}, {d_hidden_out, 4}, {d_logits, 4}});
+    if (rc) return rc;
     Plan* p = nullptr;
-    int rc = check_sessions(sessions, n, &p);
+    rc = check_sessions(sessions, n, &p);
     if (rc) return rc;
     if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
@@ -761,6 +763,7 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
                  tasp_session** out, float* d_logits_last) {
     if (!out) return fail(TASP_EINVAL, "out is NULL");
     *out = nullptr;
+    if (int rc = check_aligned({{d_embeds_bf16, 2}, {d_logits_last, 4}})) return rc;
     Plan* p = as_plan(plan);
     if (!p) return fail(TASP_EINVAL, "invalid plan handle");
     if (!d_embeds_bf16 || T < 1 || max_new_tokens < 0) return fail(TASP_EINVAL, "bad prompt (NULL or T < 1)");
@@ -789,6 +792,7 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
 }
 
 int tasp_session_prefill(tasp_session* s, const void* d_embeds_bf16, int32_t T, void* stream, float* d_logits_last) {
+    if (int rc = check_aligned({{d_embeds_bf16, 2}, {d_logits_last, 4}})) return rc;
     Session* se = as_session(s);
     if (!se) return fail(TASP_EINVAL, "invalid session handle");
     const Shape& sh = se->plan->store->sh;
@@ -932,6 +936,7 @@ int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h
 }
 
 int tasp_layer_step(tasp_session* s, int32_t layer, const float* d_x_in, float* d_x_out, void* stream) {
+    if (int rc = check_aligned({{d_x_in, 4}, {d_x_out, 4}})) return rc;
     Session* se = as_session(s);
     if (!se || !d_x_in || !d_x_out) return fail(TASP_EINVAL, "invalid session or NULL buffers");
     const Shape& sh = se->plan->store->sh;
@@ -968,8 +973,10 @@ static void prof_hook(void* c, int kind, bool before) {
 
 int tasp_profile_step(tasp_session* const* sessions, int32_t n, const void* d_x_bf16, float* d_logits, void* stream,
                       float* h_ms, int32_t* h_count) {
+    int rc = check_aligned({{d_x_bf16, 2}, {d_logits, 4}});
+    if (rc) return rc;
     Plan* p = nullptr;
-    int rc = check_sessions(sessions, n, &p);
+    rc = check_sessions(sessions, n, &p);
     if (rc) return rc;
     if (!h_ms || !h_count || !d_x_bf16) return fail(TASP_EINVAL, "NULL buffers");
     const Shape& sh = p->store->sh;

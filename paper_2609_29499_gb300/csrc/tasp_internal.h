@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <initializer_list>
 #include <string>
 #include <vector>
 
@@ -15,6 +16,20 @@ namespace tasp {
 // ---------------------------------------------------------------- errors
 void set_error(const std::string& msg);
 int fail(int code, const std::string& msg);
+
+// Caller buffers are accessed element by element: each must be aligned to its element size
+// (2 bytes for BF16, 4 for FP32). NULL passes (optional buffers are checked elsewhere).
+struct BufAlign {
+    const void* p;
+    unsigned bytes;
+};
+inline int check_aligned(std::initializer_list<BufAlign> bufs) {
+    for (const BufAlign& b : bufs)
+        if (b.p && (reinterpret_cast<uintptr_t>(b.p) % b.bytes))
+            return fail(TASP_EINVAL, "a buffer is not aligned to its element size (" + std::to_string(b.bytes) +
+                                         " bytes)");
+    return TASP_OK;
+}
 int cuda_fail(cudaError_t e, const char* what);
 
 #define TASP_CUDA(call)                                   \

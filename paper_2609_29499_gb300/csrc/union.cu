@@ -949,8 +949,10 @@ using namespace tasp;
 extern "C" int tasp_decode_step_union(tasp_session* const* sessions, int32_t n, const void* d_x_bf16,
                                       float* d_hidden_out, float* d_logits, void* stream) {
     if (!sessions || !d_x_bf16) return fail(TASP_EINVAL, "null argument");
+    int rc = check_aligned({{d_x_bf16, 2}, {d_hidden_out, 4}, {d_logits, 4}});
+    if (rc) return rc;
     Session* const* ss = reinterpret_cast<Session* const*>(sessions);
-    int rc = union_check(ss, n, true);
+    rc = union_check(ss, n, true);
     if (rc) return rc;
     const Shape& sh = ss[0]->plan->store->sh;
     if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "model has no LM head");

@@ -213,3 +213,29 @@ def test_binding_rejects_host_or_mistyped_buffers_before_any_call(lib):
         lib.decode_step_host([sess], torch.zeros((1, sh.d), dtype=torch.float32))
     with pytest.raises(ValueError):
         lib.decode_step_host([sess], torch.zeros((1, sh.d - 1), dtype=torch.bfloat16))
+
+
+def test_misaligned_device_buffers_are_refused_before_any_work(lib):
+    # element-size alignment is checked first, before the handles are even looked at
+    so = lib.load()
+    P = ctypes.c_void_p
+    none = (P * 1)()
+    odd = ctypes.c_void_p(0x1001)       # not 2-byte aligned
+    half = ctypes.c_void_p(0x1002)      # 2- but not 4-byte aligned
+    ok2 = ctypes.c_void_p(0x1000)
+    assert so.tasp_decode_step(none, 1, odd, None, None, None) == lib.EINVAL
+    assert "aligned" in so.tasp_last_error().decode()
+    assert so.tasp_decode_step(none, 1, ok2, half, None, None) == lib.EINVAL
+    assert "4 bytes" in so.tasp_last_error().decode()
+    assert so.tasp_decode_step(none, 1, ok2, None, half, None) == lib.EINVAL
+    assert so.tasp_decode_step_union(none, 1, odd, None, None, None) == lib.EINVAL
+    assert so.tasp_decode_step_static(None, odd, None, None, None) == lib.EINVAL
+    assert "aligned" in so.tasp_last_error().decode()
+    out = ctypes.c_void_p()
+    assert so.tasp_prefill(None, odd, 4, 0, None, ctypes.byref(out), None) == lib.EINVAL
+    assert so.tasp_session_prefill(None, ok2, 4, None, half) == lib.EINVAL
+    assert so.tasp_layer_step(None, 0, half, ok2, None) == lib.EINVAL
+    assert "aligned" in so.tasp_last_error().decode()
+    # aligned buffers get past the check and meet the handle check instead
+    assert so.tasp_decode_step(none, 1, ok2, None, None, None) == lib.EINVAL
+    assert "aligned" not in so.tasp_last_error().decode()
