@@ -321,6 +321,15 @@ int tasp_decode_step_union(tasp_session* const* sessions, int32_t n, const void*
 int tasp_union_status(tasp_session* const* sessions, int32_t n, int32_t* device_error, int32_t* launches);
 
 /* Thread-local description of the last failure on this thread ("" if none). */
+/* Cap on the device memory held by the library's arenas (the shared store,
+ * plan panels, sessions and step workspaces); 0 = no cap, the default. A
+ * reservation that would pass the cap fails with TASP_ENOMEM before anything
+ * is allocated, and the call that needed it fails cleanly. Prefill's per-call
+ * temporaries come from the stream-ordered pool and are not counted. Host only. */
+int tasp_set_memory_limit(int64_t bytes);
+/* Device bytes the library's arenas hold now. Host only. */
+int tasp_memory_in_use(int64_t* bytes);
+
 const char* tasp_last_error(void);
 
 /* Library version string. */

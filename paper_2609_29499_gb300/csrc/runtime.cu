@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 #include <map>
 #include <memory>
@@ -47,12 +48,26 @@ int device_info(DevInfo& out) {
 }
 
 // ---------------------------------------------------------------- arena
+// Device bytes held by all arenas, and the optional cap on them (0 = none).
+static std::atomic<int64_t> g_arena_bytes{0};
+static std::atomic<int64_t> g_arena_limit{0};
+
 int Arena::reserve(size_t bytes) {
     cap = (bytes + 255) & ~size_t(255);
     used = 0;
     if (cap == 0) return TASP_OK;
+    const int64_t lim = g_arena_limit.load();
+    const int64_t now = g_arena_bytes.fetch_add((int64_t)cap) + (int64_t)cap;
+    if (lim > 0 && now > lim) {
+        g_arena_bytes.fetch_sub((int64_t)cap);
+        const size_t want = cap;
+        cap = 0;
+        return fail(TASP_ENOMEM, "device memory limit reached (" + std::to_string(want) + " more bytes, " +
+                                     std::to_string(now - (int64_t)want) + " of " + std::to_string(lim) + " in use)");
+    }
     cudaError_t e = cudaMalloc((void**)&base, cap);
     if (e != cudaSuccess) {
+        g_arena_bytes.fetch_sub((int64_t)cap);
         base = nullptr;
         cap = 0;
         return cuda_fail(e, "cudaMalloc");
@@ -67,7 +82,10 @@ void* Arena::take(size_t bytes) {
     return p;
 }
 void Arena::release() {
-    if (base) cudaFree(base);
+    if (base) {
+        cudaFree(base);
+        g_arena_bytes.fetch_sub((int64_t)cap);
+    }
     base = nullptr;
     cap = used = 0;
 }
@@ -143,7 +161,11 @@ static int store_acquire(const Shape& sh, Store** out) {
     st->lm_head = sh.vocab ? (uint16_t*)st->arena.take((size_t)sh.vocab * d * 2) : nullptr;
     st->bytes = lay.total;
     cudaStream_t s;
-    TASP_CUDA(cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking));
+    cudaError_t ce = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+    if (ce != cudaSuccess) {
+        st->arena.release();
+        return cuda_fail(ce, "cudaStreamCreateWithFlags");
+    }
     rc = store_generate(*st, s);
     cudaError_t e = cudaStreamSynchronize(s);
     cudaStreamDestroy(s);
@@ -551,6 +573,18 @@ extern "C" {
 
 const char* tasp_last_error(void) { return g_err.c_str(); }
 const char* tasp_version(void) { return "tasp-gb300 0.1 (sm_103a)"; }
+
+int tasp_set_memory_limit(int64_t bytes) {
+    if (bytes < 0) return fail(TASP_EINVAL, "memory limit must be >= 0");
+    g_arena_limit.store(bytes);
+    return TASP_OK;
+}
+
+int tasp_memory_in_use(int64_t* bytes) {
+    if (!bytes) return fail(TASP_EINVAL, "bytes is NULL");
+    *bytes = g_arena_bytes.load();
+    return TASP_OK;
+}
 
 int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
                             int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,

@@ -28,7 +28,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 # Symbols declared in include/tasp.h (the CPU test checks they are all exported).
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
-            "tasp_mask_select_qheads",
+            "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -90,6 +90,8 @@ def load(path: str = LIB_PATH):
         "tasp_decode_step_host": (c_int32, [POINTER(P), c_int32, P, P, P, P]),
         "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
+        "tasp_set_memory_limit": (c_int32, [c_int64]),
+        "tasp_memory_in_use": (c_int32, [POINTER(c_int64)]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
         "tasp_plan_export": (c_int32, [P, c_int32, c_int32, P, c_size_t]),
@@ -232,6 +234,17 @@ def mask_select_qheads(shape, mask: _MaskArgs):
             o += counts[layer]
         out.append(lists)
     return out[0], out[1], out[2], fl
+
+
+def set_memory_limit(nbytes: int):
+    """Cap the device memory of the library's arenas (0 = no cap)."""
+    _check(load().tasp_set_memory_limit(int(nbytes)))
+
+
+def memory_in_use() -> int:
+    v = c_int64()
+    _check(load().tasp_memory_in_use(ctypes.byref(v)))
+    return v.value
 
 
 def _stream_ptr(stream):

@@ -239,3 +239,21 @@ def test_misaligned_device_buffers_are_refused_before_any_work(lib):
     # aligned buffers get past the check and meet the handle check instead
     assert so.tasp_decode_step(none, 1, ok2, None, None, None) == lib.EINVAL
     assert "aligned" not in so.tasp_last_error().decode()
+
+
+def test_memory_limit_fails_cleanly_before_allocating(lib):
+    # a cap below the store's size makes plan compilation fail with ENOMEM before any device
+    # allocation, and leaves nothing held
+    assert lib.memory_in_use() == 0
+    lib.set_memory_limit(1 << 20)
+    try:
+        with pytest.raises(lib.TaspError) as e:
+            lib.Plan(synth.LAYER1, lib.all_keep_mask())
+        assert e.value.code == lib.ENOMEM
+        assert "memory limit" in str(e.value)
+        assert lib.memory_in_use() == 0
+    finally:
+        lib.set_memory_limit(0)
+    with pytest.raises(lib.TaspError) as e:
+        lib.set_memory_limit(-1)
+    assert e.value.code == lib.EINVAL
