@@ -385,6 +385,9 @@ def run_ours(args):
             "cpu_baseline": cpu,
             "paper_context": PAPER_CONTEXT,
             "setup_s": round(setup_s, 1),
+            "memory": {"store_bytes": int(info["store_bytes"]), "plan_bytes": int(info["panel_bytes"]),
+                       "library_bytes": int(tasp.memory_in_use()),
+                       "torch_max_allocated_bytes": int(torch.cuda.max_memory_allocated())},
         }
         print(json.dumps(out), flush=True)
     if world > 1:
