@@ -163,6 +163,8 @@ def compile_mask(shape, scores, target_u24, budget=0.57, r_lo=0.35, r_hi=0.85) -
             acc[layer][u] = True
             lcost[layer] += cost[u]
             total += cost[u]
+    if total > B:
+        raise ValueError("the FLOP budget is below the forced minimum of one group and one channel unit per layer")
     groups = [[u for u in range(G) if acc[layer][u]] for layer in range(L)]
     units = [[u - G for u in range(G, G + U) if acc[layer][u]] for layer in range(L)]
     m = explicit(shape, groups, units)
@@ -261,6 +263,8 @@ def compile_mask_qheads(shape, scores, target_u24, budget=0.57, r_lo=0.35, r_hi=
         if cand is None:
             break
         total += accept(cand[0], cand[1])
+    if total > B:
+        raise ValueError("the FLOP budget is below the forced minimum of one head and one channel unit per layer")
     qheads = [[u for u in range(Hq) if kept[layer][u]] for layer in range(L)]
     units = [[u - Hq for u in range(Hq, Hq + U) if kept[layer][u]] for layer in range(L)]
     m = explicit_qheads(shape, qheads, units)

@@ -257,3 +257,49 @@ def test_memory_limit_fails_cleanly_before_allocating(lib):
     with pytest.raises(lib.TaspError) as e:
         lib.set_memory_limit(-1)
     assert e.value.code == lib.EINVAL
+
+
+def test_host_compilers_match_oracle_on_random_shapes_with_ties(lib):
+    # seeded random shapes, budgets and retention ranges, with scores drawn from a handful of
+    # values so that exact ratio ties are common: both greedy kinds agree bit for bit
+    rng = np.random.default_rng(20240611)
+    cases = 0
+    while cases < 60:
+        Hkv = int(rng.choice([1, 2, 4]))
+        g = int(rng.choice([1, 2, 4, 8]))
+        dh = int(rng.choice([16, 32, 64]))
+        cu = int(rng.choice([16, 32, 64]))
+        sh = synth.ModelShape(L=int(rng.integers(1, 6)), d=16 * int(rng.integers(2, 12)), Hq=Hkv * g, Hkv=Hkv,
+                              dh=dh, df=cu * int(rng.integers(1, 9)), vocab=0, chan_unit=cu)
+        lo = float(rng.uniform(0.05, 0.5))
+        budget = float(rng.uniform(lo, 0.95))
+        hi = float(rng.uniform(budget, 1.0))
+        tg = synth.layer_target_u24(int(rng.integers(1 << 30)), sh.L)
+        top = int(rng.choice([3, 50, 1 << 32]))
+        for kind in ("groups", "qheads"):
+            n = (sh.Hkv if kind == "groups" else sh.Hq) + sh.n_chan_units
+            sc = rng.integers(0, top, size=(sh.L, n), dtype=np.uint64).astype(np.uint32)
+            oracle_fn = maskc.compile_mask if kind == "groups" else maskc.compile_mask_qheads
+            try:
+                oracle_fn(sh, sc, tg, budget, lo, hi)
+            except ValueError:  # budget below the forced minimum: the library refuses it too
+                args = (sc, tg, budget, lo, hi)
+                with pytest.raises(lib.TaspError) as e:
+                    if kind == "groups":
+                        lib.mask_select(sh, lib.greedy_mask(*args))
+                    else:
+                        lib.mask_select_qheads(sh, lib.greedy_qhead_mask(*args))
+                assert e.value.code == lib.EINVAL and "budget" in str(e.value)
+                continue
+            if kind == "groups":
+                want = maskc.compile_mask(sh, sc, tg, budget, lo, hi)
+                groups, units, fl = lib.mask_select(sh, lib.greedy_mask(sc, tg, budget, lo, hi))
+                assert (groups, units) == (want.keep_groups, want.keep_units), (sh, budget, lo, hi)
+            else:
+                want = maskc.compile_mask_qheads(sh, sc, tg, budget, lo, hi)
+                qh, groups, units, fl = lib.mask_select_qheads(sh, lib.greedy_qhead_mask(sc, tg, budget, lo, hi))
+                assert (qh, groups, units) == (want.keep_qheads, want.keep_groups, want.keep_units), \
+                    (sh, budget, lo, hi)
+            assert fl[:sh.L].tolist() == want.info["layer_flops"]
+            assert fl[sh.L + 1] == want.info["budget_flops"]
+        cases += 1
