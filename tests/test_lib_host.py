@@ -303,3 +303,25 @@ def test_host_compilers_match_oracle_on_random_shapes_with_ties(lib):
             assert fl[:sh.L].tolist() == want.info["layer_flops"]
             assert fl[sh.L + 1] == want.info["budget_flops"]
         cases += 1
+
+
+def test_explicit_masks_fuzzed_against_the_ledger(lib):
+    rng = np.random.default_rng(99)
+    for _ in range(40):
+        Hkv, g = int(rng.choice([1, 2, 4])), int(rng.choice([1, 2, 4, 8]))
+        cu = int(rng.choice([16, 32]))
+        sh = synth.ModelShape(L=int(rng.integers(1, 5)), d=16 * int(rng.integers(2, 10)), Hq=Hkv * g, Hkv=Hkv,
+                              dh=32, df=cu * int(rng.integers(1, 7)), vocab=0, chan_unit=cu)
+        units = [sorted(rng.choice(sh.n_chan_units, int(rng.integers(0, sh.n_chan_units + 1)), replace=False).tolist())
+                 for _ in range(sh.L)]
+        heads = [sorted(rng.choice(sh.Hq, int(rng.integers(0, sh.Hq + 1)), replace=False).tolist())
+                 for _ in range(sh.L)]
+        groups = [sorted({h // g for h in hs}) for hs in heads]
+        want = maskc.explicit_qheads(sh, heads, units)
+        qh, kg, ku, fl = lib.mask_select_qheads(sh, lib.explicit_qhead_mask(heads, units))
+        assert (qh, kg, ku) == (heads, want.keep_groups, units)
+        assert fl[sh.L] == ledger.mask_flops(sh, want.keep_groups, want.keep_chans, want.keep_qheads)
+        kg2, ku2, fl2 = lib.mask_select(sh, lib.explicit_mask(groups, units))
+        wg = maskc.explicit(sh, groups, units)
+        assert (kg2, ku2) == (groups, units)
+        assert fl2[sh.L] == ledger.mask_flops(sh, wg.keep_groups, wg.keep_chans)
