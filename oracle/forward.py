@@ -19,14 +19,19 @@ teacher-forced vectors (no token feedback); new K/V are kept in FP32 here.
 
 The mask enters only through ``oracle.weights.dense_zeroed`` (mask-as-zero).
 ``compact=True`` runs the same equations on the packed panels of
-``oracle.pack`` instead; the two must agree (zero rows contribute zero).
+``oracle.pack`` instead; the two must agree (zero rows contribute zero). A mask
+may keep single query heads (``keep_qheads``): the dropped heads' Q rows and O
+columns are zero, and the compacted step maps each kept head to the position
+of its KV head among the kept groups. A shape with ``quant_group`` > 0 runs on
+groupwise-quantized weights (one BF16 scale per row and group of columns).
 
 Pins: softmax against scipy.special.softmax, rotary embedding against complex
 multiplication and its relative-position property, a single-key attention
 returning V exactly, identical keys giving uniform attention, an empty mask
 leaving the residual unchanged, all-keep equal to the unmasked forward,
 mask-as-zero equal to compacted execution, and causal prefill equal to
-step-by-step decode.
+step-by-step decode; the same two equalities with ragged query-head masks and
+on groupwise stores, and a planted wrong query-to-KV map failing them.
 """
 from __future__ import annotations
 
