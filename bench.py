@@ -164,6 +164,13 @@ def workload(args):
     return wl, wl.shape, wl.masks[0]
 
 
+def block_bounds(K: int, n: int = 5) -> list:
+    """Step indices that cut K timed steps into min(n, K) consecutive blocks (the paper reports
+    latency as mean and spread over five timing blocks); strictly increasing, first 0, last K."""
+    nb = max(1, min(n, K))
+    return [i * K // nb for i in range(nb + 1)]
+
+
 def kv_bytes(plan_dims, dh, T):
     """KV bytes of one step at context T (keys+values read for T positions, one position written)."""
     m = sum(mk for mk, _ in plan_dims)
@@ -302,15 +309,20 @@ def run_ours(args):
     barrier(world)
     torch.cuda.synchronize()
     T_start = sess.position
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
+    bounds = block_bounds(K)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in bounds]
+    evs[0].record(stream)
+    nxt = 1
     for t in range(K):
         tasp.decode_step([sess], x[Wm + t], hidden, logits)
-    ev1.record(stream)
+        if nxt < len(bounds) and t + 1 == bounds[nxt]:
+            evs[nxt].record(stream)
+            nxt += 1
     torch.cuda.synchronize()
     barrier(world)
     clocks = sampler.stop()
-    ms = ev0.elapsed_time(ev1) / K
+    ms = evs[0].elapsed_time(evs[-1]) / K
+    block_ms = [evs[i].elapsed_time(evs[i + 1]) / (bounds[i + 1] - bounds[i]) for i in range(len(bounds) - 1)]
     ms = max_over_ranks(world, ms)
 
     # per-kernel durations of one eager step (CUDA events around each launch, same stream)
@@ -379,6 +391,8 @@ def run_ours(args):
                               "unit": "GB/s", "frac": round(step_gbs / peak, 4),
                               "frac_of_8TBps": round(step_gbs / 8000.0, 4)},
             "kernels": kernels,
+            "timing_blocks": {"n": len(block_ms), "ms_per_token": [round(b, 4) for b in block_ms],
+                              "std": round(statistics.pstdev(block_ms), 4) if len(block_ms) > 1 else 0.0},
             "e2e": e2e,
             "gpu_launches": launches_per_step * K,
             "clocks": clocks,

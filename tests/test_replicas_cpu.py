@@ -68,3 +68,13 @@ def test_reference_arm_under_torchrun_prints_once():
     line = lines[0]
     assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["steps"] == 2
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_timing_block_bounds():
+    # the timed steps are cut into at most five consecutive, non-empty blocks covering all K
+    sys.path.insert(0, ROOT)
+    import bench
+    for K in range(1, 300):
+        b = bench.block_bounds(K)
+        assert b[0] == 0 and b[-1] == K and len(b) == min(5, K) + 1
+        assert all(b[i + 1] > b[i] for i in range(len(b) - 1))
