@@ -110,3 +110,19 @@ def test_all_keep_is_dense():
     m = maskc.all_keep(sh)
     assert ledger.mask_ratio(sh, m.keep_groups, m.keep_chans) == 1.0
     assert all(len(c) == sh.df for c in m.keep_chans)
+
+
+def test_synthetic_masks_overlap_like_the_papers():
+    # the five 70B masks of the mixed-turn workload overlap as the paper's task masks do
+    # (pairwise Jaccard of retained units between 0.24 and 0.81: Sec. "Spectral Scoring and Mask
+    # Diversity Are Complementary" and the appendix table of task-mask overlaps)
+    sh = synth.LLAMA3_70B
+    sets = []
+    for s in synth.MASK_SEEDS:
+        m = maskc.compile_mask(sh, synth.mask_scores_u32(s, sh.L, sh.n_units), synth.layer_target_u24(s, sh.L))
+        sets.append({(l, "g", j) for l in range(sh.L) for j in m.keep_groups[l]} |
+                    {(l, "c", u) for l in range(sh.L) for u in m.keep_units[l]})
+    for i in range(5):
+        for j in range(i + 1, 5):
+            jac = len(sets[i] & sets[j]) / len(sets[i] | sets[j])
+            assert 0.24 <= jac <= 0.81, (i, j, jac)
