@@ -321,6 +321,13 @@ int tasp_decode_step_union(tasp_session* const* sessions, int32_t n, const void*
 int tasp_union_status(tasp_session* const* sessions, int32_t n, int32_t* device_error, int32_t* launches);
 
 /* Thread-local description of the last failure on this thread ("" if none). */
+/* Per-turn plan choice (Sec. 3.3; Table 1: tau = 0.85): given the router's task
+ * distribution h_probs [n] over the n task masks, *plan = the index of the most
+ * probable task (lowest index on ties) when its probability reaches tau, else n,
+ * the dense plan. Host only; EINVAL for NULL, n < 1, tau outside [0, 1] or a
+ * negative / non-finite probability. */
+int tasp_dispatch(const float* h_probs, int32_t n, float tau, int32_t* plan);
+
 /* Cap on the device memory held by the library's arenas (the shared store,
  * plan panels, sessions and step workspaces); 0 = no cap, the default. A
  * reservation that would pass the cap fails with TASP_ENOMEM before anything

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <cstring>
 #include <map>
@@ -573,6 +574,19 @@ extern "C" {
 
 const char* tasp_last_error(void) { return g_err.c_str(); }
 const char* tasp_version(void) { return "tasp-gb300 0.1 (sm_103a)"; }
+
+int tasp_dispatch(const float* h_probs, int32_t n, float tau, int32_t* plan) {
+    if (!h_probs || !plan || n < 1) return fail(TASP_EINVAL, "dispatch needs n >= 1 probabilities and an output");
+    if (!(tau >= 0.f && tau <= 1.f)) return fail(TASP_EINVAL, "tau must lie in [0, 1]");
+    int best = 0;
+    for (int i = 0; i < n; ++i) {
+        if (!std::isfinite(h_probs[i]) || h_probs[i] < 0.f)
+            return fail(TASP_EINVAL, "probabilities must be finite and non-negative");
+        if (h_probs[i] > h_probs[best]) best = i;
+    }
+    *plan = h_probs[best] >= tau ? best : n;
+    return TASP_OK;
+}
 
 int tasp_set_memory_limit(int64_t bytes) {
     if (bytes < 0) return fail(TASP_EINVAL, "memory limit must be >= 0");

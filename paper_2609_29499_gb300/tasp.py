@@ -28,7 +28,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 # Symbols declared in include/tasp.h (the CPU test checks they are all exported).
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
-            "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use",
+            "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use", "tasp_dispatch",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -91,6 +91,7 @@ def load(path: str = LIB_PATH):
         "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_set_memory_limit": (c_int32, [c_int64]),
+        "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
         "tasp_memory_in_use": (c_int32, [POINTER(c_int64)]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
@@ -234,6 +235,15 @@ def mask_select_qheads(shape, mask: _MaskArgs):
             o += counts[layer]
         out.append(lists)
     return out[0], out[1], out[2], fl
+
+
+def dispatch(probs, tau: float = 0.85) -> int:
+    """Plan index for a turn: the most probable task's mask if its probability reaches tau, else
+    len(probs), the dense plan."""
+    p = np.ascontiguousarray(probs, dtype=np.float32)
+    v = c_int32()
+    _check(load().tasp_dispatch(p.ctypes.data, len(p), tau, ctypes.byref(v)))
+    return v.value
 
 
 def set_memory_limit(nbytes: int):

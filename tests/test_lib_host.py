@@ -325,3 +325,17 @@ def test_explicit_masks_fuzzed_against_the_ledger(lib):
         wg = maskc.explicit(sh, groups, units)
         assert (kg2, ku2) == (groups, units)
         assert fl2[sh.L] == ledger.mask_flops(sh, wg.keep_groups, wg.keep_chans)
+
+
+def test_dispatch_matches_the_oracle(lib):
+    from oracle import dispatch
+    rng = np.random.default_rng(8)
+    cases = [[0.9, 0.05, 0.05, 0.0, 0.0], [0.5, 0.3, 0.1, 0.05, 0.05], [0.2] * 5, [0.5, 0.5]]
+    cases += [rng.dirichlet(np.full(5, 0.3)).astype(np.float32).tolist() for _ in range(300)]
+    for p in cases:
+        for tau in (0.85, 0.5, 0.0, 1.0):
+            assert lib.dispatch(p, tau) == dispatch.choose_plan(np.float32(p), np.float32(tau))
+    for bad, tau in (([], 0.85), ([0.5, -0.1], 0.85), ([0.5, float("inf")], 0.85), ([0.5], 1.5)):
+        with pytest.raises(lib.TaspError) as e:
+            lib.dispatch(bad, tau)
+        assert e.value.code == lib.EINVAL
