@@ -339,3 +339,17 @@ def test_dispatch_matches_the_oracle(lib):
         with pytest.raises(lib.TaspError) as e:
             lib.dispatch(bad, tau)
         assert e.value.code == lib.EINVAL
+
+
+def test_header_is_a_plain_c_interface():
+    # the boundary is C: the header compiles as C99 on its own (the exports are checked above)
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if not cc:
+        pytest.skip("no C compiler")
+    src = "#include <tasp.h>\nint main(void) { tasp_status s = TASP_OK; tasp_model_desc m = {0};\n" \
+          "  (void)m; return (int)s + (tasp_last_error() == 0); }\n"
+    r = subprocess.run([cc, "-x", "c", "-std=c99", "-Wall", "-Werror", "-fsyntax-only",
+                        "-I", os.path.join(ROOT, "include"), "-"], input=src, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
