@@ -127,3 +127,15 @@ def test_gaussian_blocks_stay_inside_the_marchenko_pastur_edges():
         lo, hi = synth.WEIGHT_SIGMA ** 2 * (1 - r) ** 2, synth.WEIGHT_SIGMA ** 2 * (1 + r) ** 2
         assert lam.min() > 0.8 * lo and lam.max() < 1.15 * hi
         assert lam.max() > 0.85 * hi and lam.min() < 1.3 * lo
+
+
+def test_designed_power_law_spectrum_is_recovered():
+    # singular values s_i = i^(-beta) give eigenvalues lambda_i ~ i^(-2 beta), whose counting
+    # function #{lambda > x} ~ x^(-1 / (2 beta)): a Pareto tail of exponent 1 / (2 beta)
+    for beta in (0.5, 0.25):
+        n = 400
+        s = np.arange(1, n + 1, dtype=np.float64) ** (-beta)
+        W = _with_singular_values(s, n, n + 40, seed=9)
+        f = sp.features(W, n + 40, 0, 1, False)
+        assert f.alpha == pytest.approx(1.0 / (2 * beta), rel=0.15)
+        assert f.spectral_norm == pytest.approx(1.0, rel=1e-10)
