@@ -117,9 +117,8 @@ typedef struct tasp_session tasp_session;
  * identical model_desc share it), runs the host mask compiler, packs the
  * panels on the device. sync. *out receives the plan.
  * Errors: EINVAL (bad desc, mask violates closure/budget, empty layer),
- * EUNSUP (a query-head mask that keeps part of a group: the device kernels
- * take whole GQA groups; query-head masks whose groups are whole compile),
- * ENOMEM, ECUDA. */
+ * ENOMEM, ECUDA. Query-head masks may keep part of a group: the plan then
+ * carries per-layer role tables for its partial groups. */
 int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out);
 
 /* Prefill one prompt with a plan (Sec. 3.3: the plan chosen for a turn serves
@@ -224,6 +223,8 @@ int tasp_plan_info_get(const tasp_plan* plan, tasp_plan_info* out);
 
 /* Per-layer retained sizes: out[0] = m_kv (kept groups), out[1] = c (kept channels). */
 int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2);
+/* Kept query heads m_q of a layer (m_kv g unless the mask keeps part of a group). */
+int tasp_plan_layer_qheads(const tasp_plan* plan, int32_t layer, int32_t* m_q);
 
 enum tasp_export_item {
     TASP_EXPORT_KEEP_GROUPS = 0, /* int32 [m_kv] */
@@ -235,7 +236,8 @@ enum tasp_export_item {
     TASP_EXPORT_GU_W = 6,        /* int8 [2c][d], gate row then up row per kept channel */
     TASP_EXPORT_GU_S = 7,        /* float [2c] */
     TASP_EXPORT_DOWN_W = 8,      /* int8 [d][c] */
-    TASP_EXPORT_DOWN_S = 9       /* float [d] */
+    TASP_EXPORT_DOWN_S = 9,      /* float [d] */
+    TASP_EXPORT_KEEP_QHEADS = 10 /* int32 [m_q] */
 };
 
 /* Copy one packed panel (logical layout, no padding) or index list of a layer

@@ -241,6 +241,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
         }
         p.g = sh.g();
         p.dh = sh.dh;
+        p.blk_role = lp.blk_role;
         p.err = bv.err;
         gemv(K_QKV, M_QKV, p);
         // K2: split-KV attention over the retained KV heads of every session
@@ -257,6 +258,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 a.pos[b] = se.d_pos;
                 a.max_tokens[b] = se.max_tokens;
                 a.m_kv[b] = lp.m_kv;
+                a.oslot[b] = lp.oslot;
                 S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);

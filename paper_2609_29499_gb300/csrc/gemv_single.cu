@@ -48,6 +48,7 @@ struct GemvParams {
     const float2* rope;
     const int* pos;
     int g, dh;
+    const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
     float* h_out;
     float* logits;
     int* err;       // device error word (bounded waits that gave up)
@@ -431,7 +432,8 @@ __device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)
                     const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
                     float y0 = sc0 * s0, y1 = sc1 * s1;
                     const int gp2 = p.g + 2;
-                    const int jl = hb / gp2, hh = hb - jl * gp2;
+                    const int code = p.blk_role ? p.blk_role[hb] : hb;
+                    const int jl = code / gp2, hh = code - jl * gp2;
                     const int pos = es.pos;
                     if (hh <= p.g) {
                         const float2 cs = es.rope[i];
@@ -754,6 +756,7 @@ int launch_gemv_single(int mode, const gemv::Params& q, cudaStream_t s) {
     p.pos = q.pos[0];
     p.g = q.g;
     p.dh = q.dh;
+    p.blk_role = q.blk_role;
     p.h_out = q.h_out;
     p.logits = q.logits;
     return gemv1::launch_gemv(mode, p, q.err, s);

@@ -201,14 +201,16 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
     for (int l = 0; l < sh.L; ++l) {
         LayerPlan& lp = p.layers[l];
         lp.keep_groups = sel.groups[l];
+        lp.keep_qheads = sel.qheads[l];
         lp.keep_chans.clear();
         for (int u : sel.units[l])
             for (int i = 0; i < sh.cu; ++i) lp.keep_chans.push_back(u * sh.cu + i);
         lp.m_kv = (int)lp.keep_groups.size();
+        lp.m_q = (int)lp.keep_qheads.size();
         lp.c = (int)lp.keep_chans.size();
-        lp.qkv_rows = lp.m_kv * (g + 2) * dh;
+        lp.qkv_rows = (lp.m_q + 2 * lp.m_kv) * dh;
         lp.gu_rows = 2 * lp.c;
-        lp.o_K = lp.m_kv * g * dh;
+        lp.o_K = lp.m_q * dh;
         lp.dn_K = lp.c;
         lp.g_attn = st.layers[l].g_attn;
         lp.g_mlp = st.layers[l].g_mlp;
@@ -227,11 +229,17 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
         return TASP_OK;
     }
     const bool rowidx = panel_mode == TASP_PANELS_ROW_INDEXED;
+    auto ragged = [&](const LayerPlan& lp) { return lp.m_q != lp.m_kv * g; };
     // sizing pass
     Layout lay;
     for (int l = 0; l < sh.L; ++l) {
         const LayerPlan& lp = p.layers[l];
         const size_t ol = round16(lp.o_K), dl = round16(lp.dn_K);
+        if (ragged(lp)) {
+            lay.add((size_t)(lp.m_q + 2 * lp.m_kv) * 2);
+            lay.add((size_t)lp.m_kv * g * 2);
+            lay.add((size_t)lp.m_kv * (g + 2) * 2);
+        }
         lay.add((size_t)lp.qkv_rows * 4); lay.add((size_t)lp.qkv_rows * 4);  // map, scales
         lay.add((size_t)lp.gu_rows * 4); lay.add((size_t)lp.gu_rows * 4);
         lay.add(ol * 4); lay.add(dl * 4);                                       // column maps
@@ -243,16 +251,32 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
     cudaStream_t s;
     TASP_CUDA(cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking));
     std::vector<int32_t> hq, hg, ho, hd;
+    std::vector<int16_t> hrole, hslot, hblk;
     for (int l = 0; l < sh.L && !rc; ++l) {
         LayerPlan& lp = p.layers[l];
         const LayerStore& ls = st.layers[l];
         const int ol = round16(lp.o_K), dl = round16(lp.dn_K);
-        hq.clear(); hg.clear(); ho.clear(); hd.clear();
-        for (int j : lp.keep_groups)
-            for (int r = 0; r < (g + 2) * dh; ++r) hq.push_back(j * (g + 2) * dh + r);
+        hq.clear(); hg.clear(); ho.clear(); hd.clear(); hrole.clear(); hslot.assign((size_t)lp.m_kv * g, -1);
+        hblk.assign((size_t)lp.m_kv * (g + 2), -1);
+        // qkv panel: per kept group its kept heads' row blocks, then K, then V (store rows are
+        // group-major: g head blocks, K, V); O columns: the kept heads in ascending order
+        std::vector<char> keep_h(sh.Hq, 0);
+        for (int h : lp.keep_qheads) keep_h[h] = 1;
+        int slot = 0;
+        for (int jl = 0; jl < lp.m_kv; ++jl) {
+            const int j = lp.keep_groups[jl];
+            for (int hh = 0; hh < g + 2; ++hh) {
+                if (hh < g && !keep_h[j * g + hh]) continue;
+                for (int r = 0; r < dh; ++r) hq.push_back((j * (g + 2) + hh) * dh + r);
+                hblk[(size_t)jl * (g + 2) + hh] = (int16_t)hrole.size();
+                hrole.push_back((int16_t)(jl * (g + 2) + hh));
+                if (hh < g) {
+                    hslot[(size_t)jl * g + hh] = (int16_t)slot++;
+                    for (int c = 0; c < dh; ++c) ho.push_back((j * g + hh) * dh + c);
+                }
+            }
+        }
         for (int c : lp.keep_chans) { hg.push_back(2 * c); hg.push_back(2 * c + 1); }
-        for (int j : lp.keep_groups)
-            for (int c = 0; c < g * dh; ++c) ho.push_back(j * g * dh + c);
         ho.resize(ol, 0);
         hd = std::vector<int32_t>(lp.keep_chans.begin(), lp.keep_chans.end());
         hd.resize(dl, 0);
@@ -262,6 +286,17 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
         float* sg = (float*)p.arena.take(hg.size() * 4);
         int32_t* dco = (int32_t*)p.arena.take(ho.size() * 4);
         int32_t* dcd = (int32_t*)p.arena.take(hd.size() * 4);
+        if (ragged(lp)) {
+            int16_t* drole = (int16_t*)p.arena.take(hrole.size() * 2);
+            int16_t* dslot = (int16_t*)p.arena.take(hslot.size() * 2);
+            int16_t* dblk = (int16_t*)p.arena.take(hblk.size() * 2);
+            TASP_CUDA(cudaMemcpyAsync(drole, hrole.data(), hrole.size() * 2, cudaMemcpyHostToDevice, s));
+            TASP_CUDA(cudaMemcpyAsync(dslot, hslot.data(), hslot.size() * 2, cudaMemcpyHostToDevice, s));
+            TASP_CUDA(cudaMemcpyAsync(dblk, hblk.data(), hblk.size() * 2, cudaMemcpyHostToDevice, s));
+            lp.blk_role = drole;
+            lp.oslot = dslot;
+            lp.blk_of = dblk;
+        }
         if (hq.size()) TASP_CUDA(cudaMemcpyAsync(dq, hq.data(), hq.size() * 4, cudaMemcpyHostToDevice, s));
         if (hg.size()) TASP_CUDA(cudaMemcpyAsync(dg, hg.data(), hg.size() * 4, cudaMemcpyHostToDevice, s));
         if (ho.size()) TASP_CUDA(cudaMemcpyAsync(dco, ho.data(), ho.size() * 4, cudaMemcpyHostToDevice, s));
@@ -299,7 +334,7 @@ static void plan_ledger(Plan& p) {
     const Shape& sh = p.store->sh;
     int64_t fl = 0, launched = 0, bytes = 0;
     for (const LayerPlan& lp : p.layers) {
-        fl += layer_flops(sh, (int64_t)lp.m_kv * sh.g(), lp.m_kv, lp.c);
+        fl += layer_flops(sh, lp.m_q, lp.m_kv, lp.c);
         launched += 2 * (int64_t)lp.qkv_rows * sh.d + 2 * (int64_t)sh.d * lp.o_K + 2 * (int64_t)lp.gu_rows * sh.d +
                     2 * (int64_t)sh.d * lp.dn_K;
         bytes += (int64_t)lp.qkv_rows * sh.d + (int64_t)sh.d * lp.o_K + (int64_t)lp.gu_rows * sh.d +
@@ -646,9 +681,6 @@ int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, 
     for (int l = 0; l < sh.L; ++l) {
         if (sel.groups[l].empty() && sel.units[l].empty())
             return fail(TASP_EINVAL, "mask leaves a layer empty (layer " + std::to_string(l) + ")");
-        if (sel.qheads[l].size() != sel.groups[l].size() * (size_t)sh.g())
-            return fail(TASP_EUNSUP, "query-head mask keeps part of a GQA group (layer " + std::to_string(l) +
-                                         "); the device kernels take whole groups");
     }
     Store* st = nullptr;
     if ((rc = store_acquire(sh, &st))) return rc;
@@ -926,6 +958,13 @@ int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2) {
     return TASP_OK;
 }
 
+int tasp_plan_layer_qheads(const tasp_plan* plan, int32_t layer, int32_t* m_q) {
+    Plan* p = as_plan((void*)plan);
+    if (!p || !m_q || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan or layer");
+    *m_q = p->layers[layer].m_q;
+    return TASP_OK;
+}
+
 int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h_dst, size_t bytes) {
     Plan* p = as_plan((void*)plan);
     if (!p || !h_dst || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan, layer or dst");
@@ -964,6 +1003,11 @@ int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h
         case TASP_EXPORT_KEEP_GROUPS: {
             if (int rc = need(lp.keep_groups.size() * 4)) return rc;
             std::memcpy(h_dst, lp.keep_groups.data(), bytes);
+            return TASP_OK;
+        }
+        case TASP_EXPORT_KEEP_QHEADS: {
+            if (int rc = need(lp.keep_qheads.size() * 4)) return rc;
+            std::memcpy(h_dst, lp.keep_qheads.data(), bytes);
             return TASP_OK;
         }
         case TASP_EXPORT_KEEP_CHANS: {

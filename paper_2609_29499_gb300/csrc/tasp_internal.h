@@ -93,7 +93,16 @@ struct Store {
 // ---------------------------------------------------------------- plans
 struct LayerPlan {
     int m_kv = 0, c = 0;
-    std::vector<int> keep_groups, keep_chans;
+    int m_q = 0;  // kept query heads (m_kv g unless the mask keeps part of a group)
+    std::vector<int> keep_groups, keep_chans, keep_qheads;
+    // Partial groups only (NULL when every kept group keeps its g heads):
+    // blk_role[b] = role of the qkv panel's d_h-row block b as jl (g + 2) + hh, with jl the
+    // kept-group slot and hh the head within the group (< g), g for K or g + 1 for V;
+    // oslot[jl g + hh] = the compact position of that head in the O panel's columns, or -1
+    // for a dropped head (its query slot stays zero and its attention output is not written).
+    const int16_t* blk_role = nullptr;
+    const int16_t* oslot = nullptr;
+    const int16_t* blk_of = nullptr;  // inverse of blk_role: [m_kv (g + 2)] panel block or -1
     // qkv panel: rows (m_q + 2 m_kv) dh of K = d; row i at qkv_w + (qkv_map ? qkv_map[i] : i) * d
     const int8_t* qkv_w = nullptr;
     const int32_t* qkv_map = nullptr;
@@ -194,14 +203,15 @@ constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pa
 constexpr int UNION_MAX = 16;  // sessions (of any plans) in one union-of-masks step
 struct AttnParams {
     // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
-    const float* q;      // FP32 rotated queries [m_q][dh] (kept heads, group-major)
-    float* o;            // FP32 [m_q][dh]
+    const float* q;      // FP32 rotated queries [m_kv g][dh] (kept groups, all g slots)
+    float* o;            // FP32 [m_q][dh], kept heads in O-panel column order
     int64_t q_stride;
     const uint16_t* K[UNION_MAX];  // BF16 [m_kv][max_tokens][dh] of this layer
     const uint16_t* V[UNION_MAX];
     const int* pos[UNION_MAX];     // device position: the step attends to positions 0..pos
     int max_tokens[UNION_MAX];
     int m_kv[UNION_MAX];           // kept groups of the session's plan (grid y covers the largest)
+    const int16_t* oslot[UNION_MAX];  // output slot per (group slot, head), NULL = jl g + hh
     float qscale;        // log2(e) / sqrt(dh)
     float* part;         // + b * part_stride
     float* ml;           // + b * ml_stride

@@ -21,7 +21,7 @@ OK, EINVAL, EMASK, ECAP, ENOMEM, EBUSY, ECUDA, EUNSUP = 0, -1, -2, -3, -4, -5, -
 MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT, MASK_GREEDY_QHEADS, MASK_EXPLICIT_QHEADS = 0, 1, 2, 3, 4
 PANELS_COMPACT, PANELS_ROW_INDEXED = 0, 1
 (EXPORT_KEEP_GROUPS, EXPORT_KEEP_CHANS, EXPORT_QKV_W, EXPORT_QKV_S, EXPORT_O_W, EXPORT_O_S, EXPORT_GU_W,
- EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S) = range(10)
+ EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S, EXPORT_KEEP_QHEADS) = range(11)
 KERNEL_KINDS = 7
 KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "other")
 
@@ -29,6 +29,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use", "tasp_dispatch",
+            "tasp_plan_layer_qheads",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -92,6 +93,7 @@ def load(path: str = LIB_PATH):
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_set_memory_limit": (c_int32, [c_int64]),
         "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
+        "tasp_plan_layer_qheads": (c_int32, [P, c_int32, POINTER(c_int32)]),
         "tasp_memory_in_use": (c_int32, [POINTER(c_int64)]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
@@ -282,12 +284,18 @@ class Plan:
         _check(load().tasp_plan_layer_dims(self.handle, layer, out.ctypes.data))
         return int(out[0]), int(out[1])
 
+    def layer_qheads(self, layer) -> int:
+        v = c_int32()
+        _check(load().tasp_plan_layer_qheads(self.handle, layer, ctypes.byref(v)))
+        return v.value
+
     def export(self, layer, item):
         sh = self.shape
         m_kv, c = self.layer_dims(layer)
-        m_q = m_kv * (sh.Hq // sh.Hkv)
+        m_q = self.layer_qheads(layer)
         spec = {
             EXPORT_KEEP_GROUPS: (np.int32, (m_kv,)),
+            EXPORT_KEEP_QHEADS: (np.int32, (m_q,)),
             EXPORT_KEEP_CHANS: (np.int32, (c,)),
             EXPORT_QKV_W: (np.int8, ((m_q + 2 * m_kv) * sh.dh, sh.d)),
             EXPORT_QKV_S: (np.float32, ((m_q + 2 * m_kv) * sh.dh,)),

@@ -169,19 +169,6 @@ def test_explicit_qhead_masks_and_group_kinds(lib):
     assert e.value.code == lib.EINVAL
 
 
-def test_partial_group_plans_are_refused_before_device_work(lib):
-    # the device kernels take whole GQA groups: a query-head mask that keeps part of a group
-    # is refused by the host compiler before any store or panel is made
-    sh = synth.LAYER1
-    so = lib.load()
-    md = lib.model_desc(sh)
-    m = lib.explicit_qhead_mask([[0, 1, 4, 5, 6, 7]], [[0, 9]])
-    out = ctypes.c_void_p()
-    assert so.tasp_compile_mask(ctypes.byref(md), ctypes.byref(m.desc), ctypes.byref(out)) == lib.EUNSUP
-    assert "whole groups" in so.tasp_last_error().decode()
-    assert not out.value
-
-
 def test_binding_rejects_host_or_mistyped_buffers_before_any_call(lib):
     # the library takes raw device pointers it cannot check: every wrapper refuses host
     # tensors, wrong dtypes and short buffers before anything reaches the library
