@@ -202,6 +202,16 @@ int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, i
  * n_qheads [L] (ascending per layer). For the group kinds these are all g heads
  * of every kept group; for the query-head kinds keep_groups holds the KV heads
  * that the closure keeps. Host only; any output may be NULL. */
+/* Host only (test introspection): the tables a plan of `mask` uses for one layer.
+ * qkv_src [(m_q + 2 m_kv) dh]: store row of each qkv panel row (store rows are
+ * group-major: per KV group its g head blocks of dh rows, then K, then V);
+ * o_src [m_q dh]: dense O column of each panel column; role [m_q + 2 m_kv],
+ * slot [m_kv g], blk_of [m_kv (g + 2)]: the partial-group tables (role of each
+ * dh-row block as jl (g + 2) + hh; compact O position of (jl, hh) or -1; inverse
+ * of role or -1). counts [5] receives the five lengths. Any array may be NULL. */
+int tasp_plan_layout(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t layer, int32_t* qkv_src,
+                     int32_t* o_src, int16_t* role, int16_t* slot, int16_t* blk_of, int32_t* counts);
+
 int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
                             int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
                             int32_t* n_units, int64_t* flops);

@@ -193,6 +193,34 @@ static void store_release(Store* st) {
 }
 
 // ---------------------------------------------------------------- plan compilation
+// Source rows of the qkv panel in the store (per kept group its kept heads' d_h-row blocks,
+// then K, then V; store rows are group-major: g head blocks, K, V), source columns of the O
+// panel (the kept heads in ascending order), and the role / slot / block tables of partial
+// groups (see LayerPlan).
+static void layer_tables(const Shape& sh, const LayerPlan& lp, std::vector<int32_t>& hq, std::vector<int32_t>& ho,
+                         std::vector<int16_t>& hrole, std::vector<int16_t>& hslot, std::vector<int16_t>& hblk) {
+    const int g = sh.g(), dh = sh.dh;
+    hq.clear(); ho.clear(); hrole.clear();
+    hslot.assign((size_t)lp.m_kv * g, -1);
+    hblk.assign((size_t)lp.m_kv * (g + 2), -1);
+    std::vector<char> keep_h(sh.Hq, 0);
+    for (int h : lp.keep_qheads) keep_h[h] = 1;
+    int slot = 0;
+    for (int jl = 0; jl < lp.m_kv; ++jl) {
+        const int j = lp.keep_groups[jl];
+        for (int hh = 0; hh < g + 2; ++hh) {
+            if (hh < g && !keep_h[j * g + hh]) continue;
+            for (int r = 0; r < dh; ++r) hq.push_back((j * (g + 2) + hh) * dh + r);
+            hblk[(size_t)jl * (g + 2) + hh] = (int16_t)hrole.size();
+            hrole.push_back((int16_t)(jl * (g + 2) + hh));
+            if (hh < g) {
+                hslot[(size_t)jl * g + hh] = (int16_t)slot++;
+                for (int c = 0; c < dh; ++c) ho.push_back((j * g + hh) * dh + c);
+            }
+        }
+    }
+}
+
 static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep) {
     Store& st = *p.store;
     const Shape& sh = st.sh;
@@ -256,26 +284,8 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
         LayerPlan& lp = p.layers[l];
         const LayerStore& ls = st.layers[l];
         const int ol = round16(lp.o_K), dl = round16(lp.dn_K);
-        hq.clear(); hg.clear(); ho.clear(); hd.clear(); hrole.clear(); hslot.assign((size_t)lp.m_kv * g, -1);
-        hblk.assign((size_t)lp.m_kv * (g + 2), -1);
-        // qkv panel: per kept group its kept heads' row blocks, then K, then V (store rows are
-        // group-major: g head blocks, K, V); O columns: the kept heads in ascending order
-        std::vector<char> keep_h(sh.Hq, 0);
-        for (int h : lp.keep_qheads) keep_h[h] = 1;
-        int slot = 0;
-        for (int jl = 0; jl < lp.m_kv; ++jl) {
-            const int j = lp.keep_groups[jl];
-            for (int hh = 0; hh < g + 2; ++hh) {
-                if (hh < g && !keep_h[j * g + hh]) continue;
-                for (int r = 0; r < dh; ++r) hq.push_back((j * (g + 2) + hh) * dh + r);
-                hblk[(size_t)jl * (g + 2) + hh] = (int16_t)hrole.size();
-                hrole.push_back((int16_t)(jl * (g + 2) + hh));
-                if (hh < g) {
-                    hslot[(size_t)jl * g + hh] = (int16_t)slot++;
-                    for (int c = 0; c < dh; ++c) ho.push_back((j * g + hh) * dh + c);
-                }
-            }
-        }
+        layer_tables(sh, lp, hq, ho, hrole, hslot, hblk);
+        hg.clear(); hd.clear();
         for (int c : lp.keep_chans) { hg.push_back(2 * c); hg.push_back(2 * c + 1); }
         ho.resize(ol, 0);
         hd = std::vector<int32_t>(lp.keep_chans.begin(), lp.keep_chans.end());
@@ -659,6 +669,35 @@ int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* 
         flops[sh.L + 1] = sel.budget;
         flops[sh.L + 2] = sel.dense;
     }
+    return TASP_OK;
+}
+
+int tasp_plan_layout(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t layer, int32_t* qkv_src,
+                     int32_t* o_src, int16_t* role, int16_t* slot, int16_t* blk_of, int32_t* counts) {
+    Shape sh;
+    int rc = validate_shape(model, sh, false);
+    if (rc) return rc;
+    if (!mask || !counts) return fail(TASP_EINVAL, "mask_desc or counts is NULL");
+    MaskSel sel;
+    if ((rc = select_mask(sh, *mask, sel))) return rc;
+    if (layer < 0 || layer >= sh.L) return fail(TASP_EINVAL, "layer out of range");
+    LayerPlan lp;
+    lp.keep_groups = sel.groups[layer];
+    lp.keep_qheads = sel.qheads[layer];
+    lp.m_kv = (int)lp.keep_groups.size();
+    std::vector<int32_t> hq, ho;
+    std::vector<int16_t> hrole, hslot, hblk;
+    layer_tables(sh, lp, hq, ho, hrole, hslot, hblk);
+    counts[0] = (int32_t)hq.size();
+    counts[1] = (int32_t)ho.size();
+    counts[2] = (int32_t)hrole.size();
+    counts[3] = (int32_t)hslot.size();
+    counts[4] = (int32_t)hblk.size();
+    if (qkv_src) std::copy(hq.begin(), hq.end(), qkv_src);
+    if (o_src) std::copy(ho.begin(), ho.end(), o_src);
+    if (role) std::copy(hrole.begin(), hrole.end(), role);
+    if (slot) std::copy(hslot.begin(), hslot.end(), slot);
+    if (blk_of) std::copy(hblk.begin(), hblk.end(), blk_of);
     return TASP_OK;
 }
 

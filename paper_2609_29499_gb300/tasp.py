@@ -29,7 +29,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use", "tasp_dispatch",
-            "tasp_plan_layer_qheads",
+            "tasp_plan_layer_qheads", "tasp_plan_layout",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -94,6 +94,7 @@ def load(path: str = LIB_PATH):
         "tasp_set_memory_limit": (c_int32, [c_int64]),
         "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
         "tasp_plan_layer_qheads": (c_int32, [P, c_int32, POINTER(c_int32)]),
+        "tasp_plan_layout": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), c_int32, P, P, P, P, P, P]),
         "tasp_memory_in_use": (c_int32, [POINTER(c_int64)]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
@@ -257,6 +258,21 @@ def memory_in_use() -> int:
     v = c_int64()
     _check(load().tasp_memory_in_use(ctypes.byref(v)))
     return v.value
+
+
+def plan_layout(shape, mask: _MaskArgs, layer: int) -> dict:
+    """Host-only: the qkv row sources, O column sources and partial-group tables of one layer."""
+    lib = load()
+    cnt = np.zeros(5, np.int32)
+    md = model_desc(shape)
+    _check(lib.tasp_plan_layout(ctypes.byref(md), ctypes.byref(mask.desc), layer, None, None, None, None, None,
+                                cnt.ctypes.data))
+    out = {k: np.zeros(int(n), dt) for k, n, dt in zip(("qkv_src", "o_src", "role", "slot", "blk_of"), cnt,
+                                                      (np.int32, np.int32, np.int16, np.int16, np.int16))}
+    _check(lib.tasp_plan_layout(ctypes.byref(md), ctypes.byref(mask.desc), layer, out["qkv_src"].ctypes.data,
+                                out["o_src"].ctypes.data, out["role"].ctypes.data, out["slot"].ctypes.data,
+                                out["blk_of"].ctypes.data, cnt.ctypes.data))
+    return out
 
 
 def _stream_ptr(stream):

@@ -1,6 +1,7 @@
 """CPU checks of the C-ABI library: it loads, exports every declared symbol, and its
 host mask compiler matches the oracle's bit for bit (no GPU work)."""
 import ctypes
+import dataclasses
 import os
 import re
 
@@ -14,6 +15,8 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 @pytest.fixture(scope="module")
+
+
 def lib():
     from paper_2609_29499_gb300 import build
     build.build()
@@ -41,6 +44,8 @@ CASES = [(synth.LAYER1, (1000, 1001, 77)), (synth.LLAMA3_8B, synth.MASK_SEEDS), 
 
 
 @pytest.mark.parametrize("shape,seeds", CASES)
+
+
 def test_host_mask_compiler_matches_oracle(lib, shape, seeds):
     for seed in seeds:
         sc = synth.mask_scores_u32(seed, shape.L, shape.n_units)
@@ -123,6 +128,8 @@ QHEAD_CASES = [(synth.LAYER1, (1000, 1001)), (synth.LLAMA3_8B, synth.MASK_SEEDS)
 
 
 @pytest.mark.parametrize("shape,seeds", QHEAD_CASES)
+
+
 def test_host_qhead_compiler_matches_oracle(lib, shape, seeds):
     for seed in seeds:
         for budget, lo, hi in ((0.57, 0.35, 0.85), (0.3, 0.2, 0.5)):
@@ -340,3 +347,46 @@ def test_header_is_a_plain_c_interface():
     r = subprocess.run([cc, "-x", "c", "-std=c99", "-Wall", "-Werror", "-fsyntax-only",
                         "-I", os.path.join(ROOT, "include"), "-"], input=src, capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+def _store_row(shape, proj, row):
+    # the store's qkv rows are group-major: per KV group its g head blocks, then K, then V
+    g, dh = shape.g, shape.dh
+    if proj == "q":
+        h, i = divmod(row, dh)
+        j, hh = divmod(h, g)
+    else:
+        j, i = divmod(row, dh)
+        hh = g if proj == "k" else g + 1
+    return (j * (g + 2) + hh) * dh + i
+
+
+@pytest.mark.parametrize("shape,heads", [
+    (synth.LAYER1, [[1, 2, 3, 4, 6]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=2), [[0, 1, 2, 5, 9, 10, 11, 31], [3, 4, 7, 30]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=1), [list(range(32))]),
+])
+
+
+def test_partial_group_tables_match_the_oracle_packing(lib, shape, heads):
+    from oracle import pack
+    units = [[0] for _ in range(shape.L)]
+    m = maskc.explicit_qheads(shape, heads, units)
+    g, dh = shape.g, shape.dh
+    for layer in range(shape.L):
+        t = lib.plan_layout(shape, lib.explicit_qhead_mask(heads, units), layer)
+        kg, qh = m.keep_groups[layer], m.keep_qheads[layer]
+        want = [_store_row(shape, p, r) for p, r in pack.qkv_rows(shape, kg, qh)]
+        assert t["qkv_src"].tolist() == want
+        assert t["o_src"].tolist() == [h * dh + i for h in qh for i in range(dh)]
+        # role: block b of the panel holds (group slot, head or K / V); blk_of inverts it
+        nblk = len(qh) + 2 * len(kg)
+        assert len(t["role"]) == nblk and len(t["blk_of"]) == len(kg) * (g + 2)
+        for b, code in enumerate(t["role"].tolist()):
+            jl, hh = divmod(code, g + 2)
+            assert t["blk_of"][code] == b
+            assert t["qkv_src"][b * dh] == (kg[jl] * (g + 2) + hh) * dh
+        assert sorted(int(x) for x in t["blk_of"] if x >= 0) == list(range(nblk))
+        # slot: compact O position of each kept head, -1 for dropped ones
+        for jl, j in enumerate(kg):
+            for hh in range(g):
+                h = j * g + hh
+                assert t["slot"][jl * g + hh] == (qh.index(h) if h in qh else -1)
