@@ -15,8 +15,6 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 @pytest.fixture(scope="module")
-
-
 def lib():
     from paper_2609_29499_gb300 import build
     build.build()
@@ -44,8 +42,6 @@ CASES = [(synth.LAYER1, (1000, 1001, 77)), (synth.LLAMA3_8B, synth.MASK_SEEDS), 
 
 
 @pytest.mark.parametrize("shape,seeds", CASES)
-
-
 def test_host_mask_compiler_matches_oracle(lib, shape, seeds):
     for seed in seeds:
         sc = synth.mask_scores_u32(seed, shape.L, shape.n_units)
@@ -128,8 +124,6 @@ QHEAD_CASES = [(synth.LAYER1, (1000, 1001)), (synth.LLAMA3_8B, synth.MASK_SEEDS)
 
 
 @pytest.mark.parametrize("shape,seeds", QHEAD_CASES)
-
-
 def test_host_qhead_compiler_matches_oracle(lib, shape, seeds):
     for seed in seeds:
         for budget, lo, hi in ((0.57, 0.35, 0.85), (0.3, 0.2, 0.5)):
@@ -364,8 +358,6 @@ def _store_row(shape, proj, row):
     (dataclasses.replace(synth.LLAMA3_8B, L=2), [[0, 1, 2, 5, 9, 10, 11, 31], [3, 4, 7, 30]]),
     (dataclasses.replace(synth.LLAMA3_8B, L=1), [list(range(32))]),
 ])
-
-
 def test_partial_group_tables_match_the_oracle_packing(lib, shape, heads):
     from oracle import pack
     units = [[0] for _ in range(shape.L)]
