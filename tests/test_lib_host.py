@@ -382,3 +382,68 @@ def test_partial_group_tables_match_the_oracle_packing(lib, shape, heads):
             for hh in range(g):
                 h = j * g + hh
                 assert t["slot"][jl * g + hh] == (qh.index(h) if h in qh else -1)
+
+
+def _dense_of_store_row(shape, r):
+    g, dh = shape.g, shape.dh
+    blk, i = divmod(r, dh)
+    j, hh = divmod(blk, g + 2)
+    if hh < g:
+        return ("q", (j * g + hh) * dh + i)
+    return ("k" if hh == g else "v", j * dh + i)
+
+
+@pytest.mark.parametrize("shape,heads", [
+    (synth.LAYER1, [[1, 2, 3, 4, 6]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=1), [[0, 1, 2, 5, 9, 10, 11, 31]]),
+])
+def test_kernel_index_math_with_partial_group_tables(lib, shape, heads):
+    # the decode QKV epilogue, the attention output store and the prefill rotary kernel,
+    # replayed on the host with the plan's tables: every query slot, K / V row and O column
+    # receives exactly the dense row or column the oracle's mask-as-zero forward uses
+    units = [[0]]
+    m = maskc.explicit_qheads(shape, heads, units)
+    kg, qh = m.keep_groups[0], m.keep_qheads[0]
+    g, dh, half = shape.g, shape.dh, shape.dh // 2
+    t = lib.plan_layout(shape, lib.explicit_qhead_mask(heads, units), 0)
+    src, role, slot, blk_of = t["qkv_src"], t["role"], t["slot"], t["blk_of"]
+    rows = len(src)
+    # decode: work rows in pairs (w, w + 1) hold panel rows (hb dh + i, hb dh + i + d_h / 2)
+    written = {}
+    for wa in range(0, rows, 2):
+        hb = wa // dh
+        i = (wa - hb * dh) >> 1
+        pr0, pr1 = hb * dh + i, hb * dh + i + half
+        jl, hh = divmod(int(role[hb]), g + 2)
+        dest = ("q", jl * g + hh) if hh < g else ("k" if hh == g else "v", jl)
+        for off, pr in ((i, pr0), (i + half, pr1)):
+            key = (dest, off)
+            assert key not in written
+            written[key] = _dense_of_store_row(shape, int(src[pr]))
+    for jl, j in enumerate(kg):
+        for hh in range(g):
+            h = j * g + hh
+            for i in range(dh):
+                if h in qh:
+                    assert written[(("q", jl * g + hh), i)] == ("q", h * dh + i)
+                else:
+                    assert (("q", jl * g + hh), i) not in written  # the slot stays zero
+        for kv in ("k", "v"):
+            for i in range(dh):
+                assert written[((kv, jl), i)] == (kv, j * dh + i)
+    # attention output: head (jl, hh) lands in compact O columns slot * d_h, which the O panel
+    # maps back to the dense columns of head h
+    for jl, j in enumerate(kg):
+        for hh in range(g):
+            s = int(slot[jl * g + hh])
+            if s >= 0:
+                assert t["o_src"][s * dh:(s + 1) * dh].tolist() == list(range((j * g + hh) * dh, (j * g + hh + 1) * dh))
+    # prefill: the rotary kernel reads panel column block blk_of[jl (g + 2) + hh] (rows in panel order)
+    for jl, j in enumerate(kg):
+        for hh in range(g + 2):
+            b = int(blk_of[jl * (g + 2) + hh])
+            if hh < g and j * g + hh not in qh:
+                assert b == -1
+                continue
+            want = ("q", (j * g + hh) * dh) if hh < g else ("k" if hh == g else "v", j * dh)
+            assert _dense_of_store_row(shape, int(src[b * dh])) == want
