@@ -58,6 +58,11 @@ typedef struct tasp_model_desc {
     float rms_eps;     /* RMSNorm epsilon (1e-5) */
     float rope_theta;  /* rotary base (500000) */
     uint64_t seed;
+    int32_t quant_group; /* INT8 scale granularity: 0 = one FP32 scale per output row; G > 0 =
+                            one BF16 scale per output row and run of G input columns (Table 1:
+                            G = 128). G must divide d, Hq*dh, df, dh and chan_unit and be a
+                            multiple of 16. Grouped stores serve decode; prefill and the union
+                            step return EUNSUP for them. */
 } tasp_model_desc;
 
 enum tasp_mask_kind {
@@ -247,7 +252,12 @@ enum tasp_export_item {
     TASP_EXPORT_GU_S = 7,        /* float [2c] */
     TASP_EXPORT_DOWN_W = 8,      /* int8 [d][c] */
     TASP_EXPORT_DOWN_S = 9,      /* float [d] */
-    TASP_EXPORT_KEEP_QHEADS = 10 /* int32 [m_q] */
+    TASP_EXPORT_KEEP_QHEADS = 10, /* int32 [m_q] */
+    /* groupwise stores: BF16 scale bit patterns (uint16) of the panels */
+    TASP_EXPORT_QKV_G = 11,      /* [(m_q + 2 m_kv) dh][d / G] */
+    TASP_EXPORT_O_G = 12,        /* [d][m_q dh / G] */
+    TASP_EXPORT_GU_G = 13,       /* [2c][d / G] */
+    TASP_EXPORT_DOWN_G = 14      /* [d][c / G] */
 };
 
 /* Copy one packed panel (logical layout, no padding) or index list of a layer

@@ -41,6 +41,7 @@ int cuda_fail(cudaError_t e, const char* what);
 // ---------------------------------------------------------------- shape
 struct Shape {
     int L = 0, d = 0, Hq = 0, Hkv = 0, dh = 0, df = 0, vocab = 0, cu = 1;
+    int qg = 0;  // scale group (input columns per BF16 scale), 0 = one FP32 scale per row
     float eps = 1e-5f, theta = 500000.f;
     uint64_t seed = 0;
     int g() const { return Hq / Hkv; }
@@ -77,7 +78,9 @@ struct Arena {
 // channel, i.e. the packed layout of the all-keep mask.
 struct LayerStore {
     int8_t *qkv, *o, *gu, *down;
-    float *qkv_s, *o_s, *gu_s, *down_s, *g_attn, *g_mlp;
+    float *qkv_s, *o_s, *gu_s, *down_s, *g_attn, *g_mlp;  // row scales (all 1 in a grouped store)
+    // grouped store only: BF16 scales [rows][K / qg] of each projection
+    uint16_t *qkv_g = nullptr, *o_g = nullptr, *gu_g = nullptr, *down_g = nullptr;
 };
 
 struct Store {
@@ -122,6 +125,9 @@ struct LayerPlan {
     const float* dn_s = nullptr;
     int dn_K = 0, dn_ld = 0;
     const float *g_attn = nullptr, *g_mlp = nullptr;
+    // grouped store only: BF16 group scales in panel order, [rows][K / qg] (row stride gq_ld
+    // for qkv / gu, o_K / qg and dn_K / qg for the column-compacted O / down panels)
+    const uint16_t *qkv_g = nullptr, *gu_g = nullptr, *o_g = nullptr, *dn_g = nullptr;
 };
 
 // FP16 copies of a layer's panels (row strides padded to 8 elements) for the prefill GEMMs.
@@ -197,6 +203,11 @@ int gather_rows(int8_t* dst, const int8_t* src, const int32_t* map, int rows, in
 int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const int32_t* cmap, int rows, int Kc,
                 cudaStream_t s);
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
+// rows of a [*][cols] uint16 matrix (dst row r = src row map[r])
+int gather_u16_rows(uint16_t* dst, const uint16_t* src, const int32_t* map, int rows, int cols, cudaStream_t s);
+// columns of a [rows][ld_src] uint16 matrix (dst column j = src column cmap[j], j < ncols)
+int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows, int ncols,
+                    cudaStream_t s);
 
 // attention.cu
 constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pass

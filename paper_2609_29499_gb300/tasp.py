@@ -21,7 +21,8 @@ OK, EINVAL, EMASK, ECAP, ENOMEM, EBUSY, ECUDA, EUNSUP = 0, -1, -2, -3, -4, -5, -
 MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT, MASK_GREEDY_QHEADS, MASK_EXPLICIT_QHEADS = 0, 1, 2, 3, 4
 PANELS_COMPACT, PANELS_ROW_INDEXED = 0, 1
 (EXPORT_KEEP_GROUPS, EXPORT_KEEP_CHANS, EXPORT_QKV_W, EXPORT_QKV_S, EXPORT_O_W, EXPORT_O_S, EXPORT_GU_W,
- EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S, EXPORT_KEEP_QHEADS) = range(11)
+ EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S, EXPORT_KEEP_QHEADS, EXPORT_QKV_G, EXPORT_O_G, EXPORT_GU_G,
+ EXPORT_DOWN_G) = range(15)
 KERNEL_KINDS = 7
 KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "other")
 
@@ -40,7 +41,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
 class ModelDesc(ctypes.Structure):
     _fields_ = [("L", c_int32), ("d", c_int32), ("Hq", c_int32), ("Hkv", c_int32), ("dh", c_int32),
                 ("df", c_int32), ("vocab", c_int32), ("chan_unit", c_int32), ("rms_eps", c_float),
-                ("rope_theta", c_float), ("seed", c_uint64)]
+                ("rope_theta", c_float), ("seed", c_uint64), ("quant_group", c_int32)]
 
 
 class MaskDesc(ctypes.Structure):
@@ -125,11 +126,8 @@ def _check(rc):
 
 def model_desc(shape) -> ModelDesc:
     """ModelDesc from any object with L, d, Hq, Hkv, dh, df, vocab, chan_unit, eps, rope_theta, seed."""
-    if getattr(shape, "quant_group", 0):
-        raise TaspError(EUNSUP, "the device store holds one INT8 scale per output row; groupwise scales are "
-                                "not built there")
     return ModelDesc(shape.L, shape.d, shape.Hq, shape.Hkv, shape.dh, shape.df, shape.vocab, shape.chan_unit,
-                     shape.eps, shape.rope_theta, shape.seed)
+                     shape.eps, shape.rope_theta, shape.seed, getattr(shape, "quant_group", 0))
 
 
 class _MaskArgs:
@@ -312,6 +310,10 @@ class Plan:
         spec = {
             EXPORT_KEEP_GROUPS: (np.int32, (m_kv,)),
             EXPORT_KEEP_QHEADS: (np.int32, (m_q,)),
+            EXPORT_QKV_G: (np.uint16, ((m_q + 2 * m_kv) * sh.dh, sh.d // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_O_G: (np.uint16, (sh.d, m_q * sh.dh // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_GU_G: (np.uint16, (2 * c, sh.d // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_DOWN_G: (np.uint16, (sh.d, c // max(1, getattr(sh, "quant_group", 0)))),
             EXPORT_KEEP_CHANS: (np.int32, (c,)),
             EXPORT_QKV_W: (np.int8, ((m_q + 2 * m_kv) * sh.dh, sh.d)),
             EXPORT_QKV_S: (np.float32, ((m_q + 2 * m_kv) * sh.dh,)),

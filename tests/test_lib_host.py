@@ -447,3 +447,16 @@ def test_kernel_index_math_with_partial_group_tables(lib, shape, heads):
                 continue
             want = ("q", (j * g + hh) * dh) if hh < g else ("k" if hh == g else "v", j * dh)
             assert _dense_of_store_row(shape, int(src[b * dh])) == want
+
+
+def test_groupwise_shapes_are_validated_on_the_host(lib):
+    import dataclasses
+    sh = synth.LLAMA3_8B
+    sc = synth.mask_scores_u32(1000, sh.L, sh.n_units)
+    tg = synth.layer_target_u24(1000, sh.L)
+    ok = lib.mask_select(dataclasses.replace(sh, quant_group=128), lib.greedy_mask(sc, tg))
+    assert ok[0] == lib.mask_select(sh, lib.greedy_mask(sc, tg))[0]  # the mask does not depend on scales
+    for bad in (48, 100, -16, 256 * 1024):
+        with pytest.raises(lib.TaspError) as e:
+            lib.mask_select(dataclasses.replace(sh, quant_group=bad), lib.greedy_mask(sc, tg))
+        assert e.value.code == lib.EINVAL
