@@ -63,6 +63,8 @@ def parse():
                     help="mixed workload: Q/K/V and gate/up panels as row maps into the shared store "
                          "(zero copy) or materialized copies")
     ap.add_argument("--prompt", type=int, default=2048, help="prefill prompt length")
+    ap.add_argument("--quant-group", type=int, default=0,
+                    help="groupwise INT8 store with one BF16 scale per this many input columns (Table 1: 128)")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep the workload's widths but only this many layers (small cases for ncu captures)")
     return ap.parse_args()
@@ -161,6 +163,9 @@ def workload(args):
     if args.layers:
         sh = dataclasses.replace(wl.shape, L=args.layers)
         wl = dataclasses.replace(wl, shape=sh, name=f"{wl.name}_{args.layers}layers")
+    if args.quant_group:
+        sh = dataclasses.replace(wl.shape, quant_group=args.quant_group)
+        wl = dataclasses.replace(wl, shape=sh, name=f"{wl.name}_int8g{args.quant_group}")
     return wl, wl.shape, wl.masks[0]
 
 
@@ -189,6 +194,12 @@ def gemv_bytes(shape, plan_dims):
         if c:
             b["gate_up"] += 2 * c * d + 2 * c * 4 + d * 4 + d * 4 + c * 4
             b["down"] += d * c + d * 4 + c * 4 + 2 * d * 4
+        G = getattr(shape, "quant_group", 0)
+        if G:  # BF16 group scales: 2 bytes per G weights
+            b["qkv"] += 2 * rows * (d // G)
+            b["o_proj"] += 2 * d * (m_kv * g * dh // G)
+            b["gate_up"] += 2 * 2 * c * (d // G)
+            b["down"] += 2 * d * (c // G)
     b["lm_head"] = shape.vocab * d * 2 + d * 4 + shape.vocab * 4
     return b
 

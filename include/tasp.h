@@ -58,6 +58,11 @@ typedef struct tasp_model_desc {
     float rms_eps;     /* RMSNorm epsilon (1e-5) */
     float rope_theta;  /* rotary base (500000) */
     uint64_t seed;
+    int32_t quant_group; /* INT8 scale granularity: 0 = one FP32 scale per output row; G > 0 =
+                            one BF16 scale per output row and run of G input columns (Table 1:
+                            G = 128). G must divide d, Hq*dh, df, dh and chan_unit and be a
+                            multiple of 16. Grouped stores serve decode; prefill and the union
+                            step return EUNSUP for them. */
 } tasp_model_desc;
 
 enum tasp_mask_kind {
@@ -117,9 +122,8 @@ typedef struct tasp_session tasp_session;
  * identical model_desc share it), runs the host mask compiler, packs the
  * panels on the device. sync. *out receives the plan.
  * Errors: EINVAL (bad desc, mask violates closure/budget, empty layer),
- * EUNSUP (a query-head mask that keeps part of a group: the device kernels
- * take whole GQA groups; query-head masks whose groups are whole compile),
- * ENOMEM, ECUDA. */
+ * ENOMEM, ECUDA. Query-head masks may keep part of a group: the plan then
+ * carries per-layer role tables for its partial groups. */
 int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, tasp_plan** out);
 
 /* Prefill one prompt with a plan (Sec. 3.3: the plan chosen for a turn serves
@@ -203,6 +207,16 @@ int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, i
  * n_qheads [L] (ascending per layer). For the group kinds these are all g heads
  * of every kept group; for the query-head kinds keep_groups holds the KV heads
  * that the closure keeps. Host only; any output may be NULL. */
+/* Host only (test introspection): the tables a plan of `mask` uses for one layer.
+ * qkv_src [(m_q + 2 m_kv) dh]: store row of each qkv panel row (store rows are
+ * group-major: per KV group its g head blocks of dh rows, then K, then V);
+ * o_src [m_q dh]: dense O column of each panel column; role [m_q + 2 m_kv],
+ * slot [m_kv g], blk_of [m_kv (g + 2)]: the partial-group tables (role of each
+ * dh-row block as jl (g + 2) + hh; compact O position of (jl, hh) or -1; inverse
+ * of role or -1). counts [5] receives the five lengths. Any array may be NULL. */
+int tasp_plan_layout(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t layer, int32_t* qkv_src,
+                     int32_t* o_src, int16_t* role, int16_t* slot, int16_t* blk_of, int32_t* counts);
+
 int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
                             int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
                             int32_t* n_units, int64_t* flops);
@@ -224,6 +238,8 @@ int tasp_plan_info_get(const tasp_plan* plan, tasp_plan_info* out);
 
 /* Per-layer retained sizes: out[0] = m_kv (kept groups), out[1] = c (kept channels). */
 int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2);
+/* Kept query heads m_q of a layer (m_kv g unless the mask keeps part of a group). */
+int tasp_plan_layer_qheads(const tasp_plan* plan, int32_t layer, int32_t* m_q);
 
 enum tasp_export_item {
     TASP_EXPORT_KEEP_GROUPS = 0, /* int32 [m_kv] */
@@ -235,7 +251,13 @@ enum tasp_export_item {
     TASP_EXPORT_GU_W = 6,        /* int8 [2c][d], gate row then up row per kept channel */
     TASP_EXPORT_GU_S = 7,        /* float [2c] */
     TASP_EXPORT_DOWN_W = 8,      /* int8 [d][c] */
-    TASP_EXPORT_DOWN_S = 9       /* float [d] */
+    TASP_EXPORT_DOWN_S = 9,      /* float [d] */
+    TASP_EXPORT_KEEP_QHEADS = 10, /* int32 [m_q] */
+    /* groupwise stores: BF16 scale bit patterns (uint16) of the panels */
+    TASP_EXPORT_QKV_G = 11,      /* [(m_q + 2 m_kv) dh][d / G] */
+    TASP_EXPORT_O_G = 12,        /* [d][m_q dh / G] */
+    TASP_EXPORT_GU_G = 13,       /* [2c][d / G] */
+    TASP_EXPORT_DOWN_G = 14      /* [d][c / G] */
 };
 
 /* Copy one packed panel (logical layout, no padding) or index list of a layer

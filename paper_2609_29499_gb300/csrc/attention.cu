@@ -127,6 +127,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
     // session bz of the batch
     const float* const q_in = p.q + bz * p.q_stride;
     float* const o_out = p.o + bz * p.q_stride;
+    const int16_t* const oslot = p.oslot[bz];  // NULL: every head of the kept groups, in order
     float* const part = p.part + bz * p.part_stride;
     float* const ml = p.ml + bz * p.ml_stride;
     int* const cnt = p.cnt + bz * p.cnt_stride;
@@ -342,7 +343,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
 #pragma unroll
         for (int r = 0; r < CS; ++r) As = fmaf(inbox[r][it], rw[r][hh], As);
         if (NC == 1) {
-            o_out[(int64_t)(jl * G + hh) * DH + dim] = As / Lt[hh];
+            const int oh = oslot ? oslot[jl * G + hh] : jl * G + hh;
+            if (oh >= 0) o_out[(int64_t)oh * DH + dim] = As / Lt[hh];
         } else {
             part[((int64_t)(jl * NC + cid) * G + hh) * DH + dim] = As;
             if (dim == 0) {
@@ -388,7 +390,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             o.z = fmaf(a.z, w, o.z);
             o.w = fmaf(a.w, w, o.w);
         }
-        reinterpret_cast<float4*>(o_out + (int64_t)(jl * G + hh) * DH)[d4] = o;
+        const int oh = oslot ? oslot[jl * G + hh] : jl * G + hh;
+        if (oh >= 0) reinterpret_cast<float4*>(o_out + (int64_t)oh * DH)[d4] = o;
     }
     if (tid == 0) cnt[jl] = 0;
 }

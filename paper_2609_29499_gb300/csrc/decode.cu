@@ -97,6 +97,7 @@ std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 int launch_gemv(int mode, Params p, cudaStream_t s) {
     if (p.rows == 0 || p.nb == 0) return TASP_OK;
     if (p.nb > MAXNB) return fail(TASP_EINVAL, "more activation vectors than one GEMV pass takes");
+    if (p.gscale) return fail(TASP_EUNSUP, "groupwise stores decode one session per weight pass");
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
@@ -209,6 +210,15 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
         op.p = p;
         ops.push_back(op);
     };
+    // groupwise store: the row's BF16 scale of each column group of `cols` input columns
+    auto set_groups = [&](Params& q, const uint16_t* gs, int cols) {
+        if (!sh.qg) return;
+        q.gscale = gs;
+        q.gcols = cols / sh.qg;
+        int sft = 0;
+        while ((16 << sft) < sh.qg) ++sft;
+        q.gshift = sft;
+    };
     for (int l = l_begin; l < l_end; ++l) {
         const LayerPlan& lp = pl.layers[l];
         const bool first = (l == 0) && t.x_in != nullptr;
@@ -241,6 +251,8 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
         }
         p.g = sh.g();
         p.dh = sh.dh;
+        p.blk_role = lp.blk_role;
+        set_groups(p, lp.qkv_g, sh.d);
         p.err = bv.err;
         gemv(K_QKV, M_QKV, p);
         // K2: split-KV attention over the retained KV heads of every session
@@ -257,6 +269,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 a.pos[b] = se.d_pos;
                 a.max_tokens[b] = se.max_tokens;
                 a.m_kv[b] = lp.m_kv;
+                a.oslot[b] = lp.oslot;
                 S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
@@ -288,6 +301,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             o.act_stride = bv.q_stride;
             o.resid_out = bv.x;
             o.x_stride = bv.x_stride;
+            set_groups(o, lp.o_g, lp.o_K);
             o.err = bv.err;
             gemv(K_O, M_O, o);
         }
@@ -309,6 +323,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             gu.eps = sh.eps;
             gu.h_out = bv.h;
             gu.h_stride = bv.h_stride;
+            set_groups(gu, lp.gu_g, sh.d);
             gu.err = bv.err;
             gemv(K_GU, M_GU, gu);
             // K5: down projection + residual
@@ -326,6 +341,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             dn.x_stride = bv.x_stride;
             dn.hidden_out = last ? t.hidden_out : nullptr;
             dn.hid_stride = sh.d;
+            set_groups(dn, lp.dn_g, lp.dn_K);
             dn.err = bv.err;
             gemv(K_DOWN, M_DOWN, dn);
         } else if (last && t.hidden_out) {

@@ -75,6 +75,9 @@ struct Params {
     const float2* rope[MAXNB];
     const int* pos[MAXNB];
     int g, dh;
+    const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
+    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gcols] (single-vector kernels only)
+    int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
     float* h_out;          // GU: SiLU(gate) * up, stride h_stride
     int64_t h_stride;
     float* logits;         // LM: stride logit_stride
@@ -528,7 +531,8 @@ __device__ __forceinline__ void epilogue(const Params& p, const float (*red)[R *
                     const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
                     float y0 = sc0 * s0, y1 = sc1 * s1;
                     const int gp2 = p.g + 2;
-                    const int jl = hb / gp2, hh = hb - jl * gp2;
+                    const int code = p.blk_role ? p.blk_role[hb] : hb;
+                    const int jl = code / gp2, hh = code - jl * gp2;
                     if (hh <= p.g) {
                         const float2 cs = es.rope[v][i];
                         const float ya = y0 * cs.x - y1 * cs.y, yb = y1 * cs.x + y0 * cs.y;

@@ -48,6 +48,9 @@ struct GemvParams {
     const float2* rope;
     const int* pos;
     int g, dh;
+    const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
+    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gcols] (NULL = per-row only)
+    int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
     float* h_out;
     float* logits;
     int* err;       // device error word (bounded waits that gave up)
@@ -323,10 +326,12 @@ __device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
 }
 
 // INT8 rows of one stage . x: per chunk sum(w * X) = 256 sum(w * hi) + sum(w * lo) in
-// exact INT32, then acc[r] += float(sum) * scale in FP32.
-template <int R, int XC>
+// exact INT32, then acc[r] += float(sum) * scale in FP32. GS (groupwise store): the scale
+// of the chunk also carries the row's BF16 scale of the chunk's column group.
+template <int R, int XC, bool GS>
 __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC>& xd,
-                                       int nchunks, int tid, float (&acc)[R]) {
+                                       int nchunks, int tid, float (&acc)[R], const uint16_t* const (&grow)[R],
+                                       int gshift) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
@@ -341,7 +346,9 @@ __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld
                     sh = dp4a_ss(wd[k], xd.hi[j][k], sh);
                     sl = dp4a_su(wd[k], xd.lo[j][k], sl);
                 }
-                acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xd.scale[j], acc[r]);
+                float xsc = xd.scale[j];
+                if constexpr (GS) xsc *= __uint_as_float((uint32_t)__ldg(grow[r] + (c >> gshift)) << 16);
+                acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xsc, acc[r]);
             }
         }
     }
@@ -431,7 +438,8 @@ __device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)
                     const int hb = wa / p.dh, i = (wa - hb * p.dh) >> 1;
                     float y0 = sc0 * s0, y1 = sc1 * s1;
                     const int gp2 = p.g + 2;
-                    const int jl = hb / gp2, hh = hb - jl * gp2;
+                    const int code = p.blk_role ? p.blk_role[hb] : hb;
+                    const int jl = code / gp2, hh = code - jl * gp2;
                     const int pos = es.pos;
                     if (hh <= p.g) {
                         const float2 cs = es.rope[i];
@@ -481,7 +489,7 @@ __host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld,
     return g;
 }
 
-template <int MODE, int R, int XC>
+template <int MODE, int R, int XC, bool GS>
 __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams p) {
     extern __shared__ __align__(128) uint8_t sm[];
     __shared__ float red[NRB][CW][R];
@@ -610,7 +618,14 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
         } else {
 #pragma unroll
             for (int r = 0; r < R; ++r) v[r] = 0.f;
-            dot_i8<R, XC>(st, (int)p.ld, xd, p.nchunks, tid, v);
+            const uint16_t* grow[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                int w = gi * R + r;
+                if (w >= p.rows) w = 0;  // padding row of a ragged last group: never stored
+                grow[r] = GS ? p.gscale + (size_t)panel_row<MODE>(p, w) * p.gcols : nullptr;
+            }
+            dot_i8<R, XC, GS>(st, (int)p.ld, xd, p.nchunks, tid, v, grow, p.gshift);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
@@ -650,34 +665,43 @@ int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const
 
 typedef void (*GemvFn)(const GemvParams);
 
-template <int MODE>
+template <int MODE, bool GS>
 GemvFn gemv_fn(int R, int XC) {
     if (XC <= 1) {
-        if (R >= 8) return gemv_kernel<MODE, 8, 1>;
-        if (R >= 4) return gemv_kernel<MODE, 4, 1>;
-        return gemv_kernel<MODE, 2, 1>;
+        if (R >= 8) return gemv_kernel<MODE, 8, 1, GS>;
+        if (R >= 4) return gemv_kernel<MODE, 4, 1, GS>;
+        return gemv_kernel<MODE, 2, 1, GS>;
     }
     if (XC <= 2) {
-        if (R >= 4) return gemv_kernel<MODE, 4, 2>;
-        return gemv_kernel<MODE, 2, 2>;
+        if (R >= 4) return gemv_kernel<MODE, 4, 2, GS>;
+        return gemv_kernel<MODE, 2, 2, GS>;
     }
     if (XC <= 4) {
-        if (R >= 2) return gemv_kernel<MODE, 2, 4>;
+        if (R >= 2) return gemv_kernel<MODE, 2, 4, GS>;
         if constexpr (MODE == M_QKV || MODE == M_GU)
             return nullptr;  // rotary / SwiGLU pairs need two rows per stage
         else
-            return gemv_kernel<MODE, 1, 4>;
+            return gemv_kernel<MODE, 1, 4, GS>;
     }
     return nullptr;
 }
 
-GemvFn pick(int mode, int R, int XC) {
+GemvFn pick(int mode, int R, int XC, bool gs) {
+    if (gs) {
+        switch (mode) {
+            case M_QKV: return gemv_fn<M_QKV, true>(R, XC);
+            case M_O: return gemv_fn<M_O, true>(R, XC);
+            case M_GU: return gemv_fn<M_GU, true>(R, XC);
+            case M_DOWN: return gemv_fn<M_DOWN, true>(R, XC);
+            default: return nullptr;  // the LM head is BF16, never grouped
+        }
+    }
     switch (mode) {
-        case M_QKV: return gemv_fn<M_QKV>(R, XC);
-        case M_O: return gemv_fn<M_O>(R, XC);
-        case M_GU: return gemv_fn<M_GU>(R, XC);
-        case M_DOWN: return gemv_fn<M_DOWN>(R, XC);
-        default: return gemv_fn<M_LM>(R, XC);
+        case M_QKV: return gemv_fn<M_QKV, false>(R, XC);
+        case M_O: return gemv_fn<M_O, false>(R, XC);
+        case M_GU: return gemv_fn<M_GU, false>(R, XC);
+        case M_DOWN: return gemv_fn<M_DOWN, false>(R, XC);
+        default: return gemv_fn<M_LM, false>(R, XC);
     }
 }
 
@@ -703,7 +727,7 @@ int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
     if (XC > 4) return fail(TASP_EUNSUP, "row too long for the register-resident activation slice");
     if (XC == 2 && R > 4) R = 4;
     if (XC == 4 && R > 2) R = 2;
-    GemvFn fn = pick(mode, R, XC);
+    GemvFn fn = pick(mode, R, XC, p.gscale != nullptr);
     if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
     p.err = err;
     {
@@ -754,6 +778,10 @@ int launch_gemv_single(int mode, const gemv::Params& q, cudaStream_t s) {
     p.pos = q.pos[0];
     p.g = q.g;
     p.dh = q.dh;
+    p.blk_role = q.blk_role;
+    p.gscale = q.gscale;
+    p.gcols = q.gcols;
+    p.gshift = q.gshift;
     p.h_out = q.h_out;
     p.logits = q.logits;
     return gemv1::launch_gemv(mode, p, q.err, s);

@@ -33,7 +33,7 @@ int64_t layer_flops(const Shape& s, int64_t m_q, int64_t m_kv, int64_t c) {
 
 bool Shape::same(const Shape& o) const {
     return L == o.L && d == o.d && Hq == o.Hq && Hkv == o.Hkv && dh == o.dh && df == o.df && vocab == o.vocab &&
-           cu == o.cu && eps == o.eps && theta == o.theta && seed == o.seed;
+           cu == o.cu && eps == o.eps && theta == o.theta && seed == o.seed && qg == o.qg;
 }
 
 namespace {

@@ -329,13 +329,17 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_vec_kernel(const float* __re
 // keys [group][T][dh] (the transposed values come from v_transpose_kernel).
 __global__ void rope_kv_kernel(const float* __restrict__ Y, int ldy, int T, int g, int dh,
                                const float2* __restrict__ rope, float* Qf, uint16_t* Kc, uint16_t* Vc,
-                               int max_tokens, __half* Qh, float qscale, __half* Kh) {
+                               int max_tokens, __half* Qh, float qscale, __half* Kh,
+                               const int16_t* __restrict__ blk_of) {
     const int t = blockIdx.x, jl = blockIdx.y;
     const int half = dh >> 1;
     for (int w = threadIdx.x; w < (g + 2) * half; w += blockDim.x) {
         const int hh = w / half, i = w - hh * half;
-        const int col = (jl * (g + 2) + hh) * dh + i;
-        float y0 = Y[(int64_t)t * ldy + col], y1 = Y[(int64_t)t * ldy + col + half];
+        // the panel's d_h-column block of (group slot, head); -1: a dropped head, whose query
+        // slot is written as zeros (its attention output is never used)
+        const int blk = blk_of ? blk_of[jl * (g + 2) + hh] : jl * (g + 2) + hh;
+        const int col = blk * dh + i;
+        float y0 = blk >= 0 ? Y[(int64_t)t * ldy + col] : 0.f, y1 = blk >= 0 ? Y[(int64_t)t * ldy + col + half] : 0.f;
         if (hh <= g) {
             const float2 cs = rope[(int64_t)t * half + i];
             const float a = y0 * cs.x - y1 * cs.y, b = y1 * cs.x + y0 * cs.y;
@@ -451,7 +455,8 @@ struct PaCfg {
 template <int DH>
 __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const float* __restrict__ Qf, const uint16_t* K,
                                                                      const uint16_t* V, int T, int max_tokens, int g,
-                                                                     float qscale, __half* O, int ldo) {
+                                                                     float qscale, __half* O, int ldo,
+                                                                     const int16_t* __restrict__ oslot) {
     using C = PaCfg<DH>;
     constexpr int ROWB = C::ROWB, TILEB = C::TILEB, KS = DH / 16, NT = DH / 8, CPR = DH * 2 / 16;
     constexpr int SUB = PA_KT / 16;  // 16-key sub-tiles per tile
@@ -618,9 +623,10 @@ __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const fl
     for (int i = 0; i < 2; ++i) {
         l_run[i] += __shfl_xor_sync(0xffffffffu, l_run[i], 1);
         l_run[i] += __shfl_xor_sync(0xffffffffu, l_run[i], 2);
-        if (rq[i] < T) {
+        const int oh = oslot ? oslot[h] : h;  // compact O column block; -1: dropped head
+        if (rq[i] < T && oh >= 0) {
             const float inv = 1.0f / l_run[i];
-            __half* o = O + (int64_t)rq[i] * ldo + h * DH;
+            __half* o = O + (int64_t)rq[i] * ldo + oh * DH;
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
                 const int dim = nt * 8 + qc;
@@ -675,7 +681,8 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 
 __global__ void __launch_bounds__(192, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmVT, int T, int g, __half* O, int ldo, int* err) {
+                   const __grid_constant__ CUtensorMap tmVT, int T, int g, __half* O, int ldo, int* err,
+                   const int16_t* __restrict__ oslot) {
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
     uint8_t* sq = sm;
@@ -687,6 +694,7 @@ __global__ void __launch_bounds__(192, 1)
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x, jl = h / g;
+    const int oh = oslot ? oslot[h] : h;  // compact O column block of this head; -1: dropped head
     const int q0 = (gridDim.y - 1 - blockIdx.y) * 128;  // the longest query blocks of every head first
     const int kend = min(T, q0 + 128);
     const int ntile = (kend + AT_KT - 1) / AT_KT;
@@ -853,12 +861,12 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t o[32];
             tmem_ld32(trow + 128u + c0, o);
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            if (qi < T) {
+            if (qi < T && oh >= 0) {
                 uint32_t hw[16];
 #pragma unroll
                 for (int c = 0; c < 32; c += 2)
                     hw[c >> 1] = pack_h2(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv);
-                uint4* dst = reinterpret_cast<uint4*>(O + (int64_t)qi * ldo + h * 128 + c0);
+                uint4* dst = reinterpret_cast<uint4*>(O + (int64_t)qi * ldo + oh * 128 + c0);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) dst[k] = make_uint4(hw[4 * k], hw[4 * k + 1], hw[4 * k + 2], hw[4 * k + 3]);
             }
@@ -1035,7 +1043,8 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
             ga.mode = EP_STORE; ga.err = se.err;
             if ((rc = launch_gemm(Xh, ld_x, T, f.qkv, f.ld_d, lp.qkv_rows, sh.d, ga, s))) break;
             rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, tc_attn ? nullptr : Qf,
-                                                            se.K[l], se.V[l], se.max_tokens, Qh, qscale, Kh);
+                                                            se.K[l], se.V[l], se.max_tokens, Qh, qscale, Kh,
+                                                            lp.blk_of);
             if (tc_attn) {
                 v_transpose_kernel<<<dim3((T + 63) / 64, lp.m_kv), 256, 0, s>>>(se.V[l], se.max_tokens, T, VT, Tp);
                 CUtensorMap mq, mk, mv;
@@ -1044,11 +1053,11 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
                 if ((rc = make_map(&mk, Kh, lp.m_kv * T, 128, 128, AT_KT))) break;
                 if ((rc = make_map(&mv, VT, lp.m_kv * 128, Tp, Tp, 128))) break;
                 attn_tc_kernel<<<dim3(lp.m_kv * sh.g(), (T + 127) / 128), 192, AT_SMEM, s>>>(mq, mk, mv, T, sh.g(), O,
-                                                                                           ld_o, se.err);
+                                                                                           ld_o, se.err, lp.oslot);
             } else {
                 const int qb = (T + PA_QB - 1) / PA_QB;
                 attn_prefill_kernel<64><<<dim3(lp.m_kv * sh.g(), qb), PA_WARPS * 32, PaCfg<64>::SMEM, s>>>(
-                    Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o);
+                    Qf, se.K[l], se.V[l], T, se.max_tokens, sh.g(), qscale, O, ld_o, lp.oslot);
             }
             TASP_CUDA(cudaGetLastError());
             GemmArgs go{};

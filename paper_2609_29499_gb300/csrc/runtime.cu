@@ -110,12 +110,15 @@ static std::vector<Store*> g_stores;
 static int validate_shape(const tasp_model_desc* m, Shape& s, bool device = true) {
     if (!m) return fail(TASP_EINVAL, "model_desc is NULL");
     s.L = m->L; s.d = m->d; s.Hq = m->Hq; s.Hkv = m->Hkv; s.dh = m->dh; s.df = m->df; s.vocab = m->vocab;
-    s.cu = m->chan_unit; s.eps = m->rms_eps; s.theta = m->rope_theta; s.seed = m->seed;
+    s.cu = m->chan_unit; s.eps = m->rms_eps; s.theta = m->rope_theta; s.seed = m->seed; s.qg = m->quant_group;
     if (s.L < 1 || s.d < 16 || s.d % 16 || s.Hq < 1 || s.Hkv < 1 || s.Hq % s.Hkv || s.dh < 16 || s.dh % 16 ||
         s.dh > 128 || s.df < 1 || s.df % 16 || s.cu < 1 || s.df % s.cu || s.vocab < 0 || !(s.eps > 0.f) ||
         !(s.theta > 0.f))
         return fail(TASP_EINVAL, "invalid model shape (need d, df, dh multiples of 16, dh <= 128, Hq % Hkv == 0, "
                                  "df % chan_unit == 0)");
+    if (s.qg < 0 || (s.qg && (s.qg % 16 || ((s.qg / 16) & (s.qg / 16 - 1)) || s.d % s.qg || s.df % s.qg ||
+                              s.dh % s.qg || s.cu % s.qg)))
+        return fail(TASP_EINVAL, "quant_group must be 0 or 16 times a power of two dividing d, df, dh and chan_unit");
     if (!device) return TASP_OK;
     if (!attn_supported(s.dh, s.g()))
         return fail(TASP_EUNSUP, "attention kernel not built for this (head_dim, query heads per group)");
@@ -136,9 +139,11 @@ static int store_acquire(const Shape& sh, Store** out) {
     st->sh = sh;
     const size_t d = sh.d, qkv = (size_t)sh.qkv_rows_dense(), hq = (size_t)sh.Hq * sh.dh, df = sh.df;
     Layout lay;
+    const size_t G = sh.qg;
     for (int l = 0; l < sh.L; ++l) {
         lay.add(qkv * d); lay.add(d * hq); lay.add(2 * df * d); lay.add(d * df);
         lay.add(qkv * 4); lay.add(d * 4); lay.add(2 * df * 4); lay.add(d * 4); lay.add(d * 4); lay.add(d * 4);
+        if (G) { lay.add(qkv * (d / G) * 2); lay.add(d * (hq / G) * 2); lay.add(2 * df * (d / G) * 2); lay.add(d * (df / G) * 2); }
     }
     lay.add(d * 4);
     lay.add((size_t)sh.vocab * d * 2);
@@ -157,6 +162,12 @@ static int store_acquire(const Shape& sh, Store** out) {
         ls.down_s = (float*)st->arena.take(d * 4);
         ls.g_attn = (float*)st->arena.take(d * 4);
         ls.g_mlp = (float*)st->arena.take(d * 4);
+        if (G) {
+            ls.qkv_g = (uint16_t*)st->arena.take(qkv * (d / G) * 2);
+            ls.o_g = (uint16_t*)st->arena.take(d * (hq / G) * 2);
+            ls.gu_g = (uint16_t*)st->arena.take(2 * df * (d / G) * 2);
+            ls.down_g = (uint16_t*)st->arena.take(d * (df / G) * 2);
+        }
     }
     st->g_final = (float*)st->arena.take(d * 4);
     st->lm_head = sh.vocab ? (uint16_t*)st->arena.take((size_t)sh.vocab * d * 2) : nullptr;
@@ -193,6 +204,34 @@ static void store_release(Store* st) {
 }
 
 // ---------------------------------------------------------------- plan compilation
+// Source rows of the qkv panel in the store (per kept group its kept heads' d_h-row blocks,
+// then K, then V; store rows are group-major: g head blocks, K, V), source columns of the O
+// panel (the kept heads in ascending order), and the role / slot / block tables of partial
+// groups (see LayerPlan).
+static void layer_tables(const Shape& sh, const LayerPlan& lp, std::vector<int32_t>& hq, std::vector<int32_t>& ho,
+                         std::vector<int16_t>& hrole, std::vector<int16_t>& hslot, std::vector<int16_t>& hblk) {
+    const int g = sh.g(), dh = sh.dh;
+    hq.clear(); ho.clear(); hrole.clear();
+    hslot.assign((size_t)lp.m_kv * g, -1);
+    hblk.assign((size_t)lp.m_kv * (g + 2), -1);
+    std::vector<char> keep_h(sh.Hq, 0);
+    for (int h : lp.keep_qheads) keep_h[h] = 1;
+    int slot = 0;
+    for (int jl = 0; jl < lp.m_kv; ++jl) {
+        const int j = lp.keep_groups[jl];
+        for (int hh = 0; hh < g + 2; ++hh) {
+            if (hh < g && !keep_h[j * g + hh]) continue;
+            for (int r = 0; r < dh; ++r) hq.push_back((j * (g + 2) + hh) * dh + r);
+            hblk[(size_t)jl * (g + 2) + hh] = (int16_t)hrole.size();
+            hrole.push_back((int16_t)(jl * (g + 2) + hh));
+            if (hh < g) {
+                hslot[(size_t)jl * g + hh] = (int16_t)slot++;
+                for (int c = 0; c < dh; ++c) ho.push_back((j * g + hh) * dh + c);
+            }
+        }
+    }
+}
+
 static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep) {
     Store& st = *p.store;
     const Shape& sh = st.sh;
@@ -201,14 +240,16 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
     for (int l = 0; l < sh.L; ++l) {
         LayerPlan& lp = p.layers[l];
         lp.keep_groups = sel.groups[l];
+        lp.keep_qheads = sel.qheads[l];
         lp.keep_chans.clear();
         for (int u : sel.units[l])
             for (int i = 0; i < sh.cu; ++i) lp.keep_chans.push_back(u * sh.cu + i);
         lp.m_kv = (int)lp.keep_groups.size();
+        lp.m_q = (int)lp.keep_qheads.size();
         lp.c = (int)lp.keep_chans.size();
-        lp.qkv_rows = lp.m_kv * (g + 2) * dh;
+        lp.qkv_rows = (lp.m_q + 2 * lp.m_kv) * dh;
         lp.gu_rows = 2 * lp.c;
-        lp.o_K = lp.m_kv * g * dh;
+        lp.o_K = lp.m_q * dh;
         lp.dn_K = lp.c;
         lp.g_attn = st.layers[l].g_attn;
         lp.g_mlp = st.layers[l].g_mlp;
@@ -223,15 +264,28 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
             lp.o_w = ls.o; lp.o_s = ls.o_s; lp.o_ld = sh.Hq * dh;
             lp.gu_w = ls.gu; lp.gu_s = ls.gu_s;
             lp.dn_w = ls.down; lp.dn_s = ls.down_s; lp.dn_ld = sh.df;
+            lp.qkv_g = ls.qkv_g; lp.o_g = ls.o_g; lp.gu_g = ls.gu_g; lp.dn_g = ls.down_g;
         }
         return TASP_OK;
     }
+    const int G = sh.qg;  // scale group of a grouped store (0: per-row scales only)
     const bool rowidx = panel_mode == TASP_PANELS_ROW_INDEXED;
+    auto ragged = [&](const LayerPlan& lp) { return lp.m_q != lp.m_kv * g; };
     // sizing pass
     Layout lay;
     for (int l = 0; l < sh.L; ++l) {
         const LayerPlan& lp = p.layers[l];
         const size_t ol = round16(lp.o_K), dl = round16(lp.dn_K);
+        if (G) {  // group scales in panel order, and the column-group maps of O / down
+            lay.add((size_t)lp.qkv_rows * (d / G) * 2); lay.add((size_t)lp.gu_rows * (d / G) * 2);
+            lay.add((size_t)d * (lp.o_K / G) * 2); lay.add((size_t)d * (lp.dn_K / G) * 2);
+            lay.add((size_t)(lp.o_K / G) * 4); lay.add((size_t)(lp.dn_K / G) * 4);
+        }
+        if (ragged(lp)) {
+            lay.add((size_t)(lp.m_q + 2 * lp.m_kv) * 2);
+            lay.add((size_t)lp.m_kv * g * 2);
+            lay.add((size_t)lp.m_kv * (g + 2) * 2);
+        }
         lay.add((size_t)lp.qkv_rows * 4); lay.add((size_t)lp.qkv_rows * 4);  // map, scales
         lay.add((size_t)lp.gu_rows * 4); lay.add((size_t)lp.gu_rows * 4);
         lay.add(ol * 4); lay.add(dl * 4);                                       // column maps
@@ -243,16 +297,14 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
     cudaStream_t s;
     TASP_CUDA(cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking));
     std::vector<int32_t> hq, hg, ho, hd;
+    std::vector<int16_t> hrole, hslot, hblk;
     for (int l = 0; l < sh.L && !rc; ++l) {
         LayerPlan& lp = p.layers[l];
         const LayerStore& ls = st.layers[l];
         const int ol = round16(lp.o_K), dl = round16(lp.dn_K);
-        hq.clear(); hg.clear(); ho.clear(); hd.clear();
-        for (int j : lp.keep_groups)
-            for (int r = 0; r < (g + 2) * dh; ++r) hq.push_back(j * (g + 2) * dh + r);
+        layer_tables(sh, lp, hq, ho, hrole, hslot, hblk);
+        hg.clear(); hd.clear();
         for (int c : lp.keep_chans) { hg.push_back(2 * c); hg.push_back(2 * c + 1); }
-        for (int j : lp.keep_groups)
-            for (int c = 0; c < g * dh; ++c) ho.push_back(j * g * dh + c);
         ho.resize(ol, 0);
         hd = std::vector<int32_t>(lp.keep_chans.begin(), lp.keep_chans.end());
         hd.resize(dl, 0);
@@ -262,6 +314,17 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
         float* sg = (float*)p.arena.take(hg.size() * 4);
         int32_t* dco = (int32_t*)p.arena.take(ho.size() * 4);
         int32_t* dcd = (int32_t*)p.arena.take(hd.size() * 4);
+        if (ragged(lp)) {
+            int16_t* drole = (int16_t*)p.arena.take(hrole.size() * 2);
+            int16_t* dslot = (int16_t*)p.arena.take(hslot.size() * 2);
+            int16_t* dblk = (int16_t*)p.arena.take(hblk.size() * 2);
+            TASP_CUDA(cudaMemcpyAsync(drole, hrole.data(), hrole.size() * 2, cudaMemcpyHostToDevice, s));
+            TASP_CUDA(cudaMemcpyAsync(dslot, hslot.data(), hslot.size() * 2, cudaMemcpyHostToDevice, s));
+            TASP_CUDA(cudaMemcpyAsync(dblk, hblk.data(), hblk.size() * 2, cudaMemcpyHostToDevice, s));
+            lp.blk_role = drole;
+            lp.oslot = dslot;
+            lp.blk_of = dblk;
+        }
         if (hq.size()) TASP_CUDA(cudaMemcpyAsync(dq, hq.data(), hq.size() * 4, cudaMemcpyHostToDevice, s));
         if (hg.size()) TASP_CUDA(cudaMemcpyAsync(dg, hg.data(), hg.size() * 4, cudaMemcpyHostToDevice, s));
         if (ho.size()) TASP_CUDA(cudaMemcpyAsync(dco, ho.data(), ho.size() * 4, cudaMemcpyHostToDevice, s));
@@ -270,6 +333,29 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
         if ((rc = gather_f32(sg, ls.gu_s, dg, (int)hg.size(), s))) break;
         lp.qkv_s = sq;
         lp.gu_s = sg;
+        if (G) {
+            // qkv / gu: the scale rows follow their weight rows; O / down: the scale columns of
+            // the kept column groups (kept heads and channel units are whole groups)
+            std::vector<int32_t> cgo, cgd;
+            for (size_t k = 0; k < (size_t)lp.o_K; k += G) cgo.push_back(ho[k] / G);
+            for (size_t k = 0; k < (size_t)lp.dn_K; k += G) cgd.push_back(lp.keep_chans[k] / G);
+            uint16_t* gq = (uint16_t*)p.arena.take((size_t)lp.qkv_rows * (d / G) * 2);
+            uint16_t* gg = (uint16_t*)p.arena.take((size_t)lp.gu_rows * (d / G) * 2);
+            uint16_t* go = (uint16_t*)p.arena.take((size_t)d * (lp.o_K / G) * 2);
+            uint16_t* gd = (uint16_t*)p.arena.take((size_t)d * (lp.dn_K / G) * 2);
+            int32_t* dgo = (int32_t*)p.arena.take(cgo.size() * 4);
+            int32_t* dgd = (int32_t*)p.arena.take(cgd.size() * 4);
+            if (cgo.size()) TASP_CUDA(cudaMemcpyAsync(dgo, cgo.data(), cgo.size() * 4, cudaMemcpyHostToDevice, s));
+            if (cgd.size()) TASP_CUDA(cudaMemcpyAsync(dgd, cgd.data(), cgd.size() * 4, cudaMemcpyHostToDevice, s));
+            if ((rc = gather_u16_rows(gq, ls.qkv_g, dq, lp.qkv_rows, d / G, s))) break;
+            if ((rc = gather_u16_rows(gg, ls.gu_g, dg, lp.gu_rows, d / G, s))) break;
+            if ((rc = gather_u16_cols(go, ls.o_g, sh.Hq * dh / G, dgo, d, lp.o_K / G, s))) break;
+            if ((rc = gather_u16_cols(gd, ls.down_g, sh.df / G, dgd, d, lp.dn_K / G, s))) break;
+            // the host vectors above die at the end of this block: wait for their copies
+            cudaError_t ge = cudaStreamSynchronize(s);
+            if (ge != cudaSuccess) { rc = cuda_fail(ge, "group scale packing"); break; }
+            lp.qkv_g = gq; lp.gu_g = gg; lp.o_g = go; lp.dn_g = gd;
+        }
         if (rowidx) {
             lp.qkv_w = ls.qkv; lp.qkv_map = dq;
             lp.gu_w = ls.gu; lp.gu_map = dg;
@@ -299,12 +385,15 @@ static void plan_ledger(Plan& p) {
     const Shape& sh = p.store->sh;
     int64_t fl = 0, launched = 0, bytes = 0;
     for (const LayerPlan& lp : p.layers) {
-        fl += layer_flops(sh, (int64_t)lp.m_kv * sh.g(), lp.m_kv, lp.c);
+        fl += layer_flops(sh, lp.m_q, lp.m_kv, lp.c);
         launched += 2 * (int64_t)lp.qkv_rows * sh.d + 2 * (int64_t)sh.d * lp.o_K + 2 * (int64_t)lp.gu_rows * sh.d +
                     2 * (int64_t)sh.d * lp.dn_K;
         bytes += (int64_t)lp.qkv_rows * sh.d + (int64_t)sh.d * lp.o_K + (int64_t)lp.gu_rows * sh.d +
                  (int64_t)sh.d * lp.dn_K;
         bytes += 4 * ((int64_t)lp.qkv_rows + (lp.m_kv ? sh.d : 0) + lp.gu_rows + (lp.c ? sh.d : 0));
+        if (sh.qg)  // BF16 group scales, 2 bytes per qg weights
+            bytes += 2 * (((int64_t)lp.qkv_rows + lp.gu_rows) * (sh.d / sh.qg) +
+                          (int64_t)sh.d * ((lp.o_K + lp.dn_K) / sh.qg));
         bytes += 2 * 4 * (int64_t)sh.d;  // norm gains
     }
     bytes += (int64_t)sh.vocab * sh.d * 2 + 4 * (int64_t)sh.d;
@@ -627,6 +716,35 @@ int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* 
     return TASP_OK;
 }
 
+int tasp_plan_layout(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t layer, int32_t* qkv_src,
+                     int32_t* o_src, int16_t* role, int16_t* slot, int16_t* blk_of, int32_t* counts) {
+    Shape sh;
+    int rc = validate_shape(model, sh, false);
+    if (rc) return rc;
+    if (!mask || !counts) return fail(TASP_EINVAL, "mask_desc or counts is NULL");
+    MaskSel sel;
+    if ((rc = select_mask(sh, *mask, sel))) return rc;
+    if (layer < 0 || layer >= sh.L) return fail(TASP_EINVAL, "layer out of range");
+    LayerPlan lp;
+    lp.keep_groups = sel.groups[layer];
+    lp.keep_qheads = sel.qheads[layer];
+    lp.m_kv = (int)lp.keep_groups.size();
+    std::vector<int32_t> hq, ho;
+    std::vector<int16_t> hrole, hslot, hblk;
+    layer_tables(sh, lp, hq, ho, hrole, hslot, hblk);
+    counts[0] = (int32_t)hq.size();
+    counts[1] = (int32_t)ho.size();
+    counts[2] = (int32_t)hrole.size();
+    counts[3] = (int32_t)hslot.size();
+    counts[4] = (int32_t)hblk.size();
+    if (qkv_src) std::copy(hq.begin(), hq.end(), qkv_src);
+    if (o_src) std::copy(ho.begin(), ho.end(), o_src);
+    if (role) std::copy(hrole.begin(), hrole.end(), role);
+    if (slot) std::copy(hslot.begin(), hslot.end(), slot);
+    if (blk_of) std::copy(hblk.begin(), hblk.end(), blk_of);
+    return TASP_OK;
+}
+
 int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_groups,
                      int32_t* n_groups, int32_t* keep_units, int32_t* n_units, int64_t* flops) {
     return tasp_mask_select_qheads(model, mask, nullptr, nullptr, keep_groups, n_groups, keep_units, n_units, flops);
@@ -646,9 +764,6 @@ int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, 
     for (int l = 0; l < sh.L; ++l) {
         if (sel.groups[l].empty() && sel.units[l].empty())
             return fail(TASP_EINVAL, "mask leaves a layer empty (layer " + std::to_string(l) + ")");
-        if (sel.qheads[l].size() != sel.groups[l].size() * (size_t)sh.g())
-            return fail(TASP_EUNSUP, "query-head mask keeps part of a GQA group (layer " + std::to_string(l) +
-                                         "); the device kernels take whole groups");
     }
     Store* st = nullptr;
     if ((rc = store_acquire(sh, &st))) return rc;
@@ -725,6 +840,7 @@ int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_b
     if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
     if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
+    if (sh.qg && n > 1) return fail(TASP_EUNSUP, "groupwise stores decode one session per call");
     Session* const* ss = (Session* const*)sessions;
     cudaStream_t st = (cudaStream_t)stream;
     // groups of up to MAX_BATCH sessions share each weight pass
@@ -763,6 +879,7 @@ int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* 
     if (!h_x_bf16) return fail(TASP_EINVAL, "h_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
     if (h_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
+    if (sh.qg && n > 1) return fail(TASP_EUNSUP, "groupwise stores decode one session per call");
     cudaStream_t st = (cudaStream_t)stream;
     Session* const* ss = (Session* const*)sessions;
     for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {
@@ -818,6 +935,7 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
     const Shape& sh = p->store->sh;
     if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
     if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
+    if (sh.qg) return fail(TASP_EUNSUP, "prefill of a groupwise store is not built");
     Session* se = nullptr;
     int rc = session_alloc(p, T + max_new_tokens, &se);
     if (rc) return rc;
@@ -848,6 +966,7 @@ int tasp_session_prefill(tasp_session* s, const void* d_embeds_bf16, int32_t T, 
     if (T > se->max_tokens) return fail(TASP_ECAP, "prompt longer than the session capacity");
     if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
     if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
+    if (sh.qg) return fail(TASP_EUNSUP, "prefill of a groupwise store is not built");
     cudaStream_t st = (cudaStream_t)stream;
     int rc = prefill_run(*se, (const uint16_t*)d_embeds_bf16, T, st);
     if (!rc) rc = enqueue_set_pos(*se, T, st);
@@ -926,6 +1045,13 @@ int tasp_plan_layer_dims(const tasp_plan* plan, int32_t layer, int32_t* out2) {
     return TASP_OK;
 }
 
+int tasp_plan_layer_qheads(const tasp_plan* plan, int32_t layer, int32_t* m_q) {
+    Plan* p = as_plan((void*)plan);
+    if (!p || !m_q || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan or layer");
+    *m_q = p->layers[layer].m_q;
+    return TASP_OK;
+}
+
 int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h_dst, size_t bytes) {
     Plan* p = as_plan((void*)plan);
     if (!p || !h_dst || layer < 0 || layer >= (int)p->layers.size()) return fail(TASP_EINVAL, "bad plan, layer or dst");
@@ -964,6 +1090,26 @@ int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h
         case TASP_EXPORT_KEEP_GROUPS: {
             if (int rc = need(lp.keep_groups.size() * 4)) return rc;
             std::memcpy(h_dst, lp.keep_groups.data(), bytes);
+            return TASP_OK;
+        }
+        case TASP_EXPORT_QKV_G:
+        case TASP_EXPORT_O_G:
+        case TASP_EXPORT_GU_G:
+        case TASP_EXPORT_DOWN_G: {
+            if (!sh.qg) return fail(TASP_EINVAL, "the store has no group scales");
+            const uint16_t* src = item == TASP_EXPORT_QKV_G ? lp.qkv_g : item == TASP_EXPORT_O_G ? lp.o_g
+                                : item == TASP_EXPORT_GU_G ? lp.gu_g : lp.dn_g;
+            const size_t n = item == TASP_EXPORT_QKV_G ? (size_t)lp.qkv_rows * (d / sh.qg)
+                           : item == TASP_EXPORT_O_G ? d * (size_t)(lp.o_K / sh.qg)
+                           : item == TASP_EXPORT_GU_G ? (size_t)lp.gu_rows * (d / sh.qg)
+                           : d * (size_t)(lp.dn_K / sh.qg);
+            if (int rc = need(n * 2)) return rc;
+            if (n) TASP_CUDA(cudaMemcpy(h_dst, src, n * 2, cudaMemcpyDeviceToHost));
+            return TASP_OK;
+        }
+        case TASP_EXPORT_KEEP_QHEADS: {
+            if (int rc = need(lp.keep_qheads.size() * 4)) return rc;
+            std::memcpy(h_dst, lp.keep_qheads.data(), bytes);
             return TASP_OK;
         }
         case TASP_EXPORT_KEEP_CHANS: {

@@ -23,6 +23,8 @@ struct GenQuantArgs {
     int g, dh;                 // qkv row decoding
     int8_t* q;                 // [rows][cols]
     float* s;                  // [rows]
+    int qg;                    // > 0: group scales of qg columns (s is then set to 1)
+    uint16_t* gs;              // [rows][cols / qg] BF16, when qg > 0
 };
 
 __device__ __forceinline__ void row_source(const GenQuantArgs& a, int r, uint64_t& key, uint64_t& dense_row) {
@@ -69,6 +71,30 @@ __global__ void __launch_bounds__(GQ_THREADS) gen_quant_kernel(GenQuantArgs a) {
     float amax = 0.f;
 #pragma unroll
     for (int w = 0; w < GQ_THREADS / 32; ++w) amax = fmaxf(amax, red[w]);
+    if (a.qg) {
+        // groupwise (Table 1): per run of qg columns s_g = bf16(fl32(max|w| / 127)), then
+        // q = clamp(rint(fl32(w / s_g)), -127, 127); the row scale is 1
+        if (threadIdx.x == 0) a.s[r] = 1.0f;
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, ng = a.cols / a.qg;
+        int8_t* qrow = a.q + (size_t)r * a.cols;
+        for (int gi = warp; gi < ng; gi += GQ_THREADS / 32) {
+            float gm = 0.f;
+            for (int j = gi * a.qg + lane; j < (gi + 1) * a.qg; j += 32) gm = fmaxf(gm, fabsf(wrow[j]));
+            for (int o = 16; o; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
+            const __nv_bfloat16 sb = __float2bfloat16_rn(__fdiv_rn(gm, 127.0f));
+            const float sg = __bfloat162float(sb);
+            if (lane == 0) a.gs[(size_t)r * ng + gi] = *reinterpret_cast<const uint16_t*>(&sb);
+            for (int j = gi * a.qg + lane; j < (gi + 1) * a.qg; j += 32) {
+                int v = 0;
+                if (sg != 0.f) {
+                    v = __float2int_rn(__fdiv_rn(wrow[j], sg));
+                    v = v > 127 ? 127 : (v < -127 ? -127 : v);
+                }
+                qrow[j] = (int8_t)v;
+            }
+        }
+        return;
+    }
     float s = (amax == 0.f) ? 0.f : __fdiv_rn(amax, 127.0f);
     if (threadIdx.x == 0) a.s[r] = s;
     int8_t* qrow = a.q + (size_t)r * a.cols;
@@ -132,6 +158,18 @@ __global__ void gather_cols_kernel(int8_t* dst, int ld_dst, const int8_t* src, i
     for (int j = threadIdx.x; j < ld_dst; j += blockDim.x) d[j] = (j < Kc) ? s[cmap[j]] : (int8_t)0;
 }
 
+__global__ void gather_u16_rows_kernel(uint16_t* dst, const uint16_t* src, const int32_t* map, int cols) {
+    const int r = blockIdx.x;
+    const uint16_t* s = src + (size_t)map[r] * cols;
+    uint16_t* d = dst + (size_t)r * cols;
+    for (int j = threadIdx.x; j < cols; j += blockDim.x) d[j] = s[j];
+}
+
+__global__ void gather_u16_cols_kernel(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int ncols) {
+    const int r = blockIdx.x;
+    for (int j = threadIdx.x; j < ncols; j += blockDim.x) dst[(size_t)r * ncols + j] = src[(size_t)r * ld_src + cmap[j]];
+}
+
 __global__ void gather_f32_kernel(float* dst, const float* src, const int32_t* map, int n) {
     int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) dst[i] = src[map[i]];
@@ -167,6 +205,8 @@ int store_generate(Store& st, cudaStream_t s) {
         a.dh = sh.dh;
         a.q = ls.qkv;
         a.s = ls.qkv_s;
+        a.qg = sh.qg;
+        a.gs = ls.qkv_g;
         int rc = launch_gen_quant(a, s);
         if (rc) return rc;
         a = GenQuantArgs{};
@@ -176,6 +216,8 @@ int store_generate(Store& st, cudaStream_t s) {
         a.cols = sh.Hq * sh.dh;
         a.q = ls.o;
         a.s = ls.o_s;
+        a.qg = sh.qg;
+        a.gs = ls.o_g;
         if ((rc = launch_gen_quant(a, s))) return rc;
         a = GenQuantArgs{};
         a.mode = RM_GU;
@@ -185,6 +227,8 @@ int store_generate(Store& st, cudaStream_t s) {
         a.cols = sh.d;
         a.q = ls.gu;
         a.s = ls.gu_s;
+        a.qg = sh.qg;
+        a.gs = ls.gu_g;
         if ((rc = launch_gen_quant(a, s))) return rc;
         a = GenQuantArgs{};
         a.mode = RM_PLAIN;
@@ -193,6 +237,8 @@ int store_generate(Store& st, cudaStream_t s) {
         a.cols = sh.df;
         a.q = ls.down;
         a.s = ls.down_s;
+        a.qg = sh.qg;
+        a.gs = ls.down_g;
         if ((rc = launch_gen_quant(a, s))) return rc;
         int nb = (sh.d + 255) / 256;
         gamma_kernel<<<nb, 256, 0, s>>>(sm_key(sh.seed, ST_GAMMA_ATTN, l, 0), sh.d, ls.g_attn);
@@ -255,6 +301,21 @@ int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const in
                 cudaStream_t s) {
     if (rows == 0) return TASP_OK;
     gather_cols_kernel<<<rows, 256, 0, s>>>(dst, ld_dst, src, ld_src, cmap, Kc);
+    TASP_CUDA(cudaGetLastError());
+    return TASP_OK;
+}
+
+int gather_u16_rows(uint16_t* dst, const uint16_t* src, const int32_t* map, int rows, int cols, cudaStream_t s) {
+    if (rows == 0 || cols == 0) return TASP_OK;
+    gather_u16_rows_kernel<<<rows, 128, 0, s>>>(dst, src, map, cols);
+    TASP_CUDA(cudaGetLastError());
+    return TASP_OK;
+}
+
+int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows, int ncols,
+                    cudaStream_t s) {
+    if (rows == 0 || ncols == 0) return TASP_OK;
+    gather_u16_cols_kernel<<<rows, 128, 0, s>>>(dst, src, ld_src, cmap, ncols);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }

@@ -41,6 +41,7 @@ int cuda_fail(cudaError_t e, const char* what);
 // ---------------------------------------------------------------- shape
 struct Shape {
     int L = 0, d = 0, Hq = 0, Hkv = 0, dh = 0, df = 0, vocab = 0, cu = 1;
+    int qg = 0;  // scale group (input columns per BF16 scale), 0 = one FP32 scale per row
     float eps = 1e-5f, theta = 500000.f;
     uint64_t seed = 0;
     int g() const { return Hq / Hkv; }
@@ -77,7 +78,9 @@ struct Arena {
 // channel, i.e. the packed layout of the all-keep mask.
 struct LayerStore {
     int8_t *qkv, *o, *gu, *down;
-    float *qkv_s, *o_s, *gu_s, *down_s, *g_attn, *g_mlp;
+    float *qkv_s, *o_s, *gu_s, *down_s, *g_attn, *g_mlp;  // row scales (all 1 in a grouped store)
+    // grouped store only: BF16 scales [rows][K / qg] of each projection
+    uint16_t *qkv_g = nullptr, *o_g = nullptr, *gu_g = nullptr, *down_g = nullptr;
 };
 
 struct Store {
@@ -93,7 +96,16 @@ struct Store {
 // ---------------------------------------------------------------- plans
 struct LayerPlan {
     int m_kv = 0, c = 0;
-    std::vector<int> keep_groups, keep_chans;
+    int m_q = 0;  // kept query heads (m_kv g unless the mask keeps part of a group)
+    std::vector<int> keep_groups, keep_chans, keep_qheads;
+    // Partial groups only (NULL when every kept group keeps its g heads):
+    // blk_role[b] = role of the qkv panel's d_h-row block b as jl (g + 2) + hh, with jl the
+    // kept-group slot and hh the head within the group (< g), g for K or g + 1 for V;
+    // oslot[jl g + hh] = the compact position of that head in the O panel's columns, or -1
+    // for a dropped head (its query slot stays zero and its attention output is not written).
+    const int16_t* blk_role = nullptr;
+    const int16_t* oslot = nullptr;
+    const int16_t* blk_of = nullptr;  // inverse of blk_role: [m_kv (g + 2)] panel block or -1
     // qkv panel: rows (m_q + 2 m_kv) dh of K = d; row i at qkv_w + (qkv_map ? qkv_map[i] : i) * d
     const int8_t* qkv_w = nullptr;
     const int32_t* qkv_map = nullptr;
@@ -113,6 +125,9 @@ struct LayerPlan {
     const float* dn_s = nullptr;
     int dn_K = 0, dn_ld = 0;
     const float *g_attn = nullptr, *g_mlp = nullptr;
+    // grouped store only: BF16 group scales in panel order, [rows][K / qg] (row stride gq_ld
+    // for qkv / gu, o_K / qg and dn_K / qg for the column-compacted O / down panels)
+    const uint16_t *qkv_g = nullptr, *gu_g = nullptr, *o_g = nullptr, *dn_g = nullptr;
 };
 
 // FP16 copies of a layer's panels (row strides padded to 8 elements) for the prefill GEMMs.
@@ -188,20 +203,26 @@ int gather_rows(int8_t* dst, const int8_t* src, const int32_t* map, int rows, in
 int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const int32_t* cmap, int rows, int Kc,
                 cudaStream_t s);
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
+// rows of a [*][cols] uint16 matrix (dst row r = src row map[r])
+int gather_u16_rows(uint16_t* dst, const uint16_t* src, const int32_t* map, int rows, int cols, cudaStream_t s);
+// columns of a [rows][ld_src] uint16 matrix (dst column j = src column cmap[j], j < ncols)
+int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows, int ncols,
+                    cudaStream_t s);
 
 // attention.cu
 constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pass
 constexpr int UNION_MAX = 16;  // sessions (of any plans) in one union-of-masks step
 struct AttnParams {
     // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
-    const float* q;      // FP32 rotated queries [m_q][dh] (kept heads, group-major)
-    float* o;            // FP32 [m_q][dh]
+    const float* q;      // FP32 rotated queries [m_kv g][dh] (kept groups, all g slots)
+    float* o;            // FP32 [m_q][dh], kept heads in O-panel column order
     int64_t q_stride;
     const uint16_t* K[UNION_MAX];  // BF16 [m_kv][max_tokens][dh] of this layer
     const uint16_t* V[UNION_MAX];
     const int* pos[UNION_MAX];     // device position: the step attends to positions 0..pos
     int max_tokens[UNION_MAX];
     int m_kv[UNION_MAX];           // kept groups of the session's plan (grid y covers the largest)
+    const int16_t* oslot[UNION_MAX];  // output slot per (group slot, head), NULL = jl g + hh
     float qscale;        // log2(e) / sqrt(dh)
     float* part;         // + b * part_stride
     float* ml;           // + b * ml_stride

@@ -924,6 +924,11 @@ int union_check(Session* const* ss, int n, bool step) {
     const Shape& sh = st->sh;
     if (sh.d % SK_BK || (sh.Hq * sh.dh) % SK_BK || sh.df % SK_BK)
         return fail(TASP_EUNSUP, "union decode needs d, Hq*dh and d_ff that are multiples of 128");
+    if (sh.qg) return fail(TASP_EUNSUP, "union decode of a groupwise store is not built");
+    for (int b = 0; b < n; ++b)
+        for (const LayerPlan& lp : ss[b]->plan->layers)
+            if (lp.m_q != lp.m_kv * sh.g())
+                return fail(TASP_EUNSUP, "union decode takes plans of whole GQA groups only");
     return TASP_OK;
 }
 

@@ -21,7 +21,8 @@ OK, EINVAL, EMASK, ECAP, ENOMEM, EBUSY, ECUDA, EUNSUP = 0, -1, -2, -3, -4, -5, -
 MASK_ALL_KEEP, MASK_GREEDY, MASK_EXPLICIT, MASK_GREEDY_QHEADS, MASK_EXPLICIT_QHEADS = 0, 1, 2, 3, 4
 PANELS_COMPACT, PANELS_ROW_INDEXED = 0, 1
 (EXPORT_KEEP_GROUPS, EXPORT_KEEP_CHANS, EXPORT_QKV_W, EXPORT_QKV_S, EXPORT_O_W, EXPORT_O_S, EXPORT_GU_W,
- EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S) = range(10)
+ EXPORT_GU_S, EXPORT_DOWN_W, EXPORT_DOWN_S, EXPORT_KEEP_QHEADS, EXPORT_QKV_G, EXPORT_O_G, EXPORT_GU_G,
+ EXPORT_DOWN_G) = range(15)
 KERNEL_KINDS = 7
 KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "other")
 
@@ -29,6 +30,7 @@ KERNEL_NAMES = ("qkv", "attention", "o_proj", "gate_up", "down", "lm_head", "oth
 EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_release", "tasp_session_create",
             "tasp_session_fill_synthetic", "tasp_session_position", "tasp_session_status", "tasp_decode_step_host", "tasp_mask_select",
             "tasp_mask_select_qheads", "tasp_set_memory_limit", "tasp_memory_in_use", "tasp_dispatch",
+            "tasp_plan_layer_qheads", "tasp_plan_layout",
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
@@ -39,7 +41,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
 class ModelDesc(ctypes.Structure):
     _fields_ = [("L", c_int32), ("d", c_int32), ("Hq", c_int32), ("Hkv", c_int32), ("dh", c_int32),
                 ("df", c_int32), ("vocab", c_int32), ("chan_unit", c_int32), ("rms_eps", c_float),
-                ("rope_theta", c_float), ("seed", c_uint64)]
+                ("rope_theta", c_float), ("seed", c_uint64), ("quant_group", c_int32)]
 
 
 class MaskDesc(ctypes.Structure):
@@ -92,6 +94,8 @@ def load(path: str = LIB_PATH):
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_set_memory_limit": (c_int32, [c_int64]),
         "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
+        "tasp_plan_layer_qheads": (c_int32, [P, c_int32, POINTER(c_int32)]),
+        "tasp_plan_layout": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), c_int32, P, P, P, P, P, P]),
         "tasp_memory_in_use": (c_int32, [POINTER(c_int64)]),
         "tasp_plan_info_get": (c_int32, [P, POINTER(PlanInfo)]),
         "tasp_plan_layer_dims": (c_int32, [P, c_int32, P]),
@@ -122,11 +126,8 @@ def _check(rc):
 
 def model_desc(shape) -> ModelDesc:
     """ModelDesc from any object with L, d, Hq, Hkv, dh, df, vocab, chan_unit, eps, rope_theta, seed."""
-    if getattr(shape, "quant_group", 0):
-        raise TaspError(EUNSUP, "the device store holds one INT8 scale per output row; groupwise scales are "
-                                "not built there")
     return ModelDesc(shape.L, shape.d, shape.Hq, shape.Hkv, shape.dh, shape.df, shape.vocab, shape.chan_unit,
-                     shape.eps, shape.rope_theta, shape.seed)
+                     shape.eps, shape.rope_theta, shape.seed, getattr(shape, "quant_group", 0))
 
 
 class _MaskArgs:
@@ -257,6 +258,21 @@ def memory_in_use() -> int:
     return v.value
 
 
+def plan_layout(shape, mask: _MaskArgs, layer: int) -> dict:
+    """Host-only: the qkv row sources, O column sources and partial-group tables of one layer."""
+    lib = load()
+    cnt = np.zeros(5, np.int32)
+    md = model_desc(shape)
+    _check(lib.tasp_plan_layout(ctypes.byref(md), ctypes.byref(mask.desc), layer, None, None, None, None, None,
+                                cnt.ctypes.data))
+    out = {k: np.zeros(int(n), dt) for k, n, dt in zip(("qkv_src", "o_src", "role", "slot", "blk_of"), cnt,
+                                                      (np.int32, np.int32, np.int16, np.int16, np.int16))}
+    _check(lib.tasp_plan_layout(ctypes.byref(md), ctypes.byref(mask.desc), layer, out["qkv_src"].ctypes.data,
+                                out["o_src"].ctypes.data, out["role"].ctypes.data, out["slot"].ctypes.data,
+                                out["blk_of"].ctypes.data, cnt.ctypes.data))
+    return out
+
+
 def _stream_ptr(stream):
     if stream is None:
         import torch
@@ -282,12 +298,22 @@ class Plan:
         _check(load().tasp_plan_layer_dims(self.handle, layer, out.ctypes.data))
         return int(out[0]), int(out[1])
 
+    def layer_qheads(self, layer) -> int:
+        v = c_int32()
+        _check(load().tasp_plan_layer_qheads(self.handle, layer, ctypes.byref(v)))
+        return v.value
+
     def export(self, layer, item):
         sh = self.shape
         m_kv, c = self.layer_dims(layer)
-        m_q = m_kv * (sh.Hq // sh.Hkv)
+        m_q = self.layer_qheads(layer)
         spec = {
             EXPORT_KEEP_GROUPS: (np.int32, (m_kv,)),
+            EXPORT_KEEP_QHEADS: (np.int32, (m_q,)),
+            EXPORT_QKV_G: (np.uint16, ((m_q + 2 * m_kv) * sh.dh, sh.d // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_O_G: (np.uint16, (sh.d, m_q * sh.dh // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_GU_G: (np.uint16, (2 * c, sh.d // max(1, getattr(sh, "quant_group", 0)))),
+            EXPORT_DOWN_G: (np.uint16, (sh.d, c // max(1, getattr(sh, "quant_group", 0)))),
             EXPORT_KEEP_CHANS: (np.int32, (c,)),
             EXPORT_QKV_W: (np.int8, ((m_q + 2 * m_kv) * sh.dh, sh.d)),
             EXPORT_QKV_S: (np.float32, ((m_q + 2 * m_kv) * sh.dh,)),

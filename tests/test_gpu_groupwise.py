@@ -1,0 +1,131 @@
+"""GPU parity of groupwise INT8 stores (Table 1: group size 128, BF16 scales) against the
+oracle, through the C ABI: INT8 codes and BF16 group scales bit-exact on the store's panels,
+one-session decode elementwise per layer and end to end, and the paths not built for such a
+store (batches, prefill, union) refused with EUNSUP."""
+import dataclasses
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import forward, maskc, pack, weights
+from gpu_common import TOL_E2E, bf16_tensor, rel_l2, within
+
+pytestmark = pytest.mark.gpu
+
+SHAPE = dataclasses.replace(synth.LLAMA3_8B, L=2, quant_group=128)
+
+
+@pytest.fixture(scope="module")
+def tasp():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_29499_gb300 import build
+    build.build()
+    from paper_2609_29499_gb300 import tasp as t
+    t.load()
+    torch.cuda.set_device(0)
+    return t
+
+
+def _bits(a):
+    return synth.bf16_bits(np.asarray(a, np.float32))
+
+
+def check_grouped_panels(tasp, plan, sh, mask, layer):
+    lq = weights.gen_layer(sh, layer)
+    ref = pack.pack_layer(sh, lq, mask.keep_groups[layer], mask.keep_chans[layer], mask.qheads(sh, layer))
+    for item, name in ((tasp.EXPORT_QKV_W, "qkv_w"), (tasp.EXPORT_O_W, "o_w"), (tasp.EXPORT_GU_W, "gu_w"),
+                       (tasp.EXPORT_DOWN_W, "down_w")):
+        got = plan.export(layer, item)
+        assert got.shape == ref[name].shape and np.array_equal(got, ref[name]), name
+    for item, name in ((tasp.EXPORT_QKV_G, "qkv_s"), (tasp.EXPORT_O_G, "o_s"), (tasp.EXPORT_GU_G, "gu_s"),
+                       (tasp.EXPORT_DOWN_G, "down_s")):
+        got = plan.export(layer, item)
+        assert got.shape == ref[name].shape and np.array_equal(got, _bits(ref[name])), name
+
+
+def _plan(tasp, sh, seed=1000):
+    sc = synth.mask_scores_u32(seed, sh.L, sh.n_units)
+    tg = synth.layer_target_u24(seed, sh.L)
+    mask = maskc.compile_mask(sh, sc, tg)
+    return tasp.Plan(sh, tasp.greedy_mask(sc, tg)), mask
+
+
+@pytest.mark.parametrize("dense", [False, True])
+def test_grouped_panels_bit_exact(tasp, dense):
+    sh = SHAPE
+    if dense:
+        plan, mask = tasp.Plan(sh, tasp.all_keep_mask()), maskc.all_keep(sh)
+    else:
+        plan, mask = _plan(tasp, sh)
+    for layer in range(sh.L):
+        check_grouped_panels(tasp, plan, sh, mask, layer)
+    info = plan.info()
+    assert info["launched_flops"] == info["flops_retained"]
+    plan.release()
+
+
+def test_grouped_isolated_layer_and_decode(tasp):
+    import torch
+    sh = SHAPE
+    plan, mask = _plan(tasp, sh)
+    # isolated layer 1 fed the oracle's input: elementwise
+    sess = tasp.Session(plan, 701)
+    sess.fill_synthetic(700, 7)
+    x = synth.probe_f32(5, 1, sh.d, 4.0)
+    out = torch.empty(sh.d, dtype=torch.float32, device="cuda")
+    sess.layer_step(1, torch.from_numpy(x).cuda(), out)
+    torch.cuda.synchronize()
+    lq = weights.gen_layer(sh, 1)
+    W = weights.dense_zeroed(sh, lq, mask.keep_groups[1], mask.keep_chans[1])
+    Kc, Vc = forward.prior_cache(sh, 1, 7, 700)
+    ref, _, _ = forward.layer_step(sh, W, x.astype(np.float32), Kc, Vc, 700)
+    assert within(out.cpu().numpy(), ref).all()
+    sess.release()
+    # three steps through both layers with logits on sampled rows
+    sess = tasp.Session(plan, 703)
+    sess.fill_synthetic(700, 7)
+    xb = synth.step_inputs_bf16(11, 3, 1, sh.d)
+    x = bf16_tensor(xb)
+    hid = torch.empty((3, 1, sh.d), dtype=torch.float32, device="cuda")
+    logits = torch.empty((3, 1, sh.vocab), dtype=torch.float32, device="cuda")
+    for t in range(3):
+        tasp.decode_step([sess], x[t], hid[t], logits[t])
+    torch.cuda.synchronize()
+    assert sess.device_error() == 0
+    ref = forward.decode(sh, mask, synth.bf16_to_f32(xb[:, 0]), 700, 7)
+    assert rel_l2(hid.cpu().numpy()[:, 0], ref) <= TOL_E2E
+    rows = np.arange(0, sh.vocab, 997)
+    lref = forward.final_logits(sh, ref, rows=rows)
+    assert rel_l2(logits.cpu().numpy()[:, 0][:, rows], lref) <= TOL_E2E
+    # the groupwise plan reads 2 bytes of scale per 128 weights more than a per-row plan
+    row = dataclasses.replace(sh, quant_group=0)
+    prow = tasp.Plan(row, tasp.greedy_mask(synth.mask_scores_u32(1000, sh.L, sh.n_units),
+                                           synth.layer_target_u24(1000, sh.L)))
+    extra = plan.info()["weight_bytes_per_token"] - prow.info()["weight_bytes_per_token"]
+    int8 = sum(pack.pack_layer(sh, weights.gen_layer(sh, layer), mask.keep_groups[layer],
+                               mask.keep_chans[layer])["qkv_w"].size for layer in range(sh.L))
+    assert extra > 0 and extra >= 2 * int8 // 128
+    sess.release()
+    prow.release()
+    plan.release()
+
+
+def test_paths_not_built_for_grouped_stores(tasp):
+    import torch
+    sh = SHAPE
+    plan, _ = _plan(tasp, sh)
+    a, b = tasp.Session(plan, 8), tasp.Session(plan, 8)
+    for s in (a, b):
+        s.fill_synthetic(4, 1)
+    x = torch.zeros((2, sh.d), dtype=torch.bfloat16, device="cuda")
+    for call in (lambda: tasp.decode_step([a, b], x), lambda: tasp.decode_step_union([a], x[:1]),
+                 lambda: a.prefill_into(torch.zeros((4, sh.d), dtype=torch.bfloat16, device="cuda"))):
+        with pytest.raises(tasp.TaspError) as e:
+            call()
+        assert e.value.code == tasp.EUNSUP
+    a.release()
+    b.release()
+    plan.release()

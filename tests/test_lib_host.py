@@ -1,6 +1,7 @@
 """CPU checks of the C-ABI library: it loads, exports every declared symbol, and its
 host mask compiler matches the oracle's bit for bit (no GPU work)."""
 import ctypes
+import dataclasses
 import os
 import re
 
@@ -167,19 +168,6 @@ def test_explicit_qhead_masks_and_group_kinds(lib):
     with pytest.raises(lib.TaspError) as e:
         lib.mask_select_qheads(sh, lib.explicit_qhead_mask([[4], [0], [0]], u))  # head out of range
     assert e.value.code == lib.EINVAL
-
-
-def test_partial_group_plans_are_refused_before_device_work(lib):
-    # the device kernels take whole GQA groups: a query-head mask that keeps part of a group
-    # is refused by the host compiler before any store or panel is made
-    sh = synth.LAYER1
-    so = lib.load()
-    md = lib.model_desc(sh)
-    m = lib.explicit_qhead_mask([[0, 1, 4, 5, 6, 7]], [[0, 9]])
-    out = ctypes.c_void_p()
-    assert so.tasp_compile_mask(ctypes.byref(md), ctypes.byref(m.desc), ctypes.byref(out)) == lib.EUNSUP
-    assert "whole groups" in so.tasp_last_error().decode()
-    assert not out.value
 
 
 def test_binding_rejects_host_or_mistyped_buffers_before_any_call(lib):
@@ -353,3 +341,122 @@ def test_header_is_a_plain_c_interface():
     r = subprocess.run([cc, "-x", "c", "-std=c99", "-Wall", "-Werror", "-fsyntax-only",
                         "-I", os.path.join(ROOT, "include"), "-"], input=src, capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+def _store_row(shape, proj, row):
+    # the store's qkv rows are group-major: per KV group its g head blocks, then K, then V
+    g, dh = shape.g, shape.dh
+    if proj == "q":
+        h, i = divmod(row, dh)
+        j, hh = divmod(h, g)
+    else:
+        j, i = divmod(row, dh)
+        hh = g if proj == "k" else g + 1
+    return (j * (g + 2) + hh) * dh + i
+
+
+@pytest.mark.parametrize("shape,heads", [
+    (synth.LAYER1, [[1, 2, 3, 4, 6]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=2), [[0, 1, 2, 5, 9, 10, 11, 31], [3, 4, 7, 30]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=1), [list(range(32))]),
+])
+def test_partial_group_tables_match_the_oracle_packing(lib, shape, heads):
+    from oracle import pack
+    units = [[0] for _ in range(shape.L)]
+    m = maskc.explicit_qheads(shape, heads, units)
+    g, dh = shape.g, shape.dh
+    for layer in range(shape.L):
+        t = lib.plan_layout(shape, lib.explicit_qhead_mask(heads, units), layer)
+        kg, qh = m.keep_groups[layer], m.keep_qheads[layer]
+        want = [_store_row(shape, p, r) for p, r in pack.qkv_rows(shape, kg, qh)]
+        assert t["qkv_src"].tolist() == want
+        assert t["o_src"].tolist() == [h * dh + i for h in qh for i in range(dh)]
+        # role: block b of the panel holds (group slot, head or K / V); blk_of inverts it
+        nblk = len(qh) + 2 * len(kg)
+        assert len(t["role"]) == nblk and len(t["blk_of"]) == len(kg) * (g + 2)
+        for b, code in enumerate(t["role"].tolist()):
+            jl, hh = divmod(code, g + 2)
+            assert t["blk_of"][code] == b
+            assert t["qkv_src"][b * dh] == (kg[jl] * (g + 2) + hh) * dh
+        assert sorted(int(x) for x in t["blk_of"] if x >= 0) == list(range(nblk))
+        # slot: compact O position of each kept head, -1 for dropped ones
+        for jl, j in enumerate(kg):
+            for hh in range(g):
+                h = j * g + hh
+                assert t["slot"][jl * g + hh] == (qh.index(h) if h in qh else -1)
+
+
+def _dense_of_store_row(shape, r):
+    g, dh = shape.g, shape.dh
+    blk, i = divmod(r, dh)
+    j, hh = divmod(blk, g + 2)
+    if hh < g:
+        return ("q", (j * g + hh) * dh + i)
+    return ("k" if hh == g else "v", j * dh + i)
+
+
+@pytest.mark.parametrize("shape,heads", [
+    (synth.LAYER1, [[1, 2, 3, 4, 6]]),
+    (dataclasses.replace(synth.LLAMA3_8B, L=1), [[0, 1, 2, 5, 9, 10, 11, 31]]),
+])
+def test_kernel_index_math_with_partial_group_tables(lib, shape, heads):
+    # the decode QKV epilogue, the attention output store and the prefill rotary kernel,
+    # replayed on the host with the plan's tables: every query slot, K / V row and O column
+    # receives exactly the dense row or column the oracle's mask-as-zero forward uses
+    units = [[0]]
+    m = maskc.explicit_qheads(shape, heads, units)
+    kg, qh = m.keep_groups[0], m.keep_qheads[0]
+    g, dh, half = shape.g, shape.dh, shape.dh // 2
+    t = lib.plan_layout(shape, lib.explicit_qhead_mask(heads, units), 0)
+    src, role, slot, blk_of = t["qkv_src"], t["role"], t["slot"], t["blk_of"]
+    rows = len(src)
+    # decode: work rows in pairs (w, w + 1) hold panel rows (hb dh + i, hb dh + i + d_h / 2)
+    written = {}
+    for wa in range(0, rows, 2):
+        hb = wa // dh
+        i = (wa - hb * dh) >> 1
+        pr0, pr1 = hb * dh + i, hb * dh + i + half
+        jl, hh = divmod(int(role[hb]), g + 2)
+        dest = ("q", jl * g + hh) if hh < g else ("k" if hh == g else "v", jl)
+        for off, pr in ((i, pr0), (i + half, pr1)):
+            key = (dest, off)
+            assert key not in written
+            written[key] = _dense_of_store_row(shape, int(src[pr]))
+    for jl, j in enumerate(kg):
+        for hh in range(g):
+            h = j * g + hh
+            for i in range(dh):
+                if h in qh:
+                    assert written[(("q", jl * g + hh), i)] == ("q", h * dh + i)
+                else:
+                    assert (("q", jl * g + hh), i) not in written  # the slot stays zero
+        for kv in ("k", "v"):
+            for i in range(dh):
+                assert written[((kv, jl), i)] == (kv, j * dh + i)
+    # attention output: head (jl, hh) lands in compact O columns slot * d_h, which the O panel
+    # maps back to the dense columns of head h
+    for jl, j in enumerate(kg):
+        for hh in range(g):
+            s = int(slot[jl * g + hh])
+            if s >= 0:
+                assert t["o_src"][s * dh:(s + 1) * dh].tolist() == list(range((j * g + hh) * dh, (j * g + hh + 1) * dh))
+    # prefill: the rotary kernel reads panel column block blk_of[jl (g + 2) + hh] (rows in panel order)
+    for jl, j in enumerate(kg):
+        for hh in range(g + 2):
+            b = int(blk_of[jl * (g + 2) + hh])
+            if hh < g and j * g + hh not in qh:
+                assert b == -1
+                continue
+            want = ("q", (j * g + hh) * dh) if hh < g else ("k" if hh == g else "v", j * dh)
+            assert _dense_of_store_row(shape, int(src[b * dh])) == want
+
+
+def test_groupwise_shapes_are_validated_on_the_host(lib):
+    import dataclasses
+    sh = synth.LLAMA3_8B
+    sc = synth.mask_scores_u32(1000, sh.L, sh.n_units)
+    tg = synth.layer_target_u24(1000, sh.L)
+    ok = lib.mask_select(dataclasses.replace(sh, quant_group=128), lib.greedy_mask(sc, tg))
+    assert ok[0] == lib.mask_select(sh, lib.greedy_mask(sc, tg))[0]  # the mask does not depend on scales
+    for bad in (48, 100, -16, 256 * 1024):
+        with pytest.raises(lib.TaspError) as e:
+            lib.mask_select(dataclasses.replace(sh, quant_group=bad), lib.greedy_mask(sc, tg))
+        assert e.value.code == lib.EINVAL
