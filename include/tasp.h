@@ -207,6 +207,10 @@ int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, i
  * n_qheads [L] (ascending per layer). For the group kinds these are all g heads
  * of every kept group; for the query-head kinds keep_groups holds the KV heads
  * that the closure keeps. Host only; any output may be NULL. */
+int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
+                            int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
+                            int32_t* n_units, int64_t* flops);
+
 /* Host only (test introspection): the tables a plan of `mask` uses for one layer.
  * qkv_src [(m_q + 2 m_kv) dh]: store row of each qkv panel row (store rows are
  * group-major: per KV group its g head blocks of dh rows, then K, then V);
@@ -216,10 +220,6 @@ int tasp_mask_select(const tasp_model_desc* model, const tasp_mask_desc* mask, i
  * of role or -1). counts [5] receives the five lengths. Any array may be NULL. */
 int tasp_plan_layout(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t layer, int32_t* qkv_src,
                      int32_t* o_src, int16_t* role, int16_t* slot, int16_t* blk_of, int32_t* counts);
-
-int tasp_mask_select_qheads(const tasp_model_desc* model, const tasp_mask_desc* mask, int32_t* keep_qheads,
-                            int32_t* n_qheads, int32_t* keep_groups, int32_t* n_groups, int32_t* keep_units,
-                            int32_t* n_units, int64_t* flops);
 
 /* ---------------------------------------------------------------------------
  * Introspection and measurement (tests and benchmark).
@@ -342,7 +342,6 @@ int tasp_decode_step_union(tasp_session* const* sessions, int32_t n, const void*
  * union workspace of these sessions (created if absent). sync. */
 int tasp_union_status(tasp_session* const* sessions, int32_t n, int32_t* device_error, int32_t* launches);
 
-/* Thread-local description of the last failure on this thread ("" if none). */
 /* Per-turn plan choice (Sec. 3.3; Table 1: tau = 0.85): given the router's task
  * distribution h_probs [n] over the n task masks, *plan = the index of the most
  * probable task (lowest index on ties) when its probability reaches tau, else n,
@@ -359,6 +358,7 @@ int tasp_set_memory_limit(int64_t bytes);
 /* Device bytes the library's arenas hold now. Host only. */
 int tasp_memory_in_use(int64_t* bytes);
 
+/* Thread-local description of the last failure on this thread ("" if none). */
 const char* tasp_last_error(void);
 
 /* Library version string. */

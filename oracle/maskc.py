@@ -7,7 +7,7 @@ a KV head stays whenever any of its query heads stays and query heads never
 move across groups; a SwiGLU channel group keeps or drops its gate row, up
 row and down column together.
 
-Readings used here (the paper leaves them open; all are listed in the design doc):
+Readings used here (the paper leaves them open):
 
 * Unit = a whole GQA group (KV head + its g query heads) or a block of
   ``chan_unit`` channels. Closure is then satisfied by construction and is
