@@ -299,9 +299,11 @@ int tasp_step_launches(tasp_session* const* sessions, int32_t n, int32_t with_lo
  * is already handed out, another library's stream capture in progress, a serving
  * loop that forbids allocator calls). The step's kernels are launched directly (no
  * CUDA graph is built) and the attention scratch comes from one file-scope
- * device array of about 1.06 MB (8 kept KV groups x 32 partial slots x 8 query
- * heads per group x head dim 128 partial floats, plus maxima/sums and 8 merge
- * tickets) that every GPU loading the library holds until the process exits.
+ * device array of about 260 KB (8 kept KV groups x 8 attention clusters per
+ * group x 8 query heads per group x head dim 128 partial floats, plus maxima/sums
+ * and 8 merge tickets) that every GPU loading the library holds until the process
+ * exits. The clusters are used when a session's capacity exceeds one cluster's
+ * reach (about 6,100 positions at head dim 128, 12,200 at 64).
  * Arguments and outputs are those of tasp_decode_step with n = 1. The first call on
  * a device looks up the array's device address (cudaGetSymbolAddress); make that
  * first call before any stream capture. All calls share the array and it keeps the

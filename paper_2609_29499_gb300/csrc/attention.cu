@@ -33,7 +33,7 @@ namespace {
 constexpr int AT_WARPS = 8;
 constexpr int AT_THREADS = AT_WARPS * 32;
 constexpr int TILE = 16;
-constexpr int CLUSTERS_MAX = 8;  // clusters per kept group (global merge when > 1)
+constexpr int CLUSTERS_MAX = ATTN_CLUSTERS_MAX;  // clusters per kept group (global merge when > 1)
 
 template <int DH>
 struct AttCfg {

@@ -22,11 +22,13 @@ namespace tasp {
 
 namespace {
 
-// Capacity of the shared scratch, sized for up to 8 kept KV groups x 32 partial slots x 8
-// query heads per group x head dimension 128 (the Llama-3 8B/70B shapes): ~1.06 MB.
-constexpr size_t kPartFloats = 8 * 32 * 8 * 128;
-constexpr size_t kMlFloats = 8 * 32 * 8 * 2;
-constexpr size_t kTickets = 8;
+// Capacity of the shared scratch: up to 8 kept KV groups per layer, each with at most
+// ATTN_CLUSTERS_MAX attention clusters whose partial outputs (8 query heads per group x
+// head dimension 128, the Llama-3 8B/70B shapes) and (max, sum) pairs are kept: ~260 KB.
+constexpr size_t kGroups = 8;
+constexpr size_t kPartFloats = kGroups * ATTN_CLUSTERS_MAX * 8 * 128;
+constexpr size_t kMlFloats = kGroups * ATTN_CLUSTERS_MAX * 8 * 2;
+constexpr size_t kTickets = kGroups;
 constexpr size_t kScratchFloats = kPartFloats + kMlFloats + kTickets;
 
 static __device__ __align__(256) float g_tasp_static_scratch[kScratchFloats];

@@ -212,6 +212,7 @@ int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_
 // attention.cu
 constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pass
 constexpr int UNION_MAX = 16;  // sessions (of any plans) in one union-of-masks step
+constexpr int ATTN_CLUSTERS_MAX = 8;  // decode attention clusters per kept group (global merge when > 1)
 struct AttnParams {
     // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
     const float* q;      // FP32 rotated queries [m_kv g][dh] (kept groups, all g slots)
