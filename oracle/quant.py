@@ -37,7 +37,9 @@ def quantize_rows(w: np.ndarray):
 
 def dequantize_rows(q: np.ndarray, s: np.ndarray, dtype=np.float32) -> np.ndarray:
     """W~ = s * Q per output row."""
-    return (q.astype(dtype) * np.asarray(s, dtype=dtype)[:, None]).astype(dtype)
+    w = q.astype(dtype)
+    np.multiply(w, np.asarray(s, dtype=dtype)[:, None], out=w)  # in place: one product per element
+    return w
 
 
 # ------------------------------------------------------------------ groupwise variant
