@@ -82,12 +82,6 @@ __device__ __forceinline__ u64 fma2(u64 a, u64 b, u64 c) {
     return d;
 }
 
-// float4 index swizzle: F = float4s per 16-byte weight chunk (4 for INT8, 2 for BF16)
-template <int F>
-__device__ __forceinline__ int swz(int f) {
-    return f ^ ((f >> 3) & (F - 1));
-}
-
 __device__ __forceinline__ uint16_t f32_to_bf16_bits(float v) {
     __nv_bfloat16 b = __float2bfloat16_rn(v);
     return *reinterpret_cast<uint16_t*>(&b);
@@ -109,30 +103,74 @@ constexpr int ERR_WAIT_TIMEOUT = 1;
 
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(CT) : "memory"); }
 
-// ---------------------------------------------------------------- activation prologues
-// x^ = x * (1/sqrt(mean(x^2) + eps)) * gamma (FP32) into swizzled shared memory.
-// Every CTA reduces in the same fixed order, so all CTAs see identical x^.
+// ---------------------------------------------------------------- activation slices
+// Each consumer thread reads its own chunks of the activation vector straight from global
+// memory: chunk c = tid + j * CT holds elements [4F c, 4F c + 4F) (16 for the INT8 modes, 8
+// for the BF16 LM head). Nothing is staged in shared memory, so the weight ring gets all of
+// it. Elements at or beyond `len` read as zero.
 template <int F>
-__device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __restrict__ x_in, float* x_init,
-                             const float* __restrict__ gamma, int d, float eps, int nchunks, float4* xs,
-                             float* stat) {
-    const int tid = threadIdx.x;
-    const int n4 = d / 4;
-    float ss = 0.f;
-    for (int f = tid; f < n4; f += NT) {
-        float4 v;
-        if (x_in) {
-            uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
-            v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
-                            __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
-            if (x_init && blockIdx.x == 0) reinterpret_cast<float4*>(x_init)[f] = v;
-        } else {
-            v = reinterpret_cast<const float4*>(x)[f];
+__device__ __forceinline__ void chunk_f32(const float* __restrict__ a, int c, int len, float4 (&v)[F]) {
+    const int e0 = 4 * F * c;
+    if (e0 + 4 * F <= len) {
+#pragma unroll
+        for (int e = 0; e < F; ++e) v[e] = reinterpret_cast<const float4*>(a + e0)[e];
+    } else {
+#pragma unroll
+        for (int e = 0; e < F; ++e) {
+            const int b = e0 + 4 * e;
+            v[e] = make_float4(b < len ? a[b] : 0.f, b + 1 < len ? a[b + 1] : 0.f, b + 2 < len ? a[b + 2] : 0.f,
+                               b + 3 < len ? a[b + 3] : 0.f);
         }
-        ss = fmaf(v.x, v.x, ss);
-        ss = fmaf(v.y, v.y, ss);
-        ss = fmaf(v.z, v.z, ss);
-        ss = fmaf(v.w, v.w, ss);
+    }
+}
+// BF16 step input (16-byte aligned; len a multiple of 16)
+template <int F>
+__device__ __forceinline__ void chunk_bf16(const uint16_t* __restrict__ a, int c, int len, float4 (&v)[F]) {
+    const int e0 = 4 * F * c;
+#pragma unroll
+    for (int e = 0; e < F; e += 2) {
+        uint4 b = make_uint4(0u, 0u, 0u, 0u);
+        if (e0 + 4 * F <= len) b = reinterpret_cast<const uint4*>(a + e0)[e >> 1];
+        v[e] = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u), __uint_as_float(b.y << 16),
+                           __uint_as_float(b.y & 0xffff0000u));
+        if (e + 1 < F)
+            v[e + 1] = make_float4(__uint_as_float(b.z << 16), __uint_as_float(b.z & 0xffff0000u),
+                                   __uint_as_float(b.w << 16), __uint_as_float(b.w & 0xffff0000u));
+    }
+}
+
+// The residual stream's chunk c (the step input on the first layer).
+template <int F>
+__device__ __forceinline__ void chunk_resid(const GemvParams& p, int c, float4 (&v)[F]) {
+    if (p.x_in)
+        chunk_bf16<F>(p.x_in, c, p.K, v);
+    else
+        chunk_f32<F>(p.x_resid, c, p.K, v);
+}
+
+// 1 / sqrt(mean(x^2) + eps) of the residual stream. Every CTA sums in the same fixed order
+// (each thread its chunks, then the warps in index order), so all CTAs see identical x^. On
+// the first layer CTA 0 also writes the widened step input into the residual buffer.
+template <int XC, int F>
+__device__ float inv_rms(const GemvParams& p, int tid, float* stat) {
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        if (c < p.nchunks) {
+            float4 v[F];
+            chunk_resid<F>(p, c, v);
+#pragma unroll
+            for (int e = 0; e < F; ++e) {
+                ss = fmaf(v[e].x, v[e].x, ss);
+                ss = fmaf(v[e].y, v[e].y, ss);
+                ss = fmaf(v[e].z, v[e].z, ss);
+                ss = fmaf(v[e].w, v[e].w, ss);
+            }
+            if (p.x_in && p.x_resid_init && blockIdx.x == 0 && 4 * F * c < p.K)
+#pragma unroll
+                for (int e = 0; e < F; ++e) reinterpret_cast<float4*>(p.x_resid_init + 4 * F * c)[e] = v[e];
+        }
     }
     ss = warp_sum(ss);
     if ((tid & 31) == 0) stat[tid >> 5] = ss;
@@ -140,48 +178,26 @@ __device__ void norm_to_smem(const float* __restrict__ x, const uint16_t* __rest
     float tot = 0.f;
 #pragma unroll
     for (int w = 0; w < NWARP; ++w) tot += stat[w];
-    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)d) + eps);
-    const int ntot4 = nchunks * F;  // float4 slots including zero padding
-    for (int f = tid; f < ntot4; f += NT) {
-        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (f < n4) {
-            float4 v;
-            if (x_in) {
-                uint2 b = *reinterpret_cast<const uint2*>(x_in + 4 * f);
-                v = make_float4(__uint_as_float(b.x << 16), __uint_as_float(b.x & 0xffff0000u),
-                                __uint_as_float(b.y << 16), __uint_as_float(b.y & 0xffff0000u));
-            } else {
-                v = reinterpret_cast<const float4*>(x)[f];
-            }
-            float4 gm = reinterpret_cast<const float4*>(gamma)[f];
-            o.x = (v.x * inv) * gm.x;
-            o.y = (v.y * inv) * gm.y;
-            o.z = (v.z * inv) * gm.z;
-            o.w = (v.w * inv) * gm.w;
-        }
-        xs[swz<F>(f)] = o;
-    }
-    consumer_sync();
+    return 1.0f / sqrtf(__fdiv_rn(tot, (float)p.K) + p.eps);
 }
 
-// FP32 activation vector [K] -> swizzled shared memory (zero padded to nchunks*16)
-__device__ void f32_to_smem(const float* __restrict__ a, int K, int nchunks, float4* xs) {
-    const int tid = threadIdx.x;
-    const int ntot4 = nchunks * 4;
-    for (int f = tid; f < ntot4; f += NT) {
-        float4 o;
-        const int e = 4 * f;
-        if (e + 3 < K) {
-            o = *reinterpret_cast<const float4*>(a + e);
-        } else {
-            o.x = (e + 0 < K) ? a[e + 0] : 0.f;
-            o.y = (e + 1 < K) ? a[e + 1] : 0.f;
-            o.z = (e + 2 < K) ? a[e + 2] : 0.f;
-            o.w = (e + 3 < K) ? a[e + 3] : 0.f;
+// The consumer's chunk c of x^ = x * inv * gamma (norm modes) or of the plain activation.
+template <int MODE, int F>
+__device__ __forceinline__ void chunk_act(const GemvParams& p, int c, float inv, float4 (&v)[F]) {
+    if (MODE == M_QKV || MODE == M_GU || MODE == M_LM) {
+        chunk_resid<F>(p, c, v);
+        float4 gm[F];
+        chunk_f32<F>(p.gamma, c, p.K, gm);
+#pragma unroll
+        for (int e = 0; e < F; ++e) {
+            v[e].x = (v[e].x * inv) * gm[e].x;
+            v[e].y = (v[e].y * inv) * gm[e].y;
+            v[e].z = (v[e].z * inv) * gm[e].z;
+            v[e].w = (v[e].w * inv) * gm[e].w;
         }
-        xs[swz<4>(f)] = o;
+    } else {
+        chunk_f32<F>(p.act, c, p.K, v);
     }
-    consumer_sync();
 }
 
 // ---------------------------------------------------------------- row addressing
@@ -258,14 +274,15 @@ struct XRegs {
     float4 v[XC][F];
 };
 
-template <int XC, int F>
-__device__ __forceinline__ void load_x(XRegs<XC, F>& xr, const float4* xs, int nchunks, int tid) {
+template <int MODE, int XC>
+__device__ __forceinline__ void load_x(XRegs<XC, 2>& xr, const GemvParams& p, float inv, int tid) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
-#pragma unroll
-        for (int e = 0; e < F; ++e)
-            xr.v[j][e] = c < nchunks ? xs[swz<F>(F * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
+        if (c < p.nchunks)
+            chunk_act<MODE, 2>(p, c, inv, xr.v[j]);
+        else
+            xr.v[j][0] = xr.v[j][1] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
 }
 
@@ -279,19 +296,21 @@ struct XDigits {
     float scale[XC];
 };
 
-template <int XC>
-__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const float4* xs, int nchunks, int tid) {
+template <int MODE, int XC>
+__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const GemvParams& p, float inv, int tid) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
+        float4 q[4] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f),
+                       make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+        if (c < p.nchunks) chunk_act<MODE, 4>(p, c, inv, q);
         float v[16];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            const float4 q = c < nchunks ? xs[swz<4>(4 * c + e)] : make_float4(0.f, 0.f, 0.f, 0.f);
-            v[4 * e + 0] = q.x;
-            v[4 * e + 1] = q.y;
-            v[4 * e + 2] = q.z;
-            v[4 * e + 3] = q.w;
+            v[4 * e + 0] = q[e].x;
+            v[4 * e + 1] = q[e].y;
+            v[4 * e + 2] = q[e].z;
+            v[4 * e + 3] = q[e].w;
         }
         float m = 0.f;
 #pragma unroll
@@ -480,7 +499,7 @@ struct GemvSmem {
 };
 __host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap) {
     GemvSmem g;
-    g.x_bytes = ((nchunks * F * 16) + 127) & ~127;
+    g.x_bytes = 0;  // the activation slices are read from global memory
     g.stage_bytes = ((R * ld) + 127) & ~127;
     const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
     int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
@@ -498,7 +517,6 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
     const int NS = L.nstages;
-    float4* xs = reinterpret_cast<float4*>(sm);
     uint8_t* stages = sm + L.x_bytes;
     const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
     const uint32_t empty0 = full0 + 8 * MAX_STAGES;
@@ -586,19 +604,18 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     // ---- consumers
     pdl_wait();
     pdl_trigger();
+    float inv = 1.f;
     if (MODE == M_QKV || MODE == M_GU)
-        norm_to_smem<4>(p.x_resid, p.x_in, p.x_resid_init, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
+        inv = inv_rms<XC, 4>(p, tid, stat);
     else if (MODE == M_LM)
-        norm_to_smem<2>(p.x_resid, nullptr, nullptr, p.gamma, p.K, p.eps, p.nchunks, xs, stat);
-    else
-        f32_to_smem(p.act, p.K, p.nchunks, xs);
+        inv = inv_rms<XC, 2>(p, tid, stat);
 
     XRegs<XC, 2> xr;        // LM head: FP32 activation slice
     XDigits<XC> xd;         // INT8 modes: block-scaled integer digits of the slice
     if constexpr (MODE == M_LM)
-        load_x<XC, 2>(xr, xs, p.nchunks, tid);
+        load_x<MODE, XC>(xr, p, inv, tid);
     else
-        digits_x<XC>(xd, xs, p.nchunks, tid);
+        digits_x<MODE, XC>(xd, p, inv, tid);
     int s = 0, b = 0;
     uint32_t sph = 0, bph = 0;
     for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {

@@ -43,6 +43,8 @@ int device_info(DevInfo& out) {
         cached.dev = dev;
         cached.sms = pr.multiProcessorCount;
         cached.smem_optin = (int)pr.sharedMemPerBlockOptin;
+        cached.smem_per_sm = (int)pr.sharedMemPerMultiprocessor;
+        cached.smem_reserved = (int)pr.reservedSharedMemPerBlock;
     }
     out = cached;
     return TASP_OK;

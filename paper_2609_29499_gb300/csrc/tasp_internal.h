@@ -191,6 +191,7 @@ struct Session {
 // ---------------------------------------------------------------- device info
 struct DevInfo {
     int dev = -1, sms = 0, smem_optin = 0;
+    int smem_per_sm = 0, smem_reserved = 0;  // shared memory of an SM, and reserved per resident CTA
 };
 int device_info(DevInfo& out);
 
