@@ -232,25 +232,6 @@ def test_8b_batch_of_four_end_to_end(tasp):
     plan.release()
 
 
-def test_70b_batch_of_five_full_depth(tasp):
-    # the mixed-turn serving shape: 4 + 1 sessions at contexts up to 4096 with logits
-    wl = synth.CFG3
-    sh = wl.shape
-    plan = lib_plan(tasp, sh, wl.masks[0])
-    n, steps = 5, 2
-    t_priors = [4096, 3000, 2048, 1024, 256]
-    kv_seeds = [wl.kv_seed + i for i in range(n)]
-    xb = synth.step_inputs_bf16(wl.x_seed + 5, steps, n, sh.d)
-    ss = _sessions(tasp, plan, t_priors, kv_seeds, steps)
-    got, logits = _run(tasp, ss, xb, sh.vocab)
-    for i, s in enumerate(ss):
-        assert s.device_error() == 0
-        assert s.position == t_priors[i] + steps
-        s.release()
-    assert np.isfinite(got).all() and np.isfinite(logits).all()
-    plan.release()
-
-
 def test_70b_width_row_indexed_batch_is_bit_identical(tasp):
     # the mixed-turn bench's configuration: a group of four sessions on a plan whose Q/K/V and
     # gate/up panels are row maps into the shared store reads the same bytes as materialized

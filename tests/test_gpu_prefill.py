@@ -89,3 +89,10 @@ def test_prefill_8b_two_layers_bench_length(tasp):
     # head in the attention schedule) on a two-layer cut of the 8B widths
     sh = dataclasses.replace(synth.LLAMA3_8B, L=2)
     _prefill_case(tasp, sh, synth.CFG4.masks[0], 2048, 2, [0, 1], logits_rows=np.arange(0, sh.vocab, 499))
+
+
+def test_prefill_8b_two_layers_longest_prompt(tasp):
+    # the longest prompt of the prefill workload (8,192 tokens: 64 query blocks per head in the
+    # attention schedule, 64 row tiles per GEMM) on a two-layer cut of the 8B widths
+    sh = dataclasses.replace(synth.LLAMA3_8B, L=2)
+    _prefill_case(tasp, sh, synth.CFG4.masks[1], 8192, 2, [0, 1], logits_rows=np.arange(0, sh.vocab, 499), seed=9)

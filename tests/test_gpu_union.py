@@ -243,9 +243,10 @@ def test_union_is_deterministic_and_ignores_panel_layout(tasp, layer1_plans):
     assert np.array_equal(got.view(np.uint32), outs[0].view(np.uint32))
 
 
-def test_70b_width_sixteen_sessions_agree_with_per_plan(tasp):
+def test_70b_width_sixteen_sessions_agree_with_per_plan_and_oracle(tasp):
     # the 70B widths (two-layer cut): 16 sessions over the five masks and the dense plan, the
-    # down projection's 28,672-long reduction split in K slices; agreement with the per-plan path
+    # down projection's 28,672-long reduction split in K slices; agreement with the per-plan
+    # path and with the oracle
     sh = dataclasses.replace(synth.LLAMA3_70B, L=2)
     recipes = list(synth.CFG5.masks)
     plans = [lib_plan(tasp, sh, r) for r in recipes] + [tasp.Plan(sh, tasp.all_keep_mask())]
@@ -267,3 +268,14 @@ def test_70b_width_sixteen_sessions_agree_with_per_plan(tasp):
         assert rel_l2(got[:, i], ref[:, i]) <= TOL_UNION, (i, pick[i], rel_l2(got[:, i], ref[:, i]))
     for p in plans:
         p.release()
+    # and against the oracle: each plan's sessions decoded under that plan's mask as zeros
+    masks = [oracle_mask(sh, r) for r in recipes] + [maskc.all_keep(sh)]
+    xf = synth.bf16_to_f32(xb)
+    for k, mask in enumerate(masks):
+        idx = [i for i in range(n) if pick[i] == k]
+        if not idx:
+            continue
+        want = forward.decode_sessions(sh, mask, xf[:, idx], [t_priors[i] for i in idx], [kv_seeds[i] for i in idx])
+        for j, i in enumerate(idx):
+            e = rel_l2(got[:, i], want[:, j])
+            assert e <= TOL_E2E, (i, k, e)
