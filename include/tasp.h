@@ -360,6 +360,24 @@ int tasp_set_memory_limit(int64_t bytes);
 /* Device bytes the library's arenas hold now. Host only. */
 int tasp_memory_in_use(int64_t* bytes);
 
+/* ---------------------------------------------------------------------------
+ * Failure-detection test hooks (the paper has no counterpart). They let a test make
+ * a device wait run out without faulting or hanging the GPU; both are process-wide,
+ * host only, and meant for eager launches (tasp_layer_step, tasp_profile_step,
+ * tasp_decode_step_static): a CUDA graph captured while a hook is set keeps it.
+ * ------------------------------------------------------------------------- */
+
+/* Clock-cycle limit of the bounded mbarrier waits in the one-session GEMVs launched
+ * from now on (0 restores the default of ~2 s). A wait that runs out sets bit 0 of the
+ * session's device error word, every later wait of that CTA returns at once, and the
+ * kernel returns (its outputs are then invalid). EINVAL for a negative value. */
+int tasp_test_set_wait_limit(int64_t cycles);
+
+/* The next `launches` one-session GEMV launches issue no weight copies at all, so their
+ * consumers' first wait runs out (nothing is ever in flight); 0 cancels. EINVAL for a
+ * negative count. */
+int tasp_test_skip_gemv_copies(int32_t launches);
+
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char* tasp_last_error(void);
 

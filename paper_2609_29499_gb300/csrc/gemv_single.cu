@@ -55,6 +55,8 @@ struct GemvParams {
     float* logits;
     int* err;       // device error word (bounded waits that gave up)
     int smem_cap;   // dynamic shared memory available to the launch
+    long long wait_limit;  // clock cycles before a bounded wait gives up
+    int skip_copies;       // failure-detection test hook: the producer issues no copies
 };
 
 
@@ -148,56 +150,83 @@ __device__ __forceinline__ void chunk_resid(const GemvParams& p, int c, float4 (
         chunk_f32<F>(p.x_resid, c, p.K, v);
 }
 
-// 1 / sqrt(mean(x^2) + eps) of the residual stream. Every CTA sums in the same fixed order
-// (each thread its chunks, then the warps in index order), so all CTAs see identical x^. On
-// the first layer CTA 0 also writes the widened step input into the residual buffer.
+// The consumer's slice held in registers: chunk j of the thread is c = tid + j * CT.
 template <int XC, int F>
-__device__ float inv_rms(const GemvParams& p, int tid, float* stat) {
-    float ss = 0.f;
+struct Slice {
+    float4 v[XC][F];
+};
+
+// Norm gains of this thread's chunks: constant, so they are read before the dependency wait.
+template <int XC, int F>
+__device__ __forceinline__ void load_gamma(const GemvParams& p, int tid, Slice<XC, F>& g) {
+#pragma unroll
+    for (int j = 0; j < XC; ++j) {
+        const int c = tid + j * CT;
+        if (c < p.nchunks)
+            chunk_f32<F>(p.gamma, c, p.K, g.v[j]);
+        else
+#pragma unroll
+            for (int e = 0; e < F; ++e) g.v[j][e] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+}
+
+// The activation slice: x^ = x * inv * gamma with inv = 1 / sqrt(mean(x^2) + eps) for the norm
+// modes, the plain activation otherwise. One read of this thread's chunks after the dependency
+// wait; the sum of squares is taken in the same fixed order by every CTA (each thread its
+// chunks, then the warps in index order), so all CTAs see identical x^. On the first layer CTA
+// 0 also writes the widened step input into the residual buffer.
+template <int MODE, int XC, int F>
+__device__ __forceinline__ void load_slice(const GemvParams& p, int tid, float* stat, const Slice<XC, F>& g,
+                                           Slice<XC, F>& x) {
+    constexpr bool NORM = MODE == M_QKV || MODE == M_GU || MODE == M_LM;
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
         if (c < p.nchunks) {
-            float4 v[F];
-            chunk_resid<F>(p, c, v);
+            if (NORM)
+                chunk_resid<F>(p, c, x.v[j]);
+            else
+                chunk_f32<F>(p.act, c, p.K, x.v[j]);
+        } else {
 #pragma unroll
-            for (int e = 0; e < F; ++e) {
-                ss = fmaf(v[e].x, v[e].x, ss);
-                ss = fmaf(v[e].y, v[e].y, ss);
-                ss = fmaf(v[e].z, v[e].z, ss);
-                ss = fmaf(v[e].w, v[e].w, ss);
-            }
-            if (p.x_in && p.x_resid_init && blockIdx.x == 0 && 4 * F * c < p.K)
-#pragma unroll
-                for (int e = 0; e < F; ++e) reinterpret_cast<float4*>(p.x_resid_init + 4 * F * c)[e] = v[e];
+            for (int e = 0; e < F; ++e) x.v[j][e] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
     }
+    if (!NORM) return;
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < XC; ++j)
+#pragma unroll
+        for (int e = 0; e < F; ++e) {
+            ss = fmaf(x.v[j][e].x, x.v[j][e].x, ss);
+            ss = fmaf(x.v[j][e].y, x.v[j][e].y, ss);
+            ss = fmaf(x.v[j][e].z, x.v[j][e].z, ss);
+            ss = fmaf(x.v[j][e].w, x.v[j][e].w, ss);
+        }
+    if (p.x_in && p.x_resid_init && blockIdx.x == 0)
+#pragma unroll
+        for (int j = 0; j < XC; ++j) {
+            const int c = tid + j * CT;
+            if (c < p.nchunks && 4 * F * c < p.K)
+#pragma unroll
+                for (int e = 0; e < F; ++e) reinterpret_cast<float4*>(p.x_resid_init + 4 * F * c)[e] = x.v[j][e];
+        }
     ss = warp_sum(ss);
     if ((tid & 31) == 0) stat[tid >> 5] = ss;
     consumer_sync();
     float tot = 0.f;
 #pragma unroll
     for (int w = 0; w < NWARP; ++w) tot += stat[w];
-    return 1.0f / sqrtf(__fdiv_rn(tot, (float)p.K) + p.eps);
-}
-
-// The consumer's chunk c of x^ = x * inv * gamma (norm modes) or of the plain activation.
-template <int MODE, int F>
-__device__ __forceinline__ void chunk_act(const GemvParams& p, int c, float inv, float4 (&v)[F]) {
-    if (MODE == M_QKV || MODE == M_GU || MODE == M_LM) {
-        chunk_resid<F>(p, c, v);
-        float4 gm[F];
-        chunk_f32<F>(p.gamma, c, p.K, gm);
+    const float inv = 1.0f / sqrtf(__fdiv_rn(tot, (float)p.K) + p.eps);
+#pragma unroll
+    for (int j = 0; j < XC; ++j)
 #pragma unroll
         for (int e = 0; e < F; ++e) {
-            v[e].x = (v[e].x * inv) * gm[e].x;
-            v[e].y = (v[e].y * inv) * gm[e].y;
-            v[e].z = (v[e].z * inv) * gm[e].z;
-            v[e].w = (v[e].w * inv) * gm[e].w;
+            x.v[j][e].x = (x.v[j][e].x * inv) * g.v[j][e].x;
+            x.v[j][e].y = (x.v[j][e].y * inv) * g.v[j][e].y;
+            x.v[j][e].z = (x.v[j][e].z * inv) * g.v[j][e].z;
+            x.v[j][e].w = (x.v[j][e].w * inv) * g.v[j][e].w;
         }
-    } else {
-        chunk_f32<F>(p.act, c, p.K, v);
-    }
 }
 
 // ---------------------------------------------------------------- row addressing
@@ -245,16 +274,16 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Bounded wait: gives up after WAIT_LIMIT cycles, records the failure in the device
-// error word and makes every later wait of this CTA return at once (abort), so a lost
-// transfer can never hang the GPU; the host reports the error word.
-__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err,
+// Bounded wait: gives up after `limit` cycles, records the failure in the device error
+// word and makes every later wait of this CTA return at once (abort), so a lost transfer
+// can never hang the GPU; the host reports the error word.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int* abort_flag, int* err, long long limit,
                                           bool honor_abort = true) {
     if (honor_abort && *(volatile int*)abort_flag) return;
     if (mbar_try(bar, parity)) return;
     const long long t0 = clock64();
     while (!mbar_try(bar, parity)) {
-        if (clock64() - t0 > WAIT_LIMIT) {
+        if (clock64() - t0 > limit) {
             *(volatile int*)abort_flag = 1;
             if (err) atomicOr(err, ERR_WAIT_TIMEOUT);
             return;
@@ -274,18 +303,6 @@ struct XRegs {
     float4 v[XC][F];
 };
 
-template <int MODE, int XC>
-__device__ __forceinline__ void load_x(XRegs<XC, 2>& xr, const GemvParams& p, float inv, int tid) {
-#pragma unroll
-    for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-        if (c < p.nchunks)
-            chunk_act<MODE, 2>(p, c, inv, xr.v[j]);
-        else
-            xr.v[j][0] = xr.v[j][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-}
-
 // The activation slice of an INT8 GEMV as block-scaled integers: per 16-element chunk
 // one power-of-two scale 2^(e-14) with max|x| < 2^e, each element rounded to the integer
 // X in [-2^14, 2^14] and split as X = 256 hi + lo (hi signed byte, lo unsigned byte),
@@ -296,14 +313,11 @@ struct XDigits {
     float scale[XC];
 };
 
-template <int MODE, int XC>
-__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const GemvParams& p, float inv, int tid) {
+template <int XC>
+__device__ __forceinline__ void digits_x(XDigits<XC>& xd, const Slice<XC, 4>& xs) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
-        const int c = tid + j * CT;
-        float4 q[4] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f),
-                       make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
-        if (c < p.nchunks) chunk_act<MODE, 4>(p, c, inv, q);
+        const float4 (&q)[4] = xs.v[j];
         float v[16];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -543,11 +557,11 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     if (warp == CW) {
         // ---- producer: weights never depend on the previous kernel, so start at once
         pdl_trigger();
-        if (lane == 0) {
+        if (lane == 0 && !p.skip_copies) {
             int s = 0;
             uint32_t ph = 0;
             for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-                if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err);
+                if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err, p.wait_limit);
                 const int nrow = min(R, p.rows - gi * R);
                 mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
                 for (int r = 0; r < nrow; ++r)
@@ -561,7 +575,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
             // never leave while copies into this CTA's shared memory are in flight (even
             // after an abort: this second wait is bounded on its own)
             for (int gi = max(g0, g1 - NS), i = gi - g0; gi < g1; ++gi, ++i)
-                mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, false);
+                mbar_wait(full0 + 8 * (i % NS), (i / NS) & 1, &abort_flag, p.err, p.wait_limit, false);
         }
         return;
     }
@@ -589,7 +603,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
         int b = 0;
         uint32_t ph = 0;
         for (int gi = g0; gi < g1; ++gi) {
-            mbar_wait(rfull0 + 8 * b, ph, &abort_flag, p.err);
+            mbar_wait(rfull0 + 8 * b, ph, &abort_flag, p.err, p.wait_limit);
             epilogue<MODE, R>(p, red[b], gi, lane, es);
             __syncwarp();
             if (lane == 0) mbar_arrive(rempty0 + 8 * b);
@@ -602,24 +616,28 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     }
 
     // ---- consumers
+    constexpr int F = MODE == M_LM ? 2 : 4;  // float4s per 16-byte weight chunk
+    Slice<XC, F> gam, xsl;
+    if (MODE == M_QKV || MODE == M_GU || MODE == M_LM) load_gamma<XC, F>(p, tid, gam);
     pdl_wait();
     pdl_trigger();
-    float inv = 1.f;
-    if (MODE == M_QKV || MODE == M_GU)
-        inv = inv_rms<XC, 4>(p, tid, stat);
-    else if (MODE == M_LM)
-        inv = inv_rms<XC, 2>(p, tid, stat);
+    load_slice<MODE, XC, F>(p, tid, stat, gam, xsl);
 
     XRegs<XC, 2> xr;        // LM head: FP32 activation slice
     XDigits<XC> xd;         // INT8 modes: block-scaled integer digits of the slice
-    if constexpr (MODE == M_LM)
-        load_x<MODE, XC>(xr, p, inv, tid);
-    else
-        digits_x<MODE, XC>(xd, p, inv, tid);
+    if constexpr (MODE == M_LM) {
+#pragma unroll
+        for (int j = 0; j < XC; ++j) {
+            xr.v[j][0] = xsl.v[j][0];
+            xr.v[j][1] = xsl.v[j][1];
+        }
+    } else {
+        digits_x<XC>(xd, xsl);
+    }
     int s = 0, b = 0;
     uint32_t sph = 0, bph = 0;
     for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
-        mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err);
+        mbar_wait(full0 + 8 * s, sph, &abort_flag, p.err, p.wait_limit);
         const uint8_t* st = stages + (size_t)s * L.stage_bytes;
         float v[R];
         if constexpr (MODE == M_LM) {
@@ -647,7 +665,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
         const float rs = row_reduce<R>(v, lane);
-        if (i >= NRB) mbar_wait(rempty0 + 8 * b, bph ^ 1, &abort_flag, p.err);
+        if (i >= NRB) mbar_wait(rempty0 + 8 * b, bph ^ 1, &abort_flag, p.err, p.wait_limit);
         if ((lane & (32 / R - 1)) == 0) red[b][warp][lane / (32 / R)] = rs;
         __syncwarp();
         if (lane == 0) mbar_arrive(rfull0 + 8 * b);
@@ -735,6 +753,8 @@ std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 
 int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
     if (p.rows == 0) return TASP_OK;
+    p.wait_limit = test_hooks::wait_limit(WAIT_LIMIT);
+    p.skip_copies = test_hooks::take_skip() ? 1 : 0;
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;

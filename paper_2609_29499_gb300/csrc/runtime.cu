@@ -31,6 +31,21 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 // ---------------------------------------------------------------- device info
+namespace test_hooks {
+static std::atomic<long long> g_wait_limit{0};
+static std::atomic<int> g_skip{0};
+long long wait_limit(long long dflt) {
+    const long long v = g_wait_limit.load();
+    return v > 0 ? v : dflt;
+}
+bool take_skip() {
+    int v = g_skip.load();
+    while (v > 0)
+        if (g_skip.compare_exchange_weak(v, v - 1)) return true;
+    return false;
+}
+}  // namespace test_hooks
+
 int device_info(DevInfo& out) {
     static DevInfo cached;
     static std::mutex mu;
@@ -676,6 +691,18 @@ int tasp_dispatch(const float* h_probs, int32_t n, float tau, int32_t* plan) {
         if (h_probs[i] > h_probs[best]) best = i;
     }
     *plan = h_probs[best] >= tau ? best : n;
+    return TASP_OK;
+}
+
+int tasp_test_set_wait_limit(int64_t cycles) {
+    if (cycles < 0) return fail(TASP_EINVAL, "negative wait limit");
+    test_hooks::g_wait_limit.store(cycles);
+    return TASP_OK;
+}
+
+int tasp_test_skip_gemv_copies(int32_t launches) {
+    if (launches < 0) return fail(TASP_EINVAL, "negative launch count");
+    test_hooks::g_skip.store(launches);
     return TASP_OK;
 }
 

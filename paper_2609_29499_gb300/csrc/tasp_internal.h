@@ -189,6 +189,14 @@ struct Session {
 };
 
 // ---------------------------------------------------------------- device info
+// Failure-detection test hooks (tasp_test_set_wait_limit, tasp_test_skip_gemv_copies): a
+// shorter limit for the bounded waits of the one-session GEMVs, and a number of upcoming
+// one-session GEMV launches whose producer issues no copies.
+namespace test_hooks {
+long long wait_limit(long long dflt);  // the limit to launch with
+bool take_skip();                      // true (and one fewer pending) if this launch skips its copies
+}  // namespace test_hooks
+
 struct DevInfo {
     int dev = -1, sms = 0, smem_optin = 0;
     int smem_per_sm = 0, smem_reserved = 0;  // shared memory of an SM, and reserved per resident CTA

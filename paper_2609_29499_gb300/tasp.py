@@ -34,6 +34,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
+            "tasp_test_set_wait_limit", "tasp_test_skip_gemv_copies",
             "tasp_last_error",
             "tasp_version")
 
@@ -93,6 +94,8 @@ def load(path: str = LIB_PATH):
         "tasp_mask_select": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P]),
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_set_memory_limit": (c_int32, [c_int64]),
+        "tasp_test_set_wait_limit": (c_int32, [c_int64]),
+        "tasp_test_skip_gemv_copies": (c_int32, [c_int32]),
         "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
         "tasp_plan_layer_qheads": (c_int32, [P, c_int32, POINTER(c_int32)]),
         "tasp_plan_layout": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), c_int32, P, P, P, P, P, P]),
@@ -250,6 +253,18 @@ def dispatch(probs, tau: float = 0.85) -> int:
 def set_memory_limit(nbytes: int):
     """Cap the device memory of the library's arenas (0 = no cap)."""
     _check(load().tasp_set_memory_limit(int(nbytes)))
+
+
+def test_set_wait_limit(cycles: int):
+    """Failure-detection test hook: clock-cycle limit of the one-session GEMVs' bounded waits
+    (0 = the default)."""
+    _check(load().tasp_test_set_wait_limit(int(cycles)))
+
+
+def test_skip_gemv_copies(launches: int):
+    """Failure-detection test hook: the next `launches` one-session GEMV launches issue no
+    weight copies (their first wait runs out)."""
+    _check(load().tasp_test_skip_gemv_copies(int(launches)))
 
 
 def memory_in_use() -> int:
