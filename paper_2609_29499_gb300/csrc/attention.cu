@@ -25,6 +25,7 @@
 #include <algorithm>
 
 #include "tasp_internal.h"
+#include "tc_ptx.cuh"
 
 namespace tasp {
 
@@ -35,16 +36,24 @@ constexpr int AT_THREADS = AT_WARPS * 32;
 constexpr int TILE = 16;
 constexpr int CLUSTERS_MAX = ATTN_CLUSTERS_MAX;  // clusters per kept group (global merge when > 1)
 
-template <int DH>
+template <int DH, bool TMA>
 struct AttCfg {
-    static constexpr int ROWB = DH * 2 + 16;    // padded BF16 row (bytes): 16-byte rotation per row
-    static constexpr int TILEB = TILE * ROWB;   // one K or one V tile
+    // cp.async layout: rows padded by 16 bytes (a 16-byte rotation per row, read
+    // conflict-free by ldmatrix). TMA layout: per 64-dimension half a [16][128 B] box in the
+    // 128-byte swizzle (16-byte chunk j of row r stored at chunk j ^ (r & 7)).
+    static constexpr int ROWB = DH * 2 + 16;
+    static constexpr int HALFB = TILE * 128;    // one 64-dimension half of a tile (TMA layout)
+    static constexpr int TILEB = TMA ? TILE * DH * 2 : TILE * ROWB;  // one K or one V tile
     static constexpr int MAXT = DH == 128 ? 24 : 48;  // tiles resident per CTA
     static constexpr int KS = DH / 16;          // k-steps of q K^T
     static constexpr int NT = DH / 8;           // n-tiles of P V
     static constexpr int CPR = DH * 2 / 16;     // 16-byte chunks per row
-    static constexpr int SMEM = MAXT * 2 * TILEB;
+    static constexpr int SMEM = MAXT * 2 * TILEB + (TMA ? 1024 : 0);  // + alignment of the swizzle atoms
 };
+// Byte offset of 16-byte chunk c (8 dimensions) of row r in a TMA-layout tile.
+__device__ __forceinline__ uint32_t swz_off(int r, int c) {
+    return (uint32_t)((c >> 3) * (TILE * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+}
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
@@ -106,11 +115,15 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
     return r;
 }
 
-template <int DH, int G, int CS>
-__global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p) {
-    using C = AttCfg<DH>;
+template <int DH, int G, int CS, bool TMA>
+__global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const __grid_constant__ AttnParams p) {
+    using C = AttCfg<DH, TMA>;
     static_assert(G <= 8, "at most 8 query heads per KV group");
-    extern __shared__ __align__(128) uint8_t sm[];
+    extern __shared__ __align__(128) uint8_t smraw[];
+    uint8_t* const sm =
+        TMA ? reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023)) : smraw;
+    __shared__ __align__(8) uint64_t tbar[C::MAXT];  // TMA: one mbarrier per tile slot
+    __shared__ int abort_flag;
     __shared__ float red_m[AT_WARPS][8], red_l[AT_WARPS][8];
     __shared__ float cm[8], cl[8];              // this CTA's merged (max, sum) per head
     constexpr int ITEMS = G * DH / CS;          // (head, dim) outputs each CTA of the cluster finalizes
@@ -163,20 +176,47 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
         }
     };
 
+    // TMA: tile ti into slot `slot` (K then V, each DH / 64 boxes of 16 positions), completing
+    // on the slot's mbarrier. Positions past p1 hold finite cache contents (the caches start
+    // zeroed) or zeros past the capacity; their scores are masked.
+    auto issue_tma = [&](int ti, int slot) {
+        const uint32_t bar = smem_u32(&tbar[slot]);
+        const uint32_t kt = smem_u32(sm + slot * 2 * C::TILEB), vt = kt + C::TILEB;
+        tc::mbar_expect_tx(bar, 2 * C::TILEB);
+#pragma unroll
+        for (int hx = 0; hx < DH / 64; ++hx) {
+            tc::tma_load_3d(kt + hx * C::HALFB, &p.tmK[bz], hx * 64, p0 + ti * TILE, jl, bar);
+            tc::tma_load_3d(vt + hx * C::HALFB, &p.tmV[bz], hx * 64, p0 + ti * TILE, jl, bar);
+        }
+    };
+
     // first batch of tiles; the row of this step's token (written by the QKV kernel) waits
     const int nb0 = min(C::MAXT, ntiles);
-    for (int t = warp; t < nb0; t += AT_WARPS) issue(t, t, t == dep_tile ? T - 1 : -1);
-    cp_commit();
-    pdl_wait();
-    pdl_trigger();
-    if (dep_tile >= 0 && dep_tile < nb0 && dep_tile % AT_WARPS == warp && lane < C::CPR) {
-        const int r = T - 1 - (p0 + dep_tile * TILE);
-        const int64_t off = (int64_t)(T - 1) * DH + lane * 8;
-        uint8_t* kt = sm + dep_tile * 2 * C::TILEB;
-        cp_async16(smem_u32(kt + r * C::ROWB + lane * 16), Kg + off, 16);
-        cp_async16(smem_u32(kt + C::TILEB + r * C::ROWB + lane * 16), Vg + off, 16);
+    if constexpr (TMA) {
+        if (tid == 0) {
+            abort_flag = 0;
+            for (int t = 0; t < C::MAXT; ++t) tc::mbar_init(smem_u32(&tbar[t]), 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncthreads();
+        if (lane == 0)
+            for (int t = warp; t < nb0; t += AT_WARPS) issue_tma(t, t);
+        pdl_wait();
+        pdl_trigger();
+    } else {
+        for (int t = warp; t < nb0; t += AT_WARPS) issue(t, t, t == dep_tile ? T - 1 : -1);
+        cp_commit();
+        pdl_wait();
+        pdl_trigger();
+        if (dep_tile >= 0 && dep_tile < nb0 && dep_tile % AT_WARPS == warp && lane < C::CPR) {
+            const int r = T - 1 - (p0 + dep_tile * TILE);
+            const int64_t off = (int64_t)(T - 1) * DH + lane * 8;
+            uint8_t* kt = sm + dep_tile * 2 * C::TILEB;
+            cp_async16(smem_u32(kt + r * C::ROWB + lane * 16), Kg + off, 16);
+            cp_async16(smem_u32(kt + C::TILEB + r * C::ROWB + lane * 16), Vg + off, 16);
+        }
+        cp_commit();
     }
-    cp_commit();
 
     const int h = lane >> 2;        // head row of this lane's fragments
     const int qc = (lane & 3) * 2;  // column pair within an 8-column block
@@ -203,24 +243,49 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
 
     for (int b0 = 0; b0 < ntiles; b0 += C::MAXT) {
         const int nb = min(C::MAXT, ntiles - b0);
+        const uint32_t par = (uint32_t)((b0 / C::MAXT) & 1);
         if (b0 > 0) {  // later batches (very long contexts): reuse this warp's slots
-            for (int t = warp; t < nb; t += AT_WARPS) issue(b0 + t, t, -1);
-            cp_commit();
+            if constexpr (TMA) {
+                // this warp's reads of its slots are done; order them before the async writes
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0)
+                    for (int t = warp; t < nb; t += AT_WARPS) issue_tma(b0 + t, t);
+            } else {
+                for (int t = warp; t < nb; t += AT_WARPS) issue(b0 + t, t, -1);
+                cp_commit();
+            }
         }
-        cp_wait_all();
-        __syncwarp();
+        if constexpr (!TMA) {
+            cp_wait_all();
+            __syncwarp();
+        }
         for (int t = warp; t < nb; t += AT_WARPS) {
             any = true;
             const int base = p0 + (b0 + t) * TILE;
             const uint8_t* kt = sm + t * 2 * C::TILEB;
             const uint8_t* vt = kt + C::TILEB;
+            if constexpr (TMA) {
+                tc::mbar_wait(smem_u32(&tbar[t]), par, &abort_flag, p.err);
+                if (b0 == 0 && b0 + t == dep_tile) {
+                    // the box was requested before the QKV kernel wrote this step's token: copy
+                    // that row again (K by lanes 0..CPR-1, V by the next CPR lanes)
+                    const int r = T - 1 - base;
+                    if (lane < 2 * C::CPR) {
+                        const int which = lane / C::CPR, c = lane - which * C::CPR;
+                        const uint4 v = *reinterpret_cast<const uint4*>((which ? Vg : Kg) + (int64_t)(T - 1) * DH + c * 8);
+                        *reinterpret_cast<uint4*>(const_cast<uint8_t*>(which ? vt : kt) + swz_off(r, c)) = v;
+                    }
+                    __syncwarp();
+                }
+            }
             float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
-            const uint32_t krow =
-                smem_u32(kt + (8 * ((lane >> 4) & 1) + (lane & 7)) * C::ROWB + 16 * ((lane >> 3) & 1));
+            const int kr = 8 * ((lane >> 4) & 1) + (lane & 7), kh = (lane >> 3) & 1;
+            const uint32_t krow = TMA ? smem_u32(kt) : smem_u32(kt + kr * C::ROWB + 16 * kh);
 #pragma unroll
             for (int ks = 0; ks < C::KS; ++ks) {
                 uint32_t b00, b01, b10, b11;
-                ldsm_x4(krow + ks * 32, b00, b01, b10, b11);
+                ldsm_x4(TMA ? krow + swz_off(kr, 2 * ks + kh) : krow + ks * 32, b00, b01, b10, b11);
                 mma16816(s0, qa[ks], b00, b01);
                 mma16816(s1, qa[ks], b10, b11);
             }
@@ -249,19 +314,28 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
             uint32_t pa[4];
             split_pack(pv[0], pv[1], pa[0], pa[1]);
             split_pack(pv[2], pv[3], pa[2], pa[3]);
-            const uint32_t vrow =
-                smem_u32(vt + (8 * ((lane >> 3) & 1) + (lane & 7)) * C::ROWB + 16 * ((lane >> 4) & 1));
+            const int vr = 8 * ((lane >> 3) & 1) + (lane & 7), vh = (lane >> 4) & 1;
+            const uint32_t vrow = TMA ? smem_u32(vt) : smem_u32(vt + vr * C::ROWB + 16 * vh);
 #pragma unroll
             for (int nt = 0; nt < C::NT; nt += 2) {
                 uint32_t v0, v1, v2, v3;
-                ldsm_x4_t(vrow + nt * 16, v0, v1, v2, v3);
+                ldsm_x4_t(TMA ? vrow + swz_off(vr, nt + vh) : vrow + nt * 16, v0, v1, v2, v3);
                 mma16816(acc[nt], pa, v0, v1);
                 mma16816(acc[nt + 1], pa, v2, v3);
             }
         }
         __syncwarp();
     }
-    cp_wait_all();  // nothing in flight past this point (also for warps without tiles)
+    if constexpr (!TMA) cp_wait_all();  // nothing in flight past this point (also for warps without tiles)
+    if constexpr (TMA) {
+        // after a wait that gave up, wait once more (bounded on its own) for this warp's last
+        // boxes, so no copy lands in shared memory that is reused or released
+        if (*(volatile int*)&abort_flag && ntiles > 0) {
+            const int lb = (ntiles - 1) / C::MAXT * C::MAXT;
+            for (int t = warp; t < min(C::MAXT, ntiles - lb); t += AT_WARPS)
+                tc::mbar_wait(smem_u32(&tbar[t]), (uint32_t)((lb / C::MAXT) & 1), &abort_flag, p.err, false);
+        }
+    }
     l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
     l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
 
@@ -399,21 +473,25 @@ __global__ void __launch_bounds__(AT_THREADS, 1) attn_kernel(const AttnParams p)
 typedef void (*AttnFn)(const AttnParams);
 
 template <int DH, int G>
-AttnFn attn_fn(int cs) {
-    return cs == 16 ? attn_kernel<DH, G, 16> : attn_kernel<DH, G, 8>;
+AttnFn attn_fn(int cs, bool tma) {
+    if (tma) return cs == 16 ? attn_kernel<DH, G, 16, true> : attn_kernel<DH, G, 8, true>;
+    return cs == 16 ? attn_kernel<DH, G, 16, false> : attn_kernel<DH, G, 8, false>;
 }
 
-AttnFn pick(int dh, int g, int cs) {
+AttnFn pick(int dh, int g, int cs, bool tma = false) {
 #define TASP_ATT(D, GG) \
-    if (dh == D && g == GG) return attn_fn<D, GG>(cs);
+    if (dh == D && g == GG) return attn_fn<D, GG>(cs, tma);
     TASP_ATT(64, 1) TASP_ATT(64, 2) TASP_ATT(64, 4) TASP_ATT(64, 8)
     TASP_ATT(128, 1) TASP_ATT(128, 2) TASP_ATT(128, 4) TASP_ATT(128, 8)
 #undef TASP_ATT
     return nullptr;
 }
 
-int smem_of(int dh) { return dh == 128 ? AttCfg<128>::SMEM : AttCfg<64>::SMEM; }
-int maxt_of(int dh) { return dh == 128 ? AttCfg<128>::MAXT : AttCfg<64>::MAXT; }
+int smem_of(int dh, bool tma = false) {
+    if (tma) return dh == 128 ? AttCfg<128, true>::SMEM : AttCfg<64, true>::SMEM;
+    return dh == 128 ? AttCfg<128, false>::SMEM : AttCfg<64, false>::SMEM;
+}
+int maxt_of(int dh) { return dh == 128 ? AttCfg<128, false>::MAXT : AttCfg<64, false>::MAXT; }
 
 // Largest cluster size (16 when the device allows it, else 8) for a kernel.
 int cluster_size(AttnFn fn, int dh) {
@@ -465,12 +543,13 @@ int attn_splits_max() { return CLUSTERS_MAX * 16; }
 int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s,
                      int cs_cap) {
     const int cs = std::min(attn_cluster(dh, g), cs_cap);
-    AttnFn fn = pick(dh, g, cs);
+    const bool tma = a.tma != 0 && nb <= MAX_BATCH;
+    AttnFn fn = pick(dh, g, cs, tma);
     if (!fn) return fail(TASP_EUNSUP, "attention kernel not built for this (head_dim, query heads per group)");
-    static bool attr[2][9][2] = {};
-    bool& done = attr[dh == 128][g][cs == 16];
+    static bool attr[2][9][2][2] = {};
+    bool& done = attr[dh == 128][g][cs == 16][tma];
     if (!done) {
-        TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_of(dh)));
+        TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_of(dh, tma)));
         if (cs == 16) TASP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
         done = true;
     }
@@ -479,7 +558,7 @@ int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, i
     if (nb < 1 || nb > UNION_MAX) return fail(TASP_EINVAL, "attention batch of 1 to 16 sessions");
     cfg.gridDim = dim3(splits, m_kv, nb);
     cfg.blockDim = dim3(AT_THREADS);
-    cfg.dynamicSmemBytes = smem_of(dh);
+    cfg.dynamicSmemBytes = smem_of(dh, tma);
     cfg.stream = s;
     cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -273,6 +273,12 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
+            a.tma = 1;
+            for (int b = 0; b < n; ++b) {
+                a.tmK[b] = bv.ss[b]->tmK[l];
+                a.tmV[b] = bv.ss[b]->tmV[l];
+            }
+            a.err = bv.err;
             a.part = t.att_part ? t.att_part : bv.part;
             a.ml = t.att_ml ? t.att_ml : bv.ml;
             a.cnt = t.att_cnt ? t.att_cnt : bv.cnt;

@@ -974,6 +974,22 @@ int ensure_f16_panels(Plan& p, cudaStream_t s) {
 
 }  // namespace
 
+int encode_kv_map(CUtensorMap* m, const uint16_t* base, int dh, int max_tokens, int m_kv) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc;
+    int rc = encoder(&enc);
+    if (rc) return rc;
+    if (reinterpret_cast<uintptr_t>(base) & 15) return fail(TASP_EINVAL, "KV cache not 16-byte aligned");
+    cuuint64_t dims[3] = {(cuuint64_t)dh, (cuuint64_t)max_tokens, (cuuint64_t)m_kv};
+    cuuint64_t strides[2] = {(cuuint64_t)dh * 2, (cuuint64_t)max_tokens * dh * 2};
+    cuuint32_t box[3] = {64, 16, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<uint16_t*>(base), dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(TASP_ECUDA, "cuTensorMapEncodeTiled failed for a KV cache (" + std::to_string((int)r) + ")");
+    return TASP_OK;
+}
+
 int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
     Plan& pl = *se.plan;
     const Shape& sh = pl.store->sh;

@@ -467,6 +467,14 @@ static int session_alloc(Plan* p, int max_tokens, Session** out) {
     for (const LayerPlan& lp : p->layers) {
         se->K.push_back((uint16_t*)se->arena.take((size_t)lp.m_kv * max_tokens * sh.dh * 2));
         se->V.push_back((uint16_t*)se->arena.take((size_t)lp.m_kv * max_tokens * sh.dh * 2));
+        // TMA descriptors of the layer's caches for decode attention
+        CUtensorMap mk{}, mv{};
+        if (lp.m_kv > 0 && (sh.dh == 64 || sh.dh == 128)) {
+            if ((rc = encode_kv_map(&mk, se->K.back(), sh.dh, max_tokens, lp.m_kv))) return rc;
+            if ((rc = encode_kv_map(&mv, se->V.back(), sh.dh, max_tokens, lp.m_kv))) return rc;
+        }
+        se->tmK.push_back(mk);
+        se->tmV.push_back(mv);
     }
     se->rope = (float2*)se->arena.take((size_t)max_tokens * half * sizeof(float2));
     se->d_pos = (int*)se->arena.take(sizeof(int));

@@ -1,6 +1,7 @@
 // Internal structures of the TASP runtime: shared store, plans, sessions, kernel parameters.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -170,6 +171,8 @@ struct Session {
     int pos = 0;  // host mirror of the device position
     Arena arena;
     std::vector<uint16_t*> K, V;  // per layer BF16 [m_kv][max_tokens][dh]
+    // per layer TMA descriptors of K and V (boxes of 16 positions x 64 dims, 128-byte swizzle)
+    std::vector<CUtensorMap> tmK, tmV;
     float2* rope = nullptr;       // [max_tokens][dh/2] (cos, sin)
     int* d_pos = nullptr;
     // workspace of one decode step
@@ -223,6 +226,11 @@ constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pa
 constexpr int UNION_MAX = 16;  // sessions (of any plans) in one union-of-masks step
 constexpr int ATTN_CLUSTERS_MAX = 8;  // decode attention clusters per kept group (global merge when > 1)
 struct AttnParams {
+    // TMA descriptors of session b's K / V cache of this layer (tma != 0, at most MAX_BATCH
+    // sessions); otherwise the tiles are loaded with cp.async
+    CUtensorMap tmK[MAX_BATCH], tmV[MAX_BATCH];
+    int tma;
+    int* err;            // device error word (bounded waits that gave up)
     // session b of the launch (blockIdx.z) reads q + b * q_stride, writes o + b * q_stride
     const float* q;      // FP32 rotated queries [m_kv g][dh] (kept groups, all g slots)
     float* o;            // FP32 [m_q][dh], kept heads in O-panel column order
@@ -243,6 +251,9 @@ int attn_supported(int dh, int g);
 int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
 int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap = 16);
 int attn_splits_max();
+// TMA descriptor of a BF16 KV cache [m_kv][max_tokens][dh]: 16 positions x 64 dims per box,
+// 128-byte swizzle (prefill.cu)
+int encode_kv_map(CUtensorMap* m, const uint16_t* base, int dh, int max_tokens, int m_kv);
 // cs_cap: largest cluster size to use (16 or 8; many short sessions run better on 8)
 int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s,
                      int cs_cap = 16);

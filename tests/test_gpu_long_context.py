@@ -84,3 +84,24 @@ def test_union_beyond_one_cluster(tasp):
         ref = forward.decode(sh, masks[i], synth.bf16_to_f32(xb[:, i]), tps[i], seeds[i])
         assert within(got[:, i], ref).all(), (i, np.abs(got[:, i] - ref).max())
         assert rel_l2(got[:, i], ref) <= TOL_E2E
+
+
+def test_8b_layer_decode_beyond_the_resident_tiles(tasp):
+    # head dim 128, 8 clusters of 16 CTAs per kept group: past 8 x 16 x 24 tiles of 16
+    # positions each CTA holds more tiles than its shared memory, so it loads them in two
+    # batches through the same slots (one 8B layer against the oracle, elementwise)
+    import dataclasses
+    sh = dataclasses.replace(synth.LLAMA3_8B, L=1, vocab=0)
+    recipe = synth.MaskRecipe(1002)
+    plan = lib_plan(tasp, sh, recipe)
+    mask = oracle_mask(sh, recipe)
+    tp, steps = 52000, 2
+    sess = tasp.Session(plan, tp + steps)
+    sess.fill_synthetic(tp, 91)
+    xb = synth.step_inputs_bf16(92, steps, 1, sh.d)
+    got = _decode(tasp, [sess], xb, False)
+    assert sess.device_error() == 0
+    sess.release()
+    plan.release()
+    ref = forward.decode(sh, mask, synth.bf16_to_f32(xb[:, 0]), tp, 91)
+    assert within(got[:, 0], ref).all(), np.abs(got[:, 0] - ref).max()
