@@ -2,10 +2,13 @@
 //
 // One thread-block cluster of CS CTAs handles one kept KV group (all g query heads of
 // the group); its CTAs split the cached positions. Within a CTA:
-//  * every 16-position K/V tile of the CTA's range is requested at once with cp.async
-//    (16-byte chunks, zero-filled past the last position) into a padded shared-memory
-//    layout read conflict-free by ldmatrix before the programmatic-dependency wait;
-//    only the row of the token written by this step's QKV kernel waits for it;
+//  * every 16-position K/V tile of the CTA's range is requested at once, before the
+//    programmatic-dependency wait. Decode steps of one plan (TMA = true) load each tile
+//    with 3-D TMA boxes (16 positions x 64 dimensions, 128-byte swizzle, read
+//    conflict-free by ldmatrix) completing on the tile's own mbarrier, so a warp starts
+//    on a tile as soon as it lands; the row of the token this step's QKV kernel writes is
+//    copied again after the wait. The union step (up to 16 sessions, no descriptors) uses
+//    16-byte cp.async into a padded layout, where only that row waits;
 //  * S = q K^T and O += P V run on the tensor cores (mma.sync m16n8k16, BF16 in, FP32
 //    accumulate). The 16 rows of the A operand hold the g query heads twice: rows r
 //    carry bf16(x) and rows r + 8 carry bf16(x - bf16(x)), so the two halves summed in
