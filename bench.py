@@ -35,10 +35,10 @@ import synth  # noqa: E402
 
 METRIC = "decode ms/token (70B-shape, 43% mask, bs1); achieved HBM GB/s vs ~8 TB/s"
 # DRAM traffic over algorithmic bytes of one launch, from one ncu capture of the kernel
-# (dram__bytes_read.sum + dram__bytes_write.sum of a 70B-width gate/up launch with 12,288
-# kept channels: 204,765,184 B against 201,539,584 algorithmic). Re-taken whenever the
+# (dram__bytes_read.sum + dram__bytes_write.sum of a 70B-width gate/up launch with 18,432
+# kept channels: 306,268,672 B against 302,137,344 algorithmic). Re-taken whenever the
 # kernel changes.
-TRAFFIC_PER_ALGORITHMIC = {"gate_up": 204765184 / 201539584}
+TRAFFIC_PER_ALGORITHMIC = {"gate_up": 306268672 / 302137344}
 PAPER_CONTEXT = {"ms_per_token_sparse": 31.3, "ms_per_token_dense": 45.2,
                  "hardware": "1x A100 80GB SXM, real Llama-3-70B, groupwise INT8, ~2k context"}
 
@@ -65,6 +65,8 @@ def parse():
     ap.add_argument("--prompt", type=int, default=2048, help="prefill prompt length")
     ap.add_argument("--quant-group", type=int, default=0,
                     help="groupwise INT8 store with one BF16 scale per this many input columns (Table 1: 128)")
+    ap.add_argument("--no-other-workloads", action="store_true",
+                    help="decode: skip the short prefill and mixed-turn runs attached to the line")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep the workload's widths but only this many layers (small cases for ncu captures)")
     return ap.parse_args()
@@ -417,6 +419,8 @@ def run_ours(args):
                        "library_bytes": int(tasp.memory_in_use()),
                        "torch_max_allocated_bytes": int(torch.cuda.max_memory_allocated())},
         }
+        if world == 1 and not args.no_other_workloads and not args.layers and args.config == 3 and not args.dense:
+            out["other_workloads"] = other_workloads(args)
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist
@@ -432,7 +436,7 @@ def measured_tensor_peak():
         return 1900.0, "fallback"
 
 
-def run_prefill(args):
+def run_prefill(args, emit=True):
     """Configuration 4: prefill of one prompt per turn on the 8B shape, the turns rotating over
     the five masks' plans; each prefill fills its plan-shaped KV cache, which then serves 32
     decode steps on the same plan. Reports ms per prompt and tensor TFLOP/s, with the decode
@@ -533,10 +537,12 @@ def run_prefill(args):
                                     "context": T + dec_steps},
            "e2e": e2e, "clocks": clocks, "device_error": err,
            "paper_context": {"prefill_ms_2048_sparse": 1326, "prefill_ms_2048_dense": 1814, "hardware": "A100, 70B"}}
-    print(json.dumps(out), flush=True)
+    if emit:
+        print(json.dumps(out), flush=True)
+    return out
 
 
-def run_mixed(args):
+def run_mixed(args, emit=True):
     """Mixed-turn serving on the 70B shape: 16 turns, each bound to the dense plan (p = 0.1)
     or one of five masks (seeded), prompts of U[256, 2048] synthetic prior tokens; every
     step decodes one token for every turn, grouped per plan (up to four sessions share a
@@ -583,7 +589,7 @@ def run_mixed(args):
     gs = {pi: [sessions[i] for i in idx] for pi, idx in groups.items()}
     stream = torch.cuda.current_stream()
     if args.union:
-        return run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s)
+        return run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s, emit)
 
     def step(t):
         for pi in groups:
@@ -683,10 +689,12 @@ def run_mixed(args):
                              "unit": "GB/s", "frac": round(step_gbs / peak, 4)},
            "e2e": e2e, "gpu_launches": launches * K, "clocks": clocks, "cpu_baseline": cpu,
            "device_error": errs, "setup_s": round(setup_s, 1)}
-    print(json.dumps(out), flush=True)
+    if emit:
+        print(json.dumps(out), flush=True)
+    return out
 
 
-def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s):
+def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s, emit=True):
     """The mixed-turn step as one union-of-masks step over all turns: each layer's dense
     panels are read once for every session (tensor-core skinny GEMMs), each session's mask
     applied where its units meet it; the LM head (BF16) is one more skinny GEMM for all turns."""
@@ -760,7 +768,34 @@ def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s):
                              "unit": "GB/s", "frac": round(step_gbs / peak, 4), "peak_source": peak_kind},
            "e2e": e2e, "gpu_launches": launches * K, "clocks": clocks, "cpu_baseline": None,
            "device_error": errs, "setup_s": round(setup_s, 1)}
-    print(json.dumps(out), flush=True)
+    if emit:
+        print(json.dumps(out), flush=True)
+    return out
+
+
+def other_workloads(args):
+    """Configurations 4 and 5 measured in the same run as the headline decode (short, bounded):
+    the prefill of 2,048-token prompts on the 8B shape over the five masks, and the 16 mixed
+    turns on the 70B shape in one union-of-masks step per token. Each entry is the summary of
+    that workload's own line (`--workload prefill` / `--workload mixed --union`)."""
+    import copy
+    res = {}
+    for name, fn, kw in (("prefill_8b_2048", run_prefill, dict(workload="prefill", prompt=2048)),
+                         ("mixed_70b_16turns_union", run_mixed, dict(workload="mixed", union=True))):
+        a = copy.copy(args)
+        a.steps, a.warmup, a.no_cpu_baseline, a.layers = 10, 3, True, 0
+        for k, v in kw.items():
+            setattr(a, k, v)
+        t0 = time.perf_counter()
+        try:
+            d = fn(a, emit=False)
+            res[name] = {k: d.get(k) for k in ("metric", "value", "unit", "higher_is_better", "ms_per_step",
+                                                 "roofline", "step_roofline", "e2e", "clocks", "config",
+                                                 "decode_after_prefill", "device_error") if d.get(k) is not None}
+        except Exception as e:  # the headline line must still print
+            res[name] = {"error": repr(e)[:300]}
+        res[name]["wall_s"] = round(time.perf_counter() - t0, 1)
+    return res
 
 
 def main():
