@@ -53,8 +53,9 @@ def parse():
     ap.add_argument("--dense", action="store_true", help="time the dense fallback plan instead of the mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", choices=["decode", "prefill", "mixed"], default="decode",
-                    help="decode (the headline metric), the prefill of one prompt on the 8B shape, or "
+    ap.add_argument("--workload", choices=["decode", "prefill", "mixed", "spectral"], default="decode",
+                    help="decode (the headline metric), the prefill of one prompt on the 8B shape, the spectral "
+                         "descriptors of one 70B-shape layer, or "
                          "mixed-turn serving (70B shape, 16 turns over the dense plan and five masks)")
     ap.add_argument("--union", action="store_true",
                     help="mixed workload: one union-of-masks step for all turns (every weight row read once "
@@ -257,6 +258,16 @@ def cpu_oracle_sample(shape, recipe, wl, n_steps, layers=(0, None), lm_rows=1024
     return per_step, info
 
 
+def decode_config(wl, args, ratio, world):
+    """The decode workload's config, the same on both arms: the prior context is the workload's
+    (each timed step adds one token to it)."""
+    return {"workload": wl.name + ("_dense" if args.dense else ""),
+            "mask": "all-keep dense fallback" if args.dense else
+            f"greedy dependency-closed, active-FLOP ratio {ratio:.4f}",
+            "context": wl.t_prior, "batch": 1, "parallelism": "replicas" if world > 1 else "single GPU",
+            "l2": "inputs larger than L2 (each step streams the whole plan's weights)"}
+
+
 # ------------------------------------------------------------------ reference arm (the oracle)
 def run_reference(args):
     world, rank, _ = dist_setup(args)
@@ -264,6 +275,14 @@ def run_reference(args):
         return
     wl, shape, recipe = workload(args)
     per_step, info = cpu_oracle_sample(shape, recipe, wl, args.warmup + args.steps)
+    from oracle import maskc
+    if args.dense:
+        ratio = 1.0
+    else:
+        m = maskc.compile_mask(shape, synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.n_units),
+                               synth.layer_target_u24(recipe.mask_seed, shape.L), recipe.budget, recipe.r_lo,
+                               recipe.r_hi)
+        ratio = m.info["total_flops"] / m.info["dense_flops"]
     timed = per_step[args.warmup:]
     v = float(np.mean(timed))
     info["value"] = v
@@ -271,8 +290,7 @@ def run_reference(args):
     out = {"impl": "reference", "metric": METRIC, "value": v, "unit": "ms/token", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": v, "higher_is_better": False,
            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-           "config": {"workload": wl.name, "mask": "0.57 active FLOPs, seeded scores", "context": wl.t_prior,
-                      "batch": 1},
+           "config": decode_config(wl, args, ratio, world),
            "cpu_baseline": info,
            "e2e": {"value": v, "unit": "ms/token", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
@@ -393,12 +411,9 @@ def run_ours(args):
             "metric": METRIC, "value": round(ms, 4), "unit": "ms/token", "n_gpus": world, "steps": K, "warmup": Wm,
             "ms_per_step": round(ms, 4), "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
             "dtype": "int8w-f32", "data": "synthetic",
-            "config": {"workload": wl.name + ("_dense" if args.dense else ""),
-                       "mask": "all-keep dense fallback" if args.dense else
-                       f"greedy dependency-closed, active-FLOP ratio {info['flops_retained'] / info['flops_dense']:.4f}",
-                       "context": T_start, "batch": 1, "parallelism": "replicas" if world > 1 else "single GPU",
-                       "l2": "inputs larger than L2 (each step streams the whole plan's weights)",
-                       "tokens_per_s": round(1e3 / ms * world, 2)},
+            "config": decode_config(wl, args, info['flops_retained'] / info['flops_dense'], world),
+            "context_first_timed_step": T_start,
+            "tokens_per_s": round(1e3 / ms * world, 2),
             "roofline": roofline,
             "step_roofline": {"bytes_per_token": int(step_bytes), "achieved": round(step_gbs, 1), "peak": peak,
                               "unit": "GB/s", "frac": round(step_gbs / peak, 4),
@@ -773,6 +788,54 @@ def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s, emi
     return out
 
 
+def run_spectral(args, emit=True):
+    """The spectral descriptors of every candidate unit of one 70B-shape layer (64 heads of
+    [512, 8192] blocks, 28 channel groups of [3072, 8192]): ms per layer, and the Gram step's
+    tensor rate against the measured bf16 peak (FP16 operands run at the same rate)."""
+    import torch
+    from paper_2609_29499_gb300 import build
+    build.build()
+    from paper_2609_29499_gb300 import tasp
+    tasp.load()
+    sh = synth.LLAMA3_70B
+    layer = 0
+    nh, nc, nu = 4 * sh.dh, 3 * sh.chan_unit, sh.df // sh.chan_unit
+    gram_flops = 2 * sh.d * (sh.Hq * nh * nh + nu * nc * nc)
+    for _ in range(max(1, args.warmup)):
+        tasp.spectral_layer(sh, layer)
+    K = max(1, args.steps)
+    ph = np.zeros(4)
+    t_tot = 0.0
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    for _ in range(K):
+        p = np.zeros(4)
+        t0 = time.perf_counter()
+        feat, _ = tasp.spectral_layer(sh, layer, phase_ms=p)
+        t_tot += time.perf_counter() - t0
+        ph += p
+    clocks = sampler.stop()
+    ph /= K
+    ms = t_tot * 1e3 / K
+    peak, kind = measured_tensor_peak()
+    gram_tf = gram_flops / (ph[1] * 1e-3) / 1e12
+    out = {"metric": "spectral descriptors ms/layer (70B-shape, 64 head + 28 channel-group candidates)",
+           "value": round(ms, 2), "unit": "ms", "n_gpus": 1, "steps": K, "warmup": args.warmup,
+           "higher_is_better": False, "data": "synthetic", "dtype": "f16-gram-f32acc, f32 eigensolver, f64 statistics",
+           "config": {"workload": "llama3_70b_spectral_layer", "candidates": int(feat.shape[0])},
+           "phases_ms": {"blocks": round(ph[0], 3), "gram": round(ph[1], 3), "eigensolver": round(ph[2], 3),
+                         "statistics": round(ph[3], 3)},
+           "roofline": {"bound": "tensor", "kernel": "gram (gemm_persist_kernel)", "achieved": round(gram_tf, 1),
+                        "peak": peak, "unit": "TFLOP/s", "frac": round(gram_tf / peak, 4),
+                        "peak_source": f"{kind} bf16_tflops", "flops": int(gram_flops), "traffic": None,
+                        "note": "Gram FLOPs over the Gram launches' summed device time while eight worker "
+                                "streams share the GPU (the eigensolver, a library routine, sets the layer time)"},
+           "clocks": clocks}
+    if emit:
+        print(json.dumps(out), flush=True)
+    return out
+
+
 def other_workloads(args):
     """Configurations 4 and 5 measured in the same run as the headline decode (short, bounded):
     the prefill of 2,048-token prompts on the 8B shape over the five masks, and the 16 mixed
@@ -806,6 +869,8 @@ def main():
         run_prefill(args)
     elif args.workload == "mixed":
         run_mixed(args)
+    elif args.workload == "spectral":
+        run_spectral(args)
     else:
         run_ours(args)
 

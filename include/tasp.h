@@ -361,6 +361,31 @@ int tasp_set_memory_limit(int64_t bytes);
 int tasp_memory_in_use(int64_t* bytes);
 
 /* ---------------------------------------------------------------------------
+ * Spectral descriptors of the candidate units (the calibration side of the method).
+ * ------------------------------------------------------------------------- */
+
+/* Features of every candidate unit of one layer (Sec. 3.1 "Candidate Units and Spectral
+ * Features", Eqs. 1-4; Appendix "Exact candidate feature construction"): the H_q attention
+ * heads (block [4 dh][d]: the head's Q rows, the O columns it feeds transposed, its KV group's
+ * K and V rows), then the df / chan_unit channel groups (block [3 chan_unit][d]: gate rows, up
+ * rows, down columns transposed), built from the model's synthetic weights rounded to BF16.
+ * With lambda_i = s_i^2 / d the eigenvalues of a block's normalized Gram matrix:
+ * h_features FP64 [H_q + df / chan_unit][6] = (alpha: Pareto exponent of the tail
+ * lambda >= lambda_min by maximum likelihood, lambda_min chosen among the distinct eigenvalues
+ * below the largest to minimize the Kolmogorov-Smirnov distance, ties to the smaller; effective
+ * rank; spectral norm s_1; SETOL, the tail's share of sum lambda; lambda_min; the KS distance).
+ * h_lambda (optional) FP64 [H_q 4 dh + (df / chan_unit) 3 chan_unit]: each block's
+ * eigenvalues, descending, blocks in the same order. The Gram matrices run on the tensor cores
+ * (FP16 operands holding the BF16 weights, FP32 accumulation); the eigenvalues come from
+ * cuSOLVER's symmetric eigensolver, loaded at run time. Per-call device temporaries come from
+ * the stream-ordered pool. h_phase_ms (optional) FP64 [4] receives the device time summed
+ * over the candidates of the four steps: block generation, Gram matrices, eigensolver,
+ * statistics. sync. Errors: EINVAL (desc, layer, NULL), EUNSUP (4 dh or 3 chan_unit above d,
+ * d not a multiple of 64, or no eigensolver), ECUDA. */
+int tasp_spectral_layer(const tasp_model_desc* model, int32_t layer, double* h_features, double* h_lambda,
+                        double* h_phase_ms, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Failure-detection test hooks (the paper has no counterpart). They let a test make
  * a device wait run out without faulting or hanging the GPU; both are process-wide,
  * host only, and meant for eager launches (tasp_layer_step, tasp_profile_step,

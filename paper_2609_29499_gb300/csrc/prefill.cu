@@ -974,6 +974,20 @@ int ensure_f16_panels(Plan& p, cudaStream_t s) {
 
 }  // namespace
 
+int gemm_f16_nt(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, const float* scale, float* C,
+                int ldc, int* err, cudaStream_t s) {
+    GemmArgs ga{};
+    ga.M = M;
+    ga.N = N;
+    ga.K = K;
+    ga.scale = scale;
+    ga.out = C;
+    ga.ldo = ldc;
+    ga.mode = EP_STORE;
+    ga.err = err;
+    return launch_gemm(A, lda, M, B, ldb, N, K, ga, s);
+}
+
 int encode_kv_map(CUtensorMap* m, const uint16_t* base, int dh, int max_tokens, int m_kv) {
     PFN_cuTensorMapEncodeTiled_v12000 enc;
     int rc = encoder(&enc);

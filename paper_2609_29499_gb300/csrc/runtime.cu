@@ -124,7 +124,7 @@ static int round16(int v) { return (v + 15) & ~15; }
 static std::mutex g_mu;
 static std::vector<Store*> g_stores;
 
-static int validate_shape(const tasp_model_desc* m, Shape& s, bool device = true) {
+int validate_shape(const tasp_model_desc* m, Shape& s, bool device) {
     if (!m) return fail(TASP_EINVAL, "model_desc is NULL");
     s.L = m->L; s.d = m->d; s.Hq = m->Hq; s.Hkv = m->Hkv; s.dh = m->dh; s.df = m->df; s.vocab = m->vocab;
     s.cu = m->chan_unit; s.eps = m->rms_eps; s.theta = m->rope_theta; s.seed = m->seed; s.qg = m->quant_group;

@@ -205,6 +205,8 @@ struct DevInfo {
     int smem_per_sm = 0, smem_reserved = 0;  // shared memory of an SM, and reserved per resident CTA
 };
 int device_info(DevInfo& out);
+// Model description -> Shape with every requirement checked (device: also the device limits).
+int validate_shape(const tasp_model_desc* m, Shape& s, bool device = true);
 
 // ---------------------------------------------------------------- kernels (launchers)
 // store.cu
@@ -251,6 +253,10 @@ int attn_supported(int dh, int g);
 int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
 int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap = 16);
 int attn_splits_max();
+// C[m][n] = scale[n] * sum_k A[m][k] B[n][k] on the tensor cores (prefill.cu's persistent
+// tcgen05 GEMM): FP16 A [M][lda], B [N][ldb], FP32 C [M][ldc]; K a multiple of 8.
+int gemm_f16_nt(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, const float* scale, float* C,
+                int ldc, int* err, cudaStream_t s);
 // TMA descriptor of a BF16 KV cache [m_kv][max_tokens][dh]: 16 positions x 64 dims per box,
 // 128-byte swizzle (prefill.cu)
 int encode_kv_map(CUtensorMap* m, const uint16_t* base, int dh, int max_tokens, int m_kv);

@@ -34,7 +34,7 @@ EXPORTED = ("tasp_compile_mask", "tasp_prefill", "tasp_decode_step", "tasp_relea
             "tasp_plan_info_get", "tasp_plan_layer_dims", "tasp_plan_export", "tasp_layer_step",
             "tasp_profile_step", "tasp_step_launches", "tasp_decode_step_static", "tasp_session_kv_export",
             "tasp_session_prefill", "tasp_decode_step_union", "tasp_union_status",
-            "tasp_test_set_wait_limit", "tasp_test_skip_gemv_copies",
+            "tasp_test_set_wait_limit", "tasp_test_skip_gemv_copies", "tasp_spectral_layer",
             "tasp_last_error",
             "tasp_version")
 
@@ -95,6 +95,7 @@ def load(path: str = LIB_PATH):
         "tasp_mask_select_qheads": (c_int32, [POINTER(ModelDesc), POINTER(MaskDesc), P, P, P, P, P, P, P]),
         "tasp_set_memory_limit": (c_int32, [c_int64]),
         "tasp_test_set_wait_limit": (c_int32, [c_int64]),
+        "tasp_spectral_layer": (c_int32, [P, c_int32, P, P, P, P]),
         "tasp_test_skip_gemv_copies": (c_int32, [c_int32]),
         "tasp_dispatch": (c_int32, [P, c_int32, c_float, POINTER(c_int32)]),
         "tasp_plan_layer_qheads": (c_int32, [P, c_int32, POINTER(c_int32)]),
@@ -253,6 +254,30 @@ def dispatch(probs, tau: float = 0.85) -> int:
 def set_memory_limit(nbytes: int):
     """Cap the device memory of the library's arenas (0 = no cap)."""
     _check(load().tasp_set_memory_limit(int(nbytes)))
+
+
+SPECTRAL_FEATURES = ("alpha", "r_eff", "spectral_norm", "setol", "lambda_min", "ks")
+
+
+def spectral_layer(shape, layer: int, stream=None, phase_ms=None):
+    """Spectral descriptors of every candidate unit of one layer on the device: (features
+    [H_q + df / chan_unit][6] in SPECTRAL_FEATURES order, eigenvalues per block, descending).
+    ``phase_ms`` (a float64 array of 4) receives the device time of the block generation,
+    Gram matrices, eigensolver and statistics steps."""
+    nh, nc = 4 * shape.dh, 3 * shape.chan_unit
+    nu = shape.df // shape.chan_unit
+    feat = np.zeros((shape.Hq + nu, len(SPECTRAL_FEATURES)), np.float64)
+    lam = np.zeros(shape.Hq * nh + nu * nc, np.float64)
+    md = model_desc(shape)
+    ph = phase_ms.ctypes.data if phase_ms is not None else None
+    _check(load().tasp_spectral_layer(ctypes.byref(md), layer, feat.ctypes.data, lam.ctypes.data, ph,
+                                      _stream_ptr(stream)))
+    blocks, o = [], 0
+    for i in range(shape.Hq + nu):
+        n = nh if i < shape.Hq else nc
+        blocks.append(lam[o:o + n])
+        o += n
+    return feat, blocks
 
 
 def test_set_wait_limit(cycles: int):
