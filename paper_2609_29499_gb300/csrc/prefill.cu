@@ -34,14 +34,13 @@ namespace {
 using namespace tc;
 
 // ------------------------------------------------------------------ GEMM
-// Persistent GEMM on the 5th-generation tensor cores: one CTA per SM walks 128 x 256 output
-// tiles (M fastest, so the CTAs in flight share weight tiles in L2), with two 256-column
-// TMEM accumulators: the MMA warp fills one while the epilogue warps drain the other.
+// Persistent GEMM on the 5th-generation tensor cores: one CTA per SM walks 128 x BN output
+// tiles (M fastest, so the CTAs in flight share weight tiles in L2), with two BN-column TMEM
+// accumulators: the MMA warp fills one while the epilogue warps drain the other. BN = 256,
+// or 128 when 256-column tiles would not fill one wave of SMs (short prompts).
 constexpr int BM = 128, BN = 256, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
 constexpr int GEMM_THREADS = 192;
-constexpr uint32_t IDESC = idesc_f16(BM, BN);
 
 enum EpiMode { EP_STORE = 0, EP_RESID = 1, EP_SWIGLU = 2 };
 
@@ -129,15 +128,25 @@ __device__ __forceinline__ void gemm_epi32(const GemmArgs& g, int row, int nb, c
 }
 
 // Warp 0 streams the A (activation) and B (weight) k-blocks of all the CTA's tiles through a
-// 4-stage TMA ring that runs on across tile boundaries; warp 1 issues tcgen05.mma; warps 2-5
-// read an accumulator with tcgen05.ld and run the epilogue.
-constexpr int PG_STAGES = 4;
-constexpr int PG_STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int PG_SMEM = PG_STAGES * PG_STAGE_BYTES + 1024;
+// TMA ring (4 stages at BN = 256, 6 at BN = 128) that runs on across tile boundaries; warp 1
+// issues tcgen05.mma; warps 2-5 read an accumulator with tcgen05.ld and run the epilogue.
+template <int BNT>
+struct PgCfg {
+    static constexpr int B_BYTES = BNT * BK * 2;
+    static constexpr int STAGES = BNT == 256 ? 4 : 6;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024;
+    static constexpr uint32_t IDESC = idesc_f16(BM, BNT);
+    static constexpr uint32_t TMEM_COLS = 2 * BNT;
+};
 
+template <int BNT>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const GemmArgs g) {
+    using C = PgCfg<BNT>;
+    constexpr int BN = BNT, PG_STAGES = C::STAGES, PG_STAGE_BYTES = C::STAGE_BYTES;
+    constexpr uint32_t IDESC = C::IDESC;
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t bar_full[PG_STAGES], bar_empty[PG_STAGES], acc_full[2], acc_empty[2];
@@ -162,7 +171,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
-                     "r"(512)
+                     "r"(C::TMEM_COLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -207,7 +216,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                         const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
                         asm volatile(
                             "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256u * a),
+                            " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + (uint32_t)BN * a),
                             "l"(sw128_desc(sa + kk * 32)), "l"(sw128_desc(sb + kk * 32)), "r"(IDESC), "r"(accum)
                             : "memory");
                     }
@@ -240,7 +249,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                       "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
                       "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
                       "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-                    : "r"(tmem + ((uint32_t)(32 * q) << 16) + 256u * a + (uint32_t)c0));
+                    : "r"(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)BN * a + (uint32_t)c0));
                 asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
                 if (row < g.M) gemm_epi32(g, row, n0 + c0, r);
             }
@@ -253,7 +262,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     fence_before();
     __syncthreads();
     fence_after();
-    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TMEM_COLS) : "memory");
 }
 
 // ------------------------------------------------------------------ elementwise kernels
@@ -920,19 +930,29 @@ int launch_gemm(const __half* A, int lda, int M, const __half* B, int ldb, int N
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
+    // 128-column tiles when 256-column ones would leave SMs of the one wave idle
+    const int mt = (M + BM - 1) / BM;
+    const bool narrow = mt * ((N + 255) / 256) < di.sms;
+    const int bn = narrow ? 128 : 256;
     CUtensorMap ta, tb;
     if ((rc = make_map(&ta, A, M, K, lda, BM))) return rc;
-    if ((rc = make_map(&tb, B, N, K, ldb, BN))) return rc;
+    if ((rc = make_map(&tb, B, N, K, ldb, bn))) return rc;
     ga.vec = ga.mode == EP_SWIGLU ? ((reinterpret_cast<uintptr_t>(ga.hout) & 15) == 0 && ga.ldh % 8 == 0)
                                   : ((reinterpret_cast<uintptr_t>(ga.out) & 15) == 0 && ga.ldo % 4 == 0);
     ga.vec = ga.vec && (reinterpret_cast<uintptr_t>(ga.scale) & 15) == 0;
     static bool attr = false;
     if (!attr) {
-        TASP_CUDA(cudaFuncSetAttribute(gemm_persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, PG_SMEM));
+        TASP_CUDA(cudaFuncSetAttribute(gemm_persist_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       PgCfg<256>::SMEM));
+        TASP_CUDA(cudaFuncSetAttribute(gemm_persist_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       PgCfg<128>::SMEM));
         attr = true;
     }
-    const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-    gemm_persist_kernel<<<std::min(tiles, di.sms), GEMM_THREADS, PG_SMEM, s>>>(ta, tb, ga);
+    const int tiles = mt * ((N + bn - 1) / bn);
+    if (narrow)
+        gemm_persist_kernel<128><<<std::min(tiles, di.sms), GEMM_THREADS, PgCfg<128>::SMEM, s>>>(ta, tb, ga);
+    else
+        gemm_persist_kernel<256><<<std::min(tiles, di.sms), GEMM_THREADS, PgCfg<256>::SMEM, s>>>(ta, tb, ga);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }
