@@ -211,10 +211,11 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
         ops.push_back(op);
     };
     // groupwise store: the row's BF16 scale of each column group of `cols` input columns
-    auto set_groups = [&](Params& q, const uint16_t* gs, int cols) {
+    auto set_groups = [&](Params& q, const uint16_t* gs, int cols, int gld) {
         if (!sh.qg) return;
         q.gscale = gs;
         q.gcols = cols / sh.qg;
+        q.gld = gld;
         int sft = 0;
         while ((16 << sft) < sh.qg) ++sft;
         q.gshift = sft;
@@ -252,7 +253,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
         p.g = sh.g();
         p.dh = sh.dh;
         p.blk_role = lp.blk_role;
-        set_groups(p, lp.qkv_g, sh.d);
+        set_groups(p, lp.qkv_g, sh.d, lp.qkv_gld);
         p.err = bv.err;
         gemv(K_QKV, M_QKV, p);
         // K2: split-KV attention over the retained KV heads of every session
@@ -307,7 +308,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             o.act_stride = bv.q_stride;
             o.resid_out = bv.x;
             o.x_stride = bv.x_stride;
-            set_groups(o, lp.o_g, lp.o_K);
+            set_groups(o, lp.o_g, lp.o_K, lp.o_gld);
             o.err = bv.err;
             gemv(K_O, M_O, o);
         }
@@ -329,7 +330,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             gu.eps = sh.eps;
             gu.h_out = bv.h;
             gu.h_stride = bv.h_stride;
-            set_groups(gu, lp.gu_g, sh.d);
+            set_groups(gu, lp.gu_g, sh.d, lp.gu_gld);
             gu.err = bv.err;
             gemv(K_GU, M_GU, gu);
             // K5: down projection + residual
@@ -347,7 +348,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             dn.x_stride = bv.x_stride;
             dn.hidden_out = last ? t.hidden_out : nullptr;
             dn.hid_stride = sh.d;
-            set_groups(dn, lp.dn_g, lp.dn_K);
+            set_groups(dn, lp.dn_g, lp.dn_K, lp.dn_gld);
             dn.err = bv.err;
             gemv(K_DOWN, M_DOWN, dn);
         } else if (last && t.hidden_out) {

@@ -76,8 +76,9 @@ struct Params {
     const int* pos[MAXNB];
     int g, dh;
     const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
-    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gcols] (single-vector kernels only)
+    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gld] (single-vector kernels only)
     int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
+    int gld;                  // row stride of gscale (elements)
     float* h_out;          // GU: SiLU(gate) * up, stride h_stride
     int64_t h_stride;
     float* logits;         // LM: stride logit_stride

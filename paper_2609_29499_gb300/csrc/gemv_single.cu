@@ -49,8 +49,10 @@ struct GemvParams {
     const int* pos;
     int g, dh;
     const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
-    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gcols] (NULL = per-row only)
+    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gld] (NULL = per-row only)
     int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
+    int gld;                  // row stride of gscale (elements)
+    int gstage;               // the producer copies each row's scale row into the stage (gld a multiple of 8)
     float* h_out;
     float* logits;
     int* err;       // device error word (bounded waits that gave up)
@@ -364,7 +366,7 @@ __device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
 template <int R, int XC, bool GS>
 __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC>& xd,
                                        int nchunks, int tid, float (&acc)[R], const uint16_t* const (&grow)[R],
-                                       int gshift) {
+                                       int gshift, const uint16_t* __restrict__ gstage, int gld) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
@@ -380,7 +382,11 @@ __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld
                     sl = dp4a_su(wd[k], xd.lo[j][k], sl);
                 }
                 float xsc = xd.scale[j];
-                if constexpr (GS) xsc *= __uint_as_float((uint32_t)__ldg(grow[r] + (c >> gshift)) << 16);
+                if constexpr (GS) {
+                    // the row's scale of this chunk's column group: staged with the weights, or global
+                    const uint16_t sv = gstage ? gstage[r * gld + (c >> gshift)] : __ldg(grow[r] + (c >> gshift));
+                    xsc *= __uint_as_float((uint32_t)sv << 16);
+                }
                 acc[r] = fmaf(__int2float_rn(sh * 256 + sl), xsc, acc[r]);
             }
         }
@@ -511,10 +517,10 @@ __device__ __forceinline__ void epilogue(const GemvParams& p, const float (*red)
 struct GemvSmem {
     int x_bytes, stage_bytes, nstages, total;
 };
-__host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap) {
+__host__ __device__ inline GemvSmem gemv_smem(int nchunks, int F, int R, int ld, int cap, int gscale_bytes = 0) {
     GemvSmem g;
     g.x_bytes = 0;  // the activation slices are read from global memory
-    g.stage_bytes = ((R * ld) + 127) & ~127;
+    g.stage_bytes = ((R * ld + R * gscale_bytes) + 127) & ~127;  // weight rows, then their scale rows
     const int bar_bytes = (2 * MAX_STAGES + 2 * NRB) * 8 + 16;
     int ns = (cap - g.x_bytes - bar_bytes) / g.stage_bytes;
     g.nstages = ns > MAX_STAGES ? MAX_STAGES : ns;
@@ -529,7 +535,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     __shared__ float stat[CW];
     __shared__ int abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    const int gsb = GS && p.gstage ? p.gld * 2 : 0;  // bytes of one staged scale row
+    const GemvSmem L = gemv_smem(p.nchunks, MODE == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap, gsb);
     const int NS = L.nstages;
     uint8_t* stages = sm + L.x_bytes;
     const uint32_t full0 = smem_u32(stages + NS * L.stage_bytes);
@@ -563,10 +570,15 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
             for (int gi = g0, i = 0; gi < g1; ++gi, ++i) {
                 if (i >= NS) mbar_wait(empty0 + 8 * s, ph ^ 1, &abort_flag, p.err, p.wait_limit);
                 const int nrow = min(R, p.rows - gi * R);
-                mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * p.ld));
-                for (int r = 0; r < nrow; ++r)
+                mbar_expect_tx(full0 + 8 * s, (uint32_t)(nrow * (p.ld + gsb)));
+                for (int r = 0; r < nrow; ++r) {
                     bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)r * p.ld),
                              row_ptr<MODE>(p, gi * R + r), (uint32_t)p.ld, full0 + 8 * s);
+                    if (GS && gsb)  // the row's group scales, behind the stage's weight rows
+                        bulk_g2s(smem_u32(stages + (size_t)s * L.stage_bytes + (size_t)R * p.ld + (size_t)r * gsb),
+                                 p.gscale + (size_t)panel_row<MODE>(p, gi * R + r) * p.gld, (uint32_t)gsb,
+                                 full0 + 8 * s);
+                }
                 if (++s == NS) {
                     s = 0;
                     ph ^= 1;
@@ -660,7 +672,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
                 if (w >= p.rows) w = 0;  // padding row of a ragged last group: never stored
                 grow[r] = GS ? p.gscale + (size_t)panel_row<MODE>(p, w) * p.gcols : nullptr;
             }
-            dot_i8<R, XC, GS>(st, (int)p.ld, xd, p.nchunks, tid, v, grow, p.gshift);
+            dot_i8<R, XC, GS>(st, (int)p.ld, xd, p.nchunks, tid, v, grow, p.gshift,
+                              GS && gsb ? reinterpret_cast<const uint16_t*>(st + (size_t)R * p.ld) : nullptr, p.gld);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
@@ -779,7 +792,9 @@ int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
         }
         p.smem_cap = it->second;
     }
-    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap);
+    // group scales ride in the stage when their rows are 16-byte multiples (the plans pad them)
+    p.gstage = p.gscale && p.gld % 8 == 0 && (reinterpret_cast<uintptr_t>(p.gscale) & 15) == 0 ? 1 : 0;
+    const GemvSmem L = gemv_smem(p.nchunks, mode == M_LM ? 2 : 4, R, (int)p.ld, p.smem_cap, p.gstage ? p.gld * 2 : 0);
     if (L.nstages < 2) return fail(TASP_EUNSUP, "row or activation vector too long for the shared-memory ring");
     const int NG = (p.rows + R - 1) / R;
     const int grid = std::max(1, std::min(NG, di.sms));
@@ -819,6 +834,7 @@ int launch_gemv_single(int mode, const gemv::Params& q, cudaStream_t s) {
     p.gscale = q.gscale;
     p.gcols = q.gcols;
     p.gshift = q.gshift;
+    p.gld = q.gld;
     p.h_out = q.h_out;
     p.logits = q.logits;
     return gemv1::launch_gemv(mode, p, q.err, s);

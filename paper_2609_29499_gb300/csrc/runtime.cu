@@ -119,6 +119,7 @@ struct Layout {
 };
 
 static int round16(int v) { return (v + 15) & ~15; }
+static int round8(int v) { return (v + 7) & ~7; }
 
 // ---------------------------------------------------------------- store registry
 static std::mutex g_mu;
@@ -282,6 +283,11 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
             lp.gu_w = ls.gu; lp.gu_s = ls.gu_s;
             lp.dn_w = ls.down; lp.dn_s = ls.down_s; lp.dn_ld = sh.df;
             lp.qkv_g = ls.qkv_g; lp.o_g = ls.o_g; lp.gu_g = ls.gu_g; lp.dn_g = ls.down_g;
+            if (sh.qg) {
+                lp.qkv_gld = lp.gu_gld = d / sh.qg;
+                lp.o_gld = sh.Hq * dh / sh.qg;
+                lp.dn_gld = sh.df / sh.qg;
+            }
         }
         return TASP_OK;
     }
@@ -293,9 +299,9 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
     for (int l = 0; l < sh.L; ++l) {
         const LayerPlan& lp = p.layers[l];
         const size_t ol = round16(lp.o_K), dl = round16(lp.dn_K);
-        if (G) {  // group scales in panel order, and the column-group maps of O / down
-            lay.add((size_t)lp.qkv_rows * (d / G) * 2); lay.add((size_t)lp.gu_rows * (d / G) * 2);
-            lay.add((size_t)d * (lp.o_K / G) * 2); lay.add((size_t)d * (lp.dn_K / G) * 2);
+        if (G) {  // group scales in panel order (rows padded to 16 bytes), and the column-group maps of O / down
+            lay.add((size_t)lp.qkv_rows * round8(d / G) * 2); lay.add((size_t)lp.gu_rows * round8(d / G) * 2);
+            lay.add((size_t)d * round8(lp.o_K / G) * 2); lay.add((size_t)d * round8(lp.dn_K / G) * 2);
             lay.add((size_t)(lp.o_K / G) * 4); lay.add((size_t)(lp.dn_K / G) * 4);
         }
         if (ragged(lp)) {
@@ -356,18 +362,26 @@ static int build_plan(Plan& p, const MaskSel& sel, int panel_mode, bool all_keep
             std::vector<int32_t> cgo, cgd;
             for (size_t k = 0; k < (size_t)lp.o_K; k += G) cgo.push_back(ho[k] / G);
             for (size_t k = 0; k < (size_t)lp.dn_K; k += G) cgd.push_back(lp.keep_chans[k] / G);
-            uint16_t* gq = (uint16_t*)p.arena.take((size_t)lp.qkv_rows * (d / G) * 2);
-            uint16_t* gg = (uint16_t*)p.arena.take((size_t)lp.gu_rows * (d / G) * 2);
-            uint16_t* go = (uint16_t*)p.arena.take((size_t)d * (lp.o_K / G) * 2);
-            uint16_t* gd = (uint16_t*)p.arena.take((size_t)d * (lp.dn_K / G) * 2);
+            // scale rows padded to 16 bytes (zeros), so that a GEMV stage can take them by bulk copy
+            lp.qkv_gld = lp.gu_gld = round8(d / G);
+            lp.o_gld = round8(lp.o_K / G);
+            lp.dn_gld = round8(lp.dn_K / G);
+            uint16_t* gq = (uint16_t*)p.arena.take((size_t)lp.qkv_rows * lp.qkv_gld * 2);
+            uint16_t* gg = (uint16_t*)p.arena.take((size_t)lp.gu_rows * lp.gu_gld * 2);
+            uint16_t* go = (uint16_t*)p.arena.take((size_t)d * lp.o_gld * 2);
+            uint16_t* gd = (uint16_t*)p.arena.take((size_t)d * lp.dn_gld * 2);
+            TASP_CUDA(cudaMemsetAsync(gq, 0, (size_t)lp.qkv_rows * lp.qkv_gld * 2, s));
+            TASP_CUDA(cudaMemsetAsync(gg, 0, (size_t)lp.gu_rows * lp.gu_gld * 2, s));
+            TASP_CUDA(cudaMemsetAsync(go, 0, (size_t)d * lp.o_gld * 2, s));
+            TASP_CUDA(cudaMemsetAsync(gd, 0, (size_t)d * lp.dn_gld * 2, s));
             int32_t* dgo = (int32_t*)p.arena.take(cgo.size() * 4);
             int32_t* dgd = (int32_t*)p.arena.take(cgd.size() * 4);
             if (cgo.size()) TASP_CUDA(cudaMemcpyAsync(dgo, cgo.data(), cgo.size() * 4, cudaMemcpyHostToDevice, s));
             if (cgd.size()) TASP_CUDA(cudaMemcpyAsync(dgd, cgd.data(), cgd.size() * 4, cudaMemcpyHostToDevice, s));
-            if ((rc = gather_u16_rows(gq, ls.qkv_g, dq, lp.qkv_rows, d / G, s))) break;
-            if ((rc = gather_u16_rows(gg, ls.gu_g, dg, lp.gu_rows, d / G, s))) break;
-            if ((rc = gather_u16_cols(go, ls.o_g, sh.Hq * dh / G, dgo, d, lp.o_K / G, s))) break;
-            if ((rc = gather_u16_cols(gd, ls.down_g, sh.df / G, dgd, d, lp.dn_K / G, s))) break;
+            if ((rc = gather_u16_rows(gq, lp.qkv_gld, ls.qkv_g, dq, lp.qkv_rows, d / G, s))) break;
+            if ((rc = gather_u16_rows(gg, lp.gu_gld, ls.gu_g, dg, lp.gu_rows, d / G, s))) break;
+            if ((rc = gather_u16_cols(go, lp.o_gld, ls.o_g, sh.Hq * dh / G, dgo, d, lp.o_K / G, s))) break;
+            if ((rc = gather_u16_cols(gd, lp.dn_gld, ls.down_g, sh.df / G, dgd, d, lp.dn_K / G, s))) break;
             // the host vectors above die at the end of this block: wait for their copies
             cudaError_t ge = cudaStreamSynchronize(s);
             if (ge != cudaSuccess) { rc = cuda_fail(ge, "group scale packing"); break; }
@@ -1136,12 +1150,15 @@ int tasp_plan_export(const tasp_plan* plan, int32_t layer, int32_t item, void* h
             if (!sh.qg) return fail(TASP_EINVAL, "the store has no group scales");
             const uint16_t* src = item == TASP_EXPORT_QKV_G ? lp.qkv_g : item == TASP_EXPORT_O_G ? lp.o_g
                                 : item == TASP_EXPORT_GU_G ? lp.gu_g : lp.dn_g;
-            const size_t n = item == TASP_EXPORT_QKV_G ? (size_t)lp.qkv_rows * (d / sh.qg)
-                           : item == TASP_EXPORT_O_G ? d * (size_t)(lp.o_K / sh.qg)
-                           : item == TASP_EXPORT_GU_G ? (size_t)lp.gu_rows * (d / sh.qg)
-                           : d * (size_t)(lp.dn_K / sh.qg);
-            if (int rc = need(n * 2)) return rc;
-            if (n) TASP_CUDA(cudaMemcpy(h_dst, src, n * 2, cudaMemcpyDeviceToHost));
+            const int gld = item == TASP_EXPORT_QKV_G ? lp.qkv_gld : item == TASP_EXPORT_O_G ? lp.o_gld
+                          : item == TASP_EXPORT_GU_G ? lp.gu_gld : lp.dn_gld;
+            const size_t rows = item == TASP_EXPORT_QKV_G ? (size_t)lp.qkv_rows : item == TASP_EXPORT_GU_G ? (size_t)lp.gu_rows
+                                                                                                          : (size_t)d;
+            const size_t cols = item == TASP_EXPORT_QKV_G || item == TASP_EXPORT_GU_G ? (size_t)(d / sh.qg)
+                              : item == TASP_EXPORT_O_G ? (size_t)(lp.o_K / sh.qg) : (size_t)(lp.dn_K / sh.qg);
+            if (int rc = need(rows * cols * 2)) return rc;
+            if (rows * cols)
+                TASP_CUDA(cudaMemcpy2D(h_dst, cols * 2, src, (size_t)gld * 2, cols * 2, rows, cudaMemcpyDeviceToHost));
             return TASP_OK;
         }
         case TASP_EXPORT_KEEP_QHEADS: {

@@ -158,16 +158,17 @@ __global__ void gather_cols_kernel(int8_t* dst, int ld_dst, const int8_t* src, i
     for (int j = threadIdx.x; j < ld_dst; j += blockDim.x) d[j] = (j < Kc) ? s[cmap[j]] : (int8_t)0;
 }
 
-__global__ void gather_u16_rows_kernel(uint16_t* dst, const uint16_t* src, const int32_t* map, int cols) {
+__global__ void gather_u16_rows_kernel(uint16_t* dst, int ld_dst, const uint16_t* src, const int32_t* map, int cols) {
     const int r = blockIdx.x;
     const uint16_t* s = src + (size_t)map[r] * cols;
-    uint16_t* d = dst + (size_t)r * cols;
+    uint16_t* d = dst + (size_t)r * ld_dst;
     for (int j = threadIdx.x; j < cols; j += blockDim.x) d[j] = s[j];
 }
 
-__global__ void gather_u16_cols_kernel(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int ncols) {
+__global__ void gather_u16_cols_kernel(uint16_t* dst, int ld_dst, const uint16_t* src, int ld_src, const int32_t* cmap,
+                                       int ncols) {
     const int r = blockIdx.x;
-    for (int j = threadIdx.x; j < ncols; j += blockDim.x) dst[(size_t)r * ncols + j] = src[(size_t)r * ld_src + cmap[j]];
+    for (int j = threadIdx.x; j < ncols; j += blockDim.x) dst[(size_t)r * ld_dst + j] = src[(size_t)r * ld_src + cmap[j]];
 }
 
 __global__ void gather_f32_kernel(float* dst, const float* src, const int32_t* map, int n) {
@@ -305,17 +306,18 @@ int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const in
     return TASP_OK;
 }
 
-int gather_u16_rows(uint16_t* dst, const uint16_t* src, const int32_t* map, int rows, int cols, cudaStream_t s) {
+int gather_u16_rows(uint16_t* dst, int ld_dst, const uint16_t* src, const int32_t* map, int rows, int cols,
+                    cudaStream_t s) {
     if (rows == 0 || cols == 0) return TASP_OK;
-    gather_u16_rows_kernel<<<rows, 128, 0, s>>>(dst, src, map, cols);
+    gather_u16_rows_kernel<<<rows, 128, 0, s>>>(dst, ld_dst, src, map, cols);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }
 
-int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows, int ncols,
-                    cudaStream_t s) {
+int gather_u16_cols(uint16_t* dst, int ld_dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows,
+                    int ncols, cudaStream_t s) {
     if (rows == 0 || ncols == 0) return TASP_OK;
-    gather_u16_cols_kernel<<<rows, 128, 0, s>>>(dst, src, ld_src, cmap, ncols);
+    gather_u16_cols_kernel<<<rows, 128, 0, s>>>(dst, ld_dst, src, ld_src, cmap, ncols);
     TASP_CUDA(cudaGetLastError());
     return TASP_OK;
 }

@@ -129,6 +129,7 @@ struct LayerPlan {
     // grouped store only: BF16 group scales in panel order, [rows][K / qg] (row stride gq_ld
     // for qkv / gu, o_K / qg and dn_K / qg for the column-compacted O / down panels)
     const uint16_t *qkv_g = nullptr, *gu_g = nullptr, *o_g = nullptr, *dn_g = nullptr;
+    int qkv_gld = 0, gu_gld = 0, o_gld = 0, dn_gld = 0;  // their row strides (elements)
 };
 
 // FP16 copies of a layer's panels (row strides padded to 8 elements) for the prefill GEMMs.
@@ -217,11 +218,12 @@ int gather_rows(int8_t* dst, const int8_t* src, const int32_t* map, int rows, in
 int gather_cols(int8_t* dst, int ld_dst, const int8_t* src, int ld_src, const int32_t* cmap, int rows, int Kc,
                 cudaStream_t s);
 int gather_f32(float* dst, const float* src, const int32_t* map, int n, cudaStream_t s);
-// rows of a [*][cols] uint16 matrix (dst row r = src row map[r])
-int gather_u16_rows(uint16_t* dst, const uint16_t* src, const int32_t* map, int rows, int cols, cudaStream_t s);
-// columns of a [rows][ld_src] uint16 matrix (dst column j = src column cmap[j], j < ncols)
-int gather_u16_cols(uint16_t* dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows, int ncols,
+// rows of a [*][cols] uint16 matrix (dst row r, stride ld_dst, = src row map[r])
+int gather_u16_rows(uint16_t* dst, int ld_dst, const uint16_t* src, const int32_t* map, int rows, int cols,
                     cudaStream_t s);
+// columns of a [rows][ld_src] uint16 matrix (dst [rows][ld_dst] column j = src column cmap[j], j < ncols)
+int gather_u16_cols(uint16_t* dst, int ld_dst, const uint16_t* src, int ld_src, const int32_t* cmap, int rows,
+                    int ncols, cudaStream_t s);
 
 // attention.cu
 constexpr int MAX_BATCH = 4;   // sessions of one plan that share each weight pass
