@@ -51,6 +51,8 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=3, choices=[1, 2, 3])
     ap.add_argument("--dense", action="store_true", help="time the dense fallback plan instead of the mask")
+    ap.add_argument("--mask", choices=["groups", "qheads"], default="groups",
+                    help="decode: whole GQA groups (the benchmark masks) or query-head candidates with KV closure")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", choices=["decode", "prefill", "mixed", "spectral"], default="decode",
@@ -181,7 +183,7 @@ def block_bounds(K: int, n: int = 5) -> list:
 
 def kv_bytes(plan_dims, dh, T):
     """KV bytes of one step at context T (keys+values read for T positions, one position written)."""
-    m = sum(mk for mk, _ in plan_dims)
+    m = sum(dm[0] for dm in plan_dims)
     return m * 2 * T * dh * 2 + m * 2 * dh * 2
 
 
@@ -189,18 +191,20 @@ def gemv_bytes(shape, plan_dims):
     """Algorithmic bytes per launch kind, summed over layers (weights, scales, activations in/out)."""
     d, dh, g = shape.d, shape.dh, shape.Hq // shape.Hkv
     b = {"qkv": 0, "o_proj": 0, "gate_up": 0, "down": 0}
-    for m_kv, c in plan_dims:
-        rows = m_kv * (g + 2) * dh
-        b["qkv"] += rows * d + rows * 4 + d * 4 + d * 4 + m_kv * g * dh * 4 + m_kv * 2 * dh * 2
+    for dm in plan_dims:  # (kept KV groups, kept channels[, kept query heads])
+        m_kv, c = dm[0], dm[1]
+        m_q = dm[2] if len(dm) > 2 else m_kv * g
+        rows = (m_q + 2 * m_kv) * dh
+        b["qkv"] += rows * d + rows * 4 + d * 4 + d * 4 + m_q * dh * 4 + m_kv * 2 * dh * 2
         if m_kv:
-            b["o_proj"] += d * m_kv * g * dh + d * 4 + m_kv * g * dh * 4 + 2 * d * 4
+            b["o_proj"] += d * m_q * dh + d * 4 + m_q * dh * 4 + 2 * d * 4
         if c:
             b["gate_up"] += 2 * c * d + 2 * c * 4 + d * 4 + d * 4 + c * 4
             b["down"] += d * c + d * 4 + c * 4 + 2 * d * 4
         G = getattr(shape, "quant_group", 0)
         if G:  # BF16 group scales: 2 bytes per G weights
             b["qkv"] += 2 * rows * (d // G)
-            b["o_proj"] += 2 * d * (m_kv * g * dh // G)
+            b["o_proj"] += 2 * d * (m_q * dh // G)
             b["gate_up"] += 2 * 2 * c * (d // G)
             b["down"] += 2 * d * (c // G)
     b["lm_head"] = shape.vocab * d * 2 + d * 4 + shape.vocab * 4
@@ -208,7 +212,21 @@ def gemv_bytes(shape, plan_dims):
 
 
 # ------------------------------------------------------------------ CPU oracle baseline
-def cpu_oracle_sample(shape, recipe, wl, n_steps, layers=(0, None), lm_rows=1024):
+def oracle_bench_mask(shape, recipe, qheads=False, dense=False):
+    """The oracle's compiled mask for the decode workload: whole GQA groups, or query-head
+    candidates with KV closure (or everything kept, for the dense fallback)."""
+    from oracle import maskc
+    if dense:
+        return maskc.all_keep(shape)
+    tg = synth.layer_target_u24(recipe.mask_seed, shape.L)
+    if qheads:
+        sc = synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.Hq + shape.n_chan_units)
+        return maskc.compile_mask_qheads(shape, sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi)
+    sc = synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.n_units)
+    return maskc.compile_mask(shape, sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi)
+
+
+def cpu_oracle_sample(shape, recipe, wl, n_steps, layers=(0, None), lm_rows=1024, qheads=False, dense=False):
     """Time the oracle's decode arithmetic on host cores for a bounded sample.
 
     Sample: the given layers of the masked model (weights regenerated and
@@ -216,17 +234,16 @@ def cpu_oracle_sample(shape, recipe, wl, n_steps, layers=(0, None), lm_rows=1024
     decode step each per timed step, plus a slice of LM-head rows; scaled to all
     layers and the full vocabulary. Returns (ms/token per step list, info).
     """
-    from oracle import forward, maskc, weights
-    sc = synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.n_units)
-    tg = synth.layer_target_u24(recipe.mask_seed, shape.L)
-    mask = maskc.compile_mask(shape, sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi)
+    from oracle import forward, weights
+    mask = oracle_bench_mask(shape, recipe, qheads, dense)
     layers = [l if l is not None else shape.L - 1 for l in layers]
     layers = sorted(set(layers))
     t0 = time.perf_counter()
     W, KV = [], []
     for l in layers:
         lq = weights.gen_layer(shape, l)
-        W.append(weights.dense_zeroed(shape, lq, mask.keep_groups[l], mask.keep_chans[l]))
+        W.append(weights.dense_zeroed(shape, lq, mask.keep_groups[l], mask.keep_chans[l],
+                                      keep_qheads=mask.qheads(shape, l)))
         KV.append(forward.prior_cache(shape, l, wl.kv_seed, wl.t_prior))
     lm = weights.lm_head_f32(shape, 0, lm_rows) if shape.vocab else None
     gf = weights.gamma_final(shape)
@@ -261,9 +278,10 @@ def cpu_oracle_sample(shape, recipe, wl, n_steps, layers=(0, None), lm_rows=1024
 def decode_config(wl, args, ratio, world):
     """The decode workload's config, the same on both arms: the prior context is the workload's
     (each timed step adds one token to it)."""
-    return {"workload": wl.name + ("_dense" if args.dense else ""),
+    qh = getattr(args, "mask", "groups") == "qheads" and not args.dense
+    return {"workload": wl.name + ("_dense" if args.dense else "") + ("_qheads" if qh else ""),
             "mask": "all-keep dense fallback" if args.dense else
-            f"greedy dependency-closed, active-FLOP ratio {ratio:.4f}",
+            f"greedy dependency-closed{' (query-head candidates)' if qh else ''}, active-FLOP ratio {ratio:.4f}",
             "context": wl.t_prior, "batch": 1, "parallelism": "replicas" if world > 1 else "single GPU",
             "l2": "inputs larger than L2 (each step streams the whole plan's weights)"}
 
@@ -274,14 +292,12 @@ def run_reference(args):
     if rank != 0:
         return
     wl, shape, recipe = workload(args)
-    per_step, info = cpu_oracle_sample(shape, recipe, wl, args.warmup + args.steps)
-    from oracle import maskc
+    qh = args.mask == "qheads"
+    per_step, info = cpu_oracle_sample(shape, recipe, wl, args.warmup + args.steps, qheads=qh, dense=args.dense)
     if args.dense:
         ratio = 1.0
     else:
-        m = maskc.compile_mask(shape, synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.n_units),
-                               synth.layer_target_u24(recipe.mask_seed, shape.L), recipe.budget, recipe.r_lo,
-                               recipe.r_hi)
+        m = oracle_bench_mask(shape, recipe, qh)
         ratio = m.info["total_flops"] / m.info["dense_flops"]
     timed = per_step[args.warmup:]
     v = float(np.mean(timed))
@@ -314,13 +330,17 @@ def run_ours(args):
     t0 = time.perf_counter()
     if args.dense:
         plan = tasp.Plan(shape, tasp.all_keep_mask())
+    elif args.mask == "qheads":  # query-head candidates with KV closure (Sec. 3.3, Table 1)
+        sc = synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.Hq + shape.n_chan_units)
+        tg = synth.layer_target_u24(recipe.mask_seed, shape.L)
+        plan = tasp.Plan(shape, tasp.greedy_qhead_mask(sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi))
     else:
         sc = synth.mask_scores_u32(recipe.mask_seed, shape.L, shape.n_units)
         tg = synth.layer_target_u24(recipe.mask_seed, shape.L)
         plan = tasp.Plan(shape, tasp.greedy_mask(sc, tg, recipe.budget, recipe.r_lo, recipe.r_hi))
     setup_s = time.perf_counter() - t0
     info = plan.info()
-    dims = [plan.layer_dims(l) for l in range(shape.L)]
+    dims = [plan.layer_dims(l) + (plan.layer_qheads(l),) for l in range(shape.L)]
     extra = 4
     e2e_steps = 0 if args.no_e2e else K
     sess = tasp.Session(plan, wl.t_prior + Wm + K + extra + e2e_steps + 1)
@@ -401,7 +421,7 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        per_step, cinfo = cpu_oracle_sample(shape, recipe, wl, 3)
+        per_step, cinfo = cpu_oracle_sample(shape, recipe, wl, 3, qheads=args.mask == "qheads", dense=args.dense)
         cinfo["value"] = round(float(np.mean(per_step)), 1)
         cinfo["unit"] = "ms/token"
         cpu = cinfo

@@ -53,6 +53,7 @@ struct GemvParams {
     int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
     int gld;                  // row stride of gscale (elements)
     int gstage;               // the producer copies each row's scale row into the stage (gld a multiple of 8)
+    float skew;               // start-order split: CTA b takes a share 1 + skew (1 - 2 b / (grid - 1)) of the rows
     float* h_out;
     float* logits;
     int* err;       // device error word (bounded waits that gave up)
@@ -544,8 +545,20 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
     const uint32_t rfull0 = empty0 + 8 * MAX_STAGES;
     const uint32_t rempty0 = rfull0 + 8 * NRB;
     const int NG = (p.rows + R - 1) / R;
-    const int g0 = (int)((int64_t)blockIdx.x * NG / gridDim.x);
-    const int g1 = (int)((int64_t)(blockIdx.x + 1) * NG / gridDim.x);
+    // CTAs start in block-index order (each takes the SM the previous kernel frees next), so a
+    // launch whose CTAs start spread out gives the later ones a smaller share: with shares
+    // 1 + skew (1 - 2 i / (G - 1)), CTA b starts at the prefix NG S(b) / G, S(k) = k (1 + skew)
+    // - skew k (k - 1) / (G - 1), S(G) = G. skew = 0: the even split, in integers. FP32 only:
+    // FP64 runs at a few operations per clock per SM on this part, microseconds per launch here.
+    auto start_of = [&](int b) -> int {
+        if (b >= (int)gridDim.x) return NG;
+        if (p.skew == 0.f || gridDim.x < 2) return (int)((int64_t)b * NG / gridDim.x);
+        const float G = (float)gridDim.x, k = (float)b, sg = p.skew;
+        const float S = k * (1.f + sg) - sg * k * (k - 1.f) / (G - 1.f);
+        return max(0, min(NG, (int)((float)NG * S / G)));
+    };
+    const int g0 = start_of(blockIdx.x);
+    const int g1 = start_of(blockIdx.x + 1);
 
     if (tid == 0) {
         abort_flag = 0;
@@ -764,9 +777,13 @@ int rows_per_stage(int mode, int64_t ld) {
 std::mutex g_attr_mu;
 std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 
+// Start-order skew of the row split per mode (see the kernel).
+constexpr float SKEW_QKV = 0.f, SKEW_O = 0.3f, SKEW_GU = 0.f, SKEW_DOWN = 0.f;
+
 int launch_gemv(int mode, GemvParams p, int* err, cudaStream_t s) {
     if (p.rows == 0) return TASP_OK;
     p.wait_limit = test_hooks::wait_limit(WAIT_LIMIT);
+    p.skew = mode == M_O ? SKEW_O : mode == M_GU ? SKEW_GU : mode == M_DOWN ? SKEW_DOWN : mode == M_QKV ? SKEW_QKV : 0.f;
     p.skip_copies = test_hooks::take_skip() ? 1 : 0;
     DevInfo di;
     int rc = device_info(di);
