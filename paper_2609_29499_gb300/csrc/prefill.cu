@@ -649,21 +649,25 @@ __global__ void __launch_bounds__(PA_WARPS * 32, 1) attn_prefill_kernel(const fl
 // ------------------------------------------------------------------ causal attention on tcgen05
 // One CTA: 128 queries of one kept head, head dim 128. Keys stream in tiles of 64:
 //  * warp 0 loads Q once and, per tile, the FP16 key tile and the transposed FP16 value tile
-//    (TMA, 128-byte swizzle) into a 2-stage ring;
+//    (TMA, 128-byte swizzle) into two 2-slot rings: a key slot is free again once S_j has
+//    been computed, a value slot once O += P_j V_j has, so the keys run a tile further ahead
+//    (in MMA order the enabling events come as K_j, V_{j-1}, K_{j+1}, V_j, ...);
 //  * warp 1 issues S_j = Q K_j^T (M 128, N 64) into one of two TMEM score buffers, and
-//    O += P_{j-1} V_{j-1} (M 128, N 128) into the TMEM output;
+//    O += P_{j-1} V_{j-1} (M 128, N 128) into the TMEM output, with P read from TMEM;
 //  * warps 2-5 own one query row per thread: they read S_j from TMEM, apply the causal mask,
 //    keep a running maximum that may lag the true one by up to 8 (log2 units; O in TMEM is
-//    rescaled only when it would lag more), write P_j = 2^(S - m) as FP16 into shared memory
-//    in the swizzled operand layout, and finally divide O by the running sum.
+//    rescaled only when it would lag more), write P_j = 2^(S - m) as packed FP16 pairs over
+//    the first 32 columns of S_j's buffer (the MMA's A operand), and finally divide O by the
+//    running sum.
+// The MMAs of a CTA run in issue order, so S_{j+2}, issued after O += P_j V_j, cannot
+// overwrite P_j before it is read. Without a shared-memory P tile a CTA takes 97 KB and two
+// fit on an SM (8 softmax warps, one CTA's softmax overlapping the other's MMAs).
 // Every wait is bounded and reports to the device error word.
 constexpr int AT_KT = 64;
 constexpr int AT_Q_BYTES = 128 * 128 * 2;
 constexpr int AT_K_BYTES = AT_KT * 128 * 2;
 constexpr int AT_VT_BYTES = 128 * AT_KT * 2;
-constexpr int AT_STAGE_BYTES = AT_K_BYTES + AT_VT_BYTES;
-constexpr int AT_P_BYTES = 128 * AT_KT * 2;
-constexpr int AT_SMEM = AT_Q_BYTES + 2 * AT_STAGE_BYTES + 2 * AT_P_BYTES + 1024;
+constexpr int AT_SMEM = AT_Q_BYTES + 2 * (AT_K_BYTES + AT_VT_BYTES) + 1024;
 constexpr uint32_t AT_TMEM_COLS = 256;  // S0 [0, 64), S1 [64, 128), O [128, 256)
 constexpr uint32_t IDESC_S = idesc_f16(128, AT_KT), IDESC_O = idesc_f16(128, 128);
 constexpr float AT_LAZY = 8.0f;
@@ -689,17 +693,27 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
         : "memory");
 }
 
-__global__ void __launch_bounds__(192, 1)
+// O += P V with the A operand (P, M 128 x K 16 as packed FP16 pairs, row = lane) in TMEM.
+__device__ __forceinline__ void mma_f16_tmem_a(uint32_t tmem_d, uint32_t tmem_a, uint64_t bd, uint32_t idesc,
+                                               uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "r"(tmem_a), "l"(bd), "r"(idesc), "r"(accum)
+        : "memory");
+}
+
+__global__ void __launch_bounds__(192, 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmVT, int T, int g, __half* O, int ldo, int* err,
                    const int16_t* __restrict__ oslot) {
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
     uint8_t* sq = sm;
-    uint8_t* sst = sm + AT_Q_BYTES;                     // stage s: K at +0 (two 8 KB halves), VT at +AT_K_BYTES
-    uint8_t* sp = sm + AT_Q_BYTES + 2 * AT_STAGE_BYTES;  // P buffer b at + b * AT_P_BYTES
-    __shared__ __align__(8) uint64_t bar_q, kv_full[2], kv_empty[2], s_full[2], s_empty[2], p_full[2], p_empty[2],
-        o_done;
+    uint8_t* sk = sm + AT_Q_BYTES;                       // key slot s at + s * AT_K_BYTES (two 8 KB halves)
+    uint8_t* sv = sm + AT_Q_BYTES + 2 * AT_K_BYTES;      // value slot s at + s * AT_VT_BYTES
+    __shared__ __align__(8) uint64_t bar_q, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full[2],
+        p_empty[2], o_done;
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -715,10 +729,11 @@ __global__ void __launch_bounds__(192, 1)
         mbar_init(B(bar_q), 1);
         mbar_init(B(o_done), 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(B(kv_full[i]), 1);
-            mbar_init(B(kv_empty[i]), 1);
+            mbar_init(B(k_full[i]), 1);
+            mbar_init(B(k_empty[i]), 1);
+            mbar_init(B(v_full[i]), 1);
+            mbar_init(B(v_empty[i]), 1);
             mbar_init(B(s_full[i]), 1);
-            mbar_init(B(s_empty[i]), 4);
             mbar_init(B(p_full[i]), 4);
             mbar_init(B(p_empty[i]), 1);
         }
@@ -740,20 +755,29 @@ __global__ void __launch_bounds__(192, 1)
             mbar_expect_tx(B(bar_q), AT_Q_BYTES);
             tma_load_2d(smem_u32(sq), &tmQ, 0, h * T + q0, B(bar_q));
             tma_load_2d(smem_u32(sq + AT_Q_BYTES / 2), &tmQ, 64, h * T + q0, B(bar_q));
+            auto load_v = [&](int j) {
+                const int s = j & 1;
+                if (j >= 2) mbar_wait(B(v_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
+                mbar_expect_tx(B(v_full[s]), AT_VT_BYTES);
+                tma_load_2d(smem_u32(sv + s * AT_VT_BYTES), &tmVT, j * AT_KT, jl * 128, B(v_full[s]));
+            };
             for (int j = 0; j < ntile; ++j) {
                 const int s = j & 1;
-                if (j >= 2) mbar_wait(B(kv_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
-                const uint32_t fb = B(kv_full[s]);
-                mbar_expect_tx(fb, AT_STAGE_BYTES);
-                uint8_t* st = sst + s * AT_STAGE_BYTES;
+                if (j >= 2) mbar_wait(B(k_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
+                const uint32_t fb = B(k_full[s]);
+                mbar_expect_tx(fb, AT_K_BYTES);
+                uint8_t* st = sk + s * AT_K_BYTES;
                 tma_load_2d(smem_u32(st), &tmK, 0, jl * T + j * AT_KT, fb);
                 tma_load_2d(smem_u32(st + AT_K_BYTES / 2), &tmK, 64, jl * T + j * AT_KT, fb);
-                tma_load_2d(smem_u32(st + AT_K_BYTES), &tmVT, j * AT_KT, jl * 128, fb);
+                if (j >= 1) load_v(j - 1);
             }
+            load_v(ntile - 1);
             // no copy may outlive the CTA
             mbar_wait(B(bar_q), 0, &abort_flag, err, false);
-            for (int j = max(0, ntile - 2); j < ntile; ++j)
-                mbar_wait(B(kv_full[j & 1]), (j >> 1) & 1, &abort_flag, err, false);
+            for (int j = max(0, ntile - 2); j < ntile; ++j) {
+                mbar_wait(B(k_full[j & 1]), (j >> 1) & 1, &abort_flag, err, false);
+                mbar_wait(B(v_full[j & 1]), (j >> 1) & 1, &abort_flag, err, false);
+            }
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---- MMA issuer
@@ -763,10 +787,11 @@ __global__ void __launch_bounds__(192, 1)
             for (int j = 0; j <= ntile; ++j) {
                 if (j < ntile) {  // S_j = Q K_j^T into score buffer j % 2
                     const int s = j & 1;
-                    mbar_wait(B(kv_full[s]), (j >> 1) & 1, &abort_flag, err);
-                    if (j >= 2) mbar_wait(B(s_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);
+                    // score buffer s is free: S_{j-2} was read and P_{j-2} consumed by O += P_{j-2} V_{j-2},
+                    // issued (after the softmax's p_full) before this MMA, and MMAs run in order
+                    mbar_wait(B(k_full[s]), (j >> 1) & 1, &abort_flag, err);
                     fence_after();
-                    const uint32_t kb = smem_u32(sst + s * AT_STAGE_BYTES);
+                    const uint32_t kb = smem_u32(sk + s * AT_K_BYTES);
 #pragma unroll
                     for (int blk = 0; blk < 2; ++blk)
 #pragma unroll
@@ -774,19 +799,20 @@ __global__ void __launch_bounds__(192, 1)
                             mma_f16(tmem + 64u * s, sw128_desc(qa + blk * (AT_Q_BYTES / 2) + kk * 32),
                                    sw128_desc(kb + blk * (AT_K_BYTES / 2) + kk * 32), IDESC_S, (blk | kk) ? 1u : 0u);
                     commit(B(s_full[s]));
+                    commit(B(k_empty[s]));
                 }
                 if (j >= 1) {  // O += P_{j-1} V_{j-1}
                     const int jp = j - 1, s = jp & 1;
                     mbar_wait(B(p_full[s]), (jp >> 1) & 1, &abort_flag, err);
+                    mbar_wait(B(v_full[s]), (jp >> 1) & 1, &abort_flag, err);
                     fence_after();
-                    const uint32_t pa = smem_u32(sp + s * AT_P_BYTES);
-                    const uint32_t vb = smem_u32(sst + s * AT_STAGE_BYTES + AT_K_BYTES);
+                    const uint32_t vb = smem_u32(sv + s * AT_VT_BYTES);
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_f16(tmem + 128u, sw128_desc(pa + kk * 32), sw128_desc(vb + kk * 32), IDESC_O,
-                               (jp > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < 4; ++kk)  // K 16 = 8 TMEM columns of packed pairs
+                        mma_f16_tmem_a(tmem + 128u, tmem + 64u * s + 8u * kk, sw128_desc(vb + kk * 32), IDESC_O,
+                                       (jp > 0 || kk > 0) ? 1u : 0u);
                     commit(B(p_empty[s]));
-                    commit(B(kv_empty[s]));
+                    commit(B(v_empty[s]));
                 }
             }
             commit(B(o_done));
@@ -804,19 +830,21 @@ __global__ void __launch_bounds__(192, 1)
             tmem_ld32(trow + 64u * s, v0);
             tmem_ld32(trow + 64u * s + 32u, v1);
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(B(s_empty[s]));
             float x[64];
             const int k0 = j * AT_KT;
-            float mt = -INFINITY;
+            const int kv = min(qi + 1, kend) - k0;  // keys k0 + c with c < kv are visible
 #pragma unroll
             for (int c = 0; c < 64; ++c) {
                 const float v = __uint_as_float(c < 32 ? v0[c] : v1[c - 32]);
-                const int k = k0 + c;
-                x[c] = (k > qi || k >= kend) ? -INFINITY : v;  // causal
-                mt = fmaxf(mt, x[c]);
+                x[c] = c < kv ? v : -INFINITY;  // causal
             }
+            float mx[8];  // the row maximum as a tree (independent chains instead of one of 64)
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                mx[i] = fmaxf(fmaxf(fmaxf(x[i], x[i + 8]), fmaxf(x[i + 16], x[i + 24])),
+                              fmaxf(fmaxf(x[i + 32], x[i + 40]), fmaxf(x[i + 48], x[i + 56])));
+            const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                   fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
             if (j == 0) {
                 m_run = mt;  // key 0 is visible to every row
             } else {
@@ -842,23 +870,21 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
             }
-            // P_j = 2^(S - m) in FP16 (<= 2^8 by the lag bound), row-sum in FP32
+            // P_j = 2^(S - m) in FP16 (<= 2^8 by the lag bound), row-sum in FP32 (8 partial sums)
             uint32_t pw[32];
-            float ls = 0.f;
+            float lsp[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) lsp[i] = 0.f;
 #pragma unroll
             for (int c = 0; c < 64; c += 2) {
                 const float p0 = exp2f(x[c] - m_run), p1 = exp2f(x[c + 1] - m_run);
-                ls += p0 + p1;
+                lsp[(c >> 1) & 7] += p0 + p1;
                 pw[c >> 1] = pack_h2(p0, p1);
             }
-            l_run += ls;
-            if (j >= 2) mbar_wait(B(p_empty[s]), ((j >> 1) - 1) & 1, &abort_flag, err);  // P buffer free
-            uint8_t* prow = sp + s * AT_P_BYTES + row * 128;
-#pragma unroll
-            for (int c = 0; c < 8; ++c)
-                *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) =
-                    make_uint4(pw[4 * c], pw[4 * c + 1], pw[4 * c + 2], pw[4 * c + 3]);
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
+            l_run += ((lsp[0] + lsp[1]) + (lsp[2] + lsp[3])) + ((lsp[4] + lsp[5]) + (lsp[6] + lsp[7]));
+            // S_j's commit covered every earlier MMA, so O += P_{j-2} V_{j-2} has read P_{j-2}
+            tmem_st32(trow + 64u * s, pw);  // P_j over the first 32 columns of S_j's buffer
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(B(p_full[s]));
