@@ -18,11 +18,13 @@
 // FP16 (each session scaled by a power of two so its largest entry is below 2^14; exact
 // rescaling). Persistent CTAs (three per SM) walk (128-row tile, K slice) units:
 //  * warp 0 streams 128 x 128 INT8 weight tiles and the 16 x 128 FP16 activation tile of
-//    the same K range with TMA (128-byte swizzle) into a 2-stage ring;
+//    the same K range with TMA (128-byte swizzle) into a 3-stage ring;
 //  * warps 2-5 convert each INT8 tile to FP16 (exact: v + 1152 is built in the FP16 bit
-//    pattern 0x6400 | (v ^ 0x80) and 1152 subtracted) into the MMA operand buffer;
-//  * warp 1 issues tcgen05.mma (M = 128, N = 16, K = 16) into one of two 16-column TMEM
-//    accumulators;
+//    pattern 0x6400 | (v ^ 0x80) and 1152 subtracted) in registers, one weight row per
+//    thread, and store it into tensor memory (row = TMEM lane, packed FP16 pairs);
+//  * warp 1 issues tcgen05.mma (M = 128, N = 16, K = 16) with the weights as the A operand
+//    read from tensor memory and the activations from shared memory, into one of two
+//    16-column TMEM accumulators;
 //  * warps 6-9 read the accumulator (tcgen05.ld) and store the unit's FP32 partial sums.
 // The BF16 LM head runs through the same kernel: TMA writes its weight tiles straight into the
 // MMA operand layout (no conversion) and the activations are BF16.
@@ -51,24 +53,28 @@ using namespace tc;
 constexpr int US = UNION_MAX;  // sessions per union step = MMA N
 constexpr int SK_BM = 128;     // weight rows per tile (MMA M)
 constexpr int SK_BK = 128;     // K (INT8 bytes) per stage
-constexpr int SK_NST = 2;   // INT8 + activation stages
-constexpr int SK_NA = 1;    // FP16 operand buffer
+constexpr int SK_NST = 3;       // INT8 + activation stages
+constexpr int SK_NST_BF16 = 2;  // BF16 weight + activation stages (the LM head)
+constexpr int SK_NA = 1;        // FP16 operand buffers in tensor memory
 // CTAs per SM: each small MMA costs its issuing thread ~90 ns, so three CTAs (three issuing
-// threads, each with a 2-stage ring and one operand buffer) keep the tensor core busier than
-// one CTA with deep rings (measured: 1, 2, 3 CTAs per SM -> 523, 618, 711 tokens/s)
+// threads) keep the tensor core busier than one CTA with deep rings (measured with the FP16
+// operand in shared memory: 1, 2, 3 CTAs per SM -> 523, 618, 711 tokens/s)
 constexpr int SK_CTAS_PER_SM = 3;
+// Tensor memory of an INT8 CTA: accumulators at columns 0 and 16, operand buffer b (128 K
+// values = 64 columns of FP16 pairs) at 64 + 64 b; a BF16 CTA needs the accumulators only.
+constexpr uint32_t SK_TMEM_I8 = 128, SK_TMEM_BF16 = 32;
+static_assert(64 + 64 * SK_NA <= SK_TMEM_I8 && SK_CTAS_PER_SM * SK_TMEM_I8 <= 512, "tensor memory of the skinny GEMM");
 constexpr int SK_W_BYTES = SK_BM * SK_BK;      // INT8 tile
 constexpr int SK_X_BYTES = US * SK_BK * 2;     // FP16 activation tile (two 64-column boxes)
-constexpr int SK_A_HALF = SK_BM * 64 * 2;      // FP16 operand tile of 64 columns
-constexpr int SK_A_BYTES = 2 * SK_A_HALF;
+constexpr int SK_A_HALF = SK_BM * 64 * 2;      // BF16 weight box of 64 columns
 constexpr int SK_STAGE = SK_W_BYTES + SK_X_BYTES;
-constexpr int SK_SMEM = SK_NST * SK_STAGE + SK_NA * SK_A_BYTES + 1024;
+constexpr int SK_SMEM = SK_NST * SK_STAGE + 1024;
 constexpr int SK_THREADS = 320;
 constexpr uint32_t SK_IDESC = idesc_f16(SK_BM, US);
 // BF16 weights (the LM head): both operands BF16 (instruction-descriptor A/B format 1)
 constexpr uint32_t SK_IDESC_BF16 = SK_IDESC | (1u << 7) | (1u << 10);
 constexpr int SK_WB_BF16 = 2 * SK_A_HALF;  // BF16 weight tile 128 x 128 (two 64-column boxes)
-constexpr int SK_SMEM_BF16 = SK_NST * (SK_WB_BF16 + SK_X_BYTES) + 1024;
+constexpr int SK_SMEM_BF16 = SK_NST_BF16 * (SK_WB_BF16 + SK_X_BYTES) + 1024;
 constexpr int SK_UNITS_PER_CTA = 3;  // target units per CTA when choosing K slices
 constexpr int UN_ATT_CS = 8;         // attention cluster size: 16 sessions fill the GPU with 8-CTA clusters
 
@@ -103,11 +109,12 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
     skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const SkArgs a) {
     constexpr int WBYTES = BW ? SK_WB_BF16 : SK_W_BYTES;
     constexpr int STAGE = WBYTES + SK_X_BYTES;
+    constexpr int NST = BW ? SK_NST_BF16 : SK_NST;
+    constexpr uint32_t TCOLS = BW ? SK_TMEM_BF16 : SK_TMEM_I8;
     extern __shared__ uint8_t smraw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-    uint8_t* ring = sm;                      // stage s: weight tile, then the activation tile
-    uint8_t* abuf = sm + SK_NST * SK_STAGE;  // SK_NA FP16 operand buffers
-    __shared__ __align__(8) uint64_t full[SK_NST], empty[SK_NST], afull[SK_NA], aempty[SK_NA], accf[2], acce[2];
+    uint8_t* ring = sm;  // stage s: weight tile, then the activation tile
+    __shared__ __align__(8) uint64_t full[NST], empty[NST], afull[SK_NA], aempty[SK_NA], accf[2], acce[2];
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -117,7 +124,7 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
-        for (int s = 0; s < SK_NST; ++s) {
+        for (int s = 0; s < NST; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
             mbar_init(smem_u32(&empty[s]), BW ? 1 : 4 + 1);  // converter warps (INT8) + the MMAs
         }
@@ -133,7 +140,7 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
-                     "r"(32)
+                     "r"(TCOLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -149,26 +156,26 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
             // constant); activations, written by the previous kernel, after it
             int g = 0, xs = 0;  // stages issued, stages whose activation tile is issued
             auto issue_x = [&](int gx, int kb) {
-                const uint32_t st = smem_u32(ring + (gx % SK_NST) * STAGE);
-                const uint32_t fb = smem_u32(&full[gx % SK_NST]);
+                const uint32_t st = smem_u32(ring + (gx % NST) * STAGE);
+                const uint32_t fb = smem_u32(&full[gx % NST]);
                 tma_load_2d(st + WBYTES, &tmX, kb * SK_BK, 0, fb);
                 tma_load_2d(st + WBYTES + SK_X_BYTES / 2, &tmX, kb * SK_BK + 64, 0, fb);
             };
-            int pre_kb[SK_NST];
+            int pre_kb[NST];
             for (int u = blockIdx.x; u < units; u += gridDim.x) {
                 const int tile = u / a.S, ks = u - tile * a.S;
                 const int kb0 = ks * a.kbs, kb1 = min(nkb, kb0 + a.kbs);
                 for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                    const int s = g % SK_NST;
-                    if (g >= SK_NST) mbar_wait(smem_u32(&empty[s]), ((g / SK_NST) - 1) & 1, &abort_flag, a.err);
+                    const int s = g % NST;
+                    if (g >= NST) mbar_wait(smem_u32(&empty[s]), ((g / NST) - 1) & 1, &abort_flag, a.err);
                     const uint32_t fb = smem_u32(&full[s]);
                     mbar_expect_tx(fb, STAGE);
                     const uint32_t st = smem_u32(ring + s * STAGE);
                     tma_load_2d(st, &tmW, kb * SK_BK, tile * SK_BM, fb);
                     if (BW) tma_load_2d(st + SK_A_HALF, &tmW, kb * SK_BK + 64, tile * SK_BM, fb);
-                    if (g < SK_NST) {
+                    if (g < NST) {
                         pre_kb[g] = kb;
-                        if (g == SK_NST - 1) {
+                        if (g == NST - 1) {
                             grid_wait();
                             for (; xs <= g; ++xs) issue_x(xs, pre_kb[xs]);
                         }
@@ -182,8 +189,8 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
                 grid_wait();
                 for (; xs < g; ++xs) issue_x(xs, pre_kb[xs]);
             }
-            for (int k = max(0, g - SK_NST); k < g; ++k)  // no copy may outlive the CTA
-                mbar_wait(smem_u32(&full[k % SK_NST]), (k / SK_NST) & 1, &abort_flag, a.err, false);
+            for (int k = max(0, g - NST); k < g; ++k)  // no copy may outlive the CTA
+                mbar_wait(smem_u32(&full[k % NST]), (k / NST) & 1, &abort_flag, a.err, false);
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---- MMA issuer
@@ -195,54 +202,61 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
                 if (it >= 2) mbar_wait(smem_u32(&acce[acc]), ((it >> 1) - 1) & 1, &abort_flag, a.err);
                 fence_after();
                 for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                    const int s = g % SK_NST, ab = g % SK_NA;
+                    const int s = g % NST, ab = g % SK_NA;
                     if (!BW) mbar_wait(smem_u32(&afull[ab]), (g / SK_NA) & 1, &abort_flag, a.err);
-                    mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
+                    mbar_wait(smem_u32(&full[s]), (g / NST) & 1, &abort_flag, a.err);
                     fence_after();
-                    const uint32_t sa = BW ? smem_u32(ring + s * STAGE) : smem_u32(abuf + ab * SK_A_BYTES);
                     const uint32_t sx = smem_u32(ring + s * STAGE + WBYTES);
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            mma_f16(tmem + 16u * acc, sw128_desc(sa + h * SK_A_HALF + kk * 32),
-                                    sw128_desc(sx + h * (SK_X_BYTES / 2) + kk * 32), BW ? SK_IDESC_BF16 : SK_IDESC,
-                                    (kb > kb0 || h > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t bd = sw128_desc(sx + h * (SK_X_BYTES / 2) + kk * 32);
+                            const uint32_t on = (kb > kb0 || h > 0 || kk > 0) ? 1u : 0u;
+                            if constexpr (BW)
+                                mma_f16(tmem + 16u * acc, sw128_desc(smem_u32(ring + s * STAGE) + h * SK_A_HALF + kk * 32),
+                                        bd, SK_IDESC_BF16, on);
+                            else  // K 16 = 8 columns of FP16 pairs; K 64 per half
+                                mma_f16_tmem_a(tmem + 16u * acc, tmem + 64u + 64u * ab + 32u * h + 8u * kk, bd,
+                                               SK_IDESC, on);
+                        }
                     if (!BW) commit(smem_u32(&aempty[ab]));
                     commit(smem_u32(&empty[s]));
                 }
                 commit(smem_u32(&accf[acc]));
             }
         }
-    } else if (warp < 6) {  // ---- converters (INT8 weights): thread = weight row of the tile
+    } else if (warp < 6) {  // ---- converters (INT8 weights): thread = weight row = its TMEM lane
       if constexpr (!BW) {
-        const int r = (warp - 2) * 32 + lane;
+        const int r = 32 * (warp & 3) + lane;  // a warp reaches TMEM lanes 32 (warp % 4) .. + 31
+        const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
         int g = 0;
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int tile = u / a.S, ks = u - tile * a.S;
             const int kb0 = ks * a.kbs, kb1 = min(nkb, kb0 + a.kbs);
             (void)tile;
             for (int kb = kb0; kb < kb1; ++kb, ++g) {
-                const int s = g % SK_NST, ab = g % SK_NA;
-                mbar_wait(smem_u32(&full[s]), (g / SK_NST) & 1, &abort_flag, a.err);
+                const int s = g % NST, ab = g % SK_NA;
+                mbar_wait(smem_u32(&full[s]), (g / NST) & 1, &abort_flag, a.err);
                 if (g >= SK_NA) mbar_wait(smem_u32(&aempty[ab]), ((g / SK_NA) - 1) & 1, &abort_flag, a.err);
+                fence_after();  // after the MMAs that last read this operand buffer
                 const uint8_t* wrow = ring + s * STAGE + r * 128;
-                uint8_t* arow = abuf + ab * SK_A_BYTES + r * 128;
                 const int sw = r & 7;  // 128-byte swizzle: 16-byte chunk c of row r sits at c ^ (r % 8)
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const uint4 w = *reinterpret_cast<const uint4*>(wrow + ((c ^ sw) << 4));
-                    uint4 o0, o1;
-                    i8x4_to_h(w.x, o0.x, o0.y);
-                    i8x4_to_h(w.y, o0.z, o0.w);
-                    i8x4_to_h(w.z, o1.x, o1.y);
-                    i8x4_to_h(w.w, o1.z, o1.w);
-                    uint8_t* half = arow + (c >> 2) * SK_A_HALF;  // columns 0-63 / 64-127
-                    const int j = (c & 3) * 2;                     // FP16 chunk within the 64 columns
-                    *reinterpret_cast<uint4*>(half + ((j ^ sw) << 4)) = o0;
-                    *reinterpret_cast<uint4*>(half + (((j + 1) ^ sw) << 4)) = o1;
+                for (int h = 0; h < 2; ++h) {  // K columns 64 h .. 64 h + 63 -> TMEM columns 32 h ..
+                    uint32_t o[32];
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        const uint4 w = *reinterpret_cast<const uint4*>(wrow + (((4 * h + c4) ^ sw) << 4));
+                        i8x4_to_h(w.x, o[8 * c4 + 0], o[8 * c4 + 1]);
+                        i8x4_to_h(w.y, o[8 * c4 + 2], o[8 * c4 + 3]);
+                        i8x4_to_h(w.z, o[8 * c4 + 4], o[8 * c4 + 5]);
+                        i8x4_to_h(w.w, o[8 * c4 + 6], o[8 * c4 + 7]);
+                    }
+                    tmem_st32(trow + 64u + 64u * ab + 32u * h, o);
                 }
-                fence_proxy_async();
+                asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                fence_before();
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(smem_u32(&afull[ab]));
@@ -277,7 +291,7 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
     fence_before();
     __syncthreads();
     fence_after();
-    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(32) : "memory");
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TCOLS) : "memory");
 }
 
 // ------------------------------------------------------------------ activations to FP16
