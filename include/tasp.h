@@ -61,8 +61,9 @@ typedef struct tasp_model_desc {
     int32_t quant_group; /* INT8 scale granularity: 0 = one FP32 scale per output row; G > 0 =
                             one BF16 scale per output row and run of G input columns (Table 1:
                             G = 128). G must divide d, Hq*dh, df, dh and chan_unit and be a
-                            multiple of 16. Grouped stores serve decode; prefill and the union
-                            step return EUNSUP for them. */
+                            multiple of 16. Grouped stores serve one-session decode, prefill
+                            and the union step; a decode call with 2 or more sessions returns
+                            EUNSUP for them. */
 } tasp_model_desc;
 
 enum tasp_mask_kind {
@@ -321,12 +322,13 @@ int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, float* d_hidd
 /* One decode step for 1 <= n <= 16 sessions whose plans may differ (each turn keeps
  * the mask it was started with: its KV cache stays plan-shaped). Every weight row
  * of the shared store is read once for all n sessions: the projections run dense
- * for all of them on the tensor cores (INT8 rows converted to FP16 in shared
- * memory, activations in FP16 with a per-session power-of-two scale, FP32
- * accumulation), and each session's mask is applied where a unit meets it: Q/K/V of
- * a dropped group are not written, attention runs over the session's own kept
- * groups, dropped heads enter the O projection as zeros and dropped channel units
- * leave SiLU(gate) * up at zero. This equals the session's compacted plan up to
+ * for all of them on the tensor cores (INT8 rows converted to FP16 in tensor
+ * memory, times the BF16 group scale for a grouped store; activations in FP16 with a
+ * per-session power-of-two scale; FP32 accumulation), and each session's mask is
+ * applied where a unit meets it: Q/K/V of a dropped group are not written, attention
+ * runs over the session's own kept groups, dropped heads (whole groups, or single
+ * query heads of a query-head plan) enter the O projection as zeros and dropped
+ * channel units leave SiLU(gate) * up at zero. This equals the session's compacted plan up to
  * FP32 summation order and FP16 rounding of the activations (the mask-as-zero
  * reading of a plan, Sec. 3). d_x_bf16 is device BF16 [n][d]; d_hidden_out FP32
  * [n][d] and d_logits FP32 [n][vocab] are optional (NULL skips). The sessions must

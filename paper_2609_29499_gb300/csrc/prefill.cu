@@ -408,13 +408,23 @@ __global__ void __launch_bounds__(256) v_transpose_kernel(const uint16_t* __rest
     }
 }
 
-// INT8 panel rows (optionally through a row map) -> FP16 rows with a padded stride
+// INT8 panel rows (optionally through a row map) -> FP16 rows with a padded stride. A grouped
+// store's rows become q s_g 2^F16_GS_EXP, with s_g the BF16 scale of column group k / qg in
+// panel order (gs [rows][gld]): exact in FP32, one rounding to FP16.
+constexpr int F16_GS_EXP = 8;  // keeps q s_g normal in FP16 for scales down to ~2^-22
 __global__ void i8_to_f16_kernel(const int8_t* __restrict__ src, const int32_t* map, int64_t lds, int K,
-                                 __half* dst, int ldd) {
+                                 __half* dst, int ldd, const uint16_t* __restrict__ gs, int gld, int qg) {
     const int r = blockIdx.x;
     const int8_t* s = src + (int64_t)(map ? map[r] : r) * lds;
     __half* d = dst + (int64_t)r * ldd;
-    for (int k = threadIdx.x; k < ldd; k += blockDim.x) d[k] = __int2half_rn(k < K ? (int)s[k] : 0);
+    for (int k = threadIdx.x; k < ldd; k += blockDim.x) {
+        if (!gs) {
+            d[k] = __int2half_rn(k < K ? (int)s[k] : 0);
+        } else {
+            const float sg = k < K ? __uint_as_float((uint32_t)gs[(int64_t)r * gld + k / qg] << 16) : 0.f;
+            d[k] = __float2half_rn(k < K ? (float)s[k] * ldexpf(sg, F16_GS_EXP) : 0.f);
+        }
+    }
 }
 
 // ------------------------------------------------------------------ causal attention
@@ -963,6 +973,9 @@ int ensure_f16_panels(Plan& p, cudaStream_t s) {
         total += ((size_t)lp.qkv_rows * round8(sh.d) + (size_t)sh.d * round8(lp.o_K) + (size_t)lp.gu_rows * round8(sh.d) +
                   (size_t)sh.d * round8(lp.dn_K)) * 2 + 4 * 256;
     }
+    int post_n = sh.d;  // rows of the largest panel
+    for (const LayerPlan& lp : p.layers) post_n = std::max(post_n, std::max(lp.qkv_rows, lp.gu_rows));
+    if (sh.qg) total += (size_t)post_n * 4 + 256;
     int rc = p.f16_arena.reserve(total);
     if (rc) return rc;
     p.f16.resize(sh.L);
@@ -976,11 +989,27 @@ int ensure_f16_panels(Plan& p, cudaStream_t s) {
         f.o = (__half*)p.f16_arena.take((size_t)sh.d * f.ld_o * 2);
         f.gu = (__half*)p.f16_arena.take((size_t)lp.gu_rows * f.ld_d * 2);
         f.dn = (__half*)p.f16_arena.take((size_t)sh.d * f.ld_dn * 2);
-        if (lp.qkv_rows) i8_to_f16_kernel<<<lp.qkv_rows, 256, 0, s>>>(lp.qkv_w, lp.qkv_map, sh.d, sh.d, f.qkv, f.ld_d);
-        if (lp.o_K) i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.o_w, nullptr, lp.o_ld, lp.o_K, f.o, f.ld_o);
-        if (lp.gu_rows) i8_to_f16_kernel<<<lp.gu_rows, 256, 0, s>>>(lp.gu_w, lp.gu_map, sh.d, sh.d, f.gu, f.ld_d);
-        if (lp.dn_K) i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.dn_w, nullptr, lp.dn_ld, lp.dn_K, f.dn, f.ld_dn);
+        const int G = sh.qg;
+        if (lp.qkv_rows)
+            i8_to_f16_kernel<<<lp.qkv_rows, 256, 0, s>>>(lp.qkv_w, lp.qkv_map, sh.d, sh.d, f.qkv, f.ld_d,
+                                                          G ? lp.qkv_g : nullptr, lp.qkv_gld, G);
+        if (lp.o_K)
+            i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.o_w, nullptr, lp.o_ld, lp.o_K, f.o, f.ld_o, G ? lp.o_g : nullptr,
+                                                  lp.o_gld, G);
+        if (lp.gu_rows)
+            i8_to_f16_kernel<<<lp.gu_rows, 256, 0, s>>>(lp.gu_w, lp.gu_map, sh.d, sh.d, f.gu, f.ld_d,
+                                                         G ? lp.gu_g : nullptr, lp.gu_gld, G);
+        if (lp.dn_K)
+            i8_to_f16_kernel<<<sh.d, 256, 0, s>>>(lp.dn_w, nullptr, lp.dn_ld, lp.dn_K, f.dn, f.ld_dn,
+                                                  G ? lp.dn_g : nullptr, lp.dn_gld, G);
         TASP_CUDA(cudaGetLastError());
+    }
+    std::vector<float> post;
+    if (sh.qg) {
+        float* d_post = (float*)p.f16_arena.take((size_t)post_n * 4);
+        post.assign(post_n, std::ldexp(1.0f, -F16_GS_EXP));
+        TASP_CUDA(cudaMemcpyAsync(d_post, post.data(), (size_t)post_n * 4, cudaMemcpyHostToDevice, s));
+        p.f16_post = d_post;
     }
     TASP_CUDA(cudaStreamSynchronize(s));
     p.f16_ready = true;
@@ -1084,7 +1113,7 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
         TASP_CUDA(cudaGetLastError());
         if (lp.m_kv > 0) {
             GemmArgs ga{};
-            ga.M = T; ga.N = lp.qkv_rows; ga.K = sh.d; ga.scale = lp.qkv_s; ga.out = Y; ga.ldo = ld_y;
+            ga.M = T; ga.N = lp.qkv_rows; ga.K = sh.d; ga.scale = pl.f16_post ? pl.f16_post : lp.qkv_s; ga.out = Y; ga.ldo = ld_y;
             ga.mode = EP_STORE; ga.err = se.err;
             if ((rc = launch_gemm(Xh, ld_x, T, f.qkv, f.ld_d, lp.qkv_rows, sh.d, ga, s))) break;
             rope_kv_kernel<<<dim3(T, lp.m_kv), 256, 0, s>>>(Y, ld_y, T, sh.g(), sh.dh, se.rope, tc_attn ? nullptr : Qf,
@@ -1106,7 +1135,7 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
             }
             TASP_CUDA(cudaGetLastError());
             GemmArgs go{};
-            go.M = T; go.N = sh.d; go.K = lp.o_K; go.scale = lp.o_s; go.out = X; go.ldo = sh.d;
+            go.M = T; go.N = sh.d; go.K = lp.o_K; go.scale = pl.f16_post ? pl.f16_post : lp.o_s; go.out = X; go.ldo = sh.d;
             go.mode = EP_RESID; go.err = se.err;
             if ((rc = launch_gemm(O, ld_o, T, f.o, f.ld_o, sh.d, lp.o_K, go, s))) break;
         }
@@ -1117,11 +1146,11 @@ int prefill_run(Session& se, const uint16_t* d_embeds, int T, cudaStream_t s) {
                 rmsnorm_rows_kernel<<<T, 256, 0, s>>>(X, nullptr, nullptr, sh.d, lp.g_mlp, sh.eps, Xh, ld_x);
             TASP_CUDA(cudaGetLastError());
             GemmArgs gg{};
-            gg.M = T; gg.N = lp.gu_rows; gg.K = sh.d; gg.scale = lp.gu_s; gg.hout = H; gg.ldh = ld_h;
+            gg.M = T; gg.N = lp.gu_rows; gg.K = sh.d; gg.scale = pl.f16_post ? pl.f16_post : lp.gu_s; gg.hout = H; gg.ldh = ld_h;
             gg.mode = EP_SWIGLU; gg.err = se.err;
             if ((rc = launch_gemm(Xh, ld_x, T, f.gu, f.ld_d, lp.gu_rows, sh.d, gg, s))) break;
             GemmArgs gd{};
-            gd.M = T; gd.N = sh.d; gd.K = lp.c; gd.scale = lp.dn_s; gd.out = X; gd.ldo = sh.d;
+            gd.M = T; gd.N = sh.d; gd.K = lp.c; gd.scale = pl.f16_post ? pl.f16_post : lp.dn_s; gd.out = X; gd.ldo = sh.d;
             gd.mode = EP_RESID; gd.err = se.err;
             if ((rc = launch_gemm(H, ld_h, T, f.dn, f.ld_dn, sh.d, lp.c, gd, s))) break;
         }

@@ -986,7 +986,6 @@ int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t 
     const Shape& sh = p->store->sh;
     if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
     if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
-    if (sh.qg) return fail(TASP_EUNSUP, "prefill of a groupwise store is not built");
     Session* se = nullptr;
     int rc = session_alloc(p, T + max_new_tokens, &se);
     if (rc) return rc;
@@ -1017,7 +1016,6 @@ int tasp_session_prefill(tasp_session* s, const void* d_embeds_bf16, int32_t T, 
     if (T > se->max_tokens) return fail(TASP_ECAP, "prompt longer than the session capacity");
     if (d_logits_last && sh.vocab == 0) return fail(TASP_EUNSUP, "logits requested from a model without LM head");
     if (sh.d % 8) return fail(TASP_EUNSUP, "prefill needs d % 8 == 0");
-    if (sh.qg) return fail(TASP_EUNSUP, "prefill of a groupwise store is not built");
     cudaStream_t st = (cudaStream_t)stream;
     int rc = prefill_run(*se, (const uint16_t*)d_embeds_bf16, T, st);
     if (!rc) rc = enqueue_set_pos(*se, T, st);

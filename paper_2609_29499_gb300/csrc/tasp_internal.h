@@ -154,6 +154,9 @@ struct Plan {
     bool f16_ready = false;  // FP16 panels made on the first prefill
     Arena f16_arena;
     std::vector<F16Panels> f16;
+    // grouped store: the FP16 panels hold q s_g 2^F16_GS_EXP, and the prefill GEMMs scale their
+    // rows by this array of 2^-F16_GS_EXP (the store's row scales are all 1); NULL otherwise
+    const float* f16_post = nullptr;
 };
 
 // ---------------------------------------------------------------- sessions

@@ -7,9 +7,10 @@
 //  * Q/K/V: outputs of a group the session's plan drops are not written; the kept ones go
 //    to the session's plan-shaped query buffer and KV cache (rotary applied);
 //  * attention: per session over its own kept groups (the decode attention kernel, one
-//    cluster per (kept group, session));
+//    cluster per (kept group, session)); under a query-head plan the heads a kept group
+//    drops are computed but not written (the plan's output-slot table);
 //  * O: the session's attention output scattered to dense head order with zeros for the
-//    dropped heads, so their columns contribute nothing;
+//    dropped heads (whole groups or single query heads), so their columns contribute nothing;
 //  * gate/up: SiLU(gate) * up is zeroed for the channel units the plan drops, so the down
 //    projection's columns for them contribute nothing.
 //
@@ -89,7 +90,14 @@ struct SkArgs {
     int S, kbs;   // K slices and 128-column blocks per slice
     float* part;  // [S][rows][US] partial sums
     int* err;
+    // grouped store: BF16 scales [rows][gld] of qg columns each (NULL: per-row scales, applied
+    // by the finish kernels); the converters then make FP16 q s_g 2^SK_GS_EXP, one rounding
+    const uint16_t* gs;
+    int gld, qg;
 };
+// power-of-two factor on q s_g in FP16 (undone in FP32 by the finish kernels): keeps the
+// products of scales down to ~2^-22 normal in FP16 and weights up to 255 in magnitude in range
+constexpr int SK_GS_EXP = 8;
 
 // INT8 x 4 (one word) -> FP16 x 4 (two words), exact.
 __device__ __forceinline__ void i8x4_to_h(uint32_t w, uint32_t& lo, uint32_t& hi) {
@@ -104,7 +112,8 @@ __device__ __forceinline__ void i8x4_to_h(uint32_t w, uint32_t& lo, uint32_t& hi
 }
 
 // BW: BF16 weights (the LM head), read by the MMAs straight from the stage (no conversion).
-template <bool BW>
+// GS: INT8 weights of a grouped store (the converters apply the group scales).
+template <bool BW, bool GS = false>
 __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
     skinny_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const SkArgs a) {
     constexpr int WBYTES = BW ? SK_WB_BF16 : SK_W_BYTES;
@@ -234,9 +243,19 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int tile = u / a.S, ks = u - tile * a.S;
             const int kb0 = ks * a.kbs, kb1 = min(nkb, kb0 + a.kbs);
-            (void)tile;
+            const int wr = tile * SK_BM + r;  // this thread's weight row (beyond the panel: zero fill)
+            const uint16_t* gsr = GS && wr < a.rows ? a.gs + (int64_t)wr * a.gld : nullptr;
             for (int kb = kb0; kb < kb1; ++kb, ++g) {
                 const int s = g % NST, ab = g % SK_NA;
+                __half2 gsc[8];  // grouped store: the scale of each 16-column chunk, times 2^SK_GS_EXP
+                if constexpr (GS) {
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const float v = gsr ? __uint_as_float((uint32_t)__ldg(gsr + (kb * SK_BK + 16 * c) / a.qg) << 16)
+                                            : 0.f;
+                        gsc[c] = __float2half2_rn(ldexpf(v, SK_GS_EXP));
+                    }
+                }
                 mbar_wait(smem_u32(&full[s]), (g / NST) & 1, &abort_flag, a.err);
                 if (g >= SK_NA) mbar_wait(smem_u32(&aempty[ab]), ((g / SK_NA) - 1) & 1, &abort_flag, a.err);
                 fence_after();  // after the MMAs that last read this operand buffer
@@ -252,6 +271,13 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
                         i8x4_to_h(w.y, o[8 * c4 + 2], o[8 * c4 + 3]);
                         i8x4_to_h(w.z, o[8 * c4 + 4], o[8 * c4 + 5]);
                         i8x4_to_h(w.w, o[8 * c4 + 6], o[8 * c4 + 7]);
+                        if constexpr (GS) {  // exact q times an FP16 scale: one rounding of the product
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const __half2 v = __hmul2(*reinterpret_cast<const __half2*>(&o[8 * c4 + i]), gsc[4 * h + c4]);
+                                o[8 * c4 + i] = *reinterpret_cast<const uint32_t*>(&v);
+                            }
+                        }
                     }
                     tmem_st32(trow + 64u + 64u * ab + 32u * h, o);
                 }
@@ -304,6 +330,8 @@ struct PrepArgs {
     const float* gamma;        // PR_NORM
     float eps;
     const int* gmap;           // PR_HEADS: [US][Hkv] dense group -> plan group (-1: dropped)
+    const int16_t* oslot[US];  // PR_HEADS: the plan's (group slot, head) -> attention output slot, -1 for
+                               // a dropped head (NULL: every head of the kept groups, slot jl g + hh)
     int g, dh, Hkv;
     __half* x16;               // [US][ld16] (BF16 bits when bf16)
     int64_t ld16;
@@ -336,10 +364,12 @@ __device__ __forceinline__ void cluster_sync_all() {
 // RMSNorm factor): x * gamma, a copy, or the plan's heads in dense order.
 __device__ __forceinline__ float4 prep_in(const PrepArgs& p, const float* src, int b, int k) {
     if (p.mode == PR_HEADS) {
-        const int hd = k / p.dh, j = hd / p.g;
+        const int hd = k / p.dh, j = hd / p.g, hh = hd - j * p.g;
         const int lj = p.gmap[b * p.Hkv + j];
         if (lj < 0) return make_float4(0.f, 0.f, 0.f, 0.f);
-        return *reinterpret_cast<const float4*>(src + (int64_t)(lj * p.g + (hd - j * p.g)) * p.dh + (k - hd * p.dh));
+        const int slot = p.oslot[b] ? p.oslot[b][lj * p.g + hh] : lj * p.g + hh;
+        if (slot < 0) return make_float4(0.f, 0.f, 0.f, 0.f);
+        return *reinterpret_cast<const float4*>(src + (int64_t)slot * p.dh + (k - hd * p.dh));
     }
     float4 v = *reinterpret_cast<const float4*>(src + k);
     if (p.mode == PR_NORM) {
@@ -434,11 +464,12 @@ struct FinArgs {
     int S, rows, n;
     const float* scale;  // [rows]
     const float* xinv;   // [US]
+    float post;          // 2^-SK_GS_EXP for a grouped store, else 1
 };
 __device__ __forceinline__ float fin_sum(const FinArgs& f, int row, int b) {
     float acc = 0.f;
     for (int s = 0; s < f.S; ++s) acc += f.part[((int64_t)s * f.rows + row) * US + b];
-    return acc * f.scale[row] * f.xinv[b];
+    return acc * f.scale[row] * f.xinv[b] * f.post;
 }
 
 // Q/K/V: blockIdx.x = one dense head row block (group j, head hh of g + 2), blockIdx.y = a
@@ -623,7 +654,7 @@ int launch(K kern, dim3 grid, dim3 block, cudaStream_t s, const A& a) {
 
 // W: INT8 [rows][K], or BF16 [rows][K] when bw (the LM head)
 int launch_skinny(const void* W, bool bw, int rows, int K, const __half* x16, int64_t ld16, float* part, int* err,
-                  int& S_out, cudaStream_t s) {
+                  int& S_out, cudaStream_t s, const uint16_t* gs = nullptr, int qg = 0) {
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
@@ -642,12 +673,20 @@ int launch_skinny(const void* W, bool bw, int rows, int K, const __half* x16, in
     slices(rows, K, di.sms, a.S, a.kbs);
     a.part = part;
     a.err = err;
+    a.gs = gs;
+    a.qg = qg;
+    a.gld = qg ? K / qg : 0;
     const int units = ((rows + SK_BM - 1) / SK_BM) * a.S;
     const int grid = std::min(units, SK_CTAS_PER_SM * di.sms);
     if (bw) {
         if ((rc = launch_pdl(skinny_kernel<true>, dim3(grid), dim3(SK_THREADS), SK_SMEM_BF16, s, 1, tw, tx, a))) return rc;
     } else {
-        if ((rc = launch_pdl(skinny_kernel<false>, dim3(grid), dim3(SK_THREADS), SK_SMEM, s, 1, tw, tx, a))) return rc;
+        if (gs) {
+            if ((rc = launch_pdl(skinny_kernel<false, true>, dim3(grid), dim3(SK_THREADS), SK_SMEM, s, 1, tw, tx, a)))
+                return rc;
+        } else if ((rc = launch_pdl(skinny_kernel<false>, dim3(grid), dim3(SK_THREADS), SK_SMEM, s, 1, tw, tx, a))) {
+            return rc;
+        }
     }
     S_out = a.S;
     return TASP_OK;
@@ -754,6 +793,7 @@ int union_get(Session* const* ss, int n, UnionWs** out) {
     TASP_CUDA(cudaMemcpy(w->keep, kp.data(), kp.size(), cudaMemcpyHostToDevice));
     if (!g_skinny_attr) {  // before any stream capture
         TASP_CUDA(cudaFuncSetAttribute(skinny_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SK_SMEM));
+        TASP_CUDA(cudaFuncSetAttribute(skinny_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SK_SMEM));
         TASP_CUDA(cudaFuncSetAttribute(skinny_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        SK_SMEM_BF16));
         g_skinny_attr = true;
@@ -772,7 +812,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
     const int g = sh.g(), qd = sh.Hq * sh.dh, nu = sh.n_units();
     int rc = 0, nl = 0;
     auto prep = [&](int mode, const float* src, int64_t src_ld, const uint16_t* in_bf16, const float* gamma, int K,
-                    const int* gmap, int bf16 = 0) -> int {
+                    const int* gmap, int bf16 = 0, int layer = -1) -> int {
         PrepArgs p{};
         p.mode = mode;
         p.K = K;
@@ -782,6 +822,8 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         p.gamma = gamma;
         p.eps = sh.eps;
         p.gmap = gmap;
+        if (mode == PR_HEADS)
+            for (int b = 0; b < n; ++b) p.oslot[b] = w.ss[b]->plan->layers[layer].oslot;
         p.g = g;
         p.dh = sh.dh;
         p.Hkv = sh.Hkv;
@@ -800,6 +842,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         f.n = n;
         f.scale = scale;
         f.xinv = w.xinv;
+        f.post = sh.qg ? std::ldexp(1.0f, -SK_GS_EXP) : 1.0f;
         return f;
     };
     for (int l = 0; l < sh.L; ++l) {
@@ -809,7 +852,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         int S = 0;
         // Q/K/V for every session's kept groups
         if ((rc = prep(PR_NORM, w.x, sh.d, l == 0 ? w.x_stage : nullptr, ls.g_attn, sh.d, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.qkv, false, sh.qkv_rows_dense(), sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.qkv, false, sh.qkv_rows_dense(), sh.d, w.x16, w.ld16, w.part, w.err, S, s, ls.qkv_g, sh.qg))) return rc;
         ++nl;
         {
             QkvFin p{};
@@ -844,6 +887,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
                 a.pos[b] = w.ss[b]->d_pos;
                 a.max_tokens[b] = w.ss[b]->max_tokens;
                 a.m_kv[b] = w.ss[b]->plan->layers[l].m_kv;
+                a.oslot[b] = w.ss[b]->plan->layers[l].oslot;  // query-head plans: dropped heads are not written
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
             a.part = w.apart;
@@ -861,8 +905,8 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
             ++nl;
         }
         // O projection + residual (the dropped heads are zero in the scattered input)
-        if ((rc = prep(PR_HEADS, w.o, qd, nullptr, nullptr, qd, gmap))) return rc;
-        if ((rc = launch_skinny(ls.o, false, sh.d, qd, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = prep(PR_HEADS, w.o, qd, nullptr, nullptr, qd, gmap, 0, l))) return rc;
+        if ((rc = launch_skinny(ls.o, false, sh.d, qd, w.x16, w.ld16, w.part, w.err, S, s, ls.o_g, sh.qg))) return rc;
         ++nl;
         {
             ResFin p{};
@@ -875,7 +919,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         }
         // gate/up + SiLU(gate) * up, zero for the dropped channel units
         if ((rc = prep(PR_NORM, w.x, sh.d, nullptr, ls.g_mlp, sh.d, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.gu, false, 2 * sh.df, sh.d, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.gu, false, 2 * sh.df, sh.d, w.x16, w.ld16, w.part, w.err, S, s, ls.gu_g, sh.qg))) return rc;
         ++nl;
         {
             GuFin p{};
@@ -890,7 +934,7 @@ int enqueue_union(UnionWs& w, float* hidden, float* logits, cudaStream_t s, int*
         }
         // down projection + residual
         if ((rc = prep(PR_COPY, w.h, sh.df, nullptr, nullptr, sh.df, nullptr))) return rc;
-        if ((rc = launch_skinny(ls.down, false, sh.d, sh.df, w.x16, w.ld16, w.part, w.err, S, s))) return rc;
+        if ((rc = launch_skinny(ls.down, false, sh.d, sh.df, w.x16, w.ld16, w.part, w.err, S, s, ls.down_g, sh.qg))) return rc;
         ++nl;
         {
             ResFin p{};
@@ -938,11 +982,6 @@ int union_check(Session* const* ss, int n, bool step) {
     const Shape& sh = st->sh;
     if (sh.d % SK_BK || (sh.Hq * sh.dh) % SK_BK || sh.df % SK_BK)
         return fail(TASP_EUNSUP, "union decode needs d, Hq*dh and d_ff that are multiples of 128");
-    if (sh.qg) return fail(TASP_EUNSUP, "union decode of a groupwise store is not built");
-    for (int b = 0; b < n; ++b)
-        for (const LayerPlan& lp : ss[b]->plan->layers)
-            if (lp.m_q != lp.m_kv * sh.g())
-                return fail(TASP_EUNSUP, "union decode takes plans of whole GQA groups only");
     return TASP_OK;
 }
 

@@ -1,7 +1,7 @@
 """GPU parity of groupwise INT8 stores (Table 1: group size 128, BF16 scales) against the
 oracle, through the C ABI: INT8 codes and BF16 group scales bit-exact on the store's panels,
-one-session decode elementwise per layer and end to end, and the paths not built for such a
-store (batches, prefill, union) refused with EUNSUP."""
+one-session decode elementwise per layer and end to end, the union step and prefill against
+the oracle, and batches of 2-4 sessions (not built for such a store) refused with EUNSUP."""
 import dataclasses
 
 import numpy as np
@@ -113,7 +113,75 @@ def test_grouped_isolated_layer_and_decode(tasp):
     plan.release()
 
 
-def test_paths_not_built_for_grouped_stores(tasp):
+def test_grouped_union_step_matches_oracle(tasp):
+    # the union step on a grouped store: the converters scale each 16-column chunk of INT8
+    # codes by its BF16 group scale in FP16 (q s_g 2^8, one rounding); three sessions on the
+    # greedy plan and the dense plan, three steps through both layers with logits
+    import torch
+    sh = SHAPE
+    plan, mask = _plan(tasp, sh)
+    dense = tasp.Plan(sh, tasp.all_keep_mask())
+    plans, masks = [plan, dense], [mask, maskc.all_keep(sh)]
+    pick, t_priors, kv_seeds = [0, 1, 0], [700, 64, 5], [7, 8, 9]
+    ss = []
+    for k, tp, ks in zip(pick, t_priors, kv_seeds):
+        se = tasp.Session(plans[k], tp + 4)
+        se.fill_synthetic(tp, ks)
+        ss.append(se)
+    n, steps = len(pick), 3
+    xb = synth.step_inputs_bf16(13, steps, n, sh.d)
+    x = bf16_tensor(xb)
+    hid = torch.empty((steps, n, sh.d), dtype=torch.float32, device="cuda")
+    logits = torch.empty((steps, n, sh.vocab), dtype=torch.float32, device="cuda")
+    for t in range(steps):
+        tasp.decode_step_union(ss, x[t], hid[t], logits[t])
+    torch.cuda.synchronize()
+    assert tasp.union_status(ss)[0] == 0
+    rows = np.arange(0, sh.vocab, 997)
+    for i, k in enumerate(pick):
+        ref = forward.decode(sh, masks[k], synth.bf16_to_f32(xb[:, i]), t_priors[i], kv_seeds[i])
+        assert rel_l2(hid.cpu().numpy()[:, i], ref) <= TOL_E2E, i
+        lref = forward.final_logits(sh, ref, rows=rows)
+        assert rel_l2(logits.cpu().numpy()[:, i][:, rows], lref) <= TOL_E2E, i
+    for se in ss:
+        se.release()
+    dense.release()
+    plan.release()
+
+
+def test_grouped_prefill_matches_oracle(tasp):
+    # the prefill GEMMs on FP16 panels holding q s_g 2^8 (one rounding), rows scaled by 2^-8
+    import torch
+    sh = SHAPE
+    plan, mask = _plan(tasp, sh)
+    T = 300
+    emb = synth.prompt_bf16(6, 0, T, sh.d)
+    logits = torch.empty(sh.vocab, dtype=torch.float32, device="cuda")
+    sess = tasp.Session.prefill(plan, bf16_tensor(emb), 2, logits)
+    torch.cuda.synchronize()
+    Xp, kv = forward.prefill(sh, mask, synth.bf16_to_f32(emb))
+    for layer in range(sh.L):
+        for kind in (0, 1):
+            got = synth.bf16_to_f32(sess.kv(layer, kind))
+            ref = kv[layer][kind][mask.keep_groups[layer]]
+            assert rel_l2(got, ref) <= TOL_E2E, (layer, kind)
+    rows = np.arange(0, sh.vocab, 499)
+    ref = forward.final_logits(sh, Xp[-1:], rows=rows)[0]
+    assert rel_l2(logits.cpu().numpy()[rows], ref) <= TOL_E2E
+    # one decode step after the prompt reads the prefilled cache
+    xb = synth.step_inputs_bf16(3, 1, 1, sh.d)
+    hid = torch.empty((1, sh.d), dtype=torch.float32, device="cuda")
+    tasp.decode_step([sess], bf16_tensor(xb)[0], hid)
+    torch.cuda.synchronize()
+    dref = forward.decode(sh, mask, synth.bf16_to_f32(xb[:, 0]), T, 0,
+                          prior=lambda layer: (kv[layer][0], kv[layer][1]))
+    assert rel_l2(hid.cpu().numpy(), dref) <= TOL_E2E
+    assert sess.device_error() == 0
+    sess.release()
+    plan.release()
+
+
+def test_batched_gemvs_refuse_grouped_stores(tasp):
     import torch
     sh = SHAPE
     plan, _ = _plan(tasp, sh)
@@ -121,11 +189,9 @@ def test_paths_not_built_for_grouped_stores(tasp):
     for s in (a, b):
         s.fill_synthetic(4, 1)
     x = torch.zeros((2, sh.d), dtype=torch.bfloat16, device="cuda")
-    for call in (lambda: tasp.decode_step([a, b], x), lambda: tasp.decode_step_union([a], x[:1]),
-                 lambda: a.prefill_into(torch.zeros((4, sh.d), dtype=torch.bfloat16, device="cuda"))):
-        with pytest.raises(tasp.TaspError) as e:
-            call()
-        assert e.value.code == tasp.EUNSUP
+    with pytest.raises(tasp.TaspError) as e:
+        tasp.decode_step([a, b], x)
+    assert e.value.code == tasp.EUNSUP
     a.release()
     b.release()
     plan.release()

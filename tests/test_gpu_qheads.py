@@ -1,7 +1,7 @@
 """GPU parity of query-head-granular masks (Sec. 3.3: query-head candidates, a KV head kept
 whenever one of its heads is) against the oracle, through the C ABI: panels and kept lists
-bit-exact, decode and prefill elementwise, compact = row-indexed panels bit for bit, and the
-union step refusing plans with partial groups."""
+bit-exact, decode and prefill elementwise, compact = row-indexed panels bit for bit, and
+union steps that mix query-head plans with whole-group and dense plans."""
 import dataclasses
 
 import numpy as np
@@ -93,12 +93,14 @@ def test_compact_and_row_indexed_partial_groups_agree(tasp):
 
 
 def test_8b_two_layer_greedy_qhead_mask(tasp):
+    # budget 0.3: both layers keep 30 of 32 query heads over all 8 KV groups (partial groups)
     sh = dataclasses.replace(synth.LLAMA3_8B, L=2)
-    seed = 1000
+    seed = 1002
     sc = synth.mask_scores_u32(seed, sh.L, sh.Hq + sh.n_chan_units)
     tg = synth.layer_target_u24(seed, sh.L)
-    mask = maskc.compile_mask_qheads(sh, sc, tg, 0.4, 0.2, 0.6)
-    plan = tasp.Plan(sh, tasp.greedy_qhead_mask(sc, tg, 0.4, 0.2, 0.6))
+    mask = maskc.compile_mask_qheads(sh, sc, tg, 0.3, 0.1, 0.5)
+    assert all(len(mask.keep_qheads[l]) < len(mask.keep_groups[l]) * sh.g for l in range(sh.L))
+    plan = tasp.Plan(sh, tasp.greedy_qhead_mask(sc, tg, 0.3, 0.1, 0.5))
     for layer in range(sh.L):
         check_qhead_panels(tasp, plan, sh, mask, layer)
     xb = synth.step_inputs_bf16(11, 3, 1, sh.d)
@@ -136,18 +138,66 @@ def test_layer1_partial_groups_prefill(tasp, T):
     plan.release()
 
 
-def test_union_refuses_partial_groups(tasp):
+def _union(tasp, plans, t_priors, kv_seeds, xb):
     import torch
-    sh = dataclasses.replace(synth.LLAMA3_8B, L=1)
-    plan = tasp.Plan(sh, tasp.explicit_qhead_mask([[0, 1, 2, 8]], [[0, 3]]))
-    sess = tasp.Session(plan, 8)
-    sess.fill_synthetic(4, 1)
-    x = torch.zeros((1, sh.d), dtype=torch.bfloat16, device="cuda")
-    with pytest.raises(tasp.TaspError) as e:
-        tasp.decode_step_union([sess], x)
-    assert e.value.code == tasp.EUNSUP
-    sess.release()
-    plan.release()
+    S, n, d = xb.shape
+    ss = []
+    for pl, tp, ks in zip(plans, t_priors, kv_seeds):
+        s = tasp.Session(pl, tp + S + 1)
+        s.fill_synthetic(tp, ks)
+        ss.append(s)
+    x = bf16_tensor(xb)
+    hid = torch.empty((S, n, d), dtype=torch.float32, device="cuda")
+    for t in range(S):
+        tasp.decode_step_union(ss, x[t], hid[t])
+    torch.cuda.synchronize()
+    assert tasp.union_status(ss)[0] == 0
+    for i, s in enumerate(ss):
+        assert s.position == t_priors[i] + S and s.device_error() == 0
+        s.release()
+    return hid.cpu().numpy()
+
+
+def test_layer1_union_with_partial_groups_matches_oracle(tasp):
+    # one union step over a query-head plan (partial groups), a whole-group plan and the
+    # dense plan: each session against the oracle's decode under its own mask
+    wl = synth.CFG1
+    sh = wl.shape
+    units = [list(range(0, sh.df, 2))]
+    plans = [tasp.Plan(sh, tasp.explicit_qhead_mask(LAYER1_HEADS, units)),
+             tasp.Plan(sh, tasp.explicit_mask([[1]], units)), tasp.Plan(sh, tasp.all_keep_mask())]
+    masks = [maskc.explicit_qheads(sh, LAYER1_HEADS, units), maskc.explicit(sh, [[1]], units), maskc.all_keep(sh)]
+    pick = [0, 1, 2, 0, 0]
+    t_priors, kv_seeds = [128, 40, 77, 9, 300], [5, 6, 7, 8, 9]
+    xb = synth.step_inputs_bf16(21, 4, len(pick), sh.d)
+    got = _union(tasp, [plans[k] for k in pick], t_priors, kv_seeds, xb)
+    for i, k in enumerate(pick):
+        ref = forward.decode(sh, masks[k], synth.bf16_to_f32(xb[:, i]), t_priors[i], kv_seeds[i])
+        assert within(got[:, i], ref).all(), (i, np.abs(got[:, i] - ref).max())
+        assert rel_l2(got[:, i], ref) <= TOL_E2E
+    for p in plans:
+        p.release()
+
+
+def test_8b_two_layer_union_of_query_head_plans(tasp):
+    # head dim 128: two greedy query-head masks in one union step, against the oracle
+    sh = dataclasses.replace(synth.LLAMA3_8B, L=2)
+    plans, masks = [], []
+    for seed, (budget, lo, hi) in ((1002, (0.3, 0.1, 0.5)), (7, (0.2, 0.05, 0.4))):
+        sc = synth.mask_scores_u32(seed, sh.L, sh.Hq + sh.n_chan_units)
+        tg = synth.layer_target_u24(seed, sh.L)
+        masks.append(maskc.compile_mask_qheads(sh, sc, tg, budget, lo, hi))
+        plans.append(tasp.Plan(sh, tasp.greedy_qhead_mask(sc, tg, budget, lo, hi)))
+    for m in masks:  # partial groups in every layer: 30/32 heads over 8 groups; 20/6 and 25/8
+        assert all(len(m.keep_qheads[l]) < len(m.keep_groups[l]) * sh.g for l in range(sh.L))
+    pick, t_priors, kv_seeds = [0, 1, 1, 0], [300, 64, 5, 150], [41, 42, 43, 44]
+    xb = synth.step_inputs_bf16(17, 3, len(pick), sh.d)
+    got = _union(tasp, [plans[k] for k in pick], t_priors, kv_seeds, xb)
+    for i, k in enumerate(pick):
+        ref = forward.decode(sh, masks[k], synth.bf16_to_f32(xb[:, i]), t_priors[i], kv_seeds[i])
+        assert rel_l2(got[:, i], ref) <= TOL_E2E, (i, rel_l2(got[:, i], ref))
+    for p in plans:
+        p.release()
 
 
 def test_8b_two_layer_partial_groups_prefill(tasp):
