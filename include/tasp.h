@@ -61,9 +61,8 @@ typedef struct tasp_model_desc {
     int32_t quant_group; /* INT8 scale granularity: 0 = one FP32 scale per output row; G > 0 =
                             one BF16 scale per output row and run of G input columns (Table 1:
                             G = 128). G must divide d, Hq*dh, df, dh and chan_unit and be a
-                            multiple of 16. Grouped stores serve one-session decode, prefill
-                            and the union step; a decode call with 2 or more sessions returns
-                            EUNSUP for them. */
+                            multiple of 16. Grouped stores serve every path: decode (one
+                            session or batches), prefill and the union step. */
 } tasp_model_desc;
 
 enum tasp_mask_kind {

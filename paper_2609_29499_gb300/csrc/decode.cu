@@ -57,11 +57,11 @@ int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, const
     return TASP_OK;
 }
 
-Fn pick_any(int nbk, int mode, int R, int XC) {
+Fn pick_any(int nbk, int mode, int R, int XC, bool gs) {
     switch (nbk) {
-        case 1: return pick<1>(mode, R, XC);
-        case 2: return pick<2>(mode, R, XC);
-        default: return pick<4>(mode, R, XC);
+        case 1: return pick<1>(mode, R, XC, gs);
+        case 2: return pick<2>(mode, R, XC, gs);
+        default: return pick<4>(mode, R, XC, gs);
     }
 }
 
@@ -97,14 +97,15 @@ std::map<const void*, int> g_attr;  // kernel -> dynamic shared memory cap
 int launch_gemv(int mode, Params p, cudaStream_t s) {
     if (p.rows == 0 || p.nb == 0) return TASP_OK;
     if (p.nb > MAXNB) return fail(TASP_EINVAL, "more activation vectors than one GEMV pass takes");
-    if (p.gscale) return fail(TASP_EUNSUP, "groupwise stores decode one session per weight pass");
     DevInfo di;
     int rc = device_info(di);
     if (rc) return rc;
     const Variant v = variant(mode, p.nb, p.nchunks, 8);
     if ((mode == M_QKV || mode == M_GU) && v.passes > 1)
         return fail(TASP_EUNSUP, "hidden size too large for the register-resident activation slices of this batch");
-    Fn fn = pick_any(v.nbk, mode, v.R, v.XC);
+    if (p.gscale && (v.nbk == 1 || mode == M_LM))
+        return fail(TASP_EINVAL, "grouped scales on a one-vector or LM-head batched GEMV");
+    Fn fn = pick_any(v.nbk, mode, v.R, v.XC, p.gscale != nullptr);
     if (!fn) return fail(TASP_EINVAL, "no GEMV variant for this row length");
     p.seg = v.seg;
     p.passes = v.passes;

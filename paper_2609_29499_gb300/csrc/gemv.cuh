@@ -76,7 +76,7 @@ struct Params {
     const int* pos[MAXNB];
     int g, dh;
     const int16_t* blk_role;  // QKV: role of each d_h-row block (NULL = block index)
-    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gld] (single-vector kernels only)
+    const uint16_t* gscale;   // groupwise store: BF16 scales [panel row][gld] (NULL = per-row only)
     int gcols, gshift;        // scales per row; chunk c uses scale c >> gshift
     int gld;                  // row stride of gscale (elements)
     float* h_out;          // GU: SiLU(gate) * up, stride h_stride
@@ -381,10 +381,13 @@ __device__ __forceinline__ void make_xregs(const Params& p, const float (&inv)[N
 
 // ------------------------------------------------------------------ dot products
 // INT8 rows of one stage . x: per chunk sum(w X) = 256 sum(w hi) + sum(w lo) in exact
-// INT32, then acc[r][v] += float(sum) * scale in FP32.
-template <int R, int XC, int NB>
+// INT32, then acc[r][v] += float(sum) * scale in FP32. GS (grouped store): the chunk's sum
+// is also scaled by its row's BF16 group scale, grow[r][(cb + c) >> gshift] (cb = the pass's
+// first chunk), read through the cache and shared by the NB vectors.
+template <int R, int XC, int NB, bool GS = false>
 __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld, const XDigits<XC, NB>& xd,
-                                       int nvalid, int tid, float (&acc)[R][NB]) {
+                                       int nvalid, int tid, float (&acc)[R][NB],
+                                       const uint16_t* const (&grow)[R], int gshift, int cb) {
 #pragma unroll
     for (int j = 0; j < XC; ++j) {
         const int c = tid + j * CT;
@@ -393,6 +396,8 @@ __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld
             for (int r = 0; r < R; ++r) {
                 const int4 wv = *reinterpret_cast<const int4*>(stage + (size_t)r * ld + (size_t)c * 16);
                 const uint32_t wd[4] = {(uint32_t)wv.x, (uint32_t)wv.y, (uint32_t)wv.z, (uint32_t)wv.w};
+                float gsc = 1.0f;
+                if constexpr (GS) gsc = __uint_as_float((uint32_t)__ldg(grow[r] + ((cb + c) >> gshift)) << 16);
 #pragma unroll
                 for (int v = 0; v < NB; ++v) {
                     int sh = 0, sl = 0;
@@ -401,7 +406,8 @@ __device__ __forceinline__ void dot_i8(const uint8_t* __restrict__ stage, int ld
                         sh = dp4a_ss(wd[k], xd.hi[v][j][k], sh);
                         sl = dp4a_su(wd[k], xd.lo[v][j][k], sl);
                     }
-                    acc[r][v] = fmaf(__int2float_rn(sh * 256 + sl), xd.scale[v][j], acc[r][v]);
+                    const float xs = GS ? xd.scale[v][j] * gsc : xd.scale[v][j];
+                    acc[r][v] = fmaf(__int2float_rn(sh * 256 + sl), xs, acc[r][v]);
                 }
             }
         }
@@ -575,7 +581,7 @@ __device__ __forceinline__ void epilogue(const Params& p, const float (*red)[R *
 }
 
 // ------------------------------------------------------------------ the kernel
-template <int MODE, int R, int XC, int NB>
+template <int MODE, int R, int XC, int NB, bool GS = false>
 __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
     static_assert(R * NB <= 32, "row x vector entries must fit one warp");
     extern __shared__ __align__(128) uint8_t sm[];
@@ -708,7 +714,14 @@ __global__ void __launch_bounds__(THREADS, 1) gemv_kernel(const Params p) {
                 for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int v = 0; v < NB; ++v) acc[r][v] = 0.f;
-                dot_i8<R, XC, NB>(st, seg_bytes, xd, nvalid, tid, acc);
+                const uint16_t* grow[R];
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    int w = gi * R + r;
+                    if (w >= p.rows) w = 0;  // padding row of a ragged last group: never stored
+                    grow[r] = GS ? p.gscale + (size_t)panel_row<MODE>(p, w) * p.gld : nullptr;
+                }
+                dot_i8<R, XC, NB, GS>(st, seg_bytes, xd, nvalid, tid, acc, grow, p.gshift, cb);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(empty0 + 8 * s);  // this warp is done with the stage
@@ -738,10 +751,10 @@ typedef void (*Fn)(const Params);
 
 // The instantiated variants: NB * XC <= 4 keeps the digit registers of the tuned
 // single-vector kernel; R * NB <= 16 bounds the accumulators.
-template <int NB, int MODE>
+template <int NB, int MODE, bool GS = false>
 Fn pick_mode(int R, int XC) {
 #define TASP_GEMV_V(r, x) \
-    if (R == r && XC == x) return gemv_kernel<MODE, r, x, NB>;
+    if (R == r && XC == x) return gemv_kernel<MODE, r, x, NB, GS>;
     if constexpr (NB == 1) {
         TASP_GEMV_V(8, 1) TASP_GEMV_V(4, 1) TASP_GEMV_V(2, 1) TASP_GEMV_V(4, 2) TASP_GEMV_V(2, 2) TASP_GEMV_V(2, 4)
         if constexpr (MODE != M_QKV && MODE != M_GU) {
@@ -756,8 +769,23 @@ Fn pick_mode(int R, int XC) {
     return nullptr;
 }
 
+// gs: the grouped-store variant (INT8 modes with 2 or 4 vectors; one vector of a grouped
+// store runs on the single-vector kernels)
 template <int NB>
-Fn pick_nb(int mode, int R, int XC) {
+Fn pick_nb(int mode, int R, int XC, bool gs) {
+    if (gs) {
+        if constexpr (NB == 1) {
+            return nullptr;
+        } else {
+            switch (mode) {
+                case M_QKV: return pick_mode<NB, M_QKV, true>(R, XC);
+                case M_O: return pick_mode<NB, M_O, true>(R, XC);
+                case M_GU: return pick_mode<NB, M_GU, true>(R, XC);
+                case M_DOWN: return pick_mode<NB, M_DOWN, true>(R, XC);
+                default: return nullptr;
+            }
+        }
+    }
     switch (mode) {
         case M_QKV: return pick_mode<NB, M_QKV>(R, XC);
         case M_O: return pick_mode<NB, M_O>(R, XC);
@@ -767,16 +795,16 @@ Fn pick_nb(int mode, int R, int XC) {
     }
 }
 
-// Kernel variant for (mode, rows per stage R, chunks per thread XC) with NB vectors;
-// nullptr if not built. Each NB is compiled in its own translation unit.
+// Kernel variant for (mode, rows per stage R, chunks per thread XC) with NB vectors, per-row
+// or grouped scales; nullptr if not built. Each NB is compiled in its own translation unit.
 template <int NB>
-Fn pick(int mode, int R, int XC);
+Fn pick(int mode, int R, int XC, bool gs);
 template <>
-Fn pick<1>(int mode, int R, int XC);
+Fn pick<1>(int mode, int R, int XC, bool gs);
 template <>
-Fn pick<2>(int mode, int R, int XC);
+Fn pick<2>(int mode, int R, int XC, bool gs);
 template <>
-Fn pick<4>(int mode, int R, int XC);
+Fn pick<4>(int mode, int R, int XC, bool gs);
 
 }  // namespace gemv
 

@@ -5,8 +5,8 @@ namespace tasp {
 namespace gemv {
 
 template <>
-Fn pick<4>(int mode, int R, int XC) {
-    return pick_nb<4>(mode, R, XC);
+Fn pick<4>(int mode, int R, int XC, bool gs) {
+    return pick_nb<4>(mode, R, XC, gs);
 }
 
 }  // namespace gemv

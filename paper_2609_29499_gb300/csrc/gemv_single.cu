@@ -683,7 +683,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const GemvParams 
             for (int r = 0; r < R; ++r) {
                 int w = gi * R + r;
                 if (w >= p.rows) w = 0;  // padding row of a ragged last group: never stored
-                grow[r] = GS ? p.gscale + (size_t)panel_row<MODE>(p, w) * p.gcols : nullptr;
+                grow[r] = GS ? p.gscale + (size_t)panel_row<MODE>(p, w) * p.gld : nullptr;
             }
             dot_i8<R, XC, GS>(st, (int)p.ld, xd, p.nchunks, tid, v, grow, p.gshift,
                               GS && gsb ? reinterpret_cast<const uint16_t*>(st + (size_t)R * p.ld) : nullptr, p.gld);

@@ -891,7 +891,6 @@ int tasp_decode_step(tasp_session* const* sessions, int32_t n, const void* d_x_b
     if (!d_x_bf16) return fail(TASP_EINVAL, "d_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
     if (d_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
-    if (sh.qg && n > 1) return fail(TASP_EUNSUP, "groupwise stores decode one session per call");
     Session* const* ss = (Session* const*)sessions;
     cudaStream_t st = (cudaStream_t)stream;
     // groups of up to MAX_BATCH sessions share each weight pass
@@ -930,7 +929,6 @@ int tasp_decode_step_host(tasp_session* const* sessions, int32_t n, const void* 
     if (!h_x_bf16) return fail(TASP_EINVAL, "h_x_bf16 is NULL");
     const Shape& sh = p->store->sh;
     if (h_logits && sh.vocab == 0) return fail(TASP_EINVAL, "logits requested from a model without LM head");
-    if (sh.qg && n > 1) return fail(TASP_EUNSUP, "groupwise stores decode one session per call");
     cudaStream_t st = (cudaStream_t)stream;
     Session* const* ss = (Session* const*)sessions;
     for (int i0 = 0; i0 < n; i0 += MAX_BATCH) {

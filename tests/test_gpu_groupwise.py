@@ -1,7 +1,7 @@
 """GPU parity of groupwise INT8 stores (Table 1: group size 128, BF16 scales) against the
 oracle, through the C ABI: INT8 codes and BF16 group scales bit-exact on the store's panels,
-one-session decode elementwise per layer and end to end, the union step and prefill against
-the oracle, and batches of 2-4 sessions (not built for such a store) refused with EUNSUP."""
+one-session decode elementwise per layer and end to end, batches of 2-5 sessions, the union
+step and prefill against the oracle."""
 import dataclasses
 
 import numpy as np
@@ -181,17 +181,34 @@ def test_grouped_prefill_matches_oracle(tasp):
     plan.release()
 
 
-def test_batched_gemvs_refuse_grouped_stores(tasp):
+@pytest.mark.parametrize("n", [2, 4, 5])
+def test_grouped_batched_decode_matches_oracle(tasp, n):
+    # 2-4 sessions share each weight pass of the batched GEMVs (the chunk sums scaled by the
+    # row's group scale); five = a group of four plus one session on the single-vector kernels
     import torch
     sh = SHAPE
-    plan, _ = _plan(tasp, sh)
-    a, b = tasp.Session(plan, 8), tasp.Session(plan, 8)
-    for s in (a, b):
-        s.fill_synthetic(4, 1)
-    x = torch.zeros((2, sh.d), dtype=torch.bfloat16, device="cuda")
-    with pytest.raises(tasp.TaspError) as e:
-        tasp.decode_step([a, b], x)
-    assert e.value.code == tasp.EUNSUP
-    a.release()
-    b.release()
+    plan, mask = _plan(tasp, sh)
+    t_priors, kv_seeds = [700, 64, 5, 300, 33][:n], [7, 8, 9, 10, 11][:n]
+    ss = []
+    for tp, ks in zip(t_priors, kv_seeds):
+        se = tasp.Session(plan, tp + 4)
+        se.fill_synthetic(tp, ks)
+        ss.append(se)
+    steps = 3
+    xb = synth.step_inputs_bf16(19 + n, steps, n, sh.d)
+    x = bf16_tensor(xb)
+    hid = torch.empty((steps, n, sh.d), dtype=torch.float32, device="cuda")
+    logits = torch.empty((steps, n, sh.vocab), dtype=torch.float32, device="cuda")
+    for t in range(steps):
+        tasp.decode_step(ss, x[t], hid[t], logits[t])
+    torch.cuda.synchronize()
+    rows = np.arange(0, sh.vocab, 997)
+    for i in range(n):
+        assert ss[i].device_error() == 0
+        ref = forward.decode(sh, mask, synth.bf16_to_f32(xb[:, i]), t_priors[i], kv_seeds[i])
+        assert rel_l2(hid.cpu().numpy()[:, i], ref) <= TOL_E2E, i
+        lref = forward.final_logits(sh, ref, rows=rows)
+        assert rel_l2(logits.cpu().numpy()[:, i][:, rows], lref) <= TOL_E2E, i
+    for se in ss:
+        se.release()
     plan.release()
