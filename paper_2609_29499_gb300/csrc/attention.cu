@@ -26,6 +26,8 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <map>
+#include <mutex>
 
 #include "tasp_internal.h"
 #include "tc_ptx.cuh"
@@ -542,6 +544,49 @@ int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap) {
 }
 
 int attn_splits_max() { return CLUSTERS_MAX * 16; }
+
+namespace {
+// Clusters of `cs` CTAs of the attention kernel that the device holds at once (cached).
+int active_clusters(int dh, int g, int cs, bool tma) {
+    static std::mutex mu;
+    static std::map<int, int> cache;
+    const int key = ((dh * 16 + g) * 32 + cs) * 2 + (tma ? 1 : 0);
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+    int n = 0;
+    if (AttnFn fn = pick(dh, g, cs, tma)) {
+        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_of(dh, tma));
+        if (cs == 16) cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(cs, 1);
+        cfg.blockDim = dim3(AT_THREADS);
+        cfg.dynamicSmemBytes = smem_of(dh, tma);
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = cs;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
+        cudaGetLastError();
+    }
+    cache.emplace(key, n);
+    return n;
+}
+}  // namespace
+
+int attn_cluster_for(int m_kv, int nb, int max_tokens, int dh, int g, bool tma) {
+    const int c16 = attn_cluster(dh, g);
+    if (c16 < 16 || m_kv * nb <= 0) return c16;
+    auto waves = [&](int cs) {
+        const int act = active_clusters(dh, g, cs, tma);
+        const int n = m_kv * nb * (attn_splits(m_kv, max_tokens, 0, dh, g, cs) / cs);
+        return act > 0 ? (n + act - 1) / act : 1 << 20;
+    };
+    return waves(8) < waves(16) ? 8 : 16;
+}
 
 int launch_attention(const AttnParams& a, int dh, int g, int m_kv, int splits, int nb, cudaStream_t s,
                      int cs_cap) {

@@ -157,7 +157,7 @@ struct Op {
     int mode = 0;
     Params p{};
     AttnParams a{};
-    int m_kv = 0, S = 0;
+    int m_kv = 0, S = 0, cs = 16;
 };
 
 }  // namespace
@@ -186,8 +186,7 @@ int batch_attn_slots(const Plan& p, const Session* const* ss, int n, int sms) {
     int smax = 1;
     for (int b = 0; b < n; ++b)
         for (const LayerPlan& lp : p.layers)
-            smax = std::max(smax, attn_splits(lp.m_kv, ss[b]->max_tokens, sms, sh.dh, sh.g()) /
-                                      attn_cluster(sh.dh, sh.g()));
+            smax = std::max(smax, attn_splits(lp.m_kv, ss[b]->max_tokens, sms, sh.dh, sh.g(), 8) / 8);  // either size
     return smax;
 }
 
@@ -263,7 +262,9 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             a.q = bv.q;
             a.o = bv.o;
             a.q_stride = bv.q_stride;
-            int S = 0;
+            int S = 0, mt = 0;
+            for (int b = 0; b < n; ++b) mt = std::max(mt, bv.ss[b]->max_tokens);
+            const int cs = attn_cluster_for(lp.m_kv, n, mt, sh.dh, sh.g(), n <= MAX_BATCH);
             for (int b = 0; b < n; ++b) {
                 const Session& se = *bv.ss[b];
                 a.K[b] = se.K[l];
@@ -272,7 +273,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 a.max_tokens[b] = se.max_tokens;
                 a.m_kv[b] = lp.m_kv;
                 a.oslot[b] = lp.oslot;
-                S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g()));
+                S = std::max(S, attn_splits(lp.m_kv, se.max_tokens, di.sms, sh.dh, sh.g(), cs));
             }
             a.qscale = (float)(1.0 / std::sqrt((double)sh.dh) * 1.4426950408889634);
             a.tma = 1;
@@ -293,6 +294,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
             op.a = a;
             op.m_kv = lp.m_kv;
             op.S = S;
+            op.cs = cs;
             ops.push_back(op);
         }
         // K3: O-projection + residual
@@ -376,7 +378,7 @@ int enqueue_batch(const BatchView& bv, const StepTarget& t, cudaStream_t s, int 
                 rc = op.p.nb == 1 ? launch_gemv_single(op.mode, op.p, s) : launch_gemv(op.mode, op.p, s);
                 break;
             case Op::ATTN:
-                rc = launch_attention(op.a, sh.dh, sh.g(), op.m_kv, op.S, n, s);
+                rc = launch_attention(op.a, sh.dh, sh.g(), op.m_kv, op.S, n, s, op.cs);
                 break;
             case Op::COPY_HIDDEN: {
                 const cudaError_t e = cudaMemcpy2DAsync(t.hidden_out, (size_t)sh.d * 4, bv.x, (size_t)bv.x_stride * 4,

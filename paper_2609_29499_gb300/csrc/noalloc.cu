@@ -76,8 +76,7 @@ extern "C" int tasp_decode_step_static(tasp_session* s, const void* d_x_bf16, fl
     // every layer's attention partials must fit the static array
     for (const LayerPlan& lp : pl.layers) {
         // partial outputs are kept per cluster of the attention kernel
-        const size_t S = (size_t)attn_splits(lp.m_kv, se->max_tokens, di.sms, sh.dh, sh.g()) /
-                         (size_t)attn_cluster(sh.dh, sh.g());
+        const size_t S = (size_t)attn_splits(lp.m_kv, se->max_tokens, di.sms, sh.dh, sh.g(), 8) / 8;  // either size
         const size_t part = (size_t)lp.m_kv * S * sh.g() * sh.dh;
         const size_t ml = (size_t)lp.m_kv * S * sh.g() * 2;
         if (part > kPartFloats || ml > kMlFloats || (size_t)lp.m_kv > kTickets)

@@ -454,7 +454,7 @@ static int session_alloc(Plan* p, int max_tokens, Session** out) {
     se->max_tokens = max_tokens;
     int smax = 1;
     for (const LayerPlan& lp : p->layers)
-        smax = std::max(smax, attn_splits(lp.m_kv, max_tokens, di.sms, sh.dh, sh.g()) / attn_cluster(sh.dh, sh.g()));
+        smax = std::max(smax, attn_splits(lp.m_kv, max_tokens, di.sms, sh.dh, sh.g(), 8) / 8);  // either cluster size
     se->att_splits_max = smax;
     Layout lay;
     for (const LayerPlan& lp : p->layers) {

@@ -258,6 +258,9 @@ int attn_supported(int dh, int g);
 int attn_cluster(int dh, int g);  // CTAs per cluster of the attention kernel (16, else 8)
 int attn_splits(int m_kv, int max_tokens, int sms, int dh, int g, int cs_cap = 16);
 int attn_splits_max();
+// Cluster size for one launch of m_kv kept groups x nb sessions: 16, or 8 when 16-CTA clusters
+// would take more waves than 8-CTA ones (more clusters than the device holds at once)
+int attn_cluster_for(int m_kv, int nb, int max_tokens, int dh, int g, bool tma);
 // C[m][n] = scale[n] * sum_k A[m][k] B[n][k] on the tensor cores (prefill.cu's persistent
 // tcgen05 GEMM): FP16 A [M][lda], B [N][ldb], FP32 C [M][ldc]; K a multiple of 8.
 int gemm_f16_nt(const __half* A, int lda, int M, const __half* B, int ldb, int N, int K, const float* scale, float* C,
