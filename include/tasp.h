@@ -132,7 +132,8 @@ int tasp_compile_mask(const tasp_model_desc* model, const tasp_mask_desc* mask, 
  * (retained KV heads only, capacity T + max_new_tokens) holds the prompt's
  * keys/values. If d_logits_last != NULL it receives FP32 [vocab] logits of the
  * last prompt position. async on `stream`. *out receives the session.
- * Errors: EINVAL, ENOMEM, ECUDA, EUNSUP (vocab == 0 with d_logits_last). */
+ * Errors: EINVAL, ENOMEM, ECUDA, EUNSUP (vocab == 0 with d_logits_last, or d not
+ * a multiple of 8). */
 int tasp_prefill(tasp_plan* plan, const void* d_embeds_bf16, int32_t T, int32_t max_new_tokens, void* stream,
                  tasp_session** out, float* d_logits_last);
 
