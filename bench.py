@@ -12,7 +12,12 @@ Prints one JSON line (ms/token, lower is better) with the per-kernel roofline of
 the dominant kernel, an end-to-end figure through the host-buffer C-ABI call,
 clock samples, and the CPU oracle timed on the host as a baseline.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config 2|3]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config 1|2|3]
+                    [--dense | --mask groups|qheads] [--quant-group 128]
+                    [--workload decode|prefill|mixed|spectral] [--prompt T] [--union] [--layers L]
+
+The default decode line also carries the other workloads' figures (prefill of a 2,048-token
+prompt, the 16-turn union step) under "other_workloads" (--no-other-workloads skips them).
 """
 from __future__ import annotations
 
