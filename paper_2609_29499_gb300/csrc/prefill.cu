@@ -866,10 +866,15 @@ __global__ void __launch_bounds__(192, 2)
             float x[64];
             const int k0 = j * AT_KT;
             const int kv = min(qi + 1, kend) - k0;  // keys k0 + c with c < kv are visible
+            if (k0 + AT_KT <= min(q0 + 1, kend)) {  // every row of the CTA sees the whole tile
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                const float v = __uint_as_float(c < 32 ? v0[c] : v1[c - 32]);
-                x[c] = c < kv ? v : -INFINITY;  // causal
+                for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(c < 32 ? v0[c] : v1[c - 32]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 64; ++c) {
+                    const float v = __uint_as_float(c < 32 ? v0[c] : v1[c - 32]);
+                    x[c] = c < kv ? v : -INFINITY;  // causal
+                }
             }
             float mx[8];  // the row maximum as a tree (independent chains instead of one of 64)
 #pragma unroll
