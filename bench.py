@@ -490,6 +490,8 @@ def run_prefill(args, emit=True):
     tasp.load()
     wl = synth.CFG4
     sh = wl.shape if not args.layers else dataclasses.replace(wl.shape, L=args.layers)
+    if args.quant_group:  # the paper's groupwise store
+        sh = dataclasses.replace(sh, quant_group=args.quant_group)
     T, K, Wm = args.prompt, args.steps, args.warmup
     dec_steps = wl.steps
     plans, sessions, embs, flops = [], [], [], []
@@ -567,7 +569,8 @@ def run_prefill(args, emit=True):
            "unit": "ms", "n_gpus": 1, "steps": K, "warmup": Wm, "ms_per_step": round(ms, 3),
            "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f16xint8-f32acc",
            "data": "synthetic",
-           "config": {"workload": f"llama3_8b_prefill_{T}" + (f"_{args.layers}layers" if args.layers else ""),
+           "config": {"workload": f"llama3_8b_prefill_{T}" + (f"_{args.layers}layers" if args.layers else "") +
+                                  (f"_int8g{args.quant_group}" if args.quant_group else ""),
                       "masks": n, "tokens_per_s": round(T / (ms * 1e-3), 1),
                       "l2": "inputs larger than L2 (every prefill streams a plan's FP16 panels, ~8 GB)"},
            "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": peak, "unit": "TFLOP/s",
@@ -596,6 +599,8 @@ def run_mixed(args, emit=True):
     tasp.load()
     wl = synth.CFG5
     sh = wl.shape if not args.layers else dataclasses.replace(wl.shape, L=args.layers)
+    if args.quant_group:  # the paper's groupwise store
+        sh = dataclasses.replace(sh, quant_group=args.quant_group)
     K, Wm = args.steps, args.warmup
     turns = synth.turn_assignment(wl.x_seed, wl.n_turns, len(wl.masks), wl.p_dense, *wl.prompt_lens)
     n = len(turns)
@@ -718,7 +723,8 @@ def run_mixed(args, emit=True):
            "value": round(tok_s, 2), "unit": "tokens/s", "n_gpus": 1, "steps": K, "warmup": Wm,
            "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "int8w-f32", "data": "synthetic",
-           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else ""), "turns": n,
+           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else "") +
+                                  (f"_int8g{args.quant_group}" if args.quant_group else ""), "turns": n,
                       "plans": {("dense" if pi == len(wl.masks) else f"mask{pi}"): len(idx)
                                 for pi, idx in groups.items()},
                       "prompt_tokens": [T for _, T in turns], "panels": args.panels,
@@ -766,6 +772,9 @@ def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s, emi
     d, qd, df = sh.d, sh.Hq * sh.dh, sh.df
     qkv_rows = (sh.Hq + 2 * sh.Hkv) * sh.dh
     layer_w = qkv_rows * d + d * qd + 2 * df * d + d * df + 4 * (qkv_rows + d + 2 * df + d)
+    G = getattr(sh, "quant_group", 0)
+    if G:  # BF16 group scales: 2 bytes per G weights
+        layer_w += 2 * (qkv_rows * d + d * qd + 2 * df * d + d * df) // G
     lm = sh.vocab * d * 2
     kvb = 0
     for i, (pi, _) in enumerate(turns):
@@ -799,7 +808,8 @@ def run_mixed_union(args, tasp, wl, sh, turns, plans, sessions, xb, setup_s, emi
            "value": round(tok_s, 2), "unit": "tokens/s", "n_gpus": 1, "steps": K, "warmup": Wm,
            "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "int8w-f16", "data": "synthetic",
-           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else "") + "_union", "turns": n,
+           "config": {"workload": wl.name + (f"_{args.layers}layers" if args.layers else "") +
+                                  (f"_int8g{args.quant_group}" if args.quant_group else "") + "_union", "turns": n,
                       "plans": {("dense" if pi == len(wl.masks) else f"mask{pi}"): c for pi, c in groups.items()},
                       "prompt_tokens": [T for _, T in turns],
                       "l2": "inputs larger than L2 (each step streams the dense panels)"},

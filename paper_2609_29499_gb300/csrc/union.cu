@@ -249,11 +249,19 @@ __global__ void __launch_bounds__(SK_THREADS, SK_CTAS_PER_SM)
                 const int s = g % NST, ab = g % SK_NA;
                 __half2 gsc[8];  // grouped store: the scale of each 16-column chunk, times 2^SK_GS_EXP
                 if constexpr (GS) {
+                    const int gsh = __ffs(a.qg) - 1;  // the group size is a power of two
+                    if (a.qg >= SK_BK) {              // one group covers the whole k-block
+                        const float v = gsr ? __uint_as_float((uint32_t)__ldg(gsr + ((kb * SK_BK) >> gsh)) << 16) : 0.f;
+                        const __half2 h = __float2half2_rn(ldexpf(v, SK_GS_EXP));
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        const float v = gsr ? __uint_as_float((uint32_t)__ldg(gsr + (kb * SK_BK + 16 * c) / a.qg) << 16)
-                                            : 0.f;
-                        gsc[c] = __float2half2_rn(ldexpf(v, SK_GS_EXP));
+                        for (int c = 0; c < 8; ++c) gsc[c] = h;
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            const float v =
+                                gsr ? __uint_as_float((uint32_t)__ldg(gsr + ((kb * SK_BK + 16 * c) >> gsh)) << 16) : 0.f;
+                            gsc[c] = __float2half2_rn(ldexpf(v, SK_GS_EXP));
+                        }
                     }
                 }
                 mbar_wait(smem_u32(&full[s]), (g / NST) & 1, &abort_flag, a.err);
